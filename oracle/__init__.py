@@ -1,0 +1,217 @@
+"""CPU oracle of the W8A8 quantized linear layer (test infrastructure only).
+
+Only the tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
+``bench.py`` may import this package.  The product library never does, and the
+oracle never imports the product: the two share only the seeded input
+generators, which hold none of the method's arithmetic.
+
+The arithmetic lives in ``w8a8_oracle.c`` (plain C, ``-O2 -ffp-contract=off``,
+no intrinsics), compiled with gcc into ``oracle/_build/liboracle.so`` and called
+through ctypes on numpy arrays.  Each function follows the "INT8 W8A8" paragraph
+of the paper's Method section (Sec. 3); the INT8 GEMM and dequantizing epilogue
+are the fused kernel the paper lists as missing (Sec. 6, Limitations).
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+import threading
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "w8a8_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "liboracle.so")
+_lock = threading.Lock()
+_lib = None
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle with gcc (OpenMP over GEMM rows when available)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    base = ["gcc", "-O2", "-ffp-contract=off", "-fno-fast-math", "-std=c11",
+            "-shared", "-fPIC", _SRC, "-o", _LIB_PATH + ".tmp", "-lm"]
+    try:
+        subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True,
+                       capture_output=True)
+    except subprocess.CalledProcessError:
+        subprocess.run(base, check=True, capture_output=True)
+    os.replace(_LIB_PATH + ".tmp", _LIB_PATH)
+    return _LIB_PATH
+
+
+def _load():
+    global _lib
+    with _lock:
+        if _lib is None:
+            path = build()
+            lib = ctypes.CDLL(path)
+            P = ctypes.c_void_p
+            I64 = ctypes.c_int64
+            lib.oracle_channel_absmax.argtypes = [P, I64, I64, P]
+            lib.oracle_smooth_scales.argtypes = [P, P, I64, I64, ctypes.c_float, P]
+            lib.oracle_quantize_weights.argtypes = [P, P, I64, I64, P, P]
+            lib.oracle_quant_act.argtypes = [P, P, I64, I64, P, P, P]
+            lib.oracle_gemm_i32.argtypes = [P, P, I64, I64, I64, I64, I64, P]
+            lib.oracle_epilogue.argtypes = [P, P, P, P, I64, I64, P]
+            lib.oracle_linear_rows.argtypes = [P, P, P, P, P, I64, I64, I64,
+                                               I64, I64, P, P]
+            lib.oracle_f32_to_bf16_rne.argtypes = [ctypes.c_float]
+            lib.oracle_f32_to_bf16_rne.restype = ctypes.c_uint16
+            lib.oracle_bf16_to_f32.argtypes = [ctypes.c_uint16]
+            lib.oracle_bf16_to_f32.restype = ctypes.c_float
+            lib.oracle_quantize_value.argtypes = [ctypes.c_float]
+            lib.oracle_quantize_value.restype = ctypes.c_int8
+            lib.oracle_epilogue_value.argtypes = [ctypes.c_int32, ctypes.c_float,
+                                                  ctypes.c_float, P]
+            lib.oracle_epilogue_value.restype = ctypes.c_uint16
+            lib.oracle_num_threads.restype = ctypes.c_int
+            _lib = lib
+    return _lib
+
+
+def _ptr(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return None if a is None else np.ascontiguousarray(a, dtype=dtype)
+
+
+def num_threads() -> int:
+    """Threads the oracle's GEMM row loop uses."""
+    return int(_load().oracle_num_threads())
+
+
+# --------------------------------------------------------------------------
+# scalar helpers (bit patterns of bf16 are carried as uint16)
+# --------------------------------------------------------------------------
+
+def f32_to_bf16_rne(x) -> np.ndarray:
+    """fp32 -> bf16 bit pattern, round to nearest, ties to even."""
+    lib = _load()
+    x = np.asarray(x, dtype=np.float32)
+    out = np.empty(x.shape, dtype=np.uint16)
+    flat_in, flat_out = x.reshape(-1), out.reshape(-1)
+    for i in range(flat_in.size):
+        flat_out[i] = lib.oracle_f32_to_bf16_rne(float(flat_in[i]))
+    return out
+
+
+def bf16_to_f32(h) -> np.ndarray:
+    """bf16 bit pattern -> fp32 (exact)."""
+    h = np.asarray(h, dtype=np.uint16)
+    return (h.astype(np.uint32) << 16).view(np.float32)
+
+
+def quantize_value(v: float) -> int:
+    """clamp(round_half_even(v), -127, 127) in fp32."""
+    return int(_load().oracle_quantize_value(float(np.float32(v))))
+
+
+# --------------------------------------------------------------------------
+# the layer, step by step (Sec. 3, "INT8 W8A8")
+# --------------------------------------------------------------------------
+
+def channel_absmax(X_bf16: np.ndarray) -> np.ndarray:
+    """Calibration statistic s_j = max_t |X_tj| over a [T, K] bf16 batch."""
+    X = _c(X_bf16, np.uint16)
+    M, K = X.shape
+    s = np.empty(K, dtype=np.float32)
+    _load().oracle_channel_absmax(_ptr(X), M, K, _ptr(s))
+    return s
+
+
+def smooth_scales(s: np.ndarray, W: np.ndarray, alpha: float) -> np.ndarray:
+    """lambda_j = s_j^alpha / max_i |W_ij|^(1 - alpha)  (W is [N, K])."""
+    s = _c(s, np.float32)
+    W = _c(W, np.float32)
+    N, K = W.shape
+    lam = np.empty(K, dtype=np.float32)
+    _load().oracle_smooth_scales(_ptr(s), _ptr(W), N, K, float(alpha), _ptr(lam))
+    return lam
+
+
+def quantize_weights(W: np.ndarray, lam: np.ndarray | None):
+    """Per-output-row symmetric INT8 of W diag(lambda): returns (Wq, sw)."""
+    W = _c(W, np.float32)
+    lam = _c(lam, np.float32)
+    N, K = W.shape
+    Wq = np.empty((N, K), dtype=np.int8)
+    sw = np.empty(N, dtype=np.float32)
+    _load().oracle_quantize_weights(_ptr(W), _ptr(lam), N, K, _ptr(Wq), _ptr(sw))
+    return Wq, sw
+
+
+def quant_act(X_bf16: np.ndarray, lam: np.ndarray | None):
+    """Per-token dynamic INT8 of X diag(lambda)^-1: returns (Xq, sx)."""
+    X = _c(X_bf16, np.uint16)
+    lam = _c(lam, np.float32)
+    M, K = X.shape
+    Xq = np.empty((M, K), dtype=np.int8)
+    sx = np.empty(M, dtype=np.float32)
+    tmp = np.empty(K, dtype=np.float32)
+    _load().oracle_quant_act(_ptr(X), _ptr(lam), M, K, _ptr(Xq), _ptr(sx), _ptr(tmp))
+    return Xq, sx
+
+
+def gemm_i32(Xq: np.ndarray, Wq: np.ndarray, rows: tuple[int, int] | None = None):
+    """Exact acc = Xq Wq^T (int32) for the rows [m0, m1) of Xq."""
+    Xq = _c(Xq, np.int8)
+    Wq = _c(Wq, np.int8)
+    M, K = Xq.shape
+    N, K2 = Wq.shape
+    assert K == K2
+    m0, m1 = rows if rows is not None else (0, M)
+    acc = np.empty((m1 - m0, N), dtype=np.int32)
+    _load().oracle_gemm_i32(_ptr(Xq), _ptr(Wq), M, N, K, m0, m1, _ptr(acc))
+    return acc
+
+
+def epilogue(acc: np.ndarray, sx: np.ndarray, sw: np.ndarray, bias: np.ndarray | None):
+    """y = bf16_rne(((float)acc * sx_m) * sw_n + b_n), as uint16 bit patterns."""
+    acc = _c(acc, np.int32)
+    sx = _c(sx, np.float32)
+    sw = _c(sw, np.float32)
+    bias = _c(bias, np.float32)
+    rows, N = acc.shape
+    Y = np.empty((rows, N), dtype=np.uint16)
+    _load().oracle_epilogue(_ptr(acc), _ptr(sx), _ptr(sw), _ptr(bias), rows, N, _ptr(Y))
+    return Y
+
+
+def linear(Xq, sx, Wq, sw, bias, rows: tuple[int, int] | None = None):
+    """Quantized linear a4+a5 for rows [m0, m1): bf16 bit patterns [m1-m0, N]."""
+    Xq = _c(Xq, np.int8)
+    Wq = _c(Wq, np.int8)
+    sx = _c(sx, np.float32)
+    sw = _c(sw, np.float32)
+    bias = _c(bias, np.float32)
+    M, K = Xq.shape
+    N = Wq.shape[0]
+    m0, m1 = rows if rows is not None else (0, M)
+    acc = np.empty((m1 - m0, N), dtype=np.int32)
+    Y = np.empty((m1 - m0, N), dtype=np.uint16)
+    _load().oracle_linear_rows(_ptr(Xq), _ptr(sx), _ptr(Wq), _ptr(sw), _ptr(bias),
+                               M, N, K, m0, m1, _ptr(acc), _ptr(Y))
+    return Y
+
+
+def linear_dual(branches, rows=None):
+    """The dual-branch layer is the single-branch layer applied to each branch."""
+    return [linear(*br, rows=rows) for br in branches]
+
+
+def full_layer(X_bf16, W, bias, s, alpha):
+    """Offline a1+a2, then per-call a3+a4+a5; returns a dict of every stage."""
+    lam = smooth_scales(s, W, alpha)
+    Wq, sw = quantize_weights(W, lam)
+    Xq, sx = quant_act(X_bf16, lam)
+    Y = linear(Xq, sx, Wq, sw, bias)
+    return {"lambda": lam, "Wq": Wq, "sw": sw, "Xq": Xq, "sx": sx, "Y": Y}
