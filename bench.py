@@ -1,0 +1,395 @@
+"""Benchmark of the W8A8 quantized linear on GB300.
+
+One step = one pass of the per-call hot path of one quantized linear over one
+batch of tokens: per-token activation quantization (a3) followed by the INT8
+GEMM with the fused dequantizing epilogue (a4 + a5).  The offline steps (a1
+smoothing vector, a2 weight quantization) run once per layer before the timed
+region and are timed separately under "offline_ms".
+
+Default workload: the DiT attention QKV projection, M=4608 tokens, K=4096,
+N=12288 (seeded synthetic inputs).  `value` is whole-job INT8 TOPS
+(2*M*N*K per step, summed over ranks, over the max time over ranks).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+N > 1 runs N independent replicas (the layer does not shard; no collective on
+the data path); --impl reference times the CPU oracle on a bounded row sample.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import math
+import os
+import statistics
+import subprocess
+import sys
+import tempfile
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+L2_BYTES = 129 * 2**20
+PEAKS_PATH = os.path.join(ROOT, "MEASURED_PEAKS.json")
+FALLBACK_PEAKS = {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0}
+
+
+def load_peaks():
+    try:
+        with open(PEAKS_PATH) as f:
+            p = json.load(f)
+        return p, "measured"
+    except (OSError, ValueError):
+        return dict(FALLBACK_PEAKS), "fallback"
+
+
+def dist_env():
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return ws, rank, local
+
+
+def max_over_ranks(value: float, ws: int, device=None) -> float:
+    """Max of a per-rank float over all ranks (identity for one rank)."""
+    if ws <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def sum_over_ranks(value: float, ws: int, device=None) -> float:
+    if ws <= 1:
+        return value
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([value], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.SUM)
+    return float(t.item())
+
+
+class ClockSampler:
+    """nvidia-smi samples of SM clock and throttle reasons during a region."""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+        self.path = None
+
+    def start(self):
+        fd, self.path = tempfile.mkstemp(suffix=".csv")
+        os.close(fd)
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=open(self.path, "w"), stderr=subprocess.DEVNULL)
+        except OSError:
+            self.proc = None
+        time.sleep(0.25)
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except subprocess.TimeoutExpired:
+            self.proc.kill()
+        rows = []
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                rows.append((float(parts[1]), float(parts[2]), float(parts[3]), parts[5:9]))
+            except ValueError:
+                continue
+        os.unlink(self.path)
+        if not rows:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["no samples"]}
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        reasons = sorted({names[i] for r in rows for i, v in enumerate(r[3]) if v == "Active"})
+        # median over samples taken while the GPU was busy (power above idle)
+        pw = [r[2] for r in rows]
+        busy = [r for r in rows if r[2] >= 0.5 * max(pw)] or rows
+        return {"sm_mhz": statistics.median(r[0] for r in busy),
+                "sm_max_mhz": max(r[1] for r in rows),
+                "reasons": reasons, "samples": len(rows)}
+
+
+# --------------------------------------------------------------- reference
+
+def cpu_oracle_sample(case, target_s: float = 10.0, max_rows: int | None = None):
+    """Time the CPU oracle (a3 + a4 + a5) on a bounded row sample of the
+    workload.  Returns (tops, seconds, rows, cores)."""
+    import oracle
+    oracle.build()
+    s = oracle.channel_absmax(case.X_cal)
+    lam = oracle.smooth_scales(s, case.W[0], case.alpha)
+    Wq, sw = oracle.quantize_weights(case.W[0], lam)
+    M, K = case.X[0].shape
+    N = Wq.shape[0]
+    cores = oracle.num_threads()
+
+    def run(rows):
+        t0 = time.perf_counter()
+        Xq, sx = oracle.quant_act(case.X[0][:rows], lam)
+        oracle.linear(Xq, sx, Wq, sw, case.bias[0])
+        return time.perf_counter() - t0
+
+    probe = min(M, 16)
+    dt = run(probe)
+    rows = int(min(M if max_rows is None else max_rows,
+                   max(probe, probe * target_s / max(dt, 1e-6))))
+    dt = run(rows)
+    tops = 2.0 * rows * N * K / dt / 1e12
+    return tops, dt, rows, cores
+
+
+def run_reference(args):
+    from paper_2606_12280_gb300 import workloads as wl
+    ws, rank, _ = dist_env()
+    if rank != 0:
+        return 0
+    case = wl.workload_cases(args.workload)[0]
+    M, K = case.X[0].shape
+    N = case.W[0].shape[0]
+    # each step is a bounded row sample sized so the whole run ends in minutes
+    per_step_s = max(1.0, 120.0 / max(1, args.steps + args.warmup))
+    tops0, dt0, rows, cores = cpu_oracle_sample(case, target_s=per_step_s)
+    times = []
+    import oracle
+    s = oracle.channel_absmax(case.X_cal)
+    lam = oracle.smooth_scales(s, case.W[0], case.alpha)
+    Wq, sw = oracle.quantize_weights(case.W[0], lam)
+    for i in range(args.warmup + args.steps):
+        t0 = time.perf_counter()
+        Xq, sx = oracle.quant_act(case.X[0][:rows], lam)
+        oracle.linear(Xq, sx, Wq, sw, case.bias[0])
+        dt = time.perf_counter() - t0
+        if i >= args.warmup:
+            times.append(dt)
+    total = sum(times)
+    value = 2.0 * rows * N * K * len(times) / total / 1e12
+    sample = f"{rows} of {M} tokens per step (a3+a4+a5 on the CPU oracle)"
+    line = {
+        "impl": "reference", "metric": METRIC, "value": value, "unit": "TOPS",
+        "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": 1e3 * total / len(times), "higher_is_better": True,
+        "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
+        "config": {"workload": args.workload, "M": M, "K": K, "N": N},
+        "cpu_baseline": {"value": value, "unit": "TOPS", "cores": cores, "kind": "oracle",
+                         "sample": sample},
+        "e2e": {"value": value, "unit": "TOPS", "h2d_bytes_per_step": 0,
+                "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(line))
+    return 0
+
+
+METRIC = "W8A8 linear INT8 TOPS (act-quant + INT8 GEMM + fused dequant epilogue)"
+
+
+# --------------------------------------------------------------------- ours
+
+def run_ours(args):
+    import torch
+
+    from paper_2606_12280_gb300 import w8a8
+    from paper_2606_12280_gb300 import workloads as wl
+
+    ws, rank, local = dist_env()
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+    if args.engine is not None:
+        w8a8.set_gemm_engine(args.engine)
+    w8a8.lib()
+
+    case = wl.workload_cases(args.workload)[0]
+    M, K = case.X[0].shape
+    N = case.W[0].shape[0]
+
+    def bf(a):
+        return torch.from_numpy(a.view(np.int16)).view(torch.bfloat16).to(dev)
+
+    stream = torch.cuda.current_stream()
+    X_cal = bf(case.X_cal)
+    W = torch.from_numpy(case.W[0]).to(dev)
+    bias = torch.from_numpy(case.bias[0]).to(dev)
+
+    # offline: calibration statistic, smoothing vector, weight quantization
+    e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    e[0].record()
+    s = w8a8.channel_absmax(X_cal)
+    e[1].record()
+    lam = w8a8.smooth_scales(s, W, case.alpha)
+    e[2].record()
+    Wq, sw = w8a8.quantize_weights(W, lam)
+    e[3].record()
+    torch.cuda.synchronize()
+    offline = {"channel_absmax": e[0].elapsed_time(e[1]), "smooth_scales": e[1].elapsed_time(e[2]),
+               "quantize_weights": e[2].elapsed_time(e[3])}
+
+    # rotate input sets so the bytes touched between two uses of one set
+    # exceed L2 (no flush needed): each set holds its own X and Wq copy
+    set_bytes = 2 * M * K + M * K + N * K + 2 * M * N
+    n_sets = max(2, math.ceil(2 * L2_BYTES / set_bytes))
+    X0 = bf(case.X[0])
+    Xs = [X0] + [X0.clone() for _ in range(n_sets - 1)]
+    Wqs = [Wq] + [Wq.clone() for _ in range(n_sets - 1)]
+    Xqs = [torch.empty(M, K, dtype=torch.int8, device=dev) for _ in range(n_sets)]
+    sxs = [torch.empty(M, dtype=torch.float32, device=dev) for _ in range(n_sets)]
+    Ys = [torch.empty(M, N, dtype=torch.bfloat16, device=dev) for _ in range(n_sets)]
+
+    def step(i, ev=None):
+        j = i % n_sets
+        if ev is not None:
+            ev[0].record(stream)
+        w8a8.quant_act(Xs[j], lam, Xq=Xqs[j], x_scale=sxs[j], stream=stream)
+        if ev is not None:
+            ev[1].record(stream)
+        w8a8.linear(Xqs[j], sxs[j], Wqs[j], sw, bias, Y=Ys[j], stream=stream)
+        if ev is not None:
+            ev[2].record(stream)
+
+    for i in range(args.warmup):
+        step(i)
+    torch.cuda.synchronize()
+    if w8a8.device_status(stream) != 0:
+        raise RuntimeError("device error word set during warm-up")
+
+    evs = [[torch.cuda.Event(enable_timing=True) for _ in range(3)] for _ in range(args.steps)]
+    clocks = ClockSampler(local) if rank == 0 or True else None
+    clocks.start()
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    t_start = torch.cuda.Event(enable_timing=True)
+    t_end = torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    for i in range(args.steps):
+        step(args.warmup + i, evs[i])
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    if ws > 1:
+        torch.distributed.barrier()
+    torch.cuda.synchronize()
+    clk = clocks.stop()
+    total_ms = t_start.elapsed_time(t_end)
+    quant_ms = [ev[0].elapsed_time(ev[1]) for ev in evs]
+    gemm_ms = [ev[1].elapsed_time(ev[2]) for ev in evs]
+    if w8a8.device_status(stream) != 0:
+        raise RuntimeError("device error word set during the timed region")
+
+    total_ms = max_over_ranks(total_ms, ws, dev)
+    ops_step = 2.0 * M * N * K
+    all_ops = sum_over_ranks(ops_step * args.steps, ws, dev)
+    value = all_ops / (total_ms * 1e-3) / 1e12
+
+    # end to end through the public API with host buffers: H2D of X, a3, a4+a5,
+    # D2H of Y, every step
+    X_host = torch.from_numpy(case.X[0].view(np.int16)).view(torch.bfloat16).pin_memory()
+    Y_host = torch.empty(M, N, dtype=torch.bfloat16).pin_memory()
+    Xd = torch.empty(M, K, dtype=torch.bfloat16, device=dev)
+    e2e_steps = max(3, min(args.steps, 10))
+
+    def e2e_step():
+        Xd.copy_(X_host, non_blocking=True)
+        Y = w8a8.quantized_linear_forward(Xd, lam, Wq, sw, bias, stream=stream)
+        Y_host.copy_(Y, non_blocking=True)
+
+    for _ in range(2):
+        e2e_step()
+    torch.cuda.synchronize()
+    if ws > 1:
+        torch.distributed.barrier()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(e2e_steps):
+        e2e_step()
+    b.record(stream)
+    torch.cuda.synchronize()
+    e2e_ms = max_over_ranks(a.elapsed_time(b), ws, dev)
+    e2e_value = sum_over_ranks(ops_step * e2e_steps, ws, dev) / (e2e_ms * 1e-3) / 1e12
+
+    peaks, peak_kind = load_peaks()
+    gemm_avg = sum(gemm_ms) / len(gemm_ms)
+    quant_avg = sum(quant_ms) / len(quant_ms)
+    gemm_tflops = ops_step / (gemm_avg * 1e-3) / 1e12
+    engine = w8a8.get_gemm_engine()
+    peak_t = peaks["bf16_tflops"]
+    quant_bytes = 3.0 * M * K + 4.0 * M + 4.0 * K
+    quant_gbs = quant_bytes / (quant_avg * 1e-3) / 1e9
+
+    line = None
+    if rank == 0:
+        cpu = None
+        if ws == 1 and not args.no_cpu_baseline:
+            tops_cpu, dt_cpu, rows, cores = cpu_oracle_sample(case, target_s=args.cpu_seconds)
+            cpu = {"value": tops_cpu, "unit": "TOPS", "cores": cores, "kind": "oracle",
+                   "sample": f"{rows} of {M} tokens (a3+a4+a5), {dt_cpu:.1f} s of CPU work"}
+        line = {
+            "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
+            "config": {"workload": args.workload, "M": M, "K": K, "N": N, "alpha": case.alpha,
+                       "l2": f"{n_sets} rotating input sets of {set_bytes / 2**20:.0f} MiB "
+                             f"(> L2 between reuses), no flush",
+                       "gemm_engine": "tcgen05" if engine == 1 else "mma.sync"},
+            "roofline": {"bound": "tensor", "achieved": gemm_tflops, "peak": peak_t,
+                         "unit": "TFLOP/s", "frac": gemm_tflops / peak_t, "traffic": None,
+                         "kernel": "w8a8_linear (a4+a5)",
+                         "peak_source": f"{peak_kind} bf16 dense burst (the fp16/bf16 tensor "
+                                        f"datapath the exact-integer GEMM runs on)"},
+            "act_quant": {"bound": "hbm", "achieved": quant_gbs, "peak": peaks["hbm_gbs"],
+                          "unit": "GB/s", "frac": quant_gbs / peaks["hbm_gbs"],
+                          "ms": quant_avg, "bytes": quant_bytes},
+            "gemm_ms": gemm_avg, "offline_ms": offline,
+            "cpu_baseline": cpu,
+            "e2e": {"value": e2e_value, "unit": "TOPS", "h2d_bytes_per_step": 2 * M * K,
+                    "d2h_bytes_per_step": 2 * M * N},
+            "gpu_launches": 2 * args.steps,
+            "clocks": clk,
+        }
+        print(json.dumps(line))
+    if ws > 1:
+        torch.distributed.destroy_process_group()
+    return 0
+
+
+def main(argv=None):
+    p = argparse.ArgumentParser()
+    p.add_argument("--gpus", type=int, default=1)
+    p.add_argument("--steps", type=int, default=20)
+    p.add_argument("--warmup", type=int, default=5)
+    p.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    p.add_argument("--workload", default="qkv_m4608_k4096_n12288")
+    p.add_argument("--engine", type=int, default=None, help="1 tcgen05, 0 mma.sync")
+    p.add_argument("--no-cpu-baseline", action="store_true")
+    p.add_argument("--cpu-seconds", type=float, default=10.0)
+    args = p.parse_args(argv)
+    if args.warmup < 3:
+        p.error("--warmup must be >= 3")
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_ours(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -1,0 +1,188 @@
+/*
+ * w8a8.h -- C ABI of the GB300 (sm_103a) W8A8 quantized linear layer.
+ *
+ * The layer is the INT8 W8A8 recipe of "Quantizing a Dual-Branch Flow-Matching
+ * Diffusion Transformer for Consumer GPUs" (Sec. 3, Method, paragraph
+ * "INT8 W8A8"): per-output-channel symmetric INT8 weights, per-token dynamic
+ * symmetric INT8 activations, SmoothQuant outlier migration with
+ *     lambda_j = s_j^alpha / max_i |W_ij|^(1 - alpha),
+ * activations divided by lambda and weights multiplied by it before
+ * quantization.  The INT8 x INT8 -> INT32 product with a fused dequantizing
+ * epilogue is the kernel the paper reports as missing (Sec. 5, Efficiency;
+ * Sec. 6, Limitations), and the two separate-weight branches (conditional and
+ * unconditional) of its classifier-free-guidance DiT (Sec. 1; Sec. 3,
+ * Setting) run as one grouped launch.
+ *
+ * Conventions shared by every entry point
+ *   - Every pointer is a DEVICE pointer owned by the caller (for example the
+ *     data_ptr() of a CUDA tensor).  The library allocates nothing and never
+ *     frees anything.  Every base pointer must be 16-byte aligned.
+ *   - Matrices are row-major and dense (row stride = number of columns).
+ *     X [M,K] activations (tokens x input channels), W / Wq [N,K] weights
+ *     (output channels x input channels, the nn.Linear layout), Y [M,N].
+ *   - bf16 values travel as their 16-bit patterns (uint16_t).
+ *   - `stream` is a cudaStream_t (NULL = the legacy default stream).  Every
+ *     call only enqueues work on that stream and returns at once; results are
+ *     ready when the stream reaches them.  Calls on one stream are ordered.
+ *   - Shapes: M >= 0 (M == 0 is a no-op that returns W8A8_OK), N > 0 and a
+ *     multiple of 8, K > 0 and a multiple of 16, K <= 133143 (so that
+ *     K * 127^2 fits in int32).
+ *   - Arithmetic is IEEE binary32 with round-to-nearest-even on every step and
+ *     no fused multiply-add, so INT8 codes and FP32 scales are reproducible
+ *     bit for bit; rounding to INT8 is half-to-even with a symmetric clamp
+ *     to [-127, 127]; the INT32 product is exact.
+ *   - Errors: argument checks run on the host before anything is enqueued.
+ *     W8A8_ERR_INVALID_ARG (null pointer, alpha outside [0,1]),
+ *     W8A8_ERR_UNSUPPORTED_SHAPE, W8A8_ERR_MISALIGNED (a pointer not 16-byte
+ *     aligned) leave the stream untouched.  W8A8_ERR_CUDA reports a launch
+ *     failure.  The library keeps one device-side error word (see
+ *     w8a8_device_status); it holds no other state.
+ */
+#ifndef W8A8_H
+#define W8A8_H
+
+#include <stdint.h>
+
+#if defined(__GNUC__)
+#define W8A8_API __attribute__((visibility("default")))
+#else
+#define W8A8_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+    W8A8_OK = 0,
+    W8A8_ERR_INVALID_ARG = 1,
+    W8A8_ERR_UNSUPPORTED_SHAPE = 2,
+    W8A8_ERR_MISALIGNED = 3,
+    W8A8_ERR_CUDA = 4,
+    W8A8_ERR_TIMEOUT = 5
+} w8a8_status;
+
+/* Largest K for which K * 127 * 127 < 2^31. */
+#define W8A8_MAX_K 133143
+
+/* Human-readable name of a status code (static storage, never NULL). */
+W8A8_API const char *w8a8_status_string(w8a8_status status);
+
+/*
+ * Calibration statistic s_j = max_t |X_tj| over a batch of T tokens: the
+ * per-channel activation scale that feeds the smoothing vector (Sec. 3,
+ * "INT8 W8A8", where s is measured by a calibration pass over held-out
+ * prompts).
+ *   X      [T,K] bf16, read.
+ *   s      [K] fp32, written (overwritten, not accumulated).
+ */
+W8A8_API w8a8_status w8a8_channel_absmax(const uint16_t *X, int T, int K, float *s,
+                                void *stream);
+
+/*
+ * a1. Smoothing vector (Sec. 3, "INT8 W8A8"):
+ *     lambda_j = s_j^alpha / m_j^(1-alpha),  m_j = max_i |W_ij| (over output
+ *     rows i of input channel j).  s_j == 0 or m_j == 0 gives lambda_j = 1.
+ *     alpha in {0, 1/2, 1} is evaluated with correctly rounded fp32
+ *     operations (sqrt(s)/sqrt(m), 1/m, s); any other alpha in binary64 and
+ *     rounded once.
+ *   act_absmax [K] fp32 (s), read.   W [N,K] fp32, read.
+ *   smooth     [K] fp32 (lambda), written; also used as working storage for
+ *              m_j during the call.
+ *   alpha      in [0, 1], else W8A8_ERR_INVALID_ARG.
+ */
+W8A8_API w8a8_status w8a8_smooth_scales(const float *act_absmax, const float *W, int N,
+                               int K, float alpha, float *smooth, void *stream);
+
+/*
+ * a2. Per-output-channel symmetric INT8 weights of W' = W diag(lambda)
+ * (Sec. 3, "INT8 W8A8", per-channel weights; weights multiplied by lambda):
+ *     w'_ij = W_ij * lambda_j;  a_i = max_j |w'_ij|;
+ *     w_scale_i = a_i / 127;  Wq_ij = clamp(rne(w'_ij * (127 / a_i)), +-127);
+ *     an all-zero row gives w_scale_i = 0 and codes 0.
+ *   W       [N,K] fp32, read.   smooth [K] fp32 or NULL (lambda = 1).
+ *   Wq      [N,K] int8, written.   w_scale [N] fp32, written.
+ */
+W8A8_API w8a8_status w8a8_quantize_weights(const float *W, const float *smooth, int N,
+                                  int K, int8_t *Wq, float *w_scale,
+                                  void *stream);
+
+/*
+ * a3. Per-token dynamic INT8 activations of X' = X diag(lambda)^-1
+ * (Sec. 3, "INT8 W8A8", per-token dynamic activations; activations divided
+ * by lambda, implemented as a multiply by the correctly rounded 1/lambda_j):
+ *     x'_mj = X_mj * (1/lambda_j);  a_m = max_j |x'_mj|;
+ *     x_scale_m = a_m / 127;  Xq_mj = clamp(rne(x'_mj * (127 / a_m)), +-127);
+ *     an all-zero token gives x_scale_m = 0 and codes 0.
+ *   X       [M,K] bf16, read.   smooth [K] fp32 or NULL (lambda = 1).
+ *   Xq      [M,K] int8, written.   x_scale [M] fp32, written.
+ * One pass over X: reads 2MK bytes, writes MK + 4M.
+ */
+W8A8_API w8a8_status w8a8_quant_act(const uint16_t *X, const float *smooth, int M,
+                           int K, int8_t *Xq, float *x_scale, void *stream);
+
+/*
+ * a4 + a5. Quantized linear with the dequantizing epilogue fused:
+ *     acc_mn = sum_k Xq_mk * Wq_nk          (exact int32)
+ *     Y_mn   = bf16_rne(((float)acc_mn * x_scale_m) * w_scale_n + bias_n)
+ *   Xq [M,K] int8, x_scale [M] fp32, Wq [N,K] int8, w_scale [N] fp32,
+ *   bias [N] fp32 or NULL (no bias), all read.   Y [M,N] bf16, written.
+ */
+W8A8_API w8a8_status w8a8_linear(const int8_t *Xq, const float *x_scale,
+                        const int8_t *Wq, const float *w_scale,
+                        const float *bias, int M, int N, int K, uint16_t *Y,
+                        void *stream);
+
+/* One branch of the dual-branch (classifier-free guidance) layer. */
+typedef struct {
+    const int8_t *Xq;      /* [M,K] int8 */
+    const float *x_scale;  /* [M] fp32 */
+    const int8_t *Wq;      /* [N,K] int8 */
+    const float *w_scale;  /* [N] fp32 */
+    const float *bias;     /* [N] fp32 or NULL */
+    uint16_t *Y;           /* [M,N] bf16, written */
+    int M;                 /* tokens of this branch, >= 0 */
+} w8a8_branch;
+
+/*
+ * a6. The same linear layer for both separate-weight branches (conditional
+ * br[0], unconditional br[1]; Sec. 1 and Sec. 3 "Setting": two
+ * separate-weight copies of the backbone, 211 linears each) in ONE launch
+ * whose tile space covers both.  The branches share N and K; each has its
+ * own M, activations, weights, scales, bias and output.  Results are
+ * bitwise identical to two w8a8_linear calls.
+ *   br  host pointer to an array of 2 w8a8_branch (read during the call only).
+ */
+W8A8_API w8a8_status w8a8_linear_dual(const w8a8_branch *br, int N, int K,
+                             void *stream);
+
+/*
+ * Test export of a4 alone: acc = Xq Wq^T as int32 [M,N], written, so that the
+ * exact integer product can be compared bit for bit.  Same shape rules.
+ */
+W8A8_API w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int M,
+                                int N, int K, int32_t *acc, void *stream);
+
+/*
+ * The GEMM engine that w8a8_linear, w8a8_linear_dual and w8a8_debug_gemm_i32
+ * use on this device: 1 = tcgen05 tensor cores (exact integer products on the
+ * fp16 datapath, see the design notes), 0 = warp-level mma.sync s8 (legacy
+ * tensor path).  w8a8_set_gemm_engine(-1) restores the default (tcgen05);
+ * other values give W8A8_ERR_INVALID_ARG.  The setting is process-wide.
+ */
+W8A8_API w8a8_status w8a8_set_gemm_engine(int engine);
+W8A8_API int w8a8_get_gemm_engine(void);
+
+/*
+ * Waits for `stream`, then reads and clears the library's device-side error
+ * word on the current device.  Kernels that wait on barriers give up after a
+ * bounded number of polls, record a code there and return; this call then
+ * reports W8A8_ERR_TIMEOUT.  *detail (optional) receives the raw word.
+ */
+W8A8_API w8a8_status w8a8_device_status(void *stream, uint32_t *detail);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* W8A8_H */

@@ -1,0 +1,177 @@
+// api.cu -- the C ABI (include/w8a8.h): argument checks, then stream-ordered
+// launches.  No allocation, no synchronisation (except w8a8_device_status).
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "../../include/w8a8.h"
+#include "launch.h"
+
+namespace {
+
+// The library's single device-side error word: kernels with bounded waits
+// record a nonzero code here instead of spinning forever.
+__device__ unsigned int g_w8a8_device_error = 0;
+
+int g_engine = 1;   // 1 = tcgen05, 0 = mma.sync
+
+bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+w8a8_status check_mk(int M, int K) {
+    if (M < 0 || K <= 0 || (K % 16) != 0 || K > W8A8_MAX_K) return W8A8_ERR_UNSUPPORTED_SHAPE;
+    return W8A8_OK;
+}
+
+w8a8_status check_nk(int N, int K) {
+    if (N <= 0 || (N % 8) != 0 || K <= 0 || (K % 16) != 0 || K > W8A8_MAX_K)
+        return W8A8_ERR_UNSUPPORTED_SHAPE;
+    return W8A8_OK;
+}
+
+w8a8_status from_cuda(cudaError_t e) { return e == cudaSuccess ? W8A8_OK : W8A8_ERR_CUDA; }
+
+cudaStream_t as_stream(void *s) { return static_cast<cudaStream_t>(s); }
+
+unsigned int *device_error_word() {
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_w8a8_device_error) != cudaSuccess) return nullptr;
+    return static_cast<unsigned int *>(p);
+}
+
+// Validation shared by the single- and dual-branch linears.
+w8a8_status check_branch(const w8a8::GemmBranch &b, bool need_scales, int N, int K) {
+    if (b.M < 0) return W8A8_ERR_UNSUPPORTED_SHAPE;
+    if (b.M == 0) return W8A8_OK;
+    if (!b.Xq || !b.Wq || !b.out) return W8A8_ERR_INVALID_ARG;
+    if (need_scales && (!b.x_scale || !b.w_scale)) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(b.Xq) || !aligned16(b.Wq) || !aligned16(b.out)) return W8A8_ERR_MISALIGNED;
+    if (need_scales && (!aligned16(b.x_scale) || !aligned16(b.w_scale) ||
+                        (b.bias && !aligned16(b.bias))))
+        return W8A8_ERR_MISALIGNED;
+    (void)N;
+    (void)K;
+    return W8A8_OK;
+}
+
+w8a8_status run_gemm(const w8a8::GemmBranch *br, int nb, int N, int K, bool out_i32,
+                     cudaStream_t st) {
+    if (g_engine == 1) {
+        unsigned int *err = device_error_word();
+        if (!err) return W8A8_ERR_CUDA;
+        return from_cuda(w8a8::launch_gemm_tc(br, nb, N, K, out_i32, err, st));
+    }
+    return from_cuda(w8a8::launch_gemm_mma(br, nb, N, K, out_i32, st));
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *w8a8_status_string(w8a8_status status) {
+    switch (status) {
+        case W8A8_OK: return "W8A8_OK";
+        case W8A8_ERR_INVALID_ARG: return "W8A8_ERR_INVALID_ARG";
+        case W8A8_ERR_UNSUPPORTED_SHAPE: return "W8A8_ERR_UNSUPPORTED_SHAPE";
+        case W8A8_ERR_MISALIGNED: return "W8A8_ERR_MISALIGNED";
+        case W8A8_ERR_CUDA: return "W8A8_ERR_CUDA";
+        case W8A8_ERR_TIMEOUT: return "W8A8_ERR_TIMEOUT";
+    }
+    return "W8A8_ERR_UNKNOWN";
+}
+
+w8a8_status w8a8_channel_absmax(const uint16_t *X, int T, int K, float *s, void *stream) {
+    if (T < 0 || K <= 0 || (K % 16) != 0 || K > W8A8_MAX_K) return W8A8_ERR_UNSUPPORTED_SHAPE;
+    if (!s || (T > 0 && !X)) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(s) || (T > 0 && !aligned16(X))) return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_channel_absmax(X, T, K, s, as_stream(stream)));
+}
+
+w8a8_status w8a8_smooth_scales(const float *act_absmax, const float *W, int N, int K,
+                               float alpha, float *smooth, void *stream) {
+    if (w8a8_status e = check_nk(N, K)) return e;
+    if (!act_absmax || !W || !smooth) return W8A8_ERR_INVALID_ARG;
+    if (!(alpha >= 0.0f && alpha <= 1.0f)) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(act_absmax) || !aligned16(W) || !aligned16(smooth)) return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_smooth_scales(act_absmax, W, N, K, alpha, smooth,
+                                                as_stream(stream)));
+}
+
+w8a8_status w8a8_quantize_weights(const float *W, const float *smooth, int N, int K,
+                                  int8_t *Wq, float *w_scale, void *stream) {
+    if (w8a8_status e = check_nk(N, K)) return e;
+    if (!W || !Wq || !w_scale) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(W) || !aligned16(Wq) || !aligned16(w_scale) || (smooth && !aligned16(smooth)))
+        return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_quantize_weights(W, smooth, N, K, Wq, w_scale,
+                                                   as_stream(stream)));
+}
+
+w8a8_status w8a8_quant_act(const uint16_t *X, const float *smooth, int M, int K,
+                           int8_t *Xq, float *x_scale, void *stream) {
+    if (w8a8_status e = check_mk(M, K)) return e;
+    if (M == 0) return W8A8_OK;
+    if (!X || !Xq || !x_scale) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(Xq) || !aligned16(x_scale) || (smooth && !aligned16(smooth)))
+        return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_quant_act(X, smooth, M, K, Xq, x_scale, as_stream(stream)));
+}
+
+w8a8_status w8a8_linear(const int8_t *Xq, const float *x_scale, const int8_t *Wq,
+                        const float *w_scale, const float *bias, int M, int N, int K,
+                        uint16_t *Y, void *stream) {
+    if (w8a8_status e = check_nk(N, K)) return e;
+    if (w8a8_status e = check_mk(M, K)) return e;
+    w8a8::GemmBranch b{Xq, x_scale, Wq, w_scale, bias, Y, M};
+    if (w8a8_status e = check_branch(b, true, N, K)) return e;
+    if (M == 0) return W8A8_OK;
+    return run_gemm(&b, 1, N, K, false, as_stream(stream));
+}
+
+w8a8_status w8a8_linear_dual(const w8a8_branch *br, int N, int K, void *stream) {
+    if (!br) return W8A8_ERR_INVALID_ARG;
+    if (w8a8_status e = check_nk(N, K)) return e;
+    w8a8::GemmBranch b[2];
+    for (int i = 0; i < 2; ++i) {
+        b[i] = w8a8::GemmBranch{br[i].Xq, br[i].x_scale, br[i].Wq, br[i].w_scale,
+                                br[i].bias, br[i].Y, br[i].M};
+        if (w8a8_status e = check_mk(br[i].M, K)) return e;
+        if (w8a8_status e = check_branch(b[i], true, N, K)) return e;
+    }
+    if (b[0].M == 0 && b[1].M == 0) return W8A8_OK;
+    return run_gemm(b, 2, N, K, false, as_stream(stream));
+}
+
+w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int M, int N, int K,
+                                int32_t *acc, void *stream) {
+    if (w8a8_status e = check_nk(N, K)) return e;
+    if (w8a8_status e = check_mk(M, K)) return e;
+    w8a8::GemmBranch b{Xq, nullptr, Wq, nullptr, nullptr, acc, M};
+    if (w8a8_status e = check_branch(b, false, N, K)) return e;
+    if (M == 0) return W8A8_OK;
+    return run_gemm(&b, 1, N, K, true, as_stream(stream));
+}
+
+w8a8_status w8a8_set_gemm_engine(int engine) {
+    if (engine == -1) engine = 1;
+    if (engine != 0 && engine != 1) return W8A8_ERR_INVALID_ARG;
+    g_engine = engine;
+    return W8A8_OK;
+}
+
+int w8a8_get_gemm_engine(void) { return g_engine; }
+
+w8a8_status w8a8_device_status(void *stream, uint32_t *detail) {
+    cudaStream_t st = as_stream(stream);
+    if (cudaStreamSynchronize(st) != cudaSuccess) return W8A8_ERR_CUDA;
+    unsigned int word = 0;
+    if (cudaMemcpyFromSymbol(&word, g_w8a8_device_error, sizeof word) != cudaSuccess)
+        return W8A8_ERR_CUDA;
+    if (word != 0) {
+        const unsigned int zero = 0;
+        if (cudaMemcpyToSymbol(g_w8a8_device_error, &zero, sizeof zero) != cudaSuccess)
+            return W8A8_ERR_CUDA;
+    }
+    if (detail) *detail = word;
+    return word ? W8A8_ERR_TIMEOUT : W8A8_OK;
+}
+
+}  // extern "C"

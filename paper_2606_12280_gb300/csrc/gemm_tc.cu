@@ -1,0 +1,500 @@
+// gemm_tc.cu -- the W8A8 linear (a4 + a5, and the dual-branch grouping a6) on
+// the 5th-generation tensor cores of sm_103a.
+//
+// GB300's tcgen05 has no INT8 MMA kind (ptxas rejects .kind::i8 for sm_103a),
+// so the INT8 x INT8 -> INT32 product runs EXACTLY on the fp16 datapath:
+//   - every int8 value in [-127, 127] is an fp16 value,
+//   - every product (|p| <= 127^2 = 16129) is exact in fp32,
+//   - every partial sum over at most KC = 1024 products is an integer of
+//     magnitude <= 1024 * 16129 < 2^24, hence exact in the fp32 accumulator,
+// so each K chunk of 1024 is accumulated in fp32 in TMEM, then converted to
+// int32 (exact) and added to an int32 running sum held in registers by the
+// epilogue warps.  The final int32 equals sum_k Xq*Wq bit for bit.
+//
+// Per CTA (one per SM, persistent over a static tile schedule):
+//   warp 0      TMA producer: int8 tiles of Xq [128 x 64] and Wq [256 x 64]
+//               into a 4-stage ring (no swizzle, 64-byte rows)
+//   warp 1      TMEM allocator and MMA issuer: tcgen05.mma kind::f16,
+//               M=128 N=256 K=16, fp32 accumulators in TMEM, two 256-column
+//               buffers used alternately per K chunk
+//   warps 2-7   converters: int8 -> fp16 (exact, integer bit tricks) into a
+//               2-stage ring of 128-byte-swizzled K-major operand tiles
+//   warps 8-15  epilogue: TMEM -> registers per chunk, int32 running sums,
+//               then Y = bf16(((float)acc * sx) * sw + b) straight to global
+// Every mbarrier wait is bounded in time; a timeout records an error code in
+// the library's device error word and all roles stop.
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "launch.h"
+#include "tc_ptx.cuh"
+
+namespace w8a8 {
+namespace {
+
+using namespace tc;
+
+constexpr int BM = 128, BN = 256, BK = 64;          // BK in int8 bytes = fp16 elements
+constexpr int KC_BLOCKS = 16;                        // K chunk = 1024 (exactness bound)
+constexpr int S8 = 4, S16 = 2;                       // ring depths
+constexpr int STAGE8_A = BM * BK, STAGE8_B = BN * BK;
+constexpr int STAGE8 = STAGE8_A + STAGE8_B;          // 24 KB
+constexpr int STAGE16_A = BM * BK * 2, STAGE16_B = BN * BK * 2;
+constexpr int STAGE16 = STAGE16_A + STAGE16_B;       // 48 KB
+constexpr int NUM_CONV_WARPS = 6;
+constexpr int NUM_EPI_WARPS = 8;
+constexpr int THREADS = 512;
+constexpr int TMEM_COLS = 512;
+constexpr int SMEM_BARRIERS = 256;
+constexpr int SMEM_EPI = NUM_EPI_WARPS * 1024;         // per epilogue warp: 128 sw + 128 bias
+constexpr int SMEM_TOTAL = 1024 + S16 * STAGE16 + S8 * STAGE8 + SMEM_BARRIERS + SMEM_EPI;
+constexpr int LAUNCH_REGS = 128;                     // 512 threads x 128 = 65536
+constexpr int REGS_LOW = 72, REGS_HIGH = 184;        // 256*72 + 256*184 = 65536
+static_assert(256 * REGS_LOW + 256 * REGS_HIGH <= THREADS * LAUNCH_REGS, "register split");
+static_assert(KC_BLOCKS * BK * 127 * 127 < (1 << 24), "fp32 exactness bound");
+
+// error codes recorded in the device error word (bit flags)
+constexpr unsigned ERR_PRODUCER = 1u, ERR_CONVERTER = 2u, ERR_MMA = 4u, ERR_EPILOGUE = 8u,
+                   ERR_DRAIN = 16u;
+
+struct BranchArgs {
+    const float *x_scale;
+    const float *w_scale;
+    const float *bias;
+    void *out;
+    int M;
+    int m_tiles;
+    int tiles;       // m_tiles * n_tiles
+};
+
+struct Params {
+    BranchArgs br[2];
+    int N, K;
+    int n_tiles;
+    int total_tiles;
+    int k_blocks;
+    unsigned int *err;
+    uint64_t wait_limit_ns;
+};
+
+struct Tile {
+    int branch, m0, n0;
+};
+
+__device__ __forceinline__ Tile tile_coords(const Params &p, int t) {
+    Tile r;
+    r.branch = t >= p.br[0].tiles ? 1 : 0;
+    const int local = t - (r.branch ? p.br[0].tiles : 0);
+    const int mt = p.br[r.branch].m_tiles;
+    r.m0 = (local % mt) * BM;
+    r.n0 = (local / mt) * BN;
+    return r;
+}
+
+// Shared memory map (offsets from the 1024-aligned base)
+constexpr uint32_t OFF_ST16 = 0;
+constexpr uint32_t OFF_ST8 = OFF_ST16 + S16 * STAGE16;
+constexpr uint32_t OFF_BAR = OFF_ST8 + S8 * STAGE8;
+constexpr uint32_t BAR_FULL8 = OFF_BAR;
+constexpr uint32_t BAR_EMPTY8 = BAR_FULL8 + 8 * S8;
+constexpr uint32_t BAR_FULL16 = BAR_EMPTY8 + 8 * S8;
+constexpr uint32_t BAR_EMPTY16 = BAR_FULL16 + 8 * S16;
+constexpr uint32_t BAR_ACCFULL = BAR_EMPTY16 + 8 * S16;
+constexpr uint32_t BAR_ACCEMPTY = BAR_ACCFULL + 16;
+constexpr uint32_t BAR_DRAIN = BAR_ACCEMPTY + 16;
+constexpr uint32_t OFF_TMEM = BAR_DRAIN + 8;
+constexpr uint32_t OFF_ABORT = OFF_TMEM + 4;
+static_assert(OFF_ABORT + 4 - OFF_BAR <= SMEM_BARRIERS, "barrier area");
+constexpr uint32_t OFF_EPI = OFF_BAR + SMEM_BARRIERS;
+
+__device__ __forceinline__ float4 ld_shared_f4(uint32_t a) {
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(a));
+    return v;
+}
+
+__device__ __forceinline__ void st_global_v4(void *p, uint4 v) {
+    asm volatile("st.global.v4.b32 [%0], {%1,%2,%3,%4};" ::"l"(p), "r"(v.x), "r"(v.y), "r"(v.z),
+                 "r"(v.w) : "memory");
+}
+
+// int8 x4 (one 32-bit word) -> two fp16x2 words, exact: bytes u = b + 128 are
+// placed in the mantissa of 1024.0 (fp16 0x6400), then 1152 = 1024 + 128 is
+// subtracted, which is exact for every value in [1024, 1280).
+__device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
+    const uint32_t u = w ^ 0x80808080u;
+    asm("prmt.b32 %0, %1, %2, 0x4140;" : "=r"(lo) : "r"(u), "r"(0x64646464u));
+    asm("prmt.b32 %0, %1, %2, 0x4342;" : "=r"(hi) : "r"(u), "r"(0x64646464u));
+    asm("sub.f16x2 %0, %0, %1;" : "+r"(lo) : "r"(0x64806480u));
+    asm("sub.f16x2 %0, %0, %1;" : "+r"(hi) : "r"(0x64806480u));
+}
+
+template <bool OUT_I32>
+__device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint32_t tmem,
+                                              const WaitCtx &wc, int warp, int lane, int NC) {
+        // ---------------------------------------------------------- epilogue
+        const int e = warp - 8;
+        const int q = warp & 3;            // TMEM lane quarter this warp may access
+        const int h = e >> 2;              // column half of the 256-wide tile
+        uint32_t c = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+            int32_t run[128];
+#pragma unroll
+            for (int i = 0; i < 128; ++i) run[i] = 0;
+            for (int ci = 0; ci < NC; ++ci, ++c) {
+                const uint32_t buf = c & 1;
+                if (!mbar_wait(sb + BAR_ACCFULL + 8 * buf, (c >> 1) & 1, wc, ERR_EPILOGUE)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * BN + h * 128;
+#pragma unroll
+                for (int jj = 0; jj < 8; ++jj) {
+                    uint32_t v[16];
+                    tmem_ld_32x32b_x16(base + jj * 16, v);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) run[jj * 16 + i] += __float2int_rn(__uint_as_float(v[i]));
+                }
+                tc_fence_before();
+                __syncwarp();
+                if (lane == 0) mbar_arrive(sb + BAR_ACCEMPTY + 8 * buf);
+            }
+            if (!ok) break;
+            // dequantize and store this thread's row: 128 consecutive columns
+            const Tile tl = tile_coords(p, t);
+            const BranchArgs &br = p.br[tl.branch];
+            const int m = tl.m0 + q * 32 + lane;
+            const int n_base = tl.n0 + h * 128;
+            const uint32_t epi = sb + OFF_EPI + e * 1024;
+            if (!OUT_I32) {
+                // this warp's 128 per-channel scales and biases, staged once per tile
+                const int n = n_base + lane * 4;
+                float4 w = make_float4(0.f, 0.f, 0.f, 0.f), b = w;
+                if (n < p.N) {
+                    w = __ldg(reinterpret_cast<const float4 *>(br.w_scale + n));
+                    if (br.bias) b = __ldg(reinterpret_cast<const float4 *>(br.bias + n));
+                }
+                asm volatile("st.shared.v4.f32 [%0], {%1,%2,%3,%4};" ::"r"(epi + lane * 16),
+                             "f"(w.x), "f"(w.y), "f"(w.z), "f"(w.w) : "memory");
+                asm volatile("st.shared.v4.f32 [%0], {%1,%2,%3,%4};" ::"r"(epi + 512 + lane * 16),
+                             "f"(b.x), "f"(b.y), "f"(b.z), "f"(b.w) : "memory");
+                __syncwarp();
+            }
+            if (m < br.M) {
+                if (OUT_I32) {
+                    int32_t *out = static_cast<int32_t *>(br.out) + (size_t)m * p.N + n_base;
+#pragma unroll
+                    for (int g = 0; g < 16; ++g) {
+                        if (n_base + g * 8 < p.N) {
+                            *reinterpret_cast<int4 *>(out + g * 8) =
+                                make_int4(run[g * 8], run[g * 8 + 1], run[g * 8 + 2], run[g * 8 + 3]);
+                            *reinterpret_cast<int4 *>(out + g * 8 + 4) =
+                                make_int4(run[g * 8 + 4], run[g * 8 + 5], run[g * 8 + 6], run[g * 8 + 7]);
+                        }
+                    }
+                } else {
+                    const float sx = __ldg(br.x_scale + m);
+                    const bool hb = br.bias != nullptr;
+                    uint16_t *out = static_cast<uint16_t *>(br.out) + (size_t)m * p.N + n_base;
+#pragma unroll
+                    for (int g = 0; g < 16; ++g) {
+                        if (n_base + g * 8 < p.N) {
+                            const float4 w0 = ld_shared_f4(epi + g * 32);
+                            const float4 w1 = ld_shared_f4(epi + g * 32 + 16);
+                            float4 b0 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = b0;
+                            if (hb) {
+                                b0 = ld_shared_f4(epi + 512 + g * 32);
+                                b1 = ld_shared_f4(epi + 512 + g * 32 + 16);
+                            }
+                            const uint32_t y0 = epilogue_value(run[g * 8 + 0], sx, w0.x, b0.x, hb);
+                            const uint32_t y1 = epilogue_value(run[g * 8 + 1], sx, w0.y, b0.y, hb);
+                            const uint32_t y2 = epilogue_value(run[g * 8 + 2], sx, w0.z, b0.z, hb);
+                            const uint32_t y3 = epilogue_value(run[g * 8 + 3], sx, w0.w, b0.w, hb);
+                            const uint32_t y4 = epilogue_value(run[g * 8 + 4], sx, w1.x, b1.x, hb);
+                            const uint32_t y5 = epilogue_value(run[g * 8 + 5], sx, w1.y, b1.y, hb);
+                            const uint32_t y6 = epilogue_value(run[g * 8 + 6], sx, w1.z, b1.z, hb);
+                            const uint32_t y7 = epilogue_value(run[g * 8 + 7], sx, w1.w, b1.w, hb);
+                            st_global_v4(out + g * 8, make_uint4(y0 | (y1 << 16), y2 | (y3 << 16),
+                                                                 y4 | (y5 << 16), y6 | (y7 << 16)));
+                        }
+                    }
+                }
+            }
+            __syncwarp();
+        }
+    }
+
+template <bool OUT_I32>
+__global__ void __launch_bounds__(THREADS, 1)
+gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
+               const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
+               const Params p) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t sb = (smem_addr(smem_raw) + 1023u) & ~1023u;
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < S8; ++i) {
+            mbar_init(sb + BAR_FULL8 + 8 * i, 1);
+            mbar_init(sb + BAR_EMPTY8 + 8 * i, NUM_CONV_WARPS);
+        }
+        for (int i = 0; i < S16; ++i) {
+            mbar_init(sb + BAR_FULL16 + 8 * i, NUM_CONV_WARPS);
+            mbar_init(sb + BAR_EMPTY16 + 8 * i, 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(sb + BAR_ACCFULL + 8 * i, 1);
+            mbar_init(sb + BAR_ACCEMPTY + 8 * i, NUM_EPI_WARPS);
+        }
+        mbar_init(sb + BAR_DRAIN, 1);
+        st_shared_s32(sb + OFF_ABORT, 0);
+        fence_barrier_init();
+    }
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&tmA0);
+        tma_prefetch_desc(&tmB0);
+        tma_prefetch_desc(&tmA1);
+        tma_prefetch_desc(&tmB1);
+    }
+    if (warp == 1) {
+        tmem_alloc(sb + OFF_TMEM, TMEM_COLS);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = static_cast<uint32_t>(ld_shared_s32(sb + OFF_TMEM));
+    const WaitCtx wc{sb + OFF_ABORT, p.err, p.wait_limit_ns};
+    const int KB = p.k_blocks;
+    const int NC = (KB + KC_BLOCKS - 1) / KC_BLOCKS;
+
+    if (warp >= 8) {
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(REGS_HIGH));
+        epilogue_role<OUT_I32>(p, sb, tmem, wc, warp, lane, NC);
+        tc_fence_before();
+        __syncwarp();
+        asm volatile("bar.sync 1, %0;" ::"n"(THREADS) : "memory");
+    } else {
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(REGS_LOW));
+        if (warp == 0) {
+        // ------------------------------------------------------ TMA producer
+        if (lane == 0) {
+            uint32_t j = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+                const Tile tl = tile_coords(p, t);
+                const CUtensorMap *mA = tl.branch ? &tmA1 : &tmA0;
+                const CUtensorMap *mB = tl.branch ? &tmB1 : &tmB0;
+                for (int kb = 0; kb < KB; ++kb, ++j) {
+                    const uint32_t st = j % S8;
+                    if (!mbar_wait(sb + BAR_EMPTY8 + 8 * st, ((j / S8) & 1) ^ 1, wc, ERR_PRODUCER)) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t fb = sb + BAR_FULL8 + 8 * st;
+                    mbar_arrive_expect_tx(fb, STAGE8);
+                    const uint32_t dst = sb + OFF_ST8 + st * STAGE8;
+                    tma_load_2d(dst, mA, kb * BK, tl.m0, fb);
+                    tma_load_2d(dst + STAGE8_A, mB, kb * BK, tl.n0, fb);
+                }
+            }
+            // drain: every armed stage must have landed before the CTA exits
+            for (uint32_t i = (j > S8 ? j - S8 : 0); i < j; ++i)
+                mbar_wait(sb + BAR_FULL8 + 8 * (i % S8), (i / S8) & 1, wc, ERR_DRAIN, false);
+        }
+        } else if (warp == 1) {
+        // --------------------------------------------------------- MMA issue
+        if (lane == 0) {
+            constexpr uint32_t idesc = idesc_f16_f32(BM, BN);
+            uint32_t j = 0, c = 0;
+            bool ok = true;
+            for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+                for (int ci = 0; ok && ci < NC; ++ci, ++c) {
+                    const uint32_t buf = c & 1;
+                    if (!mbar_wait(sb + BAR_ACCEMPTY + 8 * buf, ((c >> 1) & 1) ^ 1, wc, ERR_MMA)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t d = tmem + buf * BN;
+                    const int kb0 = ci * KC_BLOCKS;
+                    const int kb1 = min(KB, kb0 + KC_BLOCKS);
+                    for (int kb = kb0; kb < kb1; ++kb, ++j) {
+                        const uint32_t st = j % S16;
+                        if (!mbar_wait(sb + BAR_FULL16 + 8 * st, (j / S16) & 1, wc, ERR_MMA)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t a = sb + OFF_ST16 + st * STAGE16;
+                        const uint32_t b = a + STAGE16_A;
+#pragma unroll
+                        for (int kk = 0; kk < BK / 16; ++kk) {
+                            mma_f16_ss(d, smem_desc_sw128(a + kk * 32), smem_desc_sw128(b + kk * 32),
+                                       idesc, (kb > kb0 || kk > 0) ? 1u : 0u);
+                        }
+                        mma_commit(sb + BAR_EMPTY16 + 8 * st);
+                    }
+                    if (ok) mma_commit(sb + BAR_ACCFULL + 8 * buf);
+                }
+            }
+            // every MMA this thread issued must be complete before TMEM is freed
+            mma_commit(sb + BAR_DRAIN);
+            mbar_wait(sb + BAR_DRAIN, 0, wc, ERR_DRAIN, false);
+        }
+        } else {
+        // -------------------------------------------------------- converters
+        const int cw = warp - 2;
+        const uint32_t rr = lane >> 2;     // row inside an 8-row group
+        const uint32_t c4 = lane & 3;      // 16-byte int8 chunk of the 64-byte row
+        const uint32_t src_off = rr * BK + c4 * 16;
+        const uint32_t dst_off0 = rr * 128 + (((2 * c4) ^ rr) << 4);
+        const uint32_t dst_off1 = rr * 128 + (((2 * c4 + 1) ^ rr) << 4);
+        uint32_t j = 0;
+        bool ok = true;
+        for (int t = blockIdx.x; ok && t < p.total_tiles; t += gridDim.x) {
+            for (int kb = 0; kb < KB; ++kb, ++j) {
+                const uint32_t s8 = j % S8, s16 = j % S16;
+                if (!mbar_wait(sb + BAR_FULL8 + 8 * s8, (j / S8) & 1, wc, ERR_CONVERTER) ||
+                    !mbar_wait(sb + BAR_EMPTY16 + 8 * s16, ((j / S16) & 1) ^ 1, wc, ERR_CONVERTER)) {
+                    ok = false;
+                    break;
+                }
+                const uint32_t src = sb + OFF_ST8 + s8 * STAGE8 + src_off;
+                const uint32_t dst = sb + OFF_ST16 + s16 * STAGE16;
+#pragma unroll 2
+                for (int g = cw; g < (BM + BN) / 8; g += NUM_CONV_WARPS) {
+                    const uint4 v = ld_shared_v4(src + g * 8 * BK);
+                    uint4 o0, o1;
+                    i8x4_to_f16x4(v.x, o0.x, o0.y);
+                    i8x4_to_f16x4(v.y, o0.z, o0.w);
+                    i8x4_to_f16x4(v.z, o1.x, o1.y);
+                    i8x4_to_f16x4(v.w, o1.z, o1.w);
+                    st_shared_v4(dst + g * 1024 + dst_off0, o0);
+                    st_shared_v4(dst + g * 1024 + dst_off1, o1);
+                }
+                fence_proxy_async_smem();
+                __syncwarp();
+                if (lane == 0) {
+                    mbar_arrive(sb + BAR_FULL16 + 8 * s16);
+                    mbar_arrive(sb + BAR_EMPTY8 + 8 * s8);
+                }
+            }
+        }
+        }
+        tc_fence_before();
+        __syncwarp();
+        asm volatile("bar.sync 1, %0;" ::"n"(THREADS) : "memory");
+        if (warp == 1) {
+            tc_fence_after();
+            tmem_dealloc(tmem, TMEM_COLS);
+        }
+    }
+}
+
+// ------------------------------------------------------------------ host
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    }
+    return fn;
+}
+
+// int8 row-major [rows, K] -> 2-D map with box [box_rows, 64 bytes], zero fill.
+bool make_map(CUtensorMap *m, const int8_t *base, int rows, int K, int box_rows) {
+    EncodeTiledFn enc = get_encode();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K)};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_UINT8, 2, const_cast<int8_t *>(base), dims, strides, box,
+               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int g_sms = 0;
+int g_kernel_regs[2] = {-1, -1};
+
+}  // namespace
+
+cudaError_t launch_gemm_tc(const GemmBranch *br, int nb, int N, int K, bool out_i32,
+                           unsigned int *err, cudaStream_t st) {
+    if (g_sms == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
+    }
+    const int ki = out_i32 ? 1 : 0;
+    auto kern = out_i32 ? gemm_tc_kernel<true> : gemm_tc_kernel<false>;
+    if (g_kernel_regs[ki] < 0) {
+        cudaFuncAttributes fa;
+        cudaError_t e = cudaFuncGetAttributes(&fa, kern);
+        if (e != cudaSuccess) return e;
+        g_kernel_regs[ki] = fa.numRegs;
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_TOTAL);
+        if (e != cudaSuccess) return e;
+    }
+    // the warp-group register split relies on the launch holding exactly
+    // 512 x 128 registers
+    if (g_kernel_regs[ki] != LAUNCH_REGS) return cudaErrorInvalidConfiguration;
+
+    Params p{};
+    CUtensorMap maps[4];
+    int first = -1;
+    for (int i = 0; i < 2; ++i) {
+        const GemmBranch *b = (i < nb) ? &br[i] : nullptr;
+        BranchArgs &a = p.br[i];
+        a = BranchArgs{nullptr, nullptr, nullptr, nullptr, 0, 0, 0};
+        if (b && b->M > 0) {
+            a.x_scale = b->x_scale;
+            a.w_scale = b->w_scale;
+            a.bias = b->bias;
+            a.out = b->out;
+            a.M = b->M;
+            a.m_tiles = (b->M + BM - 1) / BM;
+            a.tiles = a.m_tiles * ((N + BN - 1) / BN);
+            if (!make_map(&maps[2 * i], b->Xq, b->M, K, BM) ||
+                !make_map(&maps[2 * i + 1], b->Wq, N, K, BN))
+                return cudaErrorInvalidValue;
+            if (first < 0) first = i;
+        }
+    }
+    if (first < 0) return cudaSuccess;
+    for (int i = 0; i < 2; ++i)
+        if (p.br[i].M == 0) {
+            maps[2 * i] = maps[2 * first];
+            maps[2 * i + 1] = maps[2 * first + 1];
+        }
+    p.N = N;
+    p.K = K;
+    p.n_tiles = (N + BN - 1) / BN;
+    p.total_tiles = p.br[0].tiles + p.br[1].tiles;
+    p.k_blocks = (K + BK - 1) / BK;
+    p.err = err;
+    p.wait_limit_ns = 2000000000ull;       // 2 s per wait
+    const int grid = p.total_tiles < g_sms ? p.total_tiles : g_sms;
+    kern<<<grid, THREADS, SMEM_TOTAL, st>>>(maps[0], maps[1], maps[2], maps[3], p);
+    return cudaGetLastError();
+}
+
+}  // namespace w8a8

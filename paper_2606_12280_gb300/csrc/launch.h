@@ -1,0 +1,40 @@
+// launch.h -- host-side launchers of the library's kernels (internal).
+// Arguments are validated by the C-ABI layer before any of these is called.
+#pragma once
+
+#include <cstdint>
+#include <cuda_runtime.h>
+
+namespace w8a8 {
+
+struct GemmBranch {
+    const int8_t *Xq;
+    const float *x_scale;
+    const int8_t *Wq;
+    const float *w_scale;
+    const float *bias;
+    void *out;        // uint16_t* bf16 Y, or int32_t* acc for the debug export
+    int M;
+};
+
+cudaError_t launch_channel_absmax(const uint16_t *X, int T, int K, float *s,
+                                  cudaStream_t st);
+cudaError_t launch_smooth_scales(const float *s, const float *W, int N, int K,
+                                 float alpha, float *lambda, cudaStream_t st);
+cudaError_t launch_quantize_weights(const float *W, const float *lambda, int N,
+                                    int K, int8_t *Wq, float *w_scale,
+                                    cudaStream_t st);
+cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M,
+                             int K, int8_t *Xq, float *x_scale,
+                             cudaStream_t st);
+
+// Legacy warp-level mma.sync s8 GEMM (exact int32), nb = 1 or 2 branches.
+// out_i32: write the int32 product instead of the bf16 epilogue.
+cudaError_t launch_gemm_mma(const GemmBranch *br, int nb, int N, int K,
+                            bool out_i32, cudaStream_t st);
+
+// tcgen05 GEMM (exact integer products on the fp16 tensor datapath).
+cudaError_t launch_gemm_tc(const GemmBranch *br, int nb, int N, int K,
+                           bool out_i32, unsigned int *err, cudaStream_t st);
+
+}  // namespace w8a8

@@ -1,0 +1,361 @@
+// quant.cu -- the quantization passes of the W8A8 layer (Sec. 3, "INT8 W8A8").
+//
+//   row_quant_kernel      a3 per-token activation quant (bf16 in, x / lambda)
+//                         a2 per-output-channel weight quant (fp32 in, w * lambda)
+//   col_absmax_kernel     column max |.| of a row-major matrix: the calibration
+//                         statistic s_j and the weight column max m_j of a1
+//   smooth_finalize       a1 lambda_j = s_j^alpha / m_j^(1-alpha)
+//
+// The activation pass is HBM-bound: one read of X (2 B/elem), one write of Xq
+// (1 B/elem) and one fp32 scale per row.  A "team" of G threads owns one row at
+// a time; each thread owns CPT chunks of 8 consecutive columns (one 16-byte
+// load of bf16) at a stride of 8*G columns, so every warp-wide load is a fully
+// coalesced 512-byte segment.  The per-column factor (1/lambda_j or lambda_j)
+// is computed once per thread and kept in registers for every row the team
+// visits; the next row's data is loaded before the current row is reduced.
+#include <cstdint>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "launch.h"
+
+namespace w8a8 {
+namespace {
+
+// ---------------------------------------------------------------- loading
+
+template <typename InT> struct Chunk;
+
+template <> struct Chunk<uint16_t> {        // 8 bf16 = 16 bytes
+    uint4 v;
+    __device__ __forceinline__ void load(const uint16_t *p) {
+        v = __ldcs(reinterpret_cast<const uint4 *>(p));
+    }
+    __device__ __forceinline__ void zero() { v = make_uint4(0, 0, 0, 0); }
+    __device__ __forceinline__ float get(int e) const {
+        uint32_t w = (e < 2) ? v.x : (e < 4) ? v.y : (e < 6) ? v.z : v.w;
+        return bf16_bits_to_f32((e & 1) ? (w >> 16) : (w & 0xffffu));
+    }
+};
+
+template <> struct Chunk<float> {           // 8 fp32 = 32 bytes
+    float4 a, b;
+    __device__ __forceinline__ void load(const float *p) {
+        a = __ldcs(reinterpret_cast<const float4 *>(p));
+        b = __ldcs(reinterpret_cast<const float4 *>(p) + 1);
+    }
+    __device__ __forceinline__ void zero() {
+        a = make_float4(0.f, 0.f, 0.f, 0.f);
+        b = a;
+    }
+    __device__ __forceinline__ float get(int e) const {
+        switch (e) {
+            case 0: return a.x; case 1: return a.y; case 2: return a.z;
+            case 3: return a.w; case 4: return b.x; case 5: return b.y;
+            case 6: return b.z; default: return b.w;
+        }
+    }
+};
+
+__device__ __forceinline__ float warp_max(float v) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v = fmaxf(v, __shfl_xor_sync(0xffffffffu, v, o));
+    return v;
+}
+
+// ------------------------------------------------------------- row quant
+//
+// IS_ACT:  factor f_j = 1/lambda_j (activations are divided by lambda);
+// else:    factor f_j = lambda_j   (weights are multiplied by lambda).
+// Smoothed value x'_j = in_j * f_j (RN), absmax over the row, scale = a/127,
+// codes = clamp(rne(x'_j * (127/a)), +-127).
+template <typename InT, bool IS_ACT, int CPT>
+__global__ void __launch_bounds__(512)
+row_quant_kernel(const InT *__restrict__ in, const float *__restrict__ lam,
+                 int M, int K, int G, int8_t *__restrict__ q,
+                 float *__restrict__ scale) {
+    __shared__ float red[2][32];
+    const int tid = threadIdx.x;
+    const int teams = blockDim.x / G;
+    const int team = tid / G;
+    const int tl = tid - team * G;          // index inside the team
+    const int lane = tid & 31;
+    const int warp = tid >> 5;
+    const int team_warp0 = (team * G) >> 5;
+    const int team_warps = G >> 5;
+
+    // per-column factors, once per thread
+    float f[CPT][8];
+#pragma unroll
+    for (int c = 0; c < CPT; ++c) {
+        const int col0 = 8 * (tl + c * G);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            float fe = 1.0f;
+            if (lam != nullptr && col0 < K) {
+                const float l = __ldg(lam + col0 + e);
+                fe = IS_ACT ? __frcp_rn(l) : l;
+            }
+            f[c][e] = fe;
+        }
+    }
+
+    Chunk<InT> cur[CPT], nxt[CPT];
+    const int row_stride = gridDim.x * teams;
+    int row = blockIdx.x * teams + team;
+#pragma unroll
+    for (int c = 0; c < CPT; ++c) {
+        const int col0 = 8 * (tl + c * G);
+        if (row < M && col0 < K) cur[c].load(in + (size_t)row * K + col0);
+        else cur[c].zero();
+    }
+
+    int parity = 0;
+    for (int base = blockIdx.x * teams; base < M; base += row_stride) {
+        row = base + team;
+        const int nrow = row + row_stride;
+        // prefetch the next row this team will visit
+#pragma unroll
+        for (int c = 0; c < CPT; ++c) {
+            const int col0 = 8 * (tl + c * G);
+            if (IS_ACT && nrow < M && col0 < K) nxt[c].load(in + (size_t)nrow * K + col0);
+            else nxt[c].zero();
+        }
+        // row absmax of the smoothed values
+        float a = 0.0f;
+#pragma unroll
+        for (int c = 0; c < CPT; ++c)
+#pragma unroll
+            for (int e = 0; e < 8; ++e)
+                a = fmaxf(a, fabsf(__fmul_rn(cur[c].get(e), f[c][e])));
+        a = warp_max(a);
+        if (G > 32) {
+            if (lane == 0) red[parity][warp] = a;
+            __syncthreads();
+            a = 0.0f;
+            for (int w = 0; w < team_warps; ++w) a = fmaxf(a, red[parity][team_warp0 + w]);
+            parity ^= 1;
+        }
+        if (row < M) {
+            const bool zero_row = (a == 0.0f);
+            const float inv = zero_row ? 0.0f : __fdiv_rn(127.0f, a);
+            if (tl == 0) scale[row] = zero_row ? 0.0f : __fdiv_rn(a, 127.0f);
+#pragma unroll
+            for (int c = 0; c < CPT; ++c) {
+                const int col0 = 8 * (tl + c * G);
+                if (col0 >= K) continue;
+                uint32_t lo = 0, hi = 0;
+                if (!zero_row) {
+#pragma unroll
+                    for (int e = 0; e < 8; ++e) {
+                        const float xs = __fmul_rn(cur[c].get(e), f[c][e]);
+                        const uint32_t b = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xs, inv))) & 0xffu;
+                        if (e < 4) lo |= b << (8 * e);
+                        else hi |= b << (8 * (e - 4));
+                    }
+                }
+                *reinterpret_cast<uint2 *>(q + (size_t)row * K + col0) = make_uint2(lo, hi);
+            }
+        }
+        if (IS_ACT) {
+#pragma unroll
+            for (int c = 0; c < CPT; ++c) cur[c] = nxt[c];
+        } else {
+#pragma unroll
+            for (int c = 0; c < CPT; ++c) {
+                const int col0 = 8 * (tl + c * G);
+                if (nrow < M && col0 < K) cur[c].load(in + (size_t)nrow * K + col0);
+                else cur[c].zero();
+            }
+        }
+    }
+}
+
+// Rows too long to hold in registers (K > 4 * 512 * 8 = 16384): two passes
+// over the row, one for the absmax and one for the codes.  One block of 512
+// threads per row at a time.
+template <typename InT, bool IS_ACT>
+__global__ void __launch_bounds__(512)
+row_quant_long_kernel(const InT *__restrict__ in, const float *__restrict__ lam,
+                      int M, int K, int8_t *__restrict__ q,
+                      float *__restrict__ scale) {
+    __shared__ float red[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    for (int row = blockIdx.x; row < M; row += gridDim.x) {
+        const InT *r = in + (size_t)row * K;
+        float a = 0.0f;
+        for (int col0 = 8 * tid; col0 < K; col0 += 8 * blockDim.x) {
+            Chunk<InT> ch;
+            ch.load(r + col0);
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+                float fe = 1.0f;
+                if (lam) { const float l = __ldg(lam + col0 + e); fe = IS_ACT ? __frcp_rn(l) : l; }
+                a = fmaxf(a, fabsf(__fmul_rn(ch.get(e), fe)));
+            }
+        }
+        a = warp_max(a);
+        if (lane == 0) red[warp] = a;
+        __syncthreads();
+        a = 0.0f;
+        for (int w = 0; w < (int)(blockDim.x >> 5); ++w) a = fmaxf(a, red[w]);
+        __syncthreads();
+        const bool zero_row = (a == 0.0f);
+        const float inv = zero_row ? 0.0f : __fdiv_rn(127.0f, a);
+        if (tid == 0) scale[row] = zero_row ? 0.0f : __fdiv_rn(a, 127.0f);
+        for (int col0 = 8 * tid; col0 < K; col0 += 8 * blockDim.x) {
+            Chunk<InT> ch;
+            ch.load(r + col0);
+            uint32_t lo = 0, hi = 0;
+            if (!zero_row) {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    float fe = 1.0f;
+                    if (lam) { const float l = __ldg(lam + col0 + e); fe = IS_ACT ? __frcp_rn(l) : l; }
+                    const float xs = __fmul_rn(ch.get(e), fe);
+                    const uint32_t b = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xs, inv))) & 0xffu;
+                    if (e < 4) lo |= b << (8 * e);
+                    else hi |= b << (8 * (e - 4));
+                }
+            }
+            *reinterpret_cast<uint2 *>(q + (size_t)row * K + col0) = make_uint2(lo, hi);
+        }
+    }
+}
+
+int g_num_sms = 0;
+
+int num_sms() {
+    if (g_num_sms == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
+        if (g_num_sms <= 0) g_num_sms = 148;
+    }
+    return g_num_sms;
+}
+
+template <typename InT, bool IS_ACT, int CPT>
+cudaError_t launch_row_quant_cpt(const InT *in, const float *lam, int M, int K, int G,
+                                 int8_t *q, float *scale, cudaStream_t st) {
+    const int block = G < 256 ? 256 : G;
+    const int teams = block / G;
+    const int groups = (M + teams - 1) / teams;
+    int per_sm = 0;
+    cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, row_quant_kernel<InT, IS_ACT, CPT>,
+                                                  block, 0);
+    if (per_sm < 1) per_sm = 1;
+    int grid = num_sms() * per_sm;
+    if (grid > groups) grid = groups;
+    if (grid < 1) grid = 1;
+    row_quant_kernel<InT, IS_ACT, CPT><<<grid, block, 0, st>>>(in, lam, M, K, G, q, scale);
+    return cudaGetLastError();
+}
+
+// Team size: the smallest power of two in [32, 512] that covers the row in at
+// most 4 chunks of 8 per thread; longer rows take the two-pass kernel.
+template <typename InT, bool IS_ACT>
+cudaError_t launch_row_quant(const InT *in, const float *lam, int M, int K,
+                             int8_t *q, float *scale, cudaStream_t st) {
+    const int chunks = K / 8;
+    int G = 32;
+    while (G < 512 && G * 4 < chunks) G *= 2;
+    const int cpt = (chunks + G - 1) / G;
+    if (cpt <= 1) return launch_row_quant_cpt<InT, IS_ACT, 1>(in, lam, M, K, G, q, scale, st);
+    if (cpt <= 2) return launch_row_quant_cpt<InT, IS_ACT, 2>(in, lam, M, K, G, q, scale, st);
+    if (cpt <= 4) return launch_row_quant_cpt<InT, IS_ACT, 4>(in, lam, M, K, G, q, scale, st);
+    int g2 = num_sms() * 2;
+    if (g2 > M) g2 = M;
+    row_quant_long_kernel<InT, IS_ACT><<<g2, 512, 0, st>>>(in, lam, M, K, q, scale);
+    return cudaGetLastError();
+}
+
+// ----------------------------------------------------------- column absmax
+//
+// out_j = max_i |in_ij| over rows [0, R).  Each thread owns 8 consecutive
+// columns and a slab of rows; slabs combine with an integer atomicMax on the
+// bit patterns (non-negative floats order like their bit patterns).  `out`
+// must be zeroed first.
+template <typename InT>
+__global__ void col_absmax_kernel(const InT *__restrict__ in, int R, int C,
+                                  int rows_per_slab, float *__restrict__ out) {
+    const int cg = blockIdx.x * blockDim.x + threadIdx.x;
+    const int col0 = 8 * cg;
+    if (col0 >= C) return;
+    const int r0 = blockIdx.y * rows_per_slab;
+    int r1 = r0 + rows_per_slab;
+    if (r1 > R) r1 = R;
+    float m[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) m[e] = 0.0f;
+    for (int r = r0; r < r1; ++r) {
+        Chunk<InT> ch;
+        ch.load(in + (size_t)r * C + col0);
+#pragma unroll
+        for (int e = 0; e < 8; ++e) m[e] = fmaxf(m[e], fabsf(ch.get(e)));
+    }
+    if (r0 < r1) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+            atomicMax(reinterpret_cast<unsigned int *>(out + col0 + e), __float_as_uint(m[e]));
+    }
+}
+
+template <typename InT>
+cudaError_t launch_col_absmax(const InT *in, int R, int C, float *out, cudaStream_t st) {
+    cudaError_t e = cudaMemsetAsync(out, 0, sizeof(float) * (size_t)C, st);
+    if (e != cudaSuccess) return e;
+    if (R <= 0) return cudaSuccess;
+    const int threads = 128;
+    const int gx = (C / 8 + threads - 1) / threads;
+    int gy = (num_sms() * 8 + gx - 1) / gx;
+    if (gy > R) gy = R;
+    if (gy < 1) gy = 1;
+    const int rows_per_slab = (R + gy - 1) / gy;
+    gy = (R + rows_per_slab - 1) / rows_per_slab;
+    col_absmax_kernel<InT><<<dim3(gx, gy), threads, 0, st>>>(in, R, C, rows_per_slab, out);
+    return cudaGetLastError();
+}
+
+// lambda_j = s_j^alpha / m_j^(1-alpha), m_j already stored in lambda[j].
+__global__ void smooth_finalize_kernel(const float *__restrict__ s, float alpha,
+                                       int K, float *__restrict__ lambda) {
+    const int j = blockIdx.x * blockDim.x + threadIdx.x;
+    if (j >= K) return;
+    const float sj = s[j];
+    const float m = lambda[j];
+    float l;
+    if (sj == 0.0f || m == 0.0f) l = 1.0f;
+    else if (alpha == 0.5f) l = __fdiv_rn(__fsqrt_rn(sj), __fsqrt_rn(m));
+    else if (alpha == 1.0f) l = sj;
+    else if (alpha == 0.0f) l = __fdiv_rn(1.0f, m);
+    else l = __double2float_rn(exp2((double)alpha * log2((double)sj) -
+                                    (1.0 - (double)alpha) * log2((double)m)));
+    lambda[j] = l;
+}
+
+}  // namespace
+
+cudaError_t launch_channel_absmax(const uint16_t *X, int T, int K, float *s, cudaStream_t st) {
+    return launch_col_absmax<uint16_t>(X, T, K, s, st);
+}
+
+cudaError_t launch_smooth_scales(const float *s, const float *W, int N, int K,
+                                 float alpha, float *lambda, cudaStream_t st) {
+    cudaError_t e = launch_col_absmax<float>(W, N, K, lambda, st);
+    if (e != cudaSuccess) return e;
+    smooth_finalize_kernel<<<(K + 255) / 256, 256, 0, st>>>(s, alpha, K, lambda);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_quantize_weights(const float *W, const float *lambda, int N, int K,
+                                    int8_t *Wq, float *w_scale, cudaStream_t st) {
+    return launch_row_quant<float, false>(W, lambda, N, K, Wq, w_scale, st);
+}
+
+cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M, int K,
+                             int8_t *Xq, float *x_scale, cudaStream_t st) {
+    return launch_row_quant<uint16_t, true>(X, lambda, M, K, Xq, x_scale, st);
+}
+
+}  // namespace w8a8

@@ -1,0 +1,217 @@
+"""Python binding of the W8A8 C ABI (include/w8a8.h).
+
+Argument marshalling only: each function takes CUDA tensors, checks dtype,
+device and contiguity, and passes ``data_ptr()`` plus the current CUDA stream
+to the function of the same name in ``libw8a8.so``.  Every step of the layer
+runs in the library's CUDA kernels; there is no fallback.  If the library has
+not been built, or cannot be loaded, the first call raises.
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+import threading
+
+import torch
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "_build", "libw8a8.so")
+
+W8A8_OK = 0
+STATUS_NAMES = {0: "W8A8_OK", 1: "W8A8_ERR_INVALID_ARG", 2: "W8A8_ERR_UNSUPPORTED_SHAPE",
+                3: "W8A8_ERR_MISALIGNED", 4: "W8A8_ERR_CUDA", 5: "W8A8_ERR_TIMEOUT"}
+
+# name -> argument types, in header order
+_P, _I, _F = ctypes.c_void_p, ctypes.c_int, ctypes.c_float
+SIGNATURES = {
+    "w8a8_channel_absmax": [_P, _I, _I, _P, _P],
+    "w8a8_smooth_scales": [_P, _P, _I, _I, _F, _P, _P],
+    "w8a8_quantize_weights": [_P, _P, _I, _I, _P, _P, _P],
+    "w8a8_quant_act": [_P, _P, _I, _I, _P, _P, _P],
+    "w8a8_linear": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P],
+    "w8a8_linear_dual": [_P, _I, _I, _P],
+    "w8a8_debug_gemm_i32": [_P, _P, _I, _I, _I, _P, _P],
+    "w8a8_set_gemm_engine": [_I],
+    "w8a8_get_gemm_engine": [],
+    "w8a8_device_status": [_P, ctypes.POINTER(ctypes.c_uint32)],
+    "w8a8_status_string": [_I],
+}
+
+
+class W8A8Error(RuntimeError):
+    def __init__(self, fn: str, status: int):
+        super().__init__(f"{fn} returned {STATUS_NAMES.get(status, status)}")
+        self.status = status
+
+
+class Branch(ctypes.Structure):
+    """Mirror of ``w8a8_branch``."""
+    _fields_ = [("Xq", _P), ("x_scale", _P), ("Wq", _P), ("w_scale", _P),
+                ("bias", _P), ("Y", _P), ("M", _I)]
+
+
+_lock = threading.Lock()
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    """The loaded library (raises if it is missing: there is no fallback)."""
+    global _lib
+    with _lock:
+        if _lib is None:
+            if not os.path.exists(LIB_PATH):
+                raise RuntimeError(
+                    f"W8A8 CUDA library not built ({LIB_PATH} missing); run "
+                    "`python -c 'import __graft_entry__ as g; g.build()'`")
+            L = ctypes.CDLL(LIB_PATH)
+            for name, args in SIGNATURES.items():
+                fn = getattr(L, name)
+                fn.argtypes = args
+                fn.restype = ctypes.c_int
+            L.w8a8_status_string.restype = ctypes.c_char_p
+            _lib = L
+    return _lib
+
+
+def _check(name: str, status: int) -> None:
+    if status != W8A8_OK:
+        raise W8A8Error(name, status)
+
+
+def _stream(stream=None) -> int:
+    s = stream if stream is not None else torch.cuda.current_stream()
+    return s.cuda_stream
+
+
+def _ptr(t, dtype, name):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor) or not t.is_cuda:
+        raise TypeError(f"{name} must be a CUDA tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    return t.data_ptr()
+
+
+def channel_absmax(X, s=None, stream=None):
+    """s_j = max_t |X_tj| (calibration statistic).  X [T,K] bf16 -> s [K] fp32."""
+    T, K = X.shape
+    if s is None:
+        s = torch.empty(K, dtype=torch.float32, device=X.device)
+    _check("w8a8_channel_absmax", lib().w8a8_channel_absmax(
+        _ptr(X, torch.bfloat16, "X"), T, K, _ptr(s, torch.float32, "s"), _stream(stream)))
+    return s
+
+
+def smooth_scales(act_absmax, W, alpha: float, smooth=None, stream=None):
+    """lambda_j = s_j^alpha / max_i |W_ij|^(1-alpha).  W [N,K] fp32 -> [K] fp32."""
+    N, K = W.shape
+    if smooth is None:
+        smooth = torch.empty(K, dtype=torch.float32, device=W.device)
+    _check("w8a8_smooth_scales", lib().w8a8_smooth_scales(
+        _ptr(act_absmax, torch.float32, "act_absmax"), _ptr(W, torch.float32, "W"), N, K,
+        float(alpha), _ptr(smooth, torch.float32, "smooth"), _stream(stream)))
+    return smooth
+
+
+def quantize_weights(W, smooth=None, Wq=None, w_scale=None, stream=None):
+    """Per-output-channel INT8 of W diag(lambda): returns (Wq [N,K] int8, sw [N] fp32)."""
+    N, K = W.shape
+    if Wq is None:
+        Wq = torch.empty(N, K, dtype=torch.int8, device=W.device)
+    if w_scale is None:
+        w_scale = torch.empty(N, dtype=torch.float32, device=W.device)
+    _check("w8a8_quantize_weights", lib().w8a8_quantize_weights(
+        _ptr(W, torch.float32, "W"), _ptr(smooth, torch.float32, "smooth"), N, K,
+        _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"), _stream(stream)))
+    return Wq, w_scale
+
+
+def quant_act(X, smooth=None, Xq=None, x_scale=None, stream=None):
+    """Per-token INT8 of X diag(lambda)^-1: returns (Xq [M,K] int8, sx [M] fp32)."""
+    M, K = X.shape
+    if Xq is None:
+        Xq = torch.empty(M, K, dtype=torch.int8, device=X.device)
+    if x_scale is None:
+        x_scale = torch.empty(M, dtype=torch.float32, device=X.device)
+    _check("w8a8_quant_act", lib().w8a8_quant_act(
+        _ptr(X, torch.bfloat16, "X"), _ptr(smooth, torch.float32, "smooth"), M, K,
+        _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"), _stream(stream)))
+    return Xq, x_scale
+
+
+def linear(Xq, x_scale, Wq, w_scale, bias=None, Y=None, stream=None):
+    """Y = bf16((Xq Wq^T) * sx * sw + b): [M,N] bf16."""
+    M, K = Xq.shape
+    N = Wq.shape[0]
+    if Wq.shape[1] != K:
+        raise ValueError("Xq and Wq disagree on K")
+    if Y is None:
+        Y = torch.empty(M, N, dtype=torch.bfloat16, device=Xq.device)
+    _check("w8a8_linear", lib().w8a8_linear(
+        _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"),
+        _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
+        _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(Y, torch.bfloat16, "Y"),
+        _stream(stream)))
+    return Y
+
+
+def linear_dual(branches, Ys=None, stream=None):
+    """One grouped launch over two branches.  branches: two tuples
+    (Xq, x_scale, Wq, w_scale, bias); returns [Y_cond, Y_uncond]."""
+    if len(branches) != 2:
+        raise ValueError("linear_dual takes exactly two branches")
+    N, K = branches[0][2].shape
+    arr = (Branch * 2)()
+    out = []
+    for i, (Xq, sx, Wq, sw, b) in enumerate(branches):
+        if tuple(Wq.shape) != (N, K) or Xq.shape[1] != K:
+            raise ValueError("branches must share N and K")
+        Y = Ys[i] if Ys is not None else torch.empty(Xq.shape[0], N, dtype=torch.bfloat16,
+                                                     device=Xq.device)
+        arr[i] = Branch(_ptr(Xq, torch.int8, "Xq"), _ptr(sx, torch.float32, "x_scale"),
+                        _ptr(Wq, torch.int8, "Wq"), _ptr(sw, torch.float32, "w_scale"),
+                        _ptr(b, torch.float32, "bias"), _ptr(Y, torch.bfloat16, "Y"),
+                        Xq.shape[0])
+        out.append(Y)
+    _check("w8a8_linear_dual", lib().w8a8_linear_dual(arr, N, K, _stream(stream)))
+    return out
+
+
+def debug_gemm_i32(Xq, Wq, acc=None, stream=None):
+    """Exact int32 acc = Xq Wq^T (test export of the GEMM alone)."""
+    M, K = Xq.shape
+    N = Wq.shape[0]
+    if acc is None:
+        acc = torch.empty(M, N, dtype=torch.int32, device=Xq.device)
+    _check("w8a8_debug_gemm_i32", lib().w8a8_debug_gemm_i32(
+        _ptr(Xq, torch.int8, "Xq"), _ptr(Wq, torch.int8, "Wq"), M, N, K,
+        _ptr(acc, torch.int32, "acc"), _stream(stream)))
+    return acc
+
+
+def set_gemm_engine(engine: int) -> None:
+    """1 = tcgen05 tensor cores, 0 = legacy mma.sync s8, -1 = default."""
+    _check("w8a8_set_gemm_engine", lib().w8a8_set_gemm_engine(int(engine)))
+
+
+def get_gemm_engine() -> int:
+    return int(lib().w8a8_get_gemm_engine())
+
+
+def device_status(stream=None) -> int:
+    """Synchronise the stream and return (and clear) the device error word."""
+    detail = ctypes.c_uint32(0)
+    st = lib().w8a8_device_status(_stream(stream), ctypes.byref(detail))
+    if st not in (W8A8_OK, 5):
+        raise W8A8Error("w8a8_device_status", st)
+    return int(detail.value)
+
+
+def quantized_linear_forward(X, smooth, Wq, w_scale, bias=None, stream=None):
+    """The per-call hot path of one quantized linear: a3 then a4+a5."""
+    Xq, sx = quant_act(X, smooth, stream=stream)
+    return linear(Xq, sx, Wq, w_scale, bias, stream=stream)

@@ -1,0 +1,140 @@
+"""Host-side checks of the C ABI that need no GPU.
+
+The library must build for sm_103a, load, and export every symbol that
+include/w8a8.h declares.  Argument validation runs on the host before any CUDA
+call, so invalid calls are exercised here with fake (never dereferenced)
+pointer values and must return their status codes without touching a device.
+"""
+
+import ctypes
+import os
+import re
+
+import pytest
+
+from paper_2606_12280_gb300 import _build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "w8a8.h")
+
+OK, INVALID, SHAPE, MISALIGNED = 0, 1, 2, 3
+
+
+@pytest.fixture(scope="module")
+def L():
+    _build.build()
+    from paper_2606_12280_gb300 import w8a8
+    return w8a8.lib()
+
+
+def declared_functions():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"W8A8_API\s+[\w\s\*]*?\b(w8a8_\w+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_functions()
+    for required in ("w8a8_smooth_scales", "w8a8_quantize_weights", "w8a8_quant_act",
+                     "w8a8_linear", "w8a8_linear_dual", "w8a8_debug_gemm_i32",
+                     "w8a8_channel_absmax", "w8a8_status_string"):
+        assert required in names
+
+
+def test_library_exports_every_declared_symbol(L):
+    for name in declared_functions():
+        assert hasattr(L, name), name
+
+
+def test_binding_covers_every_symbol():
+    from paper_2606_12280_gb300 import w8a8
+    assert set(declared_functions()) == set(w8a8.SIGNATURES)
+
+
+def test_status_strings(L):
+    assert L.w8a8_status_string(0) == b"W8A8_OK"
+    assert L.w8a8_status_string(5) == b"W8A8_ERR_TIMEOUT"
+    assert L.w8a8_status_string(99) == b"W8A8_ERR_UNKNOWN"
+
+
+A = 0x100000          # a fake, 16-byte aligned "device" address (never used)
+U = A + 4             # a misaligned one
+
+
+def test_quant_act_validation(L):
+    f = L.w8a8_quant_act
+    assert f(A, None, 4, 15, A, A, None) == SHAPE        # K % 16
+    assert f(A, None, 4, 0, A, A, None) == SHAPE
+    assert f(A, None, -1, 16, A, A, None) == SHAPE
+    assert f(A, None, 4, 133152, A, A, None) == SHAPE    # K beyond the int32 bound
+    assert f(None, None, 4, 16, A, A, None) == INVALID
+    assert f(A, None, 4, 16, None, A, None) == INVALID
+    assert f(A, None, 4, 16, A, None, None) == INVALID
+    assert f(U, None, 4, 16, A, A, None) == MISALIGNED
+    assert f(A, U, 4, 16, A, A, None) == MISALIGNED
+    assert f(A, None, 0, 16, A, A, None) == OK            # empty batch: no-op
+
+
+def test_weight_and_smooth_validation(L):
+    q = L.w8a8_quantize_weights
+    assert q(A, None, 12, 16, A, A, None) == SHAPE        # N % 8
+    assert q(A, None, 8, 24, A, A, None) == SHAPE         # K % 16
+    assert q(None, None, 8, 16, A, A, None) == INVALID
+    assert q(A, None, 8, 16, U, A, None) == MISALIGNED
+    sm = L.w8a8_smooth_scales
+    assert sm(A, A, 8, 16, 1.5, A, None) == INVALID       # alpha outside [0, 1]
+    assert sm(A, A, 8, 16, -0.1, A, None) == INVALID
+    assert sm(A, A, 8, 16, float("nan"), A, None) == INVALID
+    assert sm(None, A, 8, 16, 0.5, A, None) == INVALID
+    assert sm(A, A, 8, 16, 0.5, U, None) == MISALIGNED
+    ca = L.w8a8_channel_absmax
+    assert ca(A, 4, 8, A, None) == SHAPE
+    assert ca(A, 4, 16, None, None) == INVALID
+
+
+def test_linear_validation(L):
+    f = L.w8a8_linear
+    assert f(A, A, A, A, None, 4, 12, 16, A, None) == SHAPE     # N % 8
+    assert f(A, A, A, A, None, 4, 8, 24, A, None) == SHAPE      # K % 16
+    assert f(A, A, A, A, None, -2, 8, 16, A, None) == SHAPE
+    assert f(None, A, A, A, None, 4, 8, 16, A, None) == INVALID
+    assert f(A, None, A, A, None, 4, 8, 16, A, None) == INVALID
+    assert f(A, A, A, A, None, 4, 8, 16, None, None) == INVALID
+    assert f(A, A, U, A, None, 4, 8, 16, A, None) == MISALIGNED
+    assert f(A, A, A, A, U, 4, 8, 16, A, None) == MISALIGNED    # bias
+    assert f(A, A, A, A, None, 0, 8, 16, A, None) == OK          # empty batch
+    g = L.w8a8_debug_gemm_i32
+    assert g(A, A, 4, 8, 15, A, None) == SHAPE
+    assert g(A, None, 4, 8, 16, A, None) == INVALID
+
+
+def test_dual_validation(L):
+    from paper_2606_12280_gb300.w8a8 import Branch
+    arr = (Branch * 2)()
+    for i in range(2):
+        arr[i] = Branch(A, A, A, A, None, A, 4)
+    f = L.w8a8_linear_dual
+    assert f(None, 8, 16, None) == INVALID
+    assert f(arr, 12, 16, None) == SHAPE
+    arr[1].Wq = U
+    assert f(arr, 8, 16, None) == MISALIGNED
+    arr[1].Wq = None
+    assert f(arr, 8, 16, None) == INVALID
+    arr[0].M = 0
+    arr[1] = Branch(None, None, None, None, None, None, 0)
+    assert f(arr, 8, 16, None) == OK                      # both branches empty
+
+
+def test_engine_switch(L):
+    assert L.w8a8_set_gemm_engine(7) == INVALID
+    assert L.w8a8_set_gemm_engine(0) == OK
+    assert L.w8a8_get_gemm_engine() == 0
+    assert L.w8a8_set_gemm_engine(-1) == OK
+    assert L.w8a8_get_gemm_engine() == 1
+
+
+def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
+    from paper_2606_12280_gb300 import w8a8
+    monkeypatch.setattr(w8a8, "_lib", None)
+    monkeypatch.setattr(w8a8, "LIB_PATH", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="not built"):
+        w8a8.lib()
