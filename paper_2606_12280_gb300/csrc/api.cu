@@ -31,9 +31,16 @@ w8a8_status from_cuda(cudaError_t e) { return e == cudaSuccess ? W8A8_OK : W8A8_
 
 cudaStream_t as_stream(void *s) { return static_cast<cudaStream_t>(s); }
 
+// Address of the error word on the current device, looked up once per device.
 unsigned int *device_error_word() {
+    constexpr int kMaxDevices = 64;
+    static unsigned int *cache[kMaxDevices] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
+    if (dev >= 0 && dev < kMaxDevices && cache[dev]) return cache[dev];
     void *p = nullptr;
     if (cudaGetSymbolAddress(&p, g_w8a8_device_error) != cudaSuccess) return nullptr;
+    if (dev >= 0 && dev < kMaxDevices) cache[dev] = static_cast<unsigned int *>(p);
     return static_cast<unsigned int *>(p);
 }
 
@@ -112,7 +119,9 @@ w8a8_status w8a8_quant_act(const uint16_t *X, const float *smooth, int M, int K,
     if (!X || !Xq || !x_scale) return W8A8_ERR_INVALID_ARG;
     if (!aligned16(X) || !aligned16(Xq) || !aligned16(x_scale) || (smooth && !aligned16(smooth)))
         return W8A8_ERR_MISALIGNED;
-    return from_cuda(w8a8::launch_quant_act(X, smooth, M, K, Xq, x_scale, as_stream(stream)));
+    unsigned int *err = device_error_word();
+    if (!err) return W8A8_ERR_CUDA;
+    return from_cuda(w8a8::launch_quant_act(X, smooth, M, K, Xq, x_scale, err, as_stream(stream)));
 }
 
 w8a8_status w8a8_linear(const int8_t *Xq, const float *x_scale, const int8_t *Wq,

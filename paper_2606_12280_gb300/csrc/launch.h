@@ -25,7 +25,7 @@ cudaError_t launch_quantize_weights(const float *W, const float *lambda, int N,
                                     int K, int8_t *Wq, float *w_scale,
                                     cudaStream_t st);
 cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M,
-                             int K, int8_t *Xq, float *x_scale,
+                             int K, int8_t *Xq, float *x_scale, unsigned int *err,
                              cudaStream_t st);
 
 // Legacy warp-level mma.sync s8 GEMM (exact int32), nb = 1 or 2 branches.
