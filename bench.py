@@ -201,6 +201,12 @@ def run_reference(args):
 
 METRIC = "W8A8 linear INT8 TOPS (act-quant + INT8 GEMM + fused dequant epilogue)"
 
+# DRAM bytes (read + write) of one GEMM launch from the ncu capture summarised
+# in profiles/gemm_tc_qkv_m4608_k4096_n12288.md; valid only for the kernel
+# version profiled there (set to None whenever the GEMM changes until the
+# capture is repeated).
+GEMM_TRAFFIC_BYTES = {"qkv_m4608_k4096_n12288": 135.92e6}
+
 
 # --------------------------------------------------------------------- ours
 
@@ -378,7 +384,10 @@ def run_ours(args):
                              f"(> L2 between reuses), no flush",
                        "gemm_engine": "tcgen05" if engine == 1 else "mma.sync"},
             "roofline": {"bound": "tensor", "achieved": gemm_tflops, "peak": peak_t,
-                         "unit": "TFLOP/s", "frac": gemm_tflops / peak_t, "traffic": None,
+                         "unit": "TFLOP/s", "frac": gemm_tflops / peak_t,
+                         "traffic": GEMM_TRAFFIC_BYTES.get(args.workload) if engine == 1 else None,
+                         "traffic_unit": "bytes per launch (ncu dram read + write)",
+                         "algorithmic_bytes": float(M * K + N * K + 2 * M * N + 4 * (M + 2 * N)),
                          "kernel": "w8a8_linear (a4+a5)",
                          "peak_source": f"{peak_kind} bf16 dense burst (the fp16/bf16 tensor "
                                         f"datapath the exact-integer GEMM runs on)"},
