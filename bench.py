@@ -205,7 +205,7 @@ METRIC = "W8A8 linear INT8 TOPS (act-quant + INT8 GEMM + fused dequant epilogue)
 # in profiles/gemm_tc_qkv_m4608_k4096_n12288.md; valid only for the kernel
 # version profiled there (set to None whenever the GEMM changes until the
 # capture is repeated).
-GEMM_TRAFFIC_BYTES = {"qkv_m4608_k4096_n12288": 135.92e6}
+GEMM_TRAFFIC_BYTES = {(1, "qkv_m4608_k4096_n12288"): 135.92e6}
 
 
 # --------------------------------------------------------------------- ours
@@ -382,10 +382,10 @@ def run_ours(args):
             "config": {"workload": args.workload, "M": M, "K": K, "N": N, "alpha": case.alpha,
                        "l2": f"{n_sets} rotating input sets of {set_bytes / 2**20:.0f} MiB "
                              f"(> L2 between reuses), no flush",
-                       "gemm_engine": "tcgen05" if engine == 1 else "mma.sync"},
+                       "gemm_engine": {2: "tcgen05 cta pair", 1: "tcgen05", 0: "mma.sync"}[engine]},
             "roofline": {"bound": "tensor", "achieved": gemm_tflops, "peak": peak_t,
                          "unit": "TFLOP/s", "frac": gemm_tflops / peak_t,
-                         "traffic": GEMM_TRAFFIC_BYTES.get(args.workload) if engine == 1 else None,
+                         "traffic": GEMM_TRAFFIC_BYTES.get((engine, args.workload)),
                          "traffic_unit": "bytes per launch (ncu dram read + write)",
                          "algorithmic_bytes": float(M * K + N * K + 2 * M * N + 4 * (M + 2 * N)),
                          "kernel": "w8a8_linear (a4+a5)",

@@ -165,10 +165,11 @@ W8A8_API w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int
 
 /*
  * The GEMM engine that w8a8_linear, w8a8_linear_dual and w8a8_debug_gemm_i32
- * use on this device: 1 = tcgen05 tensor cores (exact integer products on the
- * fp16 datapath, see the design notes), 0 = warp-level mma.sync s8 (legacy
- * tensor path).  w8a8_set_gemm_engine(-1) restores the default (tcgen05);
- * other values give W8A8_ERR_INVALID_ARG.  The setting is process-wide.
+ * use: 2 = tcgen05 on pairs of SMs (cta_group::2, 256x256 tiles), 1 = tcgen05
+ * on single SMs (128x256 tiles), both computing the exact integer product on
+ * the fp16 tensor datapath; 0 = warp-level mma.sync s8 (legacy INT8 tensor
+ * path).  The default is 2; w8a8_set_gemm_engine(-1) restores it; other
+ * values give W8A8_ERR_INVALID_ARG.  The setting is process-wide.
  */
 W8A8_API w8a8_status w8a8_set_gemm_engine(int engine);
 W8A8_API int w8a8_get_gemm_engine(void);

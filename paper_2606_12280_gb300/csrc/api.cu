@@ -12,7 +12,7 @@ namespace {
 // record a nonzero code here instead of spinning forever.
 __device__ unsigned int g_w8a8_device_error = 0;
 
-int g_engine = 1;   // 1 = tcgen05, 0 = mma.sync
+int g_engine = 2;   // 2 = tcgen05 CTA pairs, 1 = tcgen05, 0 = mma.sync
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -61,9 +61,10 @@ w8a8_status check_branch(const w8a8::GemmBranch &b, bool need_scales, int N, int
 
 w8a8_status run_gemm(const w8a8::GemmBranch *br, int nb, int N, int K, bool out_i32,
                      cudaStream_t st) {
-    if (g_engine == 1) {
+    if (g_engine == 1 || g_engine == 2) {
         unsigned int *err = device_error_word();
         if (!err) return W8A8_ERR_CUDA;
+        if (g_engine == 2) return from_cuda(w8a8::launch_gemm_tc2(br, nb, N, K, out_i32, err, st));
         return from_cuda(w8a8::launch_gemm_tc(br, nb, N, K, out_i32, err, st));
     }
     return from_cuda(w8a8::launch_gemm_mma(br, nb, N, K, out_i32, st));
@@ -160,8 +161,8 @@ w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int M, int N
 }
 
 w8a8_status w8a8_set_gemm_engine(int engine) {
-    if (engine == -1) engine = 1;
-    if (engine != 0 && engine != 1) return W8A8_ERR_INVALID_ARG;
+    if (engine == -1) engine = 2;
+    if (engine < 0 || engine > 2) return W8A8_ERR_INVALID_ARG;
     g_engine = engine;
     return W8A8_OK;
 }

@@ -33,6 +33,10 @@ cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M,
 cudaError_t launch_gemm_mma(const GemmBranch *br, int nb, int N, int K,
                             bool out_i32, cudaStream_t st);
 
+// tcgen05 GEMM on pairs of SMs (cta_group::2), same exact scheme.
+cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K,
+                            bool out_i32, unsigned int *err, cudaStream_t st);
+
 // tcgen05 GEMM (exact integer products on the fp16 tensor datapath).
 cudaError_t launch_gemm_tc(const GemmBranch *br, int nb, int N, int K,
                            bool out_i32, unsigned int *err, cudaStream_t st);

@@ -129,7 +129,8 @@ def test_engine_switch(L):
     assert L.w8a8_set_gemm_engine(0) == OK
     assert L.w8a8_get_gemm_engine() == 0
     assert L.w8a8_set_gemm_engine(-1) == OK
-    assert L.w8a8_get_gemm_engine() == 1
+    assert L.w8a8_get_gemm_engine() == 2
+    assert L.w8a8_set_gemm_engine(3) == INVALID
 
 
 def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):

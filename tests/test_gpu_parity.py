@@ -5,7 +5,8 @@ product bit-exact; bf16 outputs within 1 bf16 ulp (relative 2^-8), and in fact
 bit-identical because both sides follow the same pinned fp32 op order.  Sizes
 span several tiles with ragged tails; edge cases cover empty and single-row
 inputs, all-zero rows and columns, adversarial INT8 extremes and the largest K.
-Both GEMM engines (tcgen05 and mma.sync) are checked.
+All three GEMM engines (tcgen05 on SM pairs, tcgen05 on single SMs, and
+mma.sync) are checked.
 """
 
 import numpy as np
@@ -16,7 +17,7 @@ from paper_2606_12280_gb300 import workloads as wl
 
 pytestmark = pytest.mark.gpu
 
-ENGINES = [1, 0]
+ENGINES = [2, 1, 0]
 
 
 @pytest.fixture(scope="module")
@@ -29,7 +30,7 @@ def w8():
     w8a8.set_gemm_engine(-1)
 
 
-@pytest.fixture(params=ENGINES, ids=["tcgen05", "mma_sync"])
+@pytest.fixture(params=ENGINES, ids=["tcgen05_pair", "tcgen05", "mma_sync"])
 def engine(request, w8):
     w8.set_gemm_engine(request.param)
     yield request.param
