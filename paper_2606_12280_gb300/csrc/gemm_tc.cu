@@ -369,14 +369,20 @@ gemm_tc_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__
                 }
                 const uint32_t src = sb + OFF_ST8 + s8 * STAGE8 + src_off;
                 const uint32_t dst = sb + OFF_ST16 + s16 * STAGE16;
-#pragma unroll 2
-                for (int g = cw; g < (BM + BN) / 8; g += NUM_CONV_WARPS) {
-                    const uint4 v = ld_shared_v4(src + g * 8 * BK);
+                // all of this warp's 8-row groups in flight at once
+                constexpr int kPer = (BM + BN) / 8 / NUM_CONV_WARPS;
+                static_assert(kPer * NUM_CONV_WARPS * 8 == BM + BN, "even split");
+                uint4 v[kPer];
+#pragma unroll
+                for (int i = 0; i < kPer; ++i) v[i] = ld_shared_v4(src + (cw + i * NUM_CONV_WARPS) * 8 * BK);
+#pragma unroll
+                for (int i = 0; i < kPer; ++i) {
+                    const int g = cw + i * NUM_CONV_WARPS;
                     uint4 o0, o1;
-                    i8x4_to_f16x4(v.x, o0.x, o0.y);
-                    i8x4_to_f16x4(v.y, o0.z, o0.w);
-                    i8x4_to_f16x4(v.z, o1.x, o1.y);
-                    i8x4_to_f16x4(v.w, o1.z, o1.w);
+                    i8x4_to_f16x4(v[i].x, o0.x, o0.y);
+                    i8x4_to_f16x4(v[i].y, o0.z, o0.w);
+                    i8x4_to_f16x4(v[i].z, o1.x, o1.y);
+                    i8x4_to_f16x4(v[i].w, o1.z, o1.w);
                     st_shared_v4(dst + g * 1024 + dst_off0, o0);
                     st_shared_v4(dst + g * 1024 + dst_off1, o1);
                 }

@@ -377,16 +377,28 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                     }
                     const uint32_t src = sb + OFF_ST8 + s8 * STAGE8 + src_off;
                     const uint32_t dst = sb + OFF_ST16 + s16 * STAGE16;
-#pragma unroll 2
-                    for (int g = cw; g < (CTA_M + CTA_N) / 8; g += NUM_CONV_WARPS) {
-                        const uint4 v = ld_shared_v4(src + g * 8 * BK);
-                        uint4 o0, o1;
-                        i8x4_to_f16x4(v.x, o0.x, o0.y);
-                        i8x4_to_f16x4(v.y, o0.z, o0.w);
-                        i8x4_to_f16x4(v.z, o1.x, o1.y);
-                        i8x4_to_f16x4(v.w, o1.z, o1.w);
-                        st_shared_v4(dst + g * 1024 + dst_off0, o0);
-                        st_shared_v4(dst + g * 1024 + dst_off1, o1);
+                    // all of this warp's 8-row groups in flight at once: every load
+                    // is issued before the first conversion needs its data
+                    constexpr int kG = (CTA_M + CTA_N) / 8;
+                    constexpr int kPer = (kG + NUM_CONV_WARPS - 1) / NUM_CONV_WARPS;
+                    uint4 v[kPer];
+#pragma unroll
+                    for (int i = 0; i < kPer; ++i) {
+                        const int g = cw + i * NUM_CONV_WARPS;
+                        if (g < kG) v[i] = ld_shared_v4(src + g * 8 * BK);
+                    }
+#pragma unroll
+                    for (int i = 0; i < kPer; ++i) {
+                        const int g = cw + i * NUM_CONV_WARPS;
+                        if (g < kG) {
+                            uint4 o0, o1;
+                            i8x4_to_f16x4(v[i].x, o0.x, o0.y);
+                            i8x4_to_f16x4(v[i].y, o0.z, o0.w);
+                            i8x4_to_f16x4(v[i].z, o1.x, o1.y);
+                            i8x4_to_f16x4(v[i].w, o1.z, o1.w);
+                            st_shared_v4(dst + g * 1024 + dst_off0, o0);
+                            st_shared_v4(dst + g * 1024 + dst_off1, o1);
+                        }
                     }
                     fence_proxy_async_smem();
                     __syncwarp();
