@@ -502,6 +502,154 @@ cudaError_t launch_act_quant_staged(const uint16_t *X, const float *lam, int M, 
     return cudaGetLastError();
 }
 
+// ---------------------------------------------- activation quant, warp teams
+//
+// a3 with a team of TW warps per token row.  Every warp always owns the same
+// columns of the row (U chunks of 8 values per lane, chunk c = (u*TW + w)*32
+// + lane), so each lane computes its 8U factors 1/lambda_j once and keeps
+// them in registers for every row it visits, and keeps the smoothed values x'
+// in registers between the absmax and the quantization.  The bytes in flight
+// that HBM needs come from a per-warp ring of S row slices in shared memory
+// filled with cp.async (each lane reads back only the 16-byte chunks it
+// copied, so no block-level synchronisation is needed); the team combines its
+// warps' maxima through one named barrier per row.  Loads and stores are 512
+// B per warp instruction.
+__device__ __forceinline__ void cp_async_16(uint32_t dst, const void *src, bool valid) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+                 "r"(valid ? 16 : 0) : "memory");
+}
+
+template <int U, int TW, int S>
+__global__ void __launch_bounds__(TW > 8 ? 32 * TW : 256)
+act_quant_team_kernel(const uint16_t *__restrict__ X, const float *__restrict__ lam, int M, int K,
+                      int8_t *__restrict__ Xq, float *__restrict__ x_scale) {
+    constexpr int kThreads = TW > 8 ? 32 * TW : 256;
+    constexpr int kTeams = kThreads / (32 * TW);
+    extern __shared__ __align__(16) uint4 ring_s[];
+    __shared__ float red[2][kThreads / 32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int team = warp / TW, tw = warp % TW;
+    const int cpr = K / 8;                                  // 16-byte chunks per row
+    const uint32_t ring = static_cast<uint32_t>(__cvta_generic_to_shared(ring_s)) +
+                          static_cast<uint32_t>((warp * S * U * 32 + lane) * 16);
+
+    const int teams = gridDim.x * kTeams;
+    const int first = blockIdx.x * kTeams + team;
+    auto issue = [&](int k) {                               // row slice k of this team -> slot k % S
+        const int row = first + k * teams;
+        const uint32_t slot = ring + static_cast<uint32_t>((k % S) * U * 32 * 16);
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int c = (u * TW + tw) * 32 + lane;
+            const bool ok = row < M && c < cpr;
+            cp_async_16(slot + u * 32 * 16, ok ? (const void *)(X + (size_t)row * K + 8 * c) : (const void *)X, ok);
+        }
+        asm volatile("cp.async.commit_group;" ::: "memory");
+    };
+#pragma unroll
+    for (int k = 0; k < S - 1; ++k) issue(k);           // first rows in flight before the setup
+
+    float2 r[U][4];                                         // 1/lambda of this lane's columns
+#pragma unroll
+    for (int u = 0; u < U; ++u) {
+        const int c = (u * TW + tw) * 32 + lane;
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+            float f0 = 1.0f, f1 = 1.0f;
+            if (lam != nullptr && c < cpr) {
+                f0 = __frcp_rn(__ldg(lam + 8 * c + 2 * p));
+                f1 = __frcp_rn(__ldg(lam + 8 * c + 2 * p + 1));
+            }
+            r[u][p] = make_float2(f0, f1);
+        }
+    }
+
+    int parity = 0;
+    for (int k = 0;; ++k, parity ^= 1) {
+        const int row = first + k * teams;                  // uniform across the team
+        if (row >= M) break;
+        issue(k + S - 1);
+        asm volatile("cp.async.wait_group %0;" ::"n"(S - 1) : "memory");
+        const uint32_t slot = ring + static_cast<uint32_t>((k % S) * U * 32 * 16);
+        float2 xs[U][4];
+        float a = 0.0f;
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            uint4 v;
+            asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
+                         : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(slot + u * 32 * 16));
+            xs[u][0] = mul2_rn(make_float2(__uint_as_float(v.x << 16), __uint_as_float(v.x & 0xffff0000u)), r[u][0]);
+            xs[u][1] = mul2_rn(make_float2(__uint_as_float(v.y << 16), __uint_as_float(v.y & 0xffff0000u)), r[u][1]);
+            xs[u][2] = mul2_rn(make_float2(__uint_as_float(v.z << 16), __uint_as_float(v.z & 0xffff0000u)), r[u][2]);
+            xs[u][3] = mul2_rn(make_float2(__uint_as_float(v.w << 16), __uint_as_float(v.w & 0xffff0000u)), r[u][3]);
+#pragma unroll
+            for (int p = 0; p < 4; ++p) a = fmaxf(a, fmaxf(fabsf(xs[u][p].x), fabsf(xs[u][p].y)));
+        }
+        a = warp_max(a);
+        if (TW > 1) {
+            if (lane == 0) red[parity][warp] = a;
+            asm volatile("bar.sync %0, %1;" ::"r"(1 + team), "r"(TW * 32) : "memory");
+#pragma unroll
+            for (int w = 0; w < TW; ++w) a = fmaxf(a, red[parity][team * TW + w]);
+        }
+        const bool zero_row = (a == 0.0f);
+        const float inv = zero_row ? 0.0f : __fdiv_rn(127.0f, a);
+        if (tw == 0 && lane == 0) x_scale[row] = zero_row ? 0.0f : __fdiv_rn(a, 127.0f);
+        // a and 127/a finite: |x' * inv| <= 127 (1 + 2^-23), no clamp needed
+        const bool fast = (a <= 3.402823466e38f) && (inv <= 3.402823466e38f);
+        uint2 *qr = reinterpret_cast<uint2 *>(Xq + (size_t)row * K);
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+            const int c = (u * TW + tw) * 32 + lane;
+            if (c >= cpr) continue;
+            uint32_t word[2] = {0u, 0u};
+            if (zero_row) {
+            } else if (fast) {
+#pragma unroll
+                for (int h = 0; h < 2; ++h)
+                    word[h] = pack4_low_bytes(__fadd_rn(__fmul_rn(xs[u][2 * h].x, inv), kRoundMagic),
+                                              __fadd_rn(__fmul_rn(xs[u][2 * h].y, inv), kRoundMagic),
+                                              __fadd_rn(__fmul_rn(xs[u][2 * h + 1].x, inv), kRoundMagic),
+                                              __fadd_rn(__fmul_rn(xs[u][2 * h + 1].y, inv), kRoundMagic));
+            } else {
+#pragma unroll
+                for (int e = 0; e < 8; ++e) {
+                    const float xv = (e & 1) ? xs[u][e >> 1].y : xs[u][e >> 1].x;
+                    const uint32_t b = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xv, inv))) & 0xffu;
+                    word[e >> 2] |= b << (8 * (e & 3));
+                }
+            }
+            qr[c] = make_uint2(word[0], word[1]);
+        }
+    }
+    asm volatile("cp.async.wait_group 0;" ::: "memory");
+}
+
+template <int U, int TW>
+cudaError_t launch_act_quant_team(const uint16_t *X, const float *lam, int M, int K, int8_t *Xq,
+                                  float *x_scale, cudaStream_t st) {
+    constexpr int S = 4;
+    constexpr int kThreads = TW > 8 ? 32 * TW : 256;
+    constexpr int kTeams = kThreads / (32 * TW);
+    constexpr size_t smem = (size_t)(kThreads / 32) * S * U * 32 * 16;
+    static int per_sm = 0;
+    auto kern = act_quant_team_kernel<U, TW, S>;
+    if (per_sm == 0) {
+        if (smem > 48 * 1024) {
+            cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                 (int)smem);
+            if (e != cudaSuccess) return e;
+        }
+        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem);
+        if (per_sm < 1) per_sm = 1;
+    }
+    int grid = num_sms() * per_sm;
+    const int blocks_needed = (M + kTeams - 1) / kTeams;
+    if (grid > blocks_needed) grid = blocks_needed;
+    kern<<<grid, kThreads, smem, st>>>(X, lam, M, K, Xq, x_scale);
+    return cudaGetLastError();
+}
+
 // ----------------------------------------------------------- column absmax
 //
 // out_j = max_i |in_ij| over rows [0, R).  Each thread owns 8 consecutive
@@ -587,6 +735,19 @@ cudaError_t launch_quantize_weights(const float *W, const float *lambda, int N, 
 
 cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M, int K,
                              int8_t *Xq, float *x_scale, unsigned int *err, cudaStream_t st) {
+    // one warp per row, row held in registers (16 chunks of 8 per lane covers
+    // K <= 4096 in one read; wider rows are read twice, the second time from
+    // L2); 1/lambda needs K * 4 bytes of shared memory per block
+    // team of TW warps per row, U chunks of 8 values per lane: K <= 256 U TW
+    if (K <= 16384) {
+        if (K <= 256) return launch_act_quant_team<1, 1>(X, lambda, M, K, Xq, x_scale, st);
+        if (K <= 512) return launch_act_quant_team<2, 1>(X, lambda, M, K, Xq, x_scale, st);
+        if (K <= 1024) return launch_act_quant_team<2, 2>(X, lambda, M, K, Xq, x_scale, st);
+        if (K <= 2048) return launch_act_quant_team<2, 4>(X, lambda, M, K, Xq, x_scale, st);
+        if (K <= 4096) return launch_act_quant_team<2, 8>(X, lambda, M, K, Xq, x_scale, st);
+        if (K <= 8192) return launch_act_quant_team<2, 16>(X, lambda, M, K, Xq, x_scale, st);
+        return launch_act_quant_team<4, 16>(X, lambda, M, K, Xq, x_scale, st);
+    }
     // rows per slot: about 16 KB of bf16 per slot, at most 16 rows (teams of >= 16
     // threads).  Wider rows go to the register-resident kernel, which measured
     // faster there (one 32 KB slot per row leaves too few rows in flight).
