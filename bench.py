@@ -201,11 +201,11 @@ def run_reference(args):
 
 METRIC = "W8A8 linear INT8 TOPS (act-quant + INT8 GEMM + fused dequant epilogue)"
 
-# DRAM bytes (read + write) of one GEMM launch from the ncu capture summarised
-# in profiles/gemm_tc_qkv_m4608_k4096_n12288.md; valid only for the kernel
-# version profiled there (set to None whenever the GEMM changes until the
-# capture is repeated).
-GEMM_TRAFFIC_BYTES = {(1, "qkv_m4608_k4096_n12288"): 135.92e6}
+# DRAM bytes (read + write) of one GEMM launch, keyed by (engine, workload),
+# from the ncu capture summarised in profiles/gemm_tc2_qkv_m4608_k4096_n12288.md;
+# valid only for the kernel version profiled there (removed whenever that
+# kernel changes, until the capture is repeated).
+GEMM_TRAFFIC_BYTES = {(2, "qkv_m4608_k4096_n12288"): 149.08e6}
 
 
 # --------------------------------------------------------------------- ours
