@@ -1,18 +1,18 @@
 // quant.cu -- the quantization passes of the W8A8 layer (Sec. 3, "INT8 W8A8").
 //
-//   row_quant_kernel      a3 per-token activation quant (bf16 in, x / lambda)
-//                         a2 per-output-channel weight quant (fp32 in, w * lambda)
+//   act_quant_team_kernel a3 per-token activation quant (bf16 in, x / lambda),
+//                         the per-call HBM-bound pass (K <= 16384)
+//   row_quant_kernel      a2 per-output-channel weight quant (fp32 in,
+//                         w * lambda), offline; also a3 for K > 16384 through
+//   row_quant_long_kernel the two-pass variant for very long rows
 //   col_absmax_kernel     column max |.| of a row-major matrix: the calibration
 //                         statistic s_j and the weight column max m_j of a1
 //   smooth_finalize       a1 lambda_j = s_j^alpha / m_j^(1-alpha)
 //
-// The activation pass is HBM-bound: one read of X (2 B/elem), one write of Xq
-// (1 B/elem) and one fp32 scale per row.  A "team" of G threads owns one row at
-// a time; each thread owns CPT chunks of 8 consecutive columns (one 16-byte
-// load of bf16) at a stride of 8*G columns, so every warp-wide load is a fully
-// coalesced 512-byte segment.  The per-column factor (1/lambda_j or lambda_j)
-// is computed once per thread and kept in registers for every row the team
-// visits; the next row's data is loaded before the current row is reduced.
+// In row_quant_kernel a "team" of G threads owns one row at a time; each
+// thread owns CPT chunks of 8 consecutive columns at a stride of 8*G columns,
+// so every warp-wide load is a fully coalesced segment, and keeps its
+// per-column factors (1/lambda_j or lambda_j) in registers for every row.
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -273,51 +273,6 @@ cudaError_t launch_row_quant(const InT *in, const float *lam, int M, int K,
     return cudaGetLastError();
 }
 
-// ------------------------------------------------ activation quant, staged
-//
-// a3 with the rows staged in shared memory by bulk async copies (TMA engine):
-// each block owns a ring of S slots, a slot holds R consecutive rows (one
-// contiguous copy of R*K*2 bytes), and thread 0 keeps S slots in flight.  A
-// team of G = 256/R threads quantizes one row of the slot; each thread owns
-// CPT chunks of 8 columns at a stride of 8*G columns.  1/lambda is computed
-// once per block into shared memory.  One __syncthreads per slot both
-// completes the cross-warp absmax and releases the slot for the next copy.
-constexpr int AQ_THREADS = 256;
-constexpr int AQ_SLOTS = 4;
-
-__device__ __forceinline__ void aq_bar_init(uint32_t bar) {
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(bar));
-}
-__device__ __forceinline__ void aq_bulk_load(uint32_t dst, const void *src, uint32_t bytes,
-                                             uint32_t bar) {
-    asm volatile("{\n.reg .b64 st;\nmbarrier.arrive.expect_tx.shared::cta.b64 st, [%0], %1;\n}"
-                 ::"r"(bar), "r"(bytes) : "memory");
-    asm volatile("cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];"
-                 ::"r"(dst), "l"(src), "r"(bytes), "r"(bar) : "memory");
-}
-// Bounded wait for a slot's copy.  On timeout the error word gets
-// kErrActQuantTimeout and the thread carries on (control flow stays uniform,
-// so no barrier can hang); the host sees the error through w8a8_device_status.
-constexpr unsigned int kErrActQuantTimeout = 32u;
-__device__ __forceinline__ void aq_wait(uint32_t bar, uint32_t parity, unsigned int *err) {
-    uint64_t t0 = 0;
-    for (uint32_t it = 0;; ++it) {
-        uint32_t ok;
-        asm volatile("{\n.reg .pred p;\nmbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
-                     "selp.u32 %0, 1, 0, p;\n}" : "=r"(ok) : "r"(bar), "r"(parity) : "memory");
-        if (ok) return;
-        if ((it & 255u) == 0u) {
-            uint64_t t;
-            asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
-            if (it == 0) t0 = t;
-            else if (t - t0 > 1000000000ull) {        // 1 s
-                atomicOr(err, kErrActQuantTimeout);
-                return;
-            }
-        }
-    }
-}
-
 // Low byte of the fp32 sum 1.5*2^23 + y is round_half_even(y) in two's
 // complement whenever |y| < 2^22: the sum lies in [2^23, 2^24), where the
 // spacing of fp32 is exactly 1, so the addition itself rounds y to the nearest
@@ -341,165 +296,6 @@ __device__ __forceinline__ uint32_t pack4_low_bytes(float a, float b, float c, f
     const uint32_t ab = __byte_perm(__float_as_uint(a), __float_as_uint(b), 0x0040);
     const uint32_t cd = __byte_perm(__float_as_uint(c), __float_as_uint(d), 0x0040);
     return __byte_perm(ab, cd, 0x5410);
-}
-
-template <int CPT>
-__global__ void __launch_bounds__(AQ_THREADS)
-act_quant_staged_kernel(const uint16_t *__restrict__ X, const float *__restrict__ lam, int M,
-                        int K, int R, int8_t *__restrict__ Xq, float *__restrict__ x_scale,
-                        unsigned int *err) {
-    extern __shared__ __align__(128) uint8_t aq_smem[];
-    const int slot_bytes = R * K * 2;
-    float *rcp = reinterpret_cast<float *>(aq_smem + AQ_SLOTS * slot_bytes);
-    uint64_t *bars = reinterpret_cast<uint64_t *>(rcp + K);
-    __shared__ float red[2][AQ_THREADS / 32];
-
-    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int G = AQ_THREADS / R;
-    const int team = tid / G, tl = tid - team * G;
-    const int groups = (M + R - 1) / R;
-
-    for (int j = tid; j < K; j += AQ_THREADS) rcp[j] = lam ? __frcp_rn(lam[j]) : 1.0f;
-    const uint32_t smem0 = static_cast<uint32_t>(__cvta_generic_to_shared(aq_smem));
-    const uint32_t bar0 = static_cast<uint32_t>(__cvta_generic_to_shared(bars));
-    if (tid == 0) {
-        for (int i = 0; i < AQ_SLOTS; ++i) aq_bar_init(bar0 + 8 * i);
-        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-    }
-    __syncthreads();
-    if (tid == 0) {                             // first fill of the ring
-        for (int i = 0; i < AQ_SLOTS; ++i) {
-            const int g = blockIdx.x + i * gridDim.x;
-            if (g >= groups) break;
-            const int rows = min(R, M - g * R);
-            aq_bulk_load(smem0 + i * slot_bytes, X + (size_t)g * R * K, rows * K * 2, bar0 + 8 * i);
-        }
-    }
-
-    int it = 0;
-    for (int g = blockIdx.x; g < groups; g += gridDim.x, ++it) {
-        const int slot = it % AQ_SLOTS;
-        const uint32_t bar = bar0 + 8 * slot;
-        const uint32_t par = (it / AQ_SLOTS) & 1;
-        if (lane == 0) aq_wait(bar, par, err);  // one poller per warp
-        __syncwarp();
-        aq_wait(bar, par, err);                 // completes at once: acquire for every lane
-        const int row = g * R + team;
-        const bool active = row < M;
-        const uint8_t *src = aq_smem + slot * slot_bytes + team * K * 2;
-        float2 xs[CPT][4];
-        float a = 0.0f;
-#pragma unroll
-        for (int c = 0; c < CPT; ++c) {
-            const int col0 = 8 * (tl + c * G);
-            if (active && col0 < K) {
-                const uint4 v = *reinterpret_cast<const uint4 *>(src + col0 * 2);
-                const float4 f0 = *reinterpret_cast<const float4 *>(rcp + col0);
-                const float4 f1 = *reinterpret_cast<const float4 *>(rcp + col0 + 4);
-                const uint32_t w[4] = {v.x, v.y, v.z, v.w};
-                const float2 f[4] = {make_float2(f0.x, f0.y), make_float2(f0.z, f0.w),
-                                     make_float2(f1.x, f1.y), make_float2(f1.z, f1.w)};
-#pragma unroll
-                for (int p = 0; p < 4; ++p) {
-                    const float2 x = make_float2(__uint_as_float(w[p] << 16),
-                                                 __uint_as_float(w[p] & 0xffff0000u));
-                    xs[c][p] = mul2_rn(x, f[p]);
-                    a = fmaxf(a, fmaxf(fabsf(xs[c][p].x), fabsf(xs[c][p].y)));
-                }
-            } else {
-#pragma unroll
-                for (int p = 0; p < 4; ++p) xs[c][p] = make_float2(0.0f, 0.0f);
-            }
-        }
-        // team absmax: lanes, then warps of the team
-        const int width = G < 32 ? G : 32;
-        for (int o = width >> 1; o > 0; o >>= 1) a = fmaxf(a, __shfl_xor_sync(0xffffffffu, a, o));
-        if (lane == 0) red[it & 1][warp] = a;
-        __syncthreads();                       // slot fully read; partial maxima visible
-        if (tid == 0) {                         // refill this slot AQ_SLOTS groups ahead
-            const int gn = g + AQ_SLOTS * gridDim.x;
-            if (gn < groups) {
-                const int rows = min(R, M - gn * R);
-                aq_bulk_load(smem0 + slot * slot_bytes, X + (size_t)gn * R * K, rows * K * 2, bar);
-            }
-        }
-        if (G > 32) {
-            a = 0.0f;
-            const int w0 = (team * G) >> 5;
-            for (int w = 0; w < (G >> 5); ++w) a = fmaxf(a, red[it & 1][w0 + w]);
-        }
-        if (!active) continue;
-        const bool zero_row = (a == 0.0f);
-        const float inv = zero_row ? 0.0f : __fdiv_rn(127.0f, a);
-        if (tl == 0) x_scale[row] = zero_row ? 0.0f : __fdiv_rn(a, 127.0f);
-        int8_t *q = Xq + (size_t)row * K;
-        // fast path: a and 127/a finite, so |x' * inv| <= 127 (1 + 2^-23) and
-        // the rounded code is already inside [-127, 127]
-        const bool fast = (a <= 3.402823466e38f) && (inv <= 3.402823466e38f);
-#pragma unroll
-        for (int c = 0; c < CPT; ++c) {
-            const int col0 = 8 * (tl + c * G);
-            if (col0 >= K) continue;
-            uint32_t word[2] = {0u, 0u};
-            if (zero_row) {
-            } else if (fast) {
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const float2 u0 = xs[c][2 * h], u1 = xs[c][2 * h + 1];
-                    word[h] = pack4_low_bytes(__fadd_rn(__fmul_rn(u0.x, inv), kRoundMagic),
-                                              __fadd_rn(__fmul_rn(u0.y, inv), kRoundMagic),
-                                              __fadd_rn(__fmul_rn(u1.x, inv), kRoundMagic),
-                                              __fadd_rn(__fmul_rn(u1.y, inv), kRoundMagic));
-                }
-            } else {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float xv = (e & 1) ? xs[c][e >> 1].y : xs[c][e >> 1].x;
-                    const uint32_t b = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xv, inv))) & 0xffu;
-                    word[e >> 2] |= b << (8 * (e & 3));
-                }
-            }
-            *reinterpret_cast<uint2 *>(q + col0) = make_uint2(word[0], word[1]);
-        }
-    }
-}
-
-// Launch geometry of one staged-kernel instance, computed once per shared
-// memory size (attribute calls and occupancy queries cost microseconds of
-// host time, which would otherwise show up between short kernels).
-struct AqConfig {
-    size_t smem = 0;
-    int per_sm = 0;
-};
-
-template <int CPT>
-cudaError_t launch_act_quant_staged(const uint16_t *X, const float *lam, int M, int K, int R,
-                                    int8_t *Xq, float *x_scale, unsigned int *err,
-                                    cudaStream_t st) {
-    static AqConfig cache[8];
-    static size_t attr_smem = 0;
-    const size_t smem = (size_t)AQ_SLOTS * R * K * 2 + (size_t)K * 4 + AQ_SLOTS * 8;
-    auto kern = act_quant_staged_kernel<CPT>;
-    int per_sm = 0;
-    for (auto &c : cache)
-        if (c.smem == smem) { per_sm = c.per_sm; break; }
-    if (per_sm == 0) {
-        if (smem > attr_smem) {
-            cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)smem);
-            if (e != cudaSuccess) return e;
-            attr_smem = smem;
-        }
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, AQ_THREADS, smem);
-        if (per_sm < 1) per_sm = 1;
-        for (auto &c : cache)
-            if (c.smem == 0) { c.smem = smem; c.per_sm = per_sm; break; }
-    }
-    const int groups = (M + R - 1) / R;
-    int grid = num_sms() * per_sm;
-    if (grid > groups) grid = groups;
-    kern<<<grid, AQ_THREADS, smem, st>>>(X, lam, M, K, R, Xq, x_scale, err);
-    return cudaGetLastError();
 }
 
 // ---------------------------------------------- activation quant, warp teams
@@ -735,6 +531,7 @@ cudaError_t launch_quantize_weights(const float *W, const float *lambda, int N, 
 
 cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M, int K,
                              int8_t *Xq, float *x_scale, unsigned int *err, cudaStream_t st) {
+    (void)err;  // no kernel of this pass waits on a barrier
     // one warp per row, row held in registers (16 chunks of 8 per lane covers
     // K <= 4096 in one read; wider rows are read twice, the second time from
     // L2); 1/lambda needs K * 4 bytes of shared memory per block
@@ -747,21 +544,6 @@ cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M, int 
         if (K <= 4096) return launch_act_quant_team<2, 8>(X, lambda, M, K, Xq, x_scale, st);
         if (K <= 8192) return launch_act_quant_team<2, 16>(X, lambda, M, K, Xq, x_scale, st);
         return launch_act_quant_team<4, 16>(X, lambda, M, K, Xq, x_scale, st);
-    }
-    // rows per slot: about 16 KB of bf16 per slot, at most 16 rows (teams of >= 16
-    // threads).  Wider rows go to the register-resident kernel, which measured
-    // faster there (one 32 KB slot per row leaves too few rows in flight).
-    if (K <= 8192) {
-        int R = 8192 / K;
-        if (R < 1) R = 1;
-        if (R > 16) R = 16;
-        int p2 = 1;
-        while (p2 * 2 <= R) p2 *= 2;
-        R = p2;
-        const int G = AQ_THREADS / R;
-        const int cpt = (K / 8 + G - 1) / G;
-        if (cpt <= 4) return launch_act_quant_staged<4>(X, lambda, M, K, R, Xq, x_scale, err, st);
-        if (cpt <= 8) return launch_act_quant_staged<8>(X, lambda, M, K, R, Xq, x_scale, err, st);
     }
     return launch_row_quant<uint16_t, true>(X, lambda, M, K, Xq, x_scale, st);
 }
