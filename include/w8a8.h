@@ -175,6 +175,16 @@ W8A8_API w8a8_status w8a8_set_gemm_engine(int engine);
 W8A8_API int w8a8_get_gemm_engine(void);
 
 /*
+ * Test hook for failure detection (no counterpart in the paper): enqueues one
+ * small kernel whose bounded barrier wait is never satisfied, through the
+ * same wait routine the tcgen05 GEMMs use.  After limit_us microseconds
+ * (1 .. 2000000, else W8A8_ERR_INVALID_ARG) the wait records code 128 in the
+ * device error word and the kernel returns; the context stays usable and the
+ * next w8a8_device_status reports W8A8_ERR_TIMEOUT.
+ */
+W8A8_API w8a8_status w8a8_debug_wait_timeout(uint32_t limit_us, void *stream);
+
+/*
  * Waits for `stream`, then reads and clears the library's device-side error
  * word on the current device.  Kernels that wait on barriers give up after a
  * bounded number of polls, record a code there and return; this call then

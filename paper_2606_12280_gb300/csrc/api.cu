@@ -169,6 +169,13 @@ w8a8_status w8a8_set_gemm_engine(int engine) {
 
 int w8a8_get_gemm_engine(void) { return g_engine; }
 
+w8a8_status w8a8_debug_wait_timeout(uint32_t limit_us, void *stream) {
+    if (limit_us == 0 || limit_us > 2000000u) return W8A8_ERR_INVALID_ARG;
+    unsigned int *err = device_error_word();
+    if (!err) return W8A8_ERR_CUDA;
+    return from_cuda(w8a8::launch_wait_probe(err, 1000ull * limit_us, as_stream(stream)));
+}
+
 w8a8_status w8a8_device_status(void *stream, uint32_t *detail) {
     cudaStream_t st = as_stream(stream);
     if (cudaStreamSynchronize(st) != cudaSuccess) return W8A8_ERR_CUDA;

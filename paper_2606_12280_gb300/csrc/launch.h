@@ -41,4 +41,7 @@ cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K,
 cudaError_t launch_gemm_tc(const GemmBranch *br, int nb, int N, int K,
                            bool out_i32, unsigned int *err, cudaStream_t st);
 
+// Test hook: one bounded wait that is never satisfied (failure detection).
+cudaError_t launch_wait_probe(unsigned int *err, uint64_t limit_ns, cudaStream_t st);
+
 }  // namespace w8a8

@@ -35,6 +35,7 @@ SIGNATURES = {
     "w8a8_set_gemm_engine": [_I],
     "w8a8_get_gemm_engine": [],
     "w8a8_device_status": [_P, ctypes.POINTER(ctypes.c_uint32)],
+    "w8a8_debug_wait_timeout": [ctypes.c_uint32, _P],
     "w8a8_status_string": [_I],
 }
 
@@ -209,6 +210,11 @@ def device_status(stream=None) -> int:
     if st not in (W8A8_OK, 5):
         raise W8A8Error("w8a8_device_status", st)
     return int(detail.value)
+
+
+def debug_wait_timeout(limit_us: int, stream=None) -> None:
+    """Enqueue a bounded wait that can only time out (failure-detection test)."""
+    _check("w8a8_debug_wait_timeout", lib().w8a8_debug_wait_timeout(int(limit_us), _stream(stream)))
 
 
 def quantized_linear_forward(X, smooth, Wq, w_scale, bias=None, stream=None):

@@ -124,6 +124,11 @@ def test_dual_validation(L):
     assert f(arr, 8, 16, None) == OK                      # both branches empty
 
 
+def test_wait_probe_validation(L):
+    assert L.w8a8_debug_wait_timeout(0, None) == INVALID
+    assert L.w8a8_debug_wait_timeout(2000001, None) == INVALID
+
+
 def test_engine_switch(L):
     assert L.w8a8_set_gemm_engine(7) == INVALID
     assert L.w8a8_set_gemm_engine(0) == OK

@@ -242,3 +242,18 @@ def test_no_out_of_bounds_writes(w8, engine):
     torch.cuda.synchronize()
     assert torch.all(buf32[:guard] == 0x5A5A5A5A) and torch.all(buf32[guard + M * N:] == 0x5A5A5A5A)
     assert w8.device_status() == 0
+
+
+def test_bounded_wait_reports_timeout_and_context_survives(w8):
+    """A barrier wait that nothing satisfies gives up after its limit, records
+    its code in the device error word, and the context keeps working."""
+    assert w8.device_status() == 0
+    w8.debug_wait_timeout(20000)                  # 20 ms
+    assert w8.device_status() == 128             # reported once ...
+    assert w8.device_status() == 0               # ... and cleared
+    Xq = t(wl.random_int8((300, 528), seed=90))
+    Wq = t(wl.random_int8((264, 528), seed=91))
+    acc = w8.debug_gemm_i32(Xq, Wq).cpu().numpy()
+    want = Xq.cpu().numpy().astype(np.int64) @ Wq.cpu().numpy().astype(np.int64).T
+    np.testing.assert_array_equal(acc, want)
+    assert w8.device_status() == 0
