@@ -35,13 +35,29 @@ namespace {
 
 using namespace tc;
 
+#ifndef W8A8_TC2_SUB
+#define W8A8_TC2_SUB 2
+#endif
+#ifndef W8A8_TC2_S8
+#define W8A8_TC2_S8 2
+#endif
+#ifndef W8A8_TC2_S16
+#define W8A8_TC2_S16 2
+#endif
+// One pipeline stage carries SUB sub-blocks of K = 64 (one 128-byte swizzle
+// atom of fp16 per row each), so barrier hand-offs happen every 64*SUB of K.
 constexpr int PAIR_M = 256, CTA_M = 128, PAIR_N = 256, CTA_N = 128, BK = 64;
+constexpr int SUB = W8A8_TC2_SUB;
 constexpr int KC_BLOCKS = 16;                        // K chunk = 1024 (exactness bound)
-constexpr int S8 = 6, S16 = 3;
-constexpr int STAGE8_A = CTA_M * BK, STAGE8_B = CTA_N * BK;
-constexpr int STAGE8 = STAGE8_A + STAGE8_B;          // 16 KB
-constexpr int STAGE16_A = CTA_M * BK * 2, STAGE16_B = CTA_N * BK * 2;
-constexpr int STAGE16 = STAGE16_A + STAGE16_B;       // 32 KB
+constexpr int KC_STAGES = KC_BLOCKS / SUB;           // stages per K chunk
+constexpr int S8 = W8A8_TC2_S8, S16 = W8A8_TC2_S16;
+constexpr int SUB8_A = CTA_M * BK, SUB8_B = CTA_N * BK;
+constexpr int SUB8 = SUB8_A + SUB8_B;                // 16 KB int8 per sub-block
+constexpr int SUB16_A = CTA_M * BK * 2, SUB16_B = CTA_N * BK * 2;
+constexpr int SUB16 = SUB16_A + SUB16_B;             // 32 KB fp16 per sub-block
+constexpr int STAGE8 = SUB * SUB8;
+constexpr int STAGE16 = SUB * SUB16;
+static_assert(KC_BLOCKS % SUB == 0, "chunk of whole stages");
 constexpr int NUM_CONV_WARPS = 6;
 constexpr int NUM_EPI_WARPS = 8;
 constexpr int THREADS = 512;
@@ -53,6 +69,7 @@ constexpr int LAUNCH_REGS = 128;
 constexpr int REGS_LOW = 72, REGS_HIGH = 184;
 static_assert(256 * REGS_LOW + 256 * REGS_HIGH <= THREADS * LAUNCH_REGS, "register split");
 static_assert(KC_BLOCKS * BK * 127 * 127 < (1 << 24), "fp32 exactness bound");
+static_assert(1024 + S16 * STAGE16 + S8 * STAGE8 + 512 + 8192 <= 232448, "shared memory");
 
 constexpr unsigned ERR_PRODUCER = 1u, ERR_CONVERTER = 2u, ERR_MMA = 4u, ERR_EPILOGUE = 8u,
                    ERR_DRAIN = 16u, ERR_TMEM_PAIR = 64u;
@@ -276,6 +293,7 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
     if (!run_ok && threadIdx.x == 0) atomicOr(p.err, ERR_TMEM_PAIR);
     const WaitCtx wc{sb + OFF_ABORT, p.err, p.wait_limit_ns};
     const int KB = p.k_blocks;
+    const int NS = (KB + SUB - 1) / SUB;                  // pipeline stages per tile
     const int NC = (KB + KC_BLOCKS - 1) / KC_BLOCKS;
 
     if (warp >= 8) {
@@ -299,7 +317,7 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                     const CUtensorMap *mB = tl.branch ? &tmB1 : &tmB0;
                     const int arow = tl.m0 + static_cast<int>(rank) * CTA_M;
                     const int brow = tl.n0 + static_cast<int>(rank) * CTA_N;
-                    for (int kb = 0; kb < KB; ++kb, ++j) {
+                    for (int ks = 0; ks < NS; ++ks, ++j) {
                         const uint32_t st = j % S8;
                         if (!mbar_wait(sb + BAR_EMPTY8 + 8 * st, ((j / S8) & 1) ^ 1, wc, ERR_PRODUCER)) {
                             ok = false;
@@ -307,9 +325,12 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                         }
                         const uint32_t fb = sb + BAR_FULL8 + 8 * st;
                         mbar_arrive_expect_tx(fb, STAGE8);
-                        const uint32_t dst = sb + OFF_ST8 + st * STAGE8;
-                        tma_load_2d(dst, mA, kb * BK, arow, fb);
-                        tma_load_2d(dst + STAGE8_A, mB, kb * BK, brow, fb);
+#pragma unroll
+                        for (int u = 0; u < SUB; ++u) {
+                            const uint32_t dst = sb + OFF_ST8 + st * STAGE8 + u * SUB8;
+                            tma_load_2d(dst, mA, (ks * SUB + u) * BK, arow, fb);
+                            tma_load_2d(dst + SUB8_A, mB, (ks * SUB + u) * BK, brow, fb);
+                        }
                     }
                 }
                 for (uint32_t i = (j > S8 ? j - S8 : 0); i < j; ++i)
@@ -331,22 +352,25 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                         }
                         tc_fence_after();
                         const uint32_t d = tmem + buf * PAIR_N;
-                        const int kb0 = ci * KC_BLOCKS;
-                        const int kb1 = min(KB, kb0 + KC_BLOCKS);
-                        for (int kb = kb0; kb < kb1; ++kb, ++j) {
+                        const int ks0 = ci * KC_STAGES;
+                        const int ks1 = min(NS, ks0 + KC_STAGES);
+                        for (int ks = ks0; ks < ks1; ++ks, ++j) {
                             const uint32_t st = j % S16;
                             if (!mbar_wait_cluster(sb + BAR_FULL16 + 8 * st, (j / S16) & 1, wc, ERR_MMA)) {
                                 ok = false;
                                 break;
                             }
                             tc_fence_after();
-                            const uint32_t a = sb + OFF_ST16 + st * STAGE16;
-                            const uint32_t b = a + STAGE16_A;
 #pragma unroll
-                            for (int kk = 0; kk < BK / 16; ++kk) {
-                                mma_f16_ss_pair(d, smem_desc_sw128(a + kk * 32),
-                                                smem_desc_sw128(b + kk * 32), idesc,
-                                                (kb > kb0 || kk > 0) ? 1u : 0u);
+                            for (int u = 0; u < SUB; ++u) {
+                                const uint32_t a = sb + OFF_ST16 + st * STAGE16 + u * SUB16;
+                                const uint32_t b = a + SUB16_A;
+#pragma unroll
+                                for (int kk = 0; kk < BK / 16; ++kk) {
+                                    mma_f16_ss_pair(d, smem_desc_sw128(a + kk * 32),
+                                                    smem_desc_sw128(b + kk * 32), idesc,
+                                                    (ks > ks0 || u > 0 || kk > 0) ? 1u : 0u);
+                                }
                             }
                             mma_commit_pair_multicast(sb + BAR_EMPTY16 + 8 * st, 0x3);
                         }
@@ -367,7 +391,7 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
             uint32_t j = 0;
             bool ok = true;
             for (int t = pair; ok && t < p.total_tiles; t += npairs) {
-                for (int kb = 0; kb < KB; ++kb, ++j) {
+                for (int ks = 0; ks < NS; ++ks, ++j) {
                     const uint32_t s8 = j % S8, s16 = j % S16;
                     if (!mbar_wait(sb + BAR_FULL8 + 8 * s8, (j / S8) & 1, wc, ERR_CONVERTER) ||
                         !mbar_wait_cluster(sb + BAR_EMPTY16 + 8 * s16, ((j / S16) & 1) ^ 1, wc,
@@ -377,27 +401,33 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                     }
                     const uint32_t src = sb + OFF_ST8 + s8 * STAGE8 + src_off;
                     const uint32_t dst = sb + OFF_ST16 + s16 * STAGE16;
-                    // all of this warp's 8-row groups in flight at once: every load
-                    // is issued before the first conversion needs its data
-                    constexpr int kG = (CTA_M + CTA_N) / 8;
-                    constexpr int kPer = (kG + NUM_CONV_WARPS - 1) / NUM_CONV_WARPS;
-                    uint4 v[kPer];
+                    // per sub-block, all of this warp's 8-row groups in flight at
+                    // once: every load is issued before the first conversion needs
+                    // its data (group g of sub-block u sits at u * kG1 + g in both
+                    // rings: a sub-block is CTA_M + CTA_N rows of 64 int8 bytes,
+                    // 128 fp16 bytes)
+                    constexpr int kG1 = (CTA_M + CTA_N) / 8;
+                    constexpr int kPer = (kG1 + NUM_CONV_WARPS - 1) / NUM_CONV_WARPS;
 #pragma unroll
-                    for (int i = 0; i < kPer; ++i) {
-                        const int g = cw + i * NUM_CONV_WARPS;
-                        if (g < kG) v[i] = ld_shared_v4(src + g * 8 * BK);
-                    }
+                    for (int u = 0; u < SUB; ++u) {
+                        uint4 v[kPer];
 #pragma unroll
-                    for (int i = 0; i < kPer; ++i) {
-                        const int g = cw + i * NUM_CONV_WARPS;
-                        if (g < kG) {
-                            uint4 o0, o1;
-                            i8x4_to_f16x4(v[i].x, o0.x, o0.y);
-                            i8x4_to_f16x4(v[i].y, o0.z, o0.w);
-                            i8x4_to_f16x4(v[i].z, o1.x, o1.y);
-                            i8x4_to_f16x4(v[i].w, o1.z, o1.w);
-                            st_shared_v4(dst + g * 1024 + dst_off0, o0);
-                            st_shared_v4(dst + g * 1024 + dst_off1, o1);
+                        for (int i = 0; i < kPer; ++i) {
+                            const int g = cw + i * NUM_CONV_WARPS;
+                            if (g < kG1) v[i] = ld_shared_v4(src + (u * kG1 + g) * 8 * BK);
+                        }
+#pragma unroll
+                        for (int i = 0; i < kPer; ++i) {
+                            const int g = cw + i * NUM_CONV_WARPS;
+                            if (g < kG1) {
+                                uint4 o0, o1;
+                                i8x4_to_f16x4(v[i].x, o0.x, o0.y);
+                                i8x4_to_f16x4(v[i].y, o0.z, o0.w);
+                                i8x4_to_f16x4(v[i].z, o1.x, o1.y);
+                                i8x4_to_f16x4(v[i].w, o1.z, o1.w);
+                                st_shared_v4(dst + (u * kG1 + g) * 1024 + dst_off0, o0);
+                                st_shared_v4(dst + (u * kG1 + g) * 1024 + dst_off1, o1);
+                            }
                         }
                     }
                     fence_proxy_async_smem();
