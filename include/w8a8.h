@@ -9,7 +9,7 @@
  * activations divided by lambda and weights multiplied by it before
  * quantization.  The INT8 x INT8 -> INT32 product with a fused dequantizing
  * epilogue is the kernel the paper reports as missing (Sec. 5, Efficiency;
- * Sec. 6, Limitations), and the two separate-weight branches (conditional and
+ * Sec. 7, Limitations), and the two separate-weight branches (conditional and
  * unconditional) of its classifier-free-guidance DiT (Sec. 1; Sec. 3,
  * Setting) run as one grouped launch.
  *

@@ -5,11 +5,15 @@ Only the tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 oracle never imports the product: the two share only the seeded input
 generators, which hold none of the method's arithmetic.
 
-The arithmetic lives in ``w8a8_oracle.c`` (plain C, ``-O2 -ffp-contract=off``,
-no intrinsics), compiled with gcc into ``oracle/_build/liboracle.so`` and called
-through ctypes on numpy arrays.  Each function follows the "INT8 W8A8" paragraph
-of the paper's Method section (Sec. 3); the INT8 GEMM and dequantizing epilogue
-are the fused kernel the paper lists as missing (Sec. 6, Limitations).
+The arithmetic lives in ``w8a8_oracle.c`` and ``protect_oracle.c`` (plain C,
+``-O2 -ffp-contract=off``, no intrinsics), compiled with gcc into
+``oracle/_build/liboracle.so`` and called through ctypes on numpy arrays.  Each
+function follows the "INT8 W8A8" paragraph of the paper's Method section
+(Sec. 3); the INT8 GEMM and dequantizing epilogue are the fused kernel the
+paper lists as missing (Sec. 7, Limitations).  The activation statistics and
+the protected bf16 layer follow Sec. 3, "Activation-fragility profiling and
+protection"; the per-tensor activation scale is the naive arm of the
+activation-quant ablation (Sec. 5, "What drives INT8 recovery").
 """
 
 from __future__ import annotations
@@ -22,7 +26,7 @@ import threading
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRC = os.path.join(_HERE, "w8a8_oracle.c")
+_SRCS = [os.path.join(_HERE, f) for f in ("w8a8_oracle.c", "protect_oracle.c")]
 _BUILD = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD, "liboracle.so")
 _lock = threading.Lock()
@@ -33,10 +37,10 @@ def build(force: bool = False) -> str:
     """Compile the oracle with gcc (OpenMP over GEMM rows when available)."""
     os.makedirs(_BUILD, exist_ok=True)
     if (not force and os.path.exists(_LIB_PATH)
-            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+            and all(os.path.getmtime(_LIB_PATH) >= os.path.getmtime(f) for f in _SRCS)):
         return _LIB_PATH
     base = ["gcc", "-O2", "-ffp-contract=off", "-fno-fast-math", "-std=c11",
-            "-shared", "-fPIC", _SRC, "-o", _LIB_PATH + ".tmp", "-lm"]
+            "-shared", "-fPIC", *_SRCS, "-o", _LIB_PATH + ".tmp", "-lm"]
     try:
         subprocess.run(base[:1] + ["-fopenmp"] + base[1:], check=True,
                        capture_output=True)
@@ -72,6 +76,10 @@ def _load():
                                                   ctypes.c_float, P]
             lib.oracle_epilogue_value.restype = ctypes.c_uint16
             lib.oracle_num_threads.restype = ctypes.c_int
+            lib.oracle_quant_act_per_tensor.argtypes = [P, P, I64, I64, P, P, P, P]
+            lib.oracle_act_stats.argtypes = [P, I64, I64, P, P]
+            lib.oracle_shifted_power_sums.argtypes = [P, I64, I64, P, P, P]
+            lib.oracle_linear_bf16_rows.argtypes = [P, P, P, I64, I64, I64, I64, I64, P, P]
             _lib = lib
     return _lib
 
@@ -215,3 +223,76 @@ def full_layer(X_bf16, W, bias, s, alpha):
     Xq, sx = quant_act(X_bf16, lam)
     Y = linear(Xq, sx, Wq, sw, bias)
     return {"lambda": lam, "Wq": Wq, "sw": sw, "Xq": Xq, "sx": sx, "Y": Y}
+
+
+# --------------------------------------------------------------------------
+# ablation arm: per-tensor activation scale (Sec. 5, "What drives INT8
+# recovery"; the naive per-tensor INT8 of Sec. 2)
+# --------------------------------------------------------------------------
+
+def quant_act_per_tensor(X_bf16: np.ndarray, lam: np.ndarray | None):
+    """One INT8 scale for all of X diag(lambda)^-1: returns (Xq, sx [M], amax)."""
+    X = _c(X_bf16, np.uint16)
+    lam = _c(lam, np.float32)
+    M, K = X.shape
+    Xq = np.empty((M, K), dtype=np.int8)
+    sx = np.empty(M, dtype=np.float32)
+    amax = np.empty(1, dtype=np.float32)
+    tmp = np.empty(K, dtype=np.float32)
+    _load().oracle_quant_act_per_tensor(_ptr(X), _ptr(lam), M, K, _ptr(Xq), _ptr(sx),
+                                        _ptr(amax), _ptr(tmp))
+    return Xq, sx, float(amax[0])
+
+
+# --------------------------------------------------------------------------
+# fragility profiling and protection (Sec. 3, "Activation-fragility
+# profiling and protection")
+# --------------------------------------------------------------------------
+
+def act_stats(X_bf16: np.ndarray):
+    """(per-channel [4, K], whole-tensor [4]) of maxabs, mean, std, kurtosis
+    over the rows of a [T, K] bf16 batch, in binary64."""
+    X = _c(X_bf16, np.uint16)
+    T, K = X.shape
+    chan = np.empty((4, K), dtype=np.float64)
+    tensor = np.empty(4, dtype=np.float64)
+    _load().oracle_act_stats(_ptr(X), T, K, _ptr(chan), _ptr(tensor))
+    return chan, tensor
+
+
+def shifted_power_sums(X_bf16: np.ndarray, shift: np.ndarray | None):
+    """(S, A) [4, K]: S[p-1, j] = sum_t (x_tj - c_j)^p and A the same over |.|."""
+    X = _c(X_bf16, np.uint16)
+    shift = _c(shift, np.float32)
+    T, K = X.shape
+    S = np.empty((4, K), dtype=np.float64)
+    A = np.empty((4, K), dtype=np.float64)
+    _load().oracle_shifted_power_sums(_ptr(X), T, K, _ptr(shift), _ptr(S), _ptr(A))
+    return S, A
+
+
+def linear_bf16(X_bf16, W_bf16, bias, rows: tuple[int, int] | None = None):
+    """Protected layer, rows [m0, m1): (y, yabs) in binary64, y = X W^T + b exactly
+    up to binary64 summation, yabs = sum |x w| + |b|."""
+    X = _c(X_bf16, np.uint16)
+    W = _c(W_bf16, np.uint16)
+    bias = _c(bias, np.float32)
+    M, K = X.shape
+    N = W.shape[0]
+    m0, m1 = rows if rows is not None else (0, M)
+    Y = np.empty((m1 - m0, N), dtype=np.float64)
+    Ya = np.empty((m1 - m0, N), dtype=np.float64)
+    _load().oracle_linear_bf16_rows(_ptr(X), _ptr(W), _ptr(bias), M, N, K, m0, m1,
+                                    _ptr(Y), _ptr(Ya))
+    return Y, Ya
+
+
+def layer_forward(X_bf16, layer: dict, rows: tuple[int, int] | None = None):
+    """Per-layer dispatch: a protected layer is the bf16 linear (no activation
+    quantization); any other layer is a3 + a4 + a5.  Returns the bf16 result
+    for W8A8 layers (bit patterns) or the binary64 (y, yabs) pair for
+    protected ones."""
+    if layer["protect"]:
+        return linear_bf16(X_bf16, layer["W_bf16"], layer["bias"], rows=rows)
+    Xq, sx = quant_act(X_bf16, layer["smooth"])
+    return linear(Xq, sx, layer["Wq"], layer["w_scale"], layer["bias"], rows=rows)

@@ -16,7 +16,7 @@
  *     quantization,
  * plus the exact INT32 product of the two INT8 operands and the dequantizing
  * epilogue (per-token scale x per-channel scale + bias, rounded to bf16) that
- * the paper names as the missing fused INT8 GEMM (Sec. 6, Limitations).
+ * the paper names as the missing fused INT8 GEMM (Sec. 7, Limitations).
  *
  * Precision.  The quantization decisions are taken in IEEE binary32 with a
  * pinned operation order (every operation rounded to nearest-even, no fused
@@ -264,6 +264,48 @@ void oracle_linear_rows(const int8_t *Xq, const float *x_scale,
 {
     oracle_gemm_i32(Xq, Wq, M, N, K, m0, m1, acc_tmp);
     oracle_epilogue(acc_tmp, x_scale + m0, w_scale, bias, m1 - m0, N, Y);
+}
+
+/* ------------------------------------------------------------------ */
+/* ablation arm: one activation scale for the whole tensor             */
+/* (the "naive per-tensor INT8 activations" that SmoothQuant is        */
+/* contrasted with, Sec. 2 "Weight-activation PTQ"; the naive W8A8     */
+/* arm of the activation-quant ablation, Sec. 5 "What drives INT8      */
+/* recovery").  Same steps as oracle_quant_act with the max taken      */
+/* over every element of X diag(lambda)^-1 instead of one row; the     */
+/* common scale is written to every row's x_scale so that the same     */
+/* epilogue applies.                                                    */
+/* ------------------------------------------------------------------ */
+
+void oracle_quant_act_per_tensor(const uint16_t *X, const float *lambda,
+                                 int64_t M, int64_t K, int8_t *Xq,
+                                 float *x_scale, float *amax_out,
+                                 float *recip_tmp)
+{
+    for (int64_t j = 0; j < K; ++j)
+        recip_tmp[j] = lambda ? 1.0f / lambda[j] : 1.0f;
+
+    float a = 0.0f;                           /* max over the whole tensor */
+    for (int64_t t = 0; t < M; ++t)
+        for (int64_t j = 0; j < K; ++j) {
+            float ax = fabsf(oracle_bf16_to_f32(X[t * K + j]) * recip_tmp[j]);
+            if (ax > a)
+                a = ax;
+        }
+    *amax_out = a;
+    float scale = (a == 0.0f) ? 0.0f : a / 127.0f;
+    float inv = (a == 0.0f) ? 0.0f : 127.0f / a;
+    for (int64_t t = 0; t < M; ++t) {
+        x_scale[t] = scale;
+        for (int64_t j = 0; j < K; ++j) {
+            if (a == 0.0f) {
+                Xq[t * K + j] = 0;
+                continue;
+            }
+            float x = oracle_bf16_to_f32(X[t * K + j]) * recip_tmp[j];
+            Xq[t * K + j] = quantize_rne_clamp(x * inv);
+        }
+    }
 }
 
 /* threads the row loop of oracle_gemm_i32 runs on (1 without OpenMP) */

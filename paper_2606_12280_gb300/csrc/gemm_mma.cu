@@ -1,7 +1,7 @@
 // gemm_mma.cu -- INT8 x INT8 -> INT32 GEMM on the legacy warp-level tensor
 // path (mma.sync.m16n8k32 s8, native int32 accumulation) with the
 // dequantizing epilogue fused (a4 + a5 of the W8A8 layer, Sec. 3 "INT8 W8A8";
-// the fused kernel the paper lists as missing, Sec. 6 Limitations).
+// the fused kernel the paper lists as missing, Sec. 7 Limitations).
 //
 // It is the exact-integer anchor of the library and the measured "native
 // INT8" engine of this GPU.  128x128 output tile per CTA, K step 64, 8 warps

@@ -163,6 +163,12 @@ def random_f32(shape, seed: int, scale: float = 1.0) -> np.ndarray:
     return (torch.randn(tuple(shape), generator=g, dtype=torch.float32) * scale).numpy()
 
 
+def random_uniform_f32(shape, seed: int, lo: float, hi: float) -> np.ndarray:
+    """Uniform fp32 in [lo, hi) (positive smoothing vectors, shifts)."""
+    g = torch.Generator().manual_seed(seed)
+    return (torch.rand(tuple(shape), generator=g, dtype=torch.float32) * (hi - lo) + lo).numpy()
+
+
 def random_bf16(shape, seed: int, scale: float = 1.0) -> np.ndarray:
     g = torch.Generator().manual_seed(seed)
     return _bf16_bits(torch.randn(tuple(shape), generator=g, dtype=torch.float32) * scale)
