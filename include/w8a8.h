@@ -163,6 +163,113 @@ W8A8_API w8a8_status w8a8_linear_dual(const w8a8_branch *br, int N, int K,
 W8A8_API w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int M,
                                 int N, int K, int32_t *acc, void *stream);
 
+/* ------------------------------------------------------------------------
+ * Around the W8A8 layer: the ablation's per-tensor activation scale, the
+ * activation statistics of fragility profiling, and the protected (bf16)
+ * layers with per-layer dispatch.
+ * ---------------------------------------------------------------------- */
+
+/*
+ * Per-tensor INT8 activations: the naive arm of the activation-quant ablation
+ * (Sec. 5, "What drives INT8 recovery"; the naive per-tensor INT8 that
+ * SmoothQuant is contrasted with in Sec. 2).  Same arithmetic as
+ * w8a8_quant_act with the maximum taken over the whole tensor:
+ *     x'_mj = X_mj * (1/lambda_j);  a = max_mj |x'_mj|;
+ *     x_scale_m = a / 127 for every m;  Xq_mj = clamp(rne(x'_mj * (127/a)), +-127);
+ *     a == 0 gives scale 0 and codes 0.
+ * Because every row carries the same scale, w8a8_linear consumes the result
+ * unchanged.
+ *   X [M,K] bf16, read.   smooth [K] fp32 or NULL (lambda = 1), read.
+ *   Xq [M,K] int8, x_scale [M] fp32, written.   amax [1] fp32, written (a).
+ * Two passes over X (the second usually from L2): 4MK bytes read, MK + 4M
+ * written.
+ */
+W8A8_API w8a8_status w8a8_quant_act_per_tensor(const uint16_t *X, const float *smooth, int M,
+                                               int K, int8_t *Xq, float *x_scale, float *amax,
+                                               void *stream);
+
+/*
+ * Activation statistics for fragility profiling (Sec. 3, "Activation-fragility
+ * profiling and protection": every linear's input is recorded over the
+ * denoising trajectory as max-abs, standard deviation and kurtosis).
+ * Accumulates, for each input channel j over the T tokens of X,
+ *     sums[(p-1)*K + j] += sum_t (X_tj - c_j)^p     p = 1, 2, 3, 4  (fp64)
+ *     absmax[j]          = max(absmax[j], max_t |X_tj|)
+ * with c = shift (or 0 when shift is NULL).  Call it once per recorded batch
+ * (any number of times, same shift); the caller zeroes sums [4K] and absmax
+ * [K] before the first call and keeps the total token count.  A shift near
+ * each channel's mean (for example from a first batch) keeps the power sums
+ * well conditioned.  Each thread sums at most 64 of its rows in fp32 before
+ * adding into fp64: every returned sum is within (64 + 4) * 2^-24 of
+ * sum_t |X_tj - c_j|^p of its exact value.  T == 0 is a no-op.
+ *   X [T,K] bf16, read.   shift [K] fp32 or NULL, read.
+ *   sums [4,K] fp64, absmax [K] fp32: read and written (accumulators).
+ */
+W8A8_API w8a8_status w8a8_act_stats_update(const uint16_t *X, int T, int K, const float *shift,
+                                           double *sums, float *absmax, void *stream);
+
+/*
+ * Statistics from the accumulators of w8a8_act_stats_update over `count`
+ * tokens (count >= 1), in fp64, rounded to fp32 on output:
+ *   chan [4,K]: plane 0 max-abs, 1 mean, 2 population standard deviation,
+ *               3 Pearson kurtosis m4 / m2^2 (3 for a normal distribution),
+ *               per input channel;
+ *   tensor [4]: the same four over all count*K elements (channels pooled
+ *               about the grand mean).
+ * A variance within the accumulation error of zero (at most 1e-5 of the
+ * second power sum about the shift) is reported as 0, with kurtosis 0.
+ */
+W8A8_API w8a8_status w8a8_act_stats_finalize(const double *sums, const float *absmax,
+                                             const float *shift, long long count, int K,
+                                             float *chan, float *tensor, void *stream);
+
+/*
+ * Protected layer (Sec. 3, "Activation-fragility profiling and protection":
+ * the most fragile layers keep bf16 weights and no activation quantization):
+ *     Y_mn = bf16_rne(fl32(sum_k X_mk W_nk) + bias_n)
+ * with the products of bf16 values exact and the sum accumulated in fp32 by
+ * the tensor cores (order unspecified), the bias added in fp32.
+ *   X [M,K] bf16, W [N,K] bf16, bias [N] fp32 or NULL, read.  Y [M,N] bf16,
+ *   written.  Same shape rules as w8a8_linear.
+ */
+W8A8_API w8a8_status w8a8_linear_bf16(const uint16_t *X, const uint16_t *W, const float *bias,
+                                      int M, int N, int K, uint16_t *Y, void *stream);
+
+/* One linear layer of the protected-INT8 recipe. */
+typedef struct {
+    int protect;               /* nonzero: protected layer (bf16 path) */
+    int N, K;                  /* output and input channels */
+    const float *smooth;       /* W8A8: lambda [K] fp32 or NULL */
+    const int8_t *Wq;          /* W8A8: [N,K] int8 */
+    const float *w_scale;      /* W8A8: [N] fp32 */
+    const uint16_t *W_bf16;    /* protected: [N,K] bf16 */
+    const float *bias;         /* [N] fp32 or NULL, both paths */
+} w8a8_layer;
+
+/*
+ * Per-layer dispatch: a protected layer runs w8a8_linear_bf16 on X; any other
+ * layer runs w8a8_quant_act (into the caller's workspace) and w8a8_linear.
+ *   layer  host pointer, read during the call only.
+ *   X [M,K] bf16, read.   Y [M,N] bf16, written.
+ *   Xq_work [M,K] int8 and x_scale_work [M] fp32: workspace of the W8A8 path
+ *   (ignored, may be NULL, for a protected layer).
+ */
+W8A8_API w8a8_status w8a8_layer_forward(const w8a8_layer *layer, const uint16_t *X, int M,
+                                        int8_t *Xq_work, float *x_scale_work, uint16_t *Y,
+                                        void *stream);
+
+/*
+ * Choice of the protected set (Sec. 3: the N most fragile of the model's
+ * linears stay in bf16; the paper keeps 17 of 211): protect_flags[i] = 1 for
+ * the n_protect layers with the largest fragility score, 0 for the others.
+ * A NaN score ranks above every number; equal scores keep the lower index
+ * first.  How the score is formed from the statistics is the caller's
+ * choice.  Host arrays: score [L] read, protect_flags [L] written; no device
+ * work.  0 <= n_protect <= L, else W8A8_ERR_INVALID_ARG.
+ */
+W8A8_API w8a8_status w8a8_select_protected(const float *score, int L, int n_protect,
+                                           int *protect_flags);
+
 /*
  * The GEMM engine that w8a8_linear, w8a8_linear_dual and w8a8_debug_gemm_i32
  * use: 2 = tcgen05 on pairs of SMs (cta_group::2, 256x256 tiles), 1 = tcgen05

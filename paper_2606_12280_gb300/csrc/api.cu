@@ -1,6 +1,10 @@
 // api.cu -- the C ABI (include/w8a8.h): argument checks, then stream-ordered
 // launches.  No allocation, no synchronisation (except w8a8_device_status).
+#include <algorithm>
+#include <cmath>
 #include <cstdint>
+#include <numeric>
+#include <vector>
 #include <cuda_runtime.h>
 
 #include "../../include/w8a8.h"
@@ -158,6 +162,96 @@ w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int M, int N
     if (w8a8_status e = check_branch(b, false, N, K)) return e;
     if (M == 0) return W8A8_OK;
     return run_gemm(&b, 1, N, K, true, as_stream(stream));
+}
+
+w8a8_status w8a8_quant_act_per_tensor(const uint16_t *X, const float *smooth, int M, int K,
+                                      int8_t *Xq, float *x_scale, float *amax, void *stream) {
+    if (w8a8_status e = check_mk(M, K)) return e;
+    if (M == 0) return W8A8_OK;
+    if (!X || !Xq || !x_scale || !amax) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(Xq) || !aligned16(x_scale) || !aligned16(amax) ||
+        (smooth && !aligned16(smooth)))
+        return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_quant_act_per_tensor(X, smooth, M, K, Xq, x_scale, amax,
+                                                       as_stream(stream)));
+}
+
+w8a8_status w8a8_act_stats_update(const uint16_t *X, int T, int K, const float *shift,
+                                  double *sums, float *absmax, void *stream) {
+    if (w8a8_status e = check_mk(T, K)) return e;
+    if (!sums || !absmax) return W8A8_ERR_INVALID_ARG;
+    if (T == 0) return W8A8_OK;
+    if (!X) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(sums) || !aligned16(absmax) || (shift && !aligned16(shift)))
+        return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_act_stats_update(X, T, K, shift, sums, absmax,
+                                                   as_stream(stream)));
+}
+
+w8a8_status w8a8_act_stats_finalize(const double *sums, const float *absmax, const float *shift,
+                                    long long count, int K, float *chan, float *tensor,
+                                    void *stream) {
+    if (K <= 0 || (K % 16) != 0 || K > W8A8_MAX_K) return W8A8_ERR_UNSUPPORTED_SHAPE;
+    if (count <= 0 || !sums || !absmax || !chan || !tensor) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(sums) || !aligned16(absmax) || !aligned16(chan) || !aligned16(tensor) ||
+        (shift && !aligned16(shift)))
+        return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_act_stats_finalize(sums, absmax, shift, count, K, chan, tensor,
+                                                     as_stream(stream)));
+}
+
+w8a8_status w8a8_linear_bf16(const uint16_t *X, const uint16_t *W, const float *bias, int M,
+                             int N, int K, uint16_t *Y, void *stream) {
+    if (w8a8_status e = check_nk(N, K)) return e;
+    if (w8a8_status e = check_mk(M, K)) return e;
+    if (M == 0) return W8A8_OK;
+    if (!X || !W || !Y) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(W) || !aligned16(Y) || (bias && !aligned16(bias)))
+        return W8A8_ERR_MISALIGNED;
+    unsigned int *err = device_error_word();
+    if (!err) return W8A8_ERR_CUDA;
+    return from_cuda(w8a8::launch_gemm_bf16(X, W, bias, M, N, K, Y, err, as_stream(stream)));
+}
+
+w8a8_status w8a8_layer_forward(const w8a8_layer *layer, const uint16_t *X, int M, int8_t *Xq_work,
+                               float *x_scale_work, uint16_t *Y, void *stream) {
+    if (!layer) return W8A8_ERR_INVALID_ARG;
+    const int N = layer->N, K = layer->K;
+    if (w8a8_status e = check_nk(N, K)) return e;
+    if (w8a8_status e = check_mk(M, K)) return e;
+    if (layer->protect) {
+        if (!layer->W_bf16) return W8A8_ERR_INVALID_ARG;
+        return w8a8_linear_bf16(X, layer->W_bf16, layer->bias, M, N, K, Y, stream);
+    }
+    if (!layer->Wq || !layer->w_scale) return W8A8_ERR_INVALID_ARG;
+    if (M == 0) return W8A8_OK;
+    if (!Xq_work || !x_scale_work) return W8A8_ERR_INVALID_ARG;
+    // validate the GEMM's arguments before anything is enqueued
+    w8a8::GemmBranch b{Xq_work, x_scale_work, layer->Wq, layer->w_scale, layer->bias, Y, M};
+    if (w8a8_status e = check_branch(b, true, N, K)) return e;
+    if (w8a8_status e = w8a8_quant_act(X, layer->smooth, M, K, Xq_work, x_scale_work, stream))
+        return e;
+    return run_gemm(&b, 1, N, K, false, as_stream(stream));
+}
+
+w8a8_status w8a8_select_protected(const float *score, int L, int n_protect, int *protect_flags) {
+    if (L < 0 || n_protect < 0 || n_protect > L) return W8A8_ERR_INVALID_ARG;
+    if (L > 0 && (!score || !protect_flags)) return W8A8_ERR_INVALID_ARG;
+    std::vector<int> order(static_cast<size_t>(L));
+    std::iota(order.begin(), order.end(), 0);
+    // most fragile first: NaN above every number, then larger scores; equal
+    // scores keep the lower layer index first
+    auto key_greater = [&](int a, int b) {
+        const float sa = score[a], sb = score[b];
+        const bool na = std::isnan(sa), nb = std::isnan(sb);
+        if (na != nb) return na;
+        if (!na && sa != sb) return sa > sb;
+        return a < b;
+    };
+    std::stable_sort(order.begin(), order.end(), key_greater);
+    for (int i = 0; i < L; ++i) protect_flags[i] = 0;
+    for (int i = 0; i < n_protect; ++i) protect_flags[order[static_cast<size_t>(i)]] = 1;
+    return W8A8_OK;
 }
 
 w8a8_status w8a8_set_gemm_engine(int engine) {

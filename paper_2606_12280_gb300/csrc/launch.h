@@ -41,6 +41,21 @@ cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K,
 cudaError_t launch_gemm_tc(const GemmBranch *br, int nb, int N, int K,
                            bool out_i32, unsigned int *err, cudaStream_t st);
 
+// Protected (bf16) linear on tcgen05 CTA pairs: Y = bf16(X W^T + b).
+cudaError_t launch_gemm_bf16(const uint16_t *X, const uint16_t *W, const float *bias, int M,
+                             int N, int K, uint16_t *Y, unsigned int *err, cudaStream_t st);
+
+// Activation statistics: accumulate sums / absmax, then finalize.
+cudaError_t launch_act_stats_update(const uint16_t *X, int T, int K, const float *shift,
+                                    double *sums, float *absmax, cudaStream_t st);
+cudaError_t launch_act_stats_finalize(const double *sums, const float *absmax, const float *shift,
+                                      long long count, int K, float *chan, float *tensor,
+                                      cudaStream_t st);
+
+// Per-tensor activation quantization (two passes: tensor max, then codes).
+cudaError_t launch_quant_act_per_tensor(const uint16_t *X, const float *lambda, int M, int K,
+                                        int8_t *Xq, float *x_scale, float *amax, cudaStream_t st);
+
 // Test hook: one bounded wait that is never satisfied (failure detection).
 cudaError_t launch_wait_probe(unsigned int *err, uint64_t limit_ns, cudaStream_t st);
 

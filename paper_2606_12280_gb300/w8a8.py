@@ -37,6 +37,12 @@ SIGNATURES = {
     "w8a8_device_status": [_P, ctypes.POINTER(ctypes.c_uint32)],
     "w8a8_debug_wait_timeout": [ctypes.c_uint32, _P],
     "w8a8_status_string": [_I],
+    "w8a8_quant_act_per_tensor": [_P, _P, _I, _I, _P, _P, _P, _P],
+    "w8a8_act_stats_update": [_P, _I, _I, _P, _P, _P, _P],
+    "w8a8_act_stats_finalize": [_P, _P, _P, ctypes.c_longlong, _I, _P, _P, _P],
+    "w8a8_linear_bf16": [_P, _P, _P, _I, _I, _I, _P, _P],
+    "w8a8_layer_forward": [_P, _P, _I, _P, _P, _P, _P],
+    "w8a8_select_protected": [_P, _I, _I, _P],
 }
 
 
@@ -50,6 +56,12 @@ class Branch(ctypes.Structure):
     """Mirror of ``w8a8_branch``."""
     _fields_ = [("Xq", _P), ("x_scale", _P), ("Wq", _P), ("w_scale", _P),
                 ("bias", _P), ("Y", _P), ("M", _I)]
+
+
+class Layer(ctypes.Structure):
+    """Mirror of ``w8a8_layer``."""
+    _fields_ = [("protect", _I), ("N", _I), ("K", _I), ("smooth", _P), ("Wq", _P),
+                ("w_scale", _P), ("W_bf16", _P), ("bias", _P)]
 
 
 _lock = threading.Lock()
@@ -215,6 +227,90 @@ def device_status(stream=None) -> int:
 def debug_wait_timeout(limit_us: int, stream=None) -> None:
     """Enqueue a bounded wait that can only time out (failure-detection test)."""
     _check("w8a8_debug_wait_timeout", lib().w8a8_debug_wait_timeout(int(limit_us), _stream(stream)))
+
+
+def quant_act_per_tensor(X, smooth=None, Xq=None, x_scale=None, amax=None, stream=None):
+    """One INT8 scale for all of X diag(lambda)^-1: returns (Xq, sx [M], amax [1])."""
+    M, K = X.shape
+    if Xq is None:
+        Xq = torch.empty(M, K, dtype=torch.int8, device=X.device)
+    if x_scale is None:
+        x_scale = torch.empty(M, dtype=torch.float32, device=X.device)
+    if amax is None:
+        amax = torch.empty(1, dtype=torch.float32, device=X.device)
+    _check("w8a8_quant_act_per_tensor", lib().w8a8_quant_act_per_tensor(
+        _ptr(X, torch.bfloat16, "X"), _ptr(smooth, torch.float32, "smooth"), M, K,
+        _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"),
+        _ptr(amax, torch.float32, "amax"), _stream(stream)))
+    return Xq, x_scale, amax
+
+
+def act_stats_update(X, sums, absmax, shift=None, stream=None):
+    """Accumulate the per-channel power sums [4,K] fp64 and absmax [K] of X [T,K] bf16."""
+    T, K = X.shape
+    _check("w8a8_act_stats_update", lib().w8a8_act_stats_update(
+        _ptr(X, torch.bfloat16, "X"), T, K, _ptr(shift, torch.float32, "shift"),
+        _ptr(sums, torch.float64, "sums"), _ptr(absmax, torch.float32, "absmax"),
+        _stream(stream)))
+
+
+def act_stats_finalize(sums, absmax, count: int, shift=None, chan=None, tensor=None, stream=None):
+    """(chan [4,K], tensor [4]) fp32: max-abs, mean, std, kurtosis."""
+    K = absmax.shape[0]
+    if chan is None:
+        chan = torch.empty(4, K, dtype=torch.float32, device=absmax.device)
+    if tensor is None:
+        tensor = torch.empty(4, dtype=torch.float32, device=absmax.device)
+    _check("w8a8_act_stats_finalize", lib().w8a8_act_stats_finalize(
+        _ptr(sums, torch.float64, "sums"), _ptr(absmax, torch.float32, "absmax"),
+        _ptr(shift, torch.float32, "shift"), int(count), K, _ptr(chan, torch.float32, "chan"),
+        _ptr(tensor, torch.float32, "tensor"), _stream(stream)))
+    return chan, tensor
+
+
+def linear_bf16(X, W, bias=None, Y=None, stream=None):
+    """Protected layer: Y = bf16(X W^T + b), X [M,K] and W [N,K] bf16."""
+    M, K = X.shape
+    N = W.shape[0]
+    if W.shape[1] != K:
+        raise ValueError("X and W disagree on K")
+    if Y is None:
+        Y = torch.empty(M, N, dtype=torch.bfloat16, device=X.device)
+    _check("w8a8_linear_bf16", lib().w8a8_linear_bf16(
+        _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
+        _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(Y, torch.bfloat16, "Y"),
+        _stream(stream)))
+    return Y
+
+
+def layer_forward(X, protect: bool, N: int, K: int, smooth=None, Wq=None, w_scale=None,
+                  W_bf16=None, bias=None, Xq_work=None, x_scale_work=None, Y=None, stream=None):
+    """Per-layer dispatch (protected -> bf16 linear, else a3 + a4 + a5)."""
+    M = X.shape[0]
+    if Y is None:
+        Y = torch.empty(M, N, dtype=torch.bfloat16, device=X.device)
+    if not protect:
+        if Xq_work is None:
+            Xq_work = torch.empty(M, K, dtype=torch.int8, device=X.device)
+        if x_scale_work is None:
+            x_scale_work = torch.empty(M, dtype=torch.float32, device=X.device)
+    layer = Layer(1 if protect else 0, N, K, _ptr(smooth, torch.float32, "smooth"),
+                  _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
+                  _ptr(W_bf16, torch.bfloat16, "W_bf16"), _ptr(bias, torch.float32, "bias"))
+    _check("w8a8_layer_forward", lib().w8a8_layer_forward(
+        ctypes.byref(layer), _ptr(X, torch.bfloat16, "X"), M,
+        _ptr(Xq_work, torch.int8, "Xq_work"), _ptr(x_scale_work, torch.float32, "x_scale_work"),
+        _ptr(Y, torch.bfloat16, "Y"), _stream(stream)))
+    return Y
+
+
+def select_protected(scores, n_protect: int):
+    """Host: flags (list of 0/1) marking the n_protect most fragile layers."""
+    L = len(scores)
+    sc = (ctypes.c_float * L)(*[float(x) for x in scores])
+    flags = (ctypes.c_int * L)()
+    _check("w8a8_select_protected", lib().w8a8_select_protected(sc, L, int(n_protect), flags))
+    return [int(f) for f in flags]
 
 
 def quantized_linear_forward(X, smooth, Wq, w_scale, bias=None, stream=None):

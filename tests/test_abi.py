@@ -10,6 +10,7 @@ import ctypes
 import os
 import re
 
+import numpy as np
 import pytest
 
 from paper_2606_12280_gb300 import _build
@@ -144,3 +145,65 @@ def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
     monkeypatch.setattr(w8a8, "LIB_PATH", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="not built"):
         w8a8.lib()
+
+
+def test_per_tensor_and_stats_validation(L):
+    f = L.w8a8_quant_act_per_tensor
+    assert f(A, None, 4, 16, A, A, None, None) == INVALID        # amax
+    assert f(A, None, 4, 16, A, A, U, None) == MISALIGNED
+    assert f(A, None, 4, 24, A, A, A, None) == SHAPE
+    assert f(A, None, 0, 16, A, A, A, None) == OK                 # empty batch
+    u = L.w8a8_act_stats_update
+    assert u(A, 4, 16, None, None, A, None) == INVALID
+    assert u(A, 4, 16, None, A, None, None) == INVALID
+    assert u(A, 4, 15, None, A, A, None) == SHAPE
+    assert u(A, 4, 16, U, A, A, None) == MISALIGNED              # shift
+    assert u(None, 0, 16, None, A, A, None) == OK                # no tokens
+    fin = L.w8a8_act_stats_finalize
+    assert fin(A, A, None, 0, 16, A, A, None) == INVALID          # count
+    assert fin(A, A, None, 5, 16, A, None, None) == INVALID
+    assert fin(A, A, None, 5, 8, A, A, None) == SHAPE
+
+
+def test_linear_bf16_and_layer_validation(L):
+    from paper_2606_12280_gb300.w8a8 import Layer
+    f = L.w8a8_linear_bf16
+    assert f(A, A, None, 4, 12, 16, A, None) == SHAPE
+    assert f(A, None, None, 4, 8, 16, A, None) == INVALID
+    assert f(A, A, U, 4, 8, 16, A, None) == MISALIGNED
+    assert f(None, None, None, 0, 8, 16, None, None) == OK       # empty batch
+    g = L.w8a8_layer_forward
+    assert g(None, A, 4, A, A, A, None) == INVALID
+    prot = Layer(1, 8, 16, None, None, None, None, None)
+    assert g(ctypes.byref(prot), A, 4, None, None, A, None) == INVALID   # no bf16 weights
+    q = Layer(0, 8, 16, None, A, A, None, None)
+    assert g(ctypes.byref(q), A, 4, None, A, A, None) == INVALID        # no workspace
+    assert g(ctypes.byref(q), A, 4, U, A, A, None) == MISALIGNED
+    assert g(ctypes.byref(q), A, 0, None, None, A, None) == OK
+    bad = Layer(0, 12, 16, None, A, A, None, None)
+    assert g(ctypes.byref(bad), A, 4, A, A, A, None) == SHAPE
+
+
+def test_select_protected():
+    from paper_2606_12280_gb300 import w8a8
+    _build.build()
+    nan = float("nan")
+    # the n largest scores, NaN first, ties to the lower index
+    assert w8a8.select_protected([0.5, 3.0, 1.0, 3.0, 2.0], 2) == [0, 1, 0, 1, 0]
+    assert w8a8.select_protected([0.5, 3.0, 1.0, 3.0, 2.0], 1) == [0, 1, 0, 0, 0]
+    assert w8a8.select_protected([1.0, nan, 5.0], 1) == [0, 1, 0]
+    assert w8a8.select_protected([1.0, nan, 5.0], 3) == [1, 1, 1]
+    assert w8a8.select_protected([1.0, 2.0], 0) == [0, 0]
+    assert w8a8.select_protected([], 0) == []
+    # the paper's setting: 17 of 211 linears
+    rng = np.random.default_rng(0)
+    sc = rng.standard_normal(211).astype(np.float32)
+    flags = w8a8.select_protected(list(sc), 17)
+    assert sum(flags) == 17
+    assert min(sc[np.array(flags) == 1]) > max(sc[np.array(flags) == 0])
+    L = w8a8.lib()
+    assert L.w8a8_select_protected(None, 3, 1, None) == INVALID
+    arr = (ctypes.c_float * 2)(1.0, 2.0)
+    out = (ctypes.c_int * 2)()
+    assert L.w8a8_select_protected(arr, 2, 3, out) == INVALID
+    assert L.w8a8_select_protected(arr, 2, -1, out) == INVALID
