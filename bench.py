@@ -358,6 +358,24 @@ def run_ours(args):
     gemm_iso = isolated(lambda i, st: w8a8.linear(Xqs[i % n_sets], sxs[i % n_sets], Wqs[i % n_sets],
                                                   sw, bias, Y=Ys[i % n_sets], stream=st), 10)
 
+    # the pieces around the layer, each alone in a CUDA graph on the same
+    # workload: the protected bf16 linear, the statistics pass of fragility
+    # profiling and the per-tensor activation quantization of the ablation
+    Wb = [W.to(torch.bfloat16) for _ in range(2)]
+    Yb = [torch.empty(M, N, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+    bf16_iso = isolated(lambda i, st: w8a8.linear_bf16(Xs[i % n_sets], Wb[i % 2], bias,
+                                                       Y=Yb[i % 2], stream=st), 10)
+    st_sums = torch.zeros(4, K, dtype=torch.float64, device=dev)
+    st_max = torch.zeros(K, dtype=torch.float32, device=dev)
+    stats_iso = isolated(lambda i, st: w8a8.act_stats_update(Xs[i % n_sets], st_sums, st_max,
+                                                             stream=st), 40)
+    amax = torch.empty(1, dtype=torch.float32, device=dev)
+    pt_iso = isolated(lambda i, st: w8a8.quant_act_per_tensor(Xs[i % n_sets], lam, Xq=Xqs[i % n_sets],
+                                                              x_scale=sxs[i % n_sets], amax=amax,
+                                                              stream=st), 40)
+    if w8a8.device_status(stream) != 0:
+        raise RuntimeError("device error word set while timing the protection kernels")
+
     peaks, peak_kind = load_peaks()
     gemm_avg = sum(gemm_ms) / len(gemm_ms)
     quant_avg = sum(quant_ms) / len(quant_ms)
@@ -395,6 +413,24 @@ def run_ours(args):
                           "unit": "GB/s", "frac": quant_gbs / peaks["hbm_gbs"],
                           "ms_isolated": quant_iso, "ms_in_step": quant_avg, "bytes": quant_bytes,
                           "kernel": "w8a8_quant_act (a3)"},
+            "protect": {
+                "linear_bf16": {"bound": "tensor", "achieved": ops_step / (bf16_iso * 1e-3) / 1e12,
+                                "peak": peak_t, "unit": "TFLOP/s",
+                                "frac": ops_step / (bf16_iso * 1e-3) / 1e12 / peak_t,
+                                "ms_isolated": bf16_iso, "kernel": "w8a8_linear_bf16"},
+                "act_stats": {"bound": "hbm", "achieved": 2.0 * M * K / (stats_iso * 1e-3) / 1e9,
+                              "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                              "frac": 2.0 * M * K / (stats_iso * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                              "ms_isolated": stats_iso, "bytes": 2.0 * M * K,
+                              "kernel": "w8a8_act_stats_update"},
+            },
+            "ablation": {
+                "quant_act_per_tensor": {"bound": "hbm", "achieved": quant_bytes / (pt_iso * 1e-3) / 1e9,
+                                         "peak": peaks["hbm_gbs"], "unit": "GB/s",
+                                         "frac": quant_bytes / (pt_iso * 1e-3) / 1e9 / peaks["hbm_gbs"],
+                                         "ms_isolated": pt_iso, "bytes": quant_bytes,
+                                         "kernel": "w8a8_quant_act_per_tensor (two passes)"},
+            },
             "gemm_ms": gemm_avg, "gemm_ms_isolated": gemm_iso, "offline_ms": offline,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "TOPS", "h2d_bytes_per_step": 2 * M * K,

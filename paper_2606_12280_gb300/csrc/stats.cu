@@ -72,90 +72,146 @@ __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
 
 // ------------------------------------------------------------ statistics
 //
-// Lane l owns the channel pair (2l, 2l+1) of the block's 64 channels.  Each
-// thread sums (x - c)^p in fp32 over at most kGroup of its rows, then adds
-// the group sums into fp64 registers; the block combines its warps in fp64
-// through shared memory and adds into the global fp64 sums with atomics.
-// Rounding: every fp32 group sum is within (kGroup + 4) * 2^-24 of
-// sum |x - c|^p over the group, fp64 adds are exact to ~2^-53.
-constexpr int kStatsWarps = 16;
+// Lane l owns 4 consecutive channels of the block's 128 (one 8-byte load per
+// row) and the 8 warps of a block split the block's row slab.  Each thread
+// sums (x - c)^p in fp32 over groups of at most kGroup of its rows, adds the
+// group sums into fp32 level-2 sums (at most kGroup groups), and only those
+// into fp64 (at the end of the slab, or every kGroup groups); the block then
+// combines its warps in fp64 through shared memory and adds into the global
+// fp64 sums with atomics.  Rounding: every returned sum is within
+// (2 kGroup + 4) * 2^-24 of sum |x - c|^p of its exact value.
+constexpr int kStatsWarps = 8;
 constexpr int kGroup = 64;
-constexpr int kUnroll = 16;
+constexpr int kUnroll = 8;
+static_assert(kGroup % kUnroll == 0, "whole unrolled batches per group");
 
-__global__ void __launch_bounds__(32 * kStatsWarps, 2)
-stats_update_kernel(const uint32_t *__restrict__ X2, int T, int K, const float *__restrict__ shift,
+struct Acc4 {                   // one moment for the thread's 4 channels
+    float2 a, b;
+};
+
+__global__ void __launch_bounds__(32 * kStatsWarps, 3)
+stats_update_kernel(const uint2 *__restrict__ X4, int T, int K, const float *__restrict__ shift,
                     int rows_per_slab, double *__restrict__ sums, float *__restrict__ absmax) {
-    __shared__ double red_s[kStatsWarps][8][32];
-    __shared__ float red_m[kStatsWarps][2][32];
+    __shared__ double red_s[kStatsWarps][16][32];     // per-thread fp64 sums [p][e]
+    __shared__ float lvl2[kStatsWarps][16][32];       // per-thread level-2 fp32 sums,
+                                                      // then the maxima [e] (48 KB total)
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    const int pair = blockIdx.x * 32 + lane;            // channel pair index
-    const int kp = K / 2;
-    const bool active = pair < kp;
+    const int quad = blockIdx.x * 32 + lane;            // 4-channel group index
+    const int kq = K / 4;
+    const bool active = quad < kq;
     const int r0 = blockIdx.y * rows_per_slab;
     const int r1 = min(T, r0 + rows_per_slab);
+    constexpr int kStep = kStatsWarps * kUnroll;
 
-    float2 c = make_float2(0.0f, 0.0f);
-    if (active && shift) c = make_float2(-__ldg(shift + 2 * pair), -__ldg(shift + 2 * pair + 1));
-    float2 s1 = make_float2(0.f, 0.f), s2 = s1, s3 = s1, s4 = s1;
-    double S[8] = {0, 0, 0, 0, 0, 0, 0, 0};          // p-major: S[2(p-1) + e]
-    float m0 = 0.0f, m1 = 0.0f;
-    int in_group = 0;
-
-    for (int rb = r0 + w; rb < r1; rb += kStatsWarps * kUnroll) {
-        uint32_t v[kUnroll];
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-            const int r = rb + u * kStatsWarps;
-            v[u] = (active && r < r1) ? __ldcs(X2 + (size_t)r * kp + pair) : 0u;
-        }
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-            const int r = rb + u * kStatsWarps;
-            if (r < r1) {
-                const float2 x = make_float2(__uint_as_float(v[u] << 16), __uint_as_float(v[u] & 0xffff0000u));
-                m0 = fmaxf(m0, fabsf(x.x));
-                m1 = fmaxf(m1, fabsf(x.y));
-                const float2 d = add2(x, c);
-                const float2 d2 = mul2(d, d);
-                s1 = add2(s1, d);
-                s2 = add2(s2, d2);
-                s3 = fma2(d2, d, s3);
-                s4 = fma2(d2, d2, s4);
-                ++in_group;
-            }
-        }
-        if (in_group >= kGroup - kUnroll) {            // fold before kGroup rows pile up
-            S[0] += s1.x; S[1] += s1.y; S[2] += s2.x; S[3] += s2.y;
-            S[4] += s3.x; S[5] += s3.y; S[6] += s4.x; S[7] += s4.y;
-            s1 = make_float2(0.f, 0.f); s2 = s1; s3 = s1; s4 = s1;
-            in_group = 0;
-        }
+    float2 c0 = make_float2(0.0f, 0.0f), c1 = c0;     // -shift
+    if (active && shift) {
+        const float4 sh = __ldg(reinterpret_cast<const float4 *>(shift) + quad);
+        c0 = make_float2(-sh.x, -sh.y);
+        c1 = make_float2(-sh.z, -sh.w);
     }
-    S[0] += s1.x; S[1] += s1.y; S[2] += s2.x; S[3] += s2.y;
-    S[4] += s3.x; S[5] += s3.y; S[6] += s4.x; S[7] += s4.y;
+    const float2 z = make_float2(0.f, 0.f);
+    Acc4 g[4] = {{z, z}, {z, z}, {z, z}, {z, z}};      // level 1, p = 1..4
+#pragma unroll
+    for (int i = 0; i < 16; ++i) {
+        red_s[w][i][lane] = 0.0;
+        lvl2[w][i][lane] = 0.0f;
+    }
+    float mx[4] = {0.f, 0.f, 0.f, 0.f};
+    int rows_in_group = 0, groups = 0;
 
-#pragma unroll
-    for (int i = 0; i < 8; ++i) red_s[w][i][lane] = S[i];
-    red_m[w][0][lane] = m0;
-    red_m[w][1][lane] = m1;
-    __syncthreads();
-    if (w == 0 && active && r0 < r1) {
-        double tot[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-        float a0 = 0.0f, a1 = 0.0f;
-        for (int ww = 0; ww < kStatsWarps; ++ww) {
-#pragma unroll
-            for (int i = 0; i < 8; ++i) tot[i] += red_s[ww][i][lane];
-            a0 = fmaxf(a0, red_m[ww][0][lane]);
-            a1 = fmaxf(a1, red_m[ww][1][lane]);
-        }
+    // level 1 -> level 2 (every kGroup rows), level 2 -> fp64 (every kGroup
+    // groups); both live in this thread's slots of shared memory
+    auto fold_group = [&]() {
 #pragma unroll
         for (int p = 0; p < 4; ++p) {
-            atomicAdd(sums + (size_t)p * K + 2 * pair, tot[2 * p]);
-            atomicAdd(sums + (size_t)p * K + 2 * pair + 1, tot[2 * p + 1]);
+            lvl2[w][4 * p + 0][lane] += g[p].a.x;
+            lvl2[w][4 * p + 1][lane] += g[p].a.y;
+            lvl2[w][4 * p + 2][lane] += g[p].b.x;
+            lvl2[w][4 * p + 3][lane] += g[p].b.y;
+            g[p].a = z;
+            g[p].b = z;
         }
-        // non-negative floats order like their bit patterns
-        atomicMax(reinterpret_cast<unsigned int *>(absmax) + 2 * pair, __float_as_uint(a0));
-        atomicMax(reinterpret_cast<unsigned int *>(absmax) + 2 * pair + 1, __float_as_uint(a1));
+        rows_in_group = 0;
+        ++groups;
+    };
+    auto fold_level2 = [&]() {
+#pragma unroll
+        for (int i = 0; i < 16; ++i) {
+            red_s[w][i][lane] += lvl2[w][i][lane];
+            lvl2[w][i][lane] = 0.0f;
+        }
+        groups = 0;
+    };
+    auto load_batch = [&](int rb, uint2 (&v)[kUnroll]) {
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            const int r = rb + u * kStatsWarps;
+            v[u] = (active && r < r1) ? __ldcs(X4 + (size_t)r * kq + quad) : make_uint2(0u, 0u);
+        }
+    };
+
+    // two batches of kUnroll rows in flight: the next one loads while this
+    // one is summed
+    uint2 v[kUnroll];
+    load_batch(r0 + w, v);
+    for (int rb = r0 + w; rb < r1; rb += kStep) {
+        uint2 vn[kUnroll];
+        load_batch(rb + kStep, vn);
+        // rows of this batch inside the slab
+        const int valid = min(kUnroll, (r1 - rb + kStatsWarps - 1) / kStatsWarps);
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) {
+            if (u < valid) {
+                const float2 xa = make_float2(__uint_as_float(v[u].x << 16), __uint_as_float(v[u].x & 0xffff0000u));
+                const float2 xb = make_float2(__uint_as_float(v[u].y << 16), __uint_as_float(v[u].y & 0xffff0000u));
+                mx[0] = fmaxf(mx[0], fabsf(xa.x));
+                mx[1] = fmaxf(mx[1], fabsf(xa.y));
+                mx[2] = fmaxf(mx[2], fabsf(xb.x));
+                mx[3] = fmaxf(mx[3], fabsf(xb.y));
+                const float2 da = add2(xa, c0), db = add2(xb, c1);
+                const float2 da2 = mul2(da, da), db2 = mul2(db, db);
+                g[0].a = add2(g[0].a, da);
+                g[0].b = add2(g[0].b, db);
+                g[1].a = add2(g[1].a, da2);
+                g[1].b = add2(g[1].b, db2);
+                g[2].a = fma2(da2, da, g[2].a);
+                g[2].b = fma2(db2, db, g[2].b);
+                g[3].a = fma2(da2, da2, g[3].a);
+                g[3].b = fma2(db2, db2, g[3].b);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < kUnroll; ++u) v[u] = vn[u];
+        rows_in_group += kUnroll;
+        if (rows_in_group >= kGroup) {
+            fold_group();
+            if (groups >= kGroup) fold_level2();
+        }
+    }
+    fold_group();
+    fold_level2();
+#pragma unroll
+    for (int e = 0; e < 4; ++e) lvl2[w][e][lane] = mx[e];   // own slots: no other thread reads them yet
+    __syncthreads();
+    // warp p (p < 4) reduces moment p, warp 4 the maxima: 4 channels per lane
+    if (active && r0 < r1 && w < 5) {
+        if (w < 4) {
+            double tot[4] = {0, 0, 0, 0};
+            for (int ww = 0; ww < kStatsWarps; ++ww)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) tot[e] += red_s[ww][4 * w + e][lane];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) atomicAdd(sums + (size_t)w * K + 4 * quad + e, tot[e]);
+        } else {
+            float a[4] = {0.f, 0.f, 0.f, 0.f};
+            for (int ww = 0; ww < kStatsWarps; ++ww)
+#pragma unroll
+                for (int e = 0; e < 4; ++e) a[e] = fmaxf(a[e], lvl2[ww][e][lane]);
+            // non-negative floats order like their bit patterns
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+                atomicMax(reinterpret_cast<unsigned int *>(absmax) + 4 * quad + e, __float_as_uint(a[e]));
+        }
     }
 }
 
@@ -374,24 +430,42 @@ tensor_quant_kernel(const uint16_t *__restrict__ X, const float *__restrict__ la
     }
 }
 
-// Row slabs so that the grid fills the GPU about `waves` times over.
-int slabs_for(int rows, int gx, int blocks_per_sm) {
-    int gy = (num_sms() * blocks_per_sm + gx - 1) / gx;
+// Row slabs so that a (gx x gy) grid fills the GPU once: gy = the resident
+// blocks of `kern` on all SMs divided by gx, at most one slab per row.
+template <typename Kern>
+int slabs_for(Kern kern, int threads, int rows, int gx) {
+    int per_sm = 0;
+    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, 0) != cudaSuccess ||
+        per_sm < 1)
+        per_sm = 1;
+    int gy = (num_sms() * per_sm) / gx;
     if (gy > rows) gy = rows;
     if (gy < 1) gy = 1;
     return gy;
 }
 
+// Cached slab counts per (kernel, gx, rows); the grid shape depends only on
+// the launch shape.
+struct SlabCache {
+    int gx = -1, rows = -1, gy = 0;
+};
+
 }  // namespace
 
 cudaError_t launch_act_stats_update(const uint16_t *X, int T, int K, const float *shift,
                                     double *sums, float *absmax, cudaStream_t st) {
-    const int gx = (K / 2 + 31) / 32;
-    int gy = slabs_for(T, gx, 2);
+    const int gx = (K / 4 + 31) / 32;
+    static SlabCache cache;
+    if (cache.gx != gx || cache.rows != T) {
+        cache.gy = slabs_for(stats_update_kernel, 32 * kStatsWarps, T, gx);
+        cache.gx = gx;
+        cache.rows = T;
+    }
+    int gy = cache.gy;
     const int rows_per_slab = (T + gy - 1) / gy;
     gy = (T + rows_per_slab - 1) / rows_per_slab;
     stats_update_kernel<<<dim3(gx, gy), 32 * kStatsWarps, 0, st>>>(
-        reinterpret_cast<const uint32_t *>(X), T, K, shift, rows_per_slab, sums, absmax);
+        reinterpret_cast<const uint2 *>(X), T, K, shift, rows_per_slab, sums, absmax);
     return cudaGetLastError();
 }
 
@@ -408,14 +482,20 @@ cudaError_t launch_quant_act_per_tensor(const uint16_t *X, const float *lambda, 
     cudaError_t e = cudaMemsetAsync(amax, 0, sizeof(float), st);
     if (e != cudaSuccess) return e;
     const int gx = (K / 8 + 31) / 32;
-    int gy = slabs_for(M, gx, 8);
-    const int rows_per_slab = (M + gy - 1) / gy;
-    gy = (M + rows_per_slab - 1) / rows_per_slab;
-    tensor_absmax_kernel<<<dim3(gx, gy), 32 * kQWarps, 0, st>>>(X, lambda, M, K, rows_per_slab, amax);
+    static SlabCache c1, c2;
+    if (c1.gx != gx || c1.rows != M) {
+        c1.gy = slabs_for(tensor_absmax_kernel, 32 * kQWarps, M, gx);
+        c2.gy = slabs_for(tensor_quant_kernel, 32 * kQWarps, M, gx);
+        c1.gx = c2.gx = gx;
+        c1.rows = c2.rows = M;
+    }
+    const int rps1 = (M + c1.gy - 1) / c1.gy, rps2 = (M + c2.gy - 1) / c2.gy;
+    tensor_absmax_kernel<<<dim3(gx, (M + rps1 - 1) / rps1), 32 * kQWarps, 0, st>>>(X, lambda, M, K,
+                                                                                   rps1, amax);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    tensor_quant_kernel<<<dim3(gx, gy), 32 * kQWarps, 0, st>>>(X, lambda, M, K, rows_per_slab, amax,
-                                                                Xq, x_scale);
+    tensor_quant_kernel<<<dim3(gx, (M + rps2 - 1) / rps2), 32 * kQWarps, 0, st>>>(
+        X, lambda, M, K, rps2, amax, Xq, x_scale);
     return cudaGetLastError();
 }
 
