@@ -5,7 +5,8 @@ Only the tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 oracle never imports the product: the two share only the seeded input
 generators, which hold none of the method's arithmetic.
 
-The arithmetic lives in ``w8a8_oracle.c`` and ``protect_oracle.c`` (plain C,
+The arithmetic lives in ``w8a8_oracle.c``, ``protect_oracle.c`` and
+``fused_oracle.c`` (plain C,
 ``-O2 -ffp-contract=off``, no intrinsics), compiled with gcc into
 ``oracle/_build/liboracle.so`` and called through ctypes on numpy arrays.  Each
 function follows the "INT8 W8A8" paragraph of the paper's Method section
@@ -13,7 +14,9 @@ function follows the "INT8 W8A8" paragraph of the paper's Method section
 paper lists as missing (Sec. 7, Limitations).  The activation statistics and
 the protected bf16 layer follow Sec. 3, "Activation-fragility profiling and
 protection"; the per-tensor activation scale is the naive arm of the
-activation-quant ablation (Sec. 5, "What drives INT8 recovery").
+activation-quant ablation (Sec. 5, "What drives INT8 recovery"); the GELU
+fused into the quantization of the FFN down-projection input takes the exact
+erf GELU (the paper does not name the activation).
 """
 
 from __future__ import annotations
@@ -26,7 +29,7 @@ import threading
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRCS = [os.path.join(_HERE, f) for f in ("w8a8_oracle.c", "protect_oracle.c")]
+_SRCS = [os.path.join(_HERE, f) for f in ("w8a8_oracle.c", "protect_oracle.c", "fused_oracle.c")]
 _BUILD = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD, "liboracle.so")
 _lock = threading.Lock()
@@ -80,6 +83,9 @@ def _load():
             lib.oracle_act_stats.argtypes = [P, I64, I64, P, P]
             lib.oracle_shifted_power_sums.argtypes = [P, I64, I64, P, P, P]
             lib.oracle_linear_bf16_rows.argtypes = [P, P, P, I64, I64, I64, I64, I64, P, P]
+            lib.oracle_gelu_value.argtypes = [ctypes.c_float]
+            lib.oracle_gelu_value.restype = ctypes.c_float
+            lib.oracle_gelu_quant_act.argtypes = [P, P, I64, I64, P, P, P, P, P]
             _lib = lib
     return _lib
 
@@ -296,3 +302,41 @@ def layer_forward(X_bf16, layer: dict, rows: tuple[int, int] | None = None):
         return linear_bf16(X_bf16, layer["W_bf16"], layer["bias"], rows=rows)
     Xq, sx = quant_act(X_bf16, layer["smooth"])
     return linear(Xq, sx, layer["Wq"], layer["w_scale"], layer["bias"], rows=rows)
+
+
+# --------------------------------------------------------------------------
+# fused neighbours of a3: both branches in one call, GELU folded in
+# --------------------------------------------------------------------------
+
+def quant_act_dual(branches):
+    """The dual-branch activation quantization is a3 applied to each branch:
+    branches = [(X_bf16, lam), (X_bf16, lam)] -> [(Xq, sx), (Xq, sx)]."""
+    return [quant_act(X, lam) for X, lam in branches]
+
+
+def gelu_value(h) -> np.ndarray:
+    """fl32(GELU(h)), GELU(h) = (h/2) erfc(-h/sqrt(2)) in binary64."""
+    lib = _load()
+    h = np.asarray(h, dtype=np.float32)
+    out = np.empty(h.shape, dtype=np.float32)
+    fi, fo = h.reshape(-1), out.reshape(-1)
+    for i in range(fi.size):
+        fo[i] = lib.oracle_gelu_value(float(fi[i]))
+    return out
+
+
+def gelu_quant_act(H_bf16: np.ndarray, lam: np.ndarray | None, with_pre: bool = False):
+    """Per-token INT8 of GELU(H) diag(lambda)^-1 (GELU in fp32, no bf16 rounding
+    in between): returns (Xq, sx) or (Xq, sx, pre) with pre the fp32 value
+    each code is rounded from."""
+    H = _c(H_bf16, np.uint16)
+    lam = _c(lam, np.float32)
+    M, K = H.shape
+    Xq = np.empty((M, K), dtype=np.int8)
+    sx = np.empty(M, dtype=np.float32)
+    tmp = np.empty(K, dtype=np.float32)
+    row = np.empty(K, dtype=np.float32)
+    pre = np.empty((M, K), dtype=np.float32) if with_pre else None
+    _load().oracle_gelu_quant_act(_ptr(H), _ptr(lam), M, K, _ptr(Xq), _ptr(sx), _ptr(tmp),
+                                  _ptr(row), _ptr(pre))
+    return (Xq, sx, pre) if with_pre else (Xq, sx)
