@@ -164,6 +164,53 @@ W8A8_API w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int
                                 int N, int K, int32_t *acc, void *stream);
 
 /* ------------------------------------------------------------------------
+ * a3 fused with its neighbours in the DiT block.
+ * ---------------------------------------------------------------------- */
+
+/* One branch of the dual-branch activation quantization. */
+typedef struct {
+    const uint16_t *X;     /* [M,K] bf16 */
+    const float *smooth;   /* [K] fp32 (this branch's lambda) or NULL */
+    int M;                 /* tokens of this branch, >= 0 */
+    int8_t *Xq;            /* [M,K] int8, written */
+    float *x_scale;        /* [M] fp32, written */
+} w8a8_act_branch;
+
+/*
+ * a3 for both separate-weight branches (conditional br[0], unconditional
+ * br[1]; each with its own smoothing vector) in one launch whose row space
+ * covers both (two launches when K > 16384).  Results are bitwise identical
+ * to two w8a8_quant_act calls.
+ *   br  host pointer to an array of 2 w8a8_act_branch (read during the call).
+ */
+W8A8_API w8a8_status w8a8_quant_act_dual(const w8a8_act_branch *br, int K, void *stream);
+
+/*
+ * a3 of the FFN down-projection input GELU(H) in one pass over H, the
+ * up-projection's bf16 output (the down-projections are the fragile layers
+ * of Sec. 3, "Activation-fragility profiling and protection"; the paper does
+ * not name the activation, the exact erf form is taken):
+ *     g_mj = GELU(H_mj) = (H_mj / 2) * erfc(-H_mj / sqrt 2)   in fp32
+ *     then w8a8_quant_act's arithmetic on g (no rounding of g to bf16).
+ * GELU is evaluated in fp32 with a fitted approximation, log2 erfc(|h|/sqrt 2)
+ * as a degree-12 polynomial in min(|h|, 8)/4 - 1: g is within a relative
+ * 2e-6 of GELU(H) for H >= -6 and 4e-6 for H >= -8 (below -8 both have
+ * magnitude under |H| * 7e-16), so a code can differ from one computed with
+ * the correctly rounded GELU only where x' * (127/a) lies within ~3e-4 of a
+ * rounding tie (where it differs by one).
+ *   H [M,K] bf16, read.   smooth [K] fp32 or NULL.
+ *   Xq [M,K] int8, x_scale [M] fp32, written.
+ */
+W8A8_API w8a8_status w8a8_gelu_quant_act(const uint16_t *H, const float *smooth, int M, int K,
+                                         int8_t *Xq, float *x_scale, void *stream);
+
+/*
+ * Test export of the GELU that w8a8_gelu_quant_act uses: G[i] = g(H[i]) in
+ * fp32 for n values (n >= 0).  H [n] bf16, read; G [n] fp32, written.
+ */
+W8A8_API w8a8_status w8a8_debug_gelu(const uint16_t *H, int n, float *G, void *stream);
+
+/* ------------------------------------------------------------------------
  * Around the W8A8 layer: the ablation's per-tensor activation scale, the
  * activation statistics of fragility profiling, and the protected (bf16)
  * layers with per-layer dispatch.

@@ -164,6 +164,40 @@ w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int M, int N
     return run_gemm(&b, 1, N, K, true, as_stream(stream));
 }
 
+w8a8_status w8a8_quant_act_dual(const w8a8_act_branch *br, int K, void *stream) {
+    if (!br) return W8A8_ERR_INVALID_ARG;
+    w8a8::QuantActBranch b[2];
+    for (int i = 0; i < 2; ++i) {
+        if (w8a8_status e = check_mk(br[i].M, K)) return e;
+        b[i] = w8a8::QuantActBranch{br[i].X, br[i].smooth, br[i].M, br[i].Xq, br[i].x_scale};
+        if (br[i].M == 0) continue;
+        if (!br[i].X || !br[i].Xq || !br[i].x_scale) return W8A8_ERR_INVALID_ARG;
+        if (!aligned16(br[i].X) || !aligned16(br[i].Xq) || !aligned16(br[i].x_scale) ||
+            (br[i].smooth && !aligned16(br[i].smooth)))
+            return W8A8_ERR_MISALIGNED;
+    }
+    if (br[0].M == 0 && br[1].M == 0) return W8A8_OK;
+    return from_cuda(w8a8::launch_quant_act_dual(b, K, as_stream(stream)));
+}
+
+w8a8_status w8a8_gelu_quant_act(const uint16_t *H, const float *smooth, int M, int K, int8_t *Xq,
+                                float *x_scale, void *stream) {
+    if (w8a8_status e = check_mk(M, K)) return e;
+    if (M == 0) return W8A8_OK;
+    if (!H || !Xq || !x_scale) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(H) || !aligned16(Xq) || !aligned16(x_scale) || (smooth && !aligned16(smooth)))
+        return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_gelu_quant_act(H, smooth, M, K, Xq, x_scale, as_stream(stream)));
+}
+
+w8a8_status w8a8_debug_gelu(const uint16_t *H, int n, float *G, void *stream) {
+    if (n < 0) return W8A8_ERR_UNSUPPORTED_SHAPE;
+    if (n == 0) return W8A8_OK;
+    if (!H || !G) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(H) || !aligned16(G)) return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_debug_gelu(H, n, G, as_stream(stream)));
+}
+
 w8a8_status w8a8_quant_act_per_tensor(const uint16_t *X, const float *smooth, int M, int K,
                                       int8_t *Xq, float *x_scale, float *amax, void *stream) {
     if (w8a8_status e = check_mk(M, K)) return e;

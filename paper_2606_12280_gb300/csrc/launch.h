@@ -28,6 +28,26 @@ cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M,
                              int K, int8_t *Xq, float *x_scale, unsigned int *err,
                              cudaStream_t st);
 
+// One branch of the dual-branch activation quantization.
+struct QuantActBranch {
+    const uint16_t *X;
+    const float *lambda;
+    int M;
+    int8_t *Xq;
+    float *x_scale;
+};
+
+// a3 for both branches in one launch (two launches for K > 16384).
+cudaError_t launch_quant_act_dual(const QuantActBranch *br, int K, cudaStream_t st);
+
+// a3 of GELU(H): the GELU evaluated in fp32 and quantized without rounding
+// to bf16 in between.
+cudaError_t launch_gelu_quant_act(const uint16_t *H, const float *lambda, int M, int K, int8_t *Xq,
+                                  float *x_scale, cudaStream_t st);
+
+// Test export: the fp32 GELU values the fused pass uses.
+cudaError_t launch_debug_gelu(const uint16_t *H, int n, float *G, cudaStream_t st);
+
 // Legacy warp-level mma.sync s8 GEMM (exact int32), nb = 1 or 2 branches.
 // out_i32: write the int32 product instead of the bf16 epilogue.
 cudaError_t launch_gemm_mma(const GemmBranch *br, int nb, int N, int K,

@@ -63,6 +63,73 @@ __device__ __forceinline__ float warp_max(float v) {
     return v;
 }
 
+// GELU(h) = h * Phi(h) = (h/2) erfc(-h/sqrt 2), the exact (erf) form, for
+// the FFN down-projection input.  With a = min(|h|, 8),
+//     log2 erfc(a/sqrt 2) ~= P(u),   u = a/4 - 1   (exact in fp32),
+// P of degree 12 fitted by least squares over a in [0, 8]
+// (fit_gelu_erfc.py beside this file), evaluated by Horner in fp32 with the
+// constant term lowered by 1, so that d = 2^P'(u) = erfc(a/sqrt 2)/2 =
+// Phi(-a); then GELU(h) = h d for h < 0 and h - h d for h >= 0 (one ex2, no
+// division).  Relative error of the result: below 2e-6 for h >= -6 and 4e-6
+// for h >= -8; below -8 the result has magnitude below |h| * 7e-16 like
+// GELU(h) itself.
+__device__ __forceinline__ float ex2_approx(float x) {
+    float r;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t pk(float a, float b) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
+    return r;
+}
+
+__device__ __forceinline__ float2 upk(uint64_t v) {
+    float2 r;
+    asm("mov.b64 {%0, %1}, %2;" : "=f"(r.x), "=f"(r.y) : "l"(v));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t fma_pk(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t mul_pk(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t splat(float c) { return pk(c, c); }
+
+// GELU of two values with packed fp32 instructions (each packed operation
+// rounds like its scalar form).
+__device__ __forceinline__ float2 gelu_erf2(float2 h) {
+    const uint64_t u = fma_pk(pk(fminf(fabsf(h.x), 8.0f), fminf(fabsf(h.y), 8.0f)), splat(0.25f),
+                              splat(-1.0f));
+    uint64_t p = splat(-0.00130923442f);
+    p = fma_pk(p, u, splat(0.00208183355f));
+    p = fma_pk(p, u, splat(0.00157369743f));
+    p = fma_pk(p, u, splat(-0.00497690868f));
+    p = fma_pk(p, u, splat(0.00688785873f));
+    p = fma_pk(p, u, splat(-0.0167602543f));
+    p = fma_pk(p, u, splat(0.039086014f));
+    p = fma_pk(p, u, splat(-0.0774176419f));
+    p = fma_pk(p, u, splat(0.146253109f));
+    p = fma_pk(p, u, splat(-0.274731398f));
+    p = fma_pk(p, u, splat(-11.0028801f));
+    p = fma_pk(p, u, splat(-24.3850517f));
+    p = fma_pk(p, u, splat(-14.9464674f));                  // C0 - 1: halves erfc
+    const float2 lg = upk(p);
+    const float2 q = upk(mul_pk(pk(h.x, h.y), pk(ex2_approx(lg.x), ex2_approx(lg.y))));   // h Phi(-|h|)
+    return make_float2(h.x >= 0.0f ? h.x - q.x : q.x, h.y >= 0.0f ? h.y - q.y : q.y);
+}
+
+__device__ __forceinline__ float gelu_erf(float h) { return gelu_erf2(make_float2(h, 0.0f)).x; }
+
 // ------------------------------------------------------------- row quant
 //
 // IS_ACT:  factor f_j = 1/lambda_j (activations are divided by lambda);
@@ -174,7 +241,7 @@ row_quant_kernel(const InT *__restrict__ in, const float *__restrict__ lam,
 // Rows too long to hold in registers (K > 4 * 512 * 8 = 16384): two passes
 // over the row, one for the absmax and one for the codes.  One block of 512
 // threads per row at a time.
-template <typename InT, bool IS_ACT>
+template <typename InT, bool IS_ACT, bool GELU = false>
 __global__ void __launch_bounds__(512)
 row_quant_long_kernel(const InT *__restrict__ in, const float *__restrict__ lam,
                       int M, int K, int8_t *__restrict__ q,
@@ -191,7 +258,7 @@ row_quant_long_kernel(const InT *__restrict__ in, const float *__restrict__ lam,
             for (int e = 0; e < 8; ++e) {
                 float fe = 1.0f;
                 if (lam) { const float l = __ldg(lam + col0 + e); fe = IS_ACT ? __frcp_rn(l) : l; }
-                a = fmaxf(a, fabsf(__fmul_rn(ch.get(e), fe)));
+                a = fmaxf(a, fabsf(__fmul_rn(GELU ? gelu_erf(ch.get(e)) : ch.get(e), fe)));
             }
         }
         a = warp_max(a);
@@ -212,7 +279,7 @@ row_quant_long_kernel(const InT *__restrict__ in, const float *__restrict__ lam,
                 for (int e = 0; e < 8; ++e) {
                     float fe = 1.0f;
                     if (lam) { const float l = __ldg(lam + col0 + e); fe = IS_ACT ? __frcp_rn(l) : l; }
-                    const float xs = __fmul_rn(ch.get(e), fe);
+                    const float xs = __fmul_rn(GELU ? gelu_erf(ch.get(e)) : ch.get(e), fe);
                     const uint32_t b = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xs, inv))) & 0xffu;
                     if (e < 4) lo |= b << (8 * e);
                     else hi |= b << (8 * (e - 4));
@@ -315,22 +382,44 @@ __device__ __forceinline__ void cp_async_16(uint32_t dst, const void *src, bool 
                  "r"(valid ? 16 : 0) : "memory");
 }
 
-template <int U, int TW, int S>
+struct ActBranch {
+    const uint16_t *X;
+    const float *lam;
+    int8_t *Xq;
+    float *x_scale;
+    int M;
+};
+
+// One launch covers up to two independent row sets (the conditional and
+// unconditional branches): teams [0, teams0) of the grid take branch 0, the
+// others branch 1, so every team keeps one branch's 1/lambda in registers.
+struct ActParams {
+    ActBranch br[2];
+    int K;
+    int teams0;
+};
+
+template <int U, int TW, int S, bool GELU>
 __global__ void __launch_bounds__(TW > 8 ? 32 * TW : 256)
-act_quant_team_kernel(const uint16_t *__restrict__ X, const float *__restrict__ lam, int M, int K,
-                      int8_t *__restrict__ Xq, float *__restrict__ x_scale) {
+act_quant_team_kernel(const __grid_constant__ ActParams p) {
     constexpr int kThreads = TW > 8 ? 32 * TW : 256;
     constexpr int kTeams = kThreads / (32 * TW);
     extern __shared__ __align__(16) uint4 ring_s[];
     __shared__ float red[2][kThreads / 32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int team = warp / TW, tw = warp % TW;
+    const int K = p.K;
     const int cpr = K / 8;                                  // 16-byte chunks per row
     const uint32_t ring = static_cast<uint32_t>(__cvta_generic_to_shared(ring_s)) +
                           static_cast<uint32_t>((warp * S * U * 32 + lane) * 16);
 
-    const int teams = gridDim.x * kTeams;
-    const int first = blockIdx.x * kTeams + team;
+    const int gteam = blockIdx.x * kTeams + team;
+    const bool second = gteam >= p.teams0;
+    const ActBranch b = second ? p.br[1] : p.br[0];
+    const uint16_t *__restrict__ X = b.X;
+    const int M = b.M;
+    const int teams = second ? gridDim.x * kTeams - p.teams0 : p.teams0;
+    const int first = second ? gteam - p.teams0 : gteam;
     auto issue = [&](int k) {                               // row slice k of this team -> slot k % S
         const int row = first + k * teams;
         const uint32_t slot = ring + static_cast<uint32_t>((k % S) * U * 32 * 16);
@@ -350,13 +439,13 @@ act_quant_team_kernel(const uint16_t *__restrict__ X, const float *__restrict__ 
     for (int u = 0; u < U; ++u) {
         const int c = (u * TW + tw) * 32 + lane;
 #pragma unroll
-        for (int p = 0; p < 4; ++p) {
+        for (int q = 0; q < 4; ++q) {
             float f0 = 1.0f, f1 = 1.0f;
-            if (lam != nullptr && c < cpr) {
-                f0 = __frcp_rn(__ldg(lam + 8 * c + 2 * p));
-                f1 = __frcp_rn(__ldg(lam + 8 * c + 2 * p + 1));
+            if (b.lam != nullptr && c < cpr) {
+                f0 = __frcp_rn(__ldg(b.lam + 8 * c + 2 * q));
+                f1 = __frcp_rn(__ldg(b.lam + 8 * c + 2 * q + 1));
             }
-            r[u][p] = make_float2(f0, f1);
+            r[u][q] = make_float2(f0, f1);
         }
     }
 
@@ -374,12 +463,15 @@ act_quant_team_kernel(const uint16_t *__restrict__ X, const float *__restrict__ 
             uint4 v;
             asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
                          : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(slot + u * 32 * 16));
-            xs[u][0] = mul2_rn(make_float2(__uint_as_float(v.x << 16), __uint_as_float(v.x & 0xffff0000u)), r[u][0]);
-            xs[u][1] = mul2_rn(make_float2(__uint_as_float(v.y << 16), __uint_as_float(v.y & 0xffff0000u)), r[u][1]);
-            xs[u][2] = mul2_rn(make_float2(__uint_as_float(v.z << 16), __uint_as_float(v.z & 0xffff0000u)), r[u][2]);
-            xs[u][3] = mul2_rn(make_float2(__uint_as_float(v.w << 16), __uint_as_float(v.w & 0xffff0000u)), r[u][3]);
+            const uint32_t wd[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-            for (int p = 0; p < 4; ++p) a = fmaxf(a, fmaxf(fabsf(xs[u][p].x), fabsf(xs[u][p].y)));
+            for (int q = 0; q < 4; ++q) {
+                float2 h = make_float2(__uint_as_float(wd[q] << 16), __uint_as_float(wd[q] & 0xffff0000u));
+                if (GELU) h = gelu_erf2(h);
+                xs[u][q] = mul2_rn(h, r[u][q]);
+            }
+#pragma unroll
+            for (int q = 0; q < 4; ++q) a = fmaxf(a, fmaxf(fabsf(xs[u][q].x), fabsf(xs[u][q].y)));
         }
         a = warp_max(a);
         if (TW > 1) {
@@ -390,10 +482,10 @@ act_quant_team_kernel(const uint16_t *__restrict__ X, const float *__restrict__ 
         }
         const bool zero_row = (a == 0.0f);
         const float inv = zero_row ? 0.0f : __fdiv_rn(127.0f, a);
-        if (tw == 0 && lane == 0) x_scale[row] = zero_row ? 0.0f : __fdiv_rn(a, 127.0f);
+        if (tw == 0 && lane == 0) b.x_scale[row] = zero_row ? 0.0f : __fdiv_rn(a, 127.0f);
         // a and 127/a finite: |x' * inv| <= 127 (1 + 2^-23), no clamp needed
         const bool fast = (a <= 3.402823466e38f) && (inv <= 3.402823466e38f);
-        uint2 *qr = reinterpret_cast<uint2 *>(Xq + (size_t)row * K);
+        uint2 *qr = reinterpret_cast<uint2 *>(b.Xq + (size_t)row * K);
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const int c = (u * TW + tw) * 32 + lane;
@@ -411,8 +503,8 @@ act_quant_team_kernel(const uint16_t *__restrict__ X, const float *__restrict__ 
 #pragma unroll
                 for (int e = 0; e < 8; ++e) {
                     const float xv = (e & 1) ? xs[u][e >> 1].y : xs[u][e >> 1].x;
-                    const uint32_t b = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xv, inv))) & 0xffu;
-                    word[e >> 2] |= b << (8 * (e & 3));
+                    const uint32_t q8 = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xv, inv))) & 0xffu;
+                    word[e >> 2] |= q8 << (8 * (e & 3));
                 }
             }
             qr[c] = make_uint2(word[0], word[1]);
@@ -421,15 +513,14 @@ act_quant_team_kernel(const uint16_t *__restrict__ X, const float *__restrict__ 
     asm volatile("cp.async.wait_group 0;" ::: "memory");
 }
 
-template <int U, int TW>
-cudaError_t launch_act_quant_team(const uint16_t *X, const float *lam, int M, int K, int8_t *Xq,
-                                  float *x_scale, cudaStream_t st) {
+template <int U, int TW, bool GELU>
+cudaError_t launch_act_quant_team(ActParams p, cudaStream_t st) {
     constexpr int S = 4;
     constexpr int kThreads = TW > 8 ? 32 * TW : 256;
     constexpr int kTeams = kThreads / (32 * TW);
     constexpr size_t smem = (size_t)(kThreads / 32) * S * U * 32 * 16;
     static int per_sm = 0;
-    auto kern = act_quant_team_kernel<U, TW, S>;
+    auto kern = act_quant_team_kernel<U, TW, S, GELU>;
     if (per_sm == 0) {
         if (smem > 48 * 1024) {
             cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -439,11 +530,34 @@ cudaError_t launch_act_quant_team(const uint16_t *X, const float *lam, int M, in
         cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem);
         if (per_sm < 1) per_sm = 1;
     }
+    const int M0 = p.br[0].M, M1 = p.br[1].M;
     int grid = num_sms() * per_sm;
-    const int blocks_needed = (M + kTeams - 1) / kTeams;
+    const int blocks_needed = (M0 + M1 + kTeams - 1) / kTeams;
     if (grid > blocks_needed) grid = blocks_needed;
-    kern<<<grid, kThreads, smem, st>>>(X, lam, M, K, Xq, x_scale);
+    const bool both = M0 > 0 && M1 > 0;
+    if (both && grid * kTeams < 2) grid = 2;            // at least one team per branch
+    const int nteams = grid * kTeams;
+    if (!both) {
+        p.teams0 = M1 == 0 ? nteams : 0;
+    } else {
+        int t0 = static_cast<int>((static_cast<long long>(nteams) * M0 + (M0 + M1) / 2) / (M0 + M1));
+        p.teams0 = t0 < 1 ? 1 : (t0 > nteams - 1 ? nteams - 1 : t0);
+    }
+    kern<<<grid, kThreads, smem, st>>>(p);
     return cudaGetLastError();
+}
+
+template <bool GELU>
+cudaError_t launch_act_quant_teams(const ActParams &p, cudaStream_t st) {
+    // team of TW warps per row, U chunks of 8 values per lane: K <= 256 U TW
+    const int K = p.K;
+    if (K <= 256) return launch_act_quant_team<1, 1, GELU>(p, st);
+    if (K <= 512) return launch_act_quant_team<2, 1, GELU>(p, st);
+    if (K <= 1024) return launch_act_quant_team<2, 2, GELU>(p, st);
+    if (K <= 2048) return launch_act_quant_team<2, 4, GELU>(p, st);
+    if (K <= 4096) return launch_act_quant_team<2, 8, GELU>(p, st);
+    if (K <= 8192) return launch_act_quant_team<2, 16, GELU>(p, st);
+    return launch_act_quant_team<4, 16, GELU>(p, st);
 }
 
 // ----------------------------------------------------------- column absmax
@@ -532,20 +646,59 @@ cudaError_t launch_quantize_weights(const float *W, const float *lambda, int N, 
 cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M, int K,
                              int8_t *Xq, float *x_scale, unsigned int *err, cudaStream_t st) {
     (void)err;  // no kernel of this pass waits on a barrier
-    // one warp per row, row held in registers (16 chunks of 8 per lane covers
-    // K <= 4096 in one read; wider rows are read twice, the second time from
-    // L2); 1/lambda needs K * 4 bytes of shared memory per block
-    // team of TW warps per row, U chunks of 8 values per lane: K <= 256 U TW
     if (K <= 16384) {
-        if (K <= 256) return launch_act_quant_team<1, 1>(X, lambda, M, K, Xq, x_scale, st);
-        if (K <= 512) return launch_act_quant_team<2, 1>(X, lambda, M, K, Xq, x_scale, st);
-        if (K <= 1024) return launch_act_quant_team<2, 2>(X, lambda, M, K, Xq, x_scale, st);
-        if (K <= 2048) return launch_act_quant_team<2, 4>(X, lambda, M, K, Xq, x_scale, st);
-        if (K <= 4096) return launch_act_quant_team<2, 8>(X, lambda, M, K, Xq, x_scale, st);
-        if (K <= 8192) return launch_act_quant_team<2, 16>(X, lambda, M, K, Xq, x_scale, st);
-        return launch_act_quant_team<4, 16>(X, lambda, M, K, Xq, x_scale, st);
+        ActParams p{};
+        p.br[0] = ActBranch{X, lambda, Xq, x_scale, M};
+        p.K = K;
+        return launch_act_quant_teams<false>(p, st);
     }
     return launch_row_quant<uint16_t, true>(X, lambda, M, K, Xq, x_scale, st);
+}
+
+cudaError_t launch_quant_act_dual(const QuantActBranch *br, int K, cudaStream_t st) {
+    if (K <= 16384) {
+        ActParams p{};
+        for (int i = 0; i < 2; ++i)
+            p.br[i] = ActBranch{br[i].X, br[i].lambda, br[i].Xq, br[i].x_scale, br[i].M};
+        p.K = K;
+        return launch_act_quant_teams<false>(p, st);
+    }
+    for (int i = 0; i < 2; ++i) {
+        if (br[i].M == 0) continue;
+        cudaError_t e = launch_row_quant<uint16_t, true>(br[i].X, br[i].lambda, br[i].M, K, br[i].Xq,
+                                                         br[i].x_scale, st);
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+}
+
+namespace {
+__global__ void gelu_values_kernel(const uint16_t *__restrict__ H, int n, float *__restrict__ G) {
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
+        G[i] = gelu_erf(bf16_bits_to_f32(H[i]));
+}
+}  // namespace
+
+cudaError_t launch_debug_gelu(const uint16_t *H, int n, float *G, cudaStream_t st) {
+    if (n == 0) return cudaSuccess;
+    int grid = (n + 255) / 256;
+    if (grid > num_sms() * 8) grid = num_sms() * 8;
+    gelu_values_kernel<<<grid, 256, 0, st>>>(H, n, G);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gelu_quant_act(const uint16_t *H, const float *lambda, int M, int K, int8_t *Xq,
+                                  float *x_scale, cudaStream_t st) {
+    if (K <= 16384) {
+        ActParams p{};
+        p.br[0] = ActBranch{H, lambda, Xq, x_scale, M};
+        p.K = K;
+        return launch_act_quant_teams<true>(p, st);
+    }
+    int g2 = num_sms() * 2;
+    if (g2 > M) g2 = M;
+    row_quant_long_kernel<uint16_t, true, true><<<g2, 512, 0, st>>>(H, lambda, M, K, Xq, x_scale);
+    return cudaGetLastError();
 }
 
 }  // namespace w8a8

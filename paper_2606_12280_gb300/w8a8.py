@@ -43,6 +43,9 @@ SIGNATURES = {
     "w8a8_linear_bf16": [_P, _P, _P, _I, _I, _I, _P, _P],
     "w8a8_layer_forward": [_P, _P, _I, _P, _P, _P, _P],
     "w8a8_select_protected": [_P, _I, _I, _P],
+    "w8a8_quant_act_dual": [_P, _I, _P],
+    "w8a8_gelu_quant_act": [_P, _P, _I, _I, _P, _P, _P],
+    "w8a8_debug_gelu": [_P, _I, _P, _P],
 }
 
 
@@ -56,6 +59,11 @@ class Branch(ctypes.Structure):
     """Mirror of ``w8a8_branch``."""
     _fields_ = [("Xq", _P), ("x_scale", _P), ("Wq", _P), ("w_scale", _P),
                 ("bias", _P), ("Y", _P), ("M", _I)]
+
+
+class ActBranch(ctypes.Structure):
+    """Mirror of ``w8a8_act_branch``."""
+    _fields_ = [("X", _P), ("smooth", _P), ("M", _I), ("Xq", _P), ("x_scale", _P)]
 
 
 class Layer(ctypes.Structure):
@@ -227,6 +235,54 @@ def device_status(stream=None) -> int:
 def debug_wait_timeout(limit_us: int, stream=None) -> None:
     """Enqueue a bounded wait that can only time out (failure-detection test)."""
     _check("w8a8_debug_wait_timeout", lib().w8a8_debug_wait_timeout(int(limit_us), _stream(stream)))
+
+
+def quant_act_dual(branches, out=None, stream=None):
+    """a3 for two branches in one launch: branches = [(X, smooth), (X, smooth)]
+    (smooth may be None); returns [(Xq, sx), (Xq, sx)] (written into `out`
+    when given)."""
+    if len(branches) != 2:
+        raise ValueError("quant_act_dual takes exactly two branches")
+    K = branches[0][0].shape[1]
+    arr = (ActBranch * 2)()
+    res = []
+    for i, (X, sm) in enumerate(branches):
+        if X.shape[1] != K:
+            raise ValueError("branches must share K")
+        M = X.shape[0]
+        if out is not None:
+            Xq, sx = out[i]
+        else:
+            Xq = torch.empty(M, K, dtype=torch.int8, device=X.device)
+            sx = torch.empty(M, dtype=torch.float32, device=X.device)
+        arr[i] = ActBranch(_ptr(X, torch.bfloat16, "X"), _ptr(sm, torch.float32, "smooth"), M,
+                           _ptr(Xq, torch.int8, "Xq"), _ptr(sx, torch.float32, "x_scale"))
+        res.append((Xq, sx))
+    _check("w8a8_quant_act_dual", lib().w8a8_quant_act_dual(arr, K, _stream(stream)))
+    return res
+
+
+def gelu_quant_act(H, smooth=None, Xq=None, x_scale=None, stream=None):
+    """Per-token INT8 of GELU(H) diag(lambda)^-1 in one pass: returns (Xq, sx)."""
+    M, K = H.shape
+    if Xq is None:
+        Xq = torch.empty(M, K, dtype=torch.int8, device=H.device)
+    if x_scale is None:
+        x_scale = torch.empty(M, dtype=torch.float32, device=H.device)
+    _check("w8a8_gelu_quant_act", lib().w8a8_gelu_quant_act(
+        _ptr(H, torch.bfloat16, "H"), _ptr(smooth, torch.float32, "smooth"), M, K,
+        _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"), _stream(stream)))
+    return Xq, x_scale
+
+
+def debug_gelu(H, G=None, stream=None):
+    """The fp32 GELU values of the fused pass, for a flat bf16 tensor H."""
+    n = H.numel()
+    if G is None:
+        G = torch.empty(n, dtype=torch.float32, device=H.device)
+    _check("w8a8_debug_gelu", lib().w8a8_debug_gelu(
+        _ptr(H, torch.bfloat16, "H"), n, _ptr(G, torch.float32, "G"), _stream(stream)))
+    return G
 
 
 def quant_act_per_tensor(X, smooth=None, Xq=None, x_scale=None, amax=None, stream=None):

@@ -97,15 +97,26 @@ def _activations(g: torch.Generator, M: int, K: int, outliers: torch.Tensor,
         x = torch.randn(M, K, generator=g, dtype=torch.float32)
         x[:, outliers] *= mult
         return _bf16_bits(x)
-    if act == "gelu_t":
+    if act in ("gelu_t", "heavy_t"):
         z = torch.randn(M, K, generator=g, dtype=torch.float32)
         # Student-t(3) on the outlier channels: z / sqrt(chi2_3 / 3)
         n = outliers.numel()
         zt = torch.randn(M, n, generator=g, dtype=torch.float32)
         chi2 = (torch.randn(M, n, 3, generator=g, dtype=torch.float32) ** 2).sum(-1)
         z[:, outliers] = zt / torch.sqrt(chi2 / 3.0)
-        return _bf16_bits(torch.nn.functional.gelu(z))
+        # "heavy_t" is the pre-activation itself (the up-projection output
+        # that the GELU-fused quantization reads); "gelu_t" is the FFN
+        # down-projection input built from it outside the method
+        return _bf16_bits(z if act == "heavy_t" else torch.nn.functional.gelu(z))
     raise ValueError(act)
+
+
+def ffn_preactivation(M: int, K: int, seed: int, frac: float = 0.01) -> np.ndarray:
+    """Stand-in for the FFN up-projection output [M, K] bf16: N(0, 1) with a
+    Student-t(3) on max(1, round(frac*K)) channels (outlier set drawn first)."""
+    g = torch.Generator().manual_seed(seed)
+    outliers = torch.randperm(K, generator=g)[:n_outliers(K, frac)]
+    return _activations(g, M, K, outliers, 1.0, "heavy_t")
 
 
 @dataclasses.dataclass

@@ -207,3 +207,25 @@ def test_select_protected():
     out = (ctypes.c_int * 2)()
     assert L.w8a8_select_protected(arr, 2, 3, out) == INVALID
     assert L.w8a8_select_protected(arr, 2, -1, out) == INVALID
+
+
+def test_fused_quant_validation(L):
+    from paper_2606_12280_gb300.w8a8 import ActBranch
+    arr = (ActBranch * 2)()
+    for i in range(2):
+        arr[i] = ActBranch(A, None, 4, A, A)
+    f = L.w8a8_quant_act_dual
+    assert f(None, 16, None) == INVALID
+    assert f(arr, 24, None) == SHAPE
+    arr[1].Xq = U
+    assert f(arr, 16, None) == MISALIGNED
+    arr[1].Xq = None
+    assert f(arr, 16, None) == INVALID
+    arr[0] = ActBranch(None, None, 0, None, None)
+    arr[1] = ActBranch(None, None, 0, None, None)
+    assert f(arr, 16, None) == OK                        # both branches empty
+    g = L.w8a8_gelu_quant_act
+    assert g(A, None, 4, 15, A, A, None) == SHAPE
+    assert g(None, None, 4, 16, A, A, None) == INVALID
+    assert g(A, U, 4, 16, A, A, None) == MISALIGNED
+    assert g(None, None, 0, 16, None, None, None) == OK  # empty batch
