@@ -5,8 +5,8 @@ Only the tests, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
 oracle never imports the product: the two share only the seeded input
 generators, which hold none of the method's arithmetic.
 
-The arithmetic lives in ``w8a8_oracle.c``, ``protect_oracle.c`` and
-``fused_oracle.c`` (plain C,
+The arithmetic lives in ``w8a8_oracle.c``, ``protect_oracle.c``,
+``fused_oracle.c`` and ``gguf_oracle.c`` (plain C,
 ``-O2 -ffp-contract=off``, no intrinsics), compiled with gcc into
 ``oracle/_build/liboracle.so`` and called through ctypes on numpy arrays.  Each
 function follows the "INT8 W8A8" paragraph of the paper's Method section
@@ -16,7 +16,8 @@ the protected bf16 layer follow Sec. 3, "Activation-fragility profiling and
 protection"; the per-tensor activation scale is the naive arm of the
 activation-quant ablation (Sec. 5, "What drives INT8 recovery"); the GELU
 fused into the quantization of the FFN down-projection input takes the exact
-erf GELU (the paper does not name the activation).
+erf GELU (the paper does not name the activation); the GGUF Q8_0 / Q4_K
+weight-only layer decodes the public block formats (Sec. 3, "GGUF k-quants").
 """
 
 from __future__ import annotations
@@ -29,7 +30,8 @@ import threading
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRCS = [os.path.join(_HERE, f) for f in ("w8a8_oracle.c", "protect_oracle.c", "fused_oracle.c")]
+_SRCS = [os.path.join(_HERE, f) for f in ("w8a8_oracle.c", "protect_oracle.c", "fused_oracle.c",
+                                          "gguf_oracle.c")]
 _BUILD = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD, "liboracle.so")
 _lock = threading.Lock()
@@ -86,6 +88,11 @@ def _load():
             lib.oracle_gelu_value.argtypes = [ctypes.c_float]
             lib.oracle_gelu_value.restype = ctypes.c_float
             lib.oracle_gelu_quant_act.argtypes = [P, P, I64, I64, P, P, P, P, P]
+            lib.oracle_f32_to_bf16_rne_array.argtypes = [P, I64, P]
+            lib.oracle_f16_to_f32.argtypes = [ctypes.c_uint16]
+            lib.oracle_f16_to_f32.restype = ctypes.c_float
+            lib.oracle_dequant_q8_0.argtypes = [P, I64, I64, P]
+            lib.oracle_dequant_q4_k.argtypes = [P, I64, I64, P]
             _lib = lib
     return _lib
 
@@ -340,3 +347,47 @@ def gelu_quant_act(H_bf16: np.ndarray, lam: np.ndarray | None, with_pre: bool = 
     _load().oracle_gelu_quant_act(_ptr(H), _ptr(lam), M, K, _ptr(Xq), _ptr(sx), _ptr(tmp),
                                   _ptr(row), _ptr(pre))
     return (Xq, sx, pre) if with_pre else (Xq, sx)
+
+
+# --------------------------------------------------------------------------
+# GGUF weight-only layer (Sec. 3, "GGUF k-quants")
+# --------------------------------------------------------------------------
+
+GGUF_Q8_0, GGUF_Q4_K = 0, 1
+GGUF_BLOCK = {GGUF_Q8_0: (32, 34), GGUF_Q4_K: (256, 144)}   # weights, bytes
+
+
+def f32_to_bf16_array(x: np.ndarray) -> np.ndarray:
+    """fp32 -> bf16 bit patterns (round to nearest even), any shape."""
+    x = np.ascontiguousarray(x, dtype=np.float32)
+    out = np.empty(x.shape, dtype=np.uint16)
+    _load().oracle_f32_to_bf16_rne_array(_ptr(x), x.size, _ptr(out))
+    return out
+
+
+def f16_to_f32(h) -> np.ndarray:
+    lib = _load()
+    h = np.asarray(h, dtype=np.uint16)
+    return np.array([lib.oracle_f16_to_f32(int(v)) for v in h.ravel()], np.float32).reshape(h.shape)
+
+
+def gguf_dequant(raw: np.ndarray, fmt: int, N: int, K: int) -> np.ndarray:
+    """Decode N rows of K weights from raw GGUF blocks (uint8 [N, K/QK*bytes]) to fp32."""
+    qk, nbytes = GGUF_BLOCK[fmt]
+    raw = np.ascontiguousarray(raw, dtype=np.uint8).reshape(N, K // qk * nbytes)
+    out = np.empty((N, K), dtype=np.float32)
+    fn = _load().oracle_dequant_q8_0 if fmt == GGUF_Q8_0 else _load().oracle_dequant_q4_k
+    fn(_ptr(raw), N, K, _ptr(out))
+    return out
+
+
+def gguf_dequant_bf16(raw, fmt, N, K) -> np.ndarray:
+    """The decoded weights as the layer consumes them: bf16 (nearest even)."""
+    return f32_to_bf16_array(gguf_dequant(raw, fmt, N, K))
+
+
+def linear_gguf(X_bf16, raw, fmt, N, bias, rows=None):
+    """Weight-only layer: y = X dequant(W)^T + b with the decoded weights in
+    bf16, as (y, yabs) in binary64 for rows [m0, m1)."""
+    K = X_bf16.shape[1]
+    return linear_bf16(X_bf16, gguf_dequant_bf16(raw, fmt, N, K), bias, rows=rows)

@@ -79,6 +79,13 @@ uint16_t oracle_f32_to_bf16_rne(float t)
     return (uint16_t)(u >> 16);
 }
 
+/* the same rounding over an array */
+void oracle_f32_to_bf16_rne_array(const float *x, int64_t n, uint16_t *out)
+{
+    for (int64_t i = 0; i < n; ++i)
+        out[i] = oracle_f32_to_bf16_rne(x[i]);
+}
+
 /* q = clamp(round_half_even(v), -127, 127); a NaN product gives 0. */
 static int8_t quantize_rne_clamp(float v)
 {

@@ -183,3 +183,26 @@ def random_uniform_f32(shape, seed: int, lo: float, hi: float) -> np.ndarray:
 def random_bf16(shape, seed: int, scale: float = 1.0) -> np.ndarray:
     g = torch.Generator().manual_seed(seed)
     return _bf16_bits(torch.randn(tuple(shape), generator=g, dtype=torch.float32) * scale)
+
+
+def random_gguf(fmt: int, N: int, K: int, seed: int) -> np.ndarray:
+    """Random but well-formed GGUF weight blocks, uint8 [N, bytes per row]:
+    fmt 0 = Q8_0 (fp16 d in [1e-4, 4e-3), int8 quants), fmt 1 = Q4_K (fp16 d
+    and dmin in [1e-5, 4e-4), random 6-bit scale/min bytes, random 4-bit
+    quants).  Only random draws: decoding is the method's business."""
+    g = torch.Generator().manual_seed(seed)
+    if fmt == 0:
+        nb = K // 32
+        d = (torch.rand(N, nb, generator=g) * 3.9e-3 + 1e-4).to(torch.float16)
+        q = torch.randint(-127, 128, (N, nb, 32), generator=g, dtype=torch.int16).to(torch.int8)
+        raw = np.empty((N, nb, 34), np.uint8)
+        raw[..., 0:2] = d.view(torch.int16).numpy().view(np.uint8).reshape(N, nb, 2)
+        raw[..., 2:] = q.numpy().view(np.uint8)
+        return raw.reshape(N, nb * 34)
+    nb = K // 256
+    dd = (torch.rand(N, nb, 2, generator=g) * 3.9e-4 + 1e-5).to(torch.float16)
+    rest = torch.randint(0, 256, (N, nb, 140), generator=g, dtype=torch.int16).to(torch.uint8)
+    raw = np.empty((N, nb, 144), np.uint8)
+    raw[..., 0:4] = dd.view(torch.int16).numpy().view(np.uint8).reshape(N, nb, 4)
+    raw[..., 4:] = rest.numpy()
+    return raw.reshape(N, nb * 144)
