@@ -395,6 +395,15 @@ def run_ours(args):
     gelu_iso = isolated(lambda i, st: w8a8.gelu_quant_act(Hg[i % 2], lam_g, Xq=Xqg[i % 2],
                                                           x_scale=sxg[i % 2], stream=st), 20)
     del Xd2, Hg, Xqg, outd
+    # the GGUF weight-only layer on the same QKV shape (bf16 activations,
+    # Q8_0 / Q4_K weight blocks decoded next to the MMA)
+    gguf_iso = {}
+    for fmt, name in ((0, "q8_0"), (1, "q4_k")):
+        raws = [torch.from_numpy(wl.random_gguf(fmt, N, K, seed=20 + fmt + i)).to(dev) for i in range(2)]
+        gguf_iso[name] = (isolated(lambda i, st: w8a8.linear_gguf(Xs[i % n_sets], raws[i % 2], fmt, N, bias,
+                                                                   Y=Yb[i % 2], stream=st), 10),
+                          raws[0].numel())
+        del raws
     if w8a8.device_status(stream) != 0:
         raise RuntimeError("device error word set while timing the protection kernels")
 
@@ -469,6 +478,11 @@ def run_ours(args):
                                    "ms_isolated": gelu_iso, "shape": [Mg, Kg],
                                    "kernel": "w8a8_gelu_quant_act"},
             },
+            "gguf": {name: {"bound": "tensor", "achieved": ops_step / (ms * 1e-3) / 1e12, "peak": peak_t,
+                            "unit": "TFLOP/s", "frac": ops_step / (ms * 1e-3) / 1e12 / peak_t,
+                            "ms_isolated": ms, "weight_bytes": nbytes,
+                            "kernel": f"w8a8_linear_gguf ({name})"}
+                     for name, (ms, nbytes) in gguf_iso.items()},
             "gemm_ms": gemm_avg, "gemm_ms_isolated": gemm_iso, "offline_ms": offline,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "TOPS", "h2d_bytes_per_step": 2 * M * K,

@@ -164,6 +164,47 @@ W8A8_API w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int
                                 int N, int K, int32_t *acc, void *stream);
 
 /* ------------------------------------------------------------------------
+ * GGUF weight-only layers (Sec. 3, "GGUF k-quants": the DiT serialized to
+ * Q8_0, 8.5 bits per weight, and Q4_K, 4.5 bits, the paper's memory-Pareto
+ * variant, which it ran with a Torch dequantization).
+ * ---------------------------------------------------------------------- */
+
+#define W8A8_GGUF_Q8_0 0
+#define W8A8_GGUF_Q4_K 1
+
+/*
+ * Weight blocks in the public GGUF/ggml layouts, little-endian, each weight
+ * row [K] a run of consecutive blocks (row stride = K/32*34 bytes for Q8_0,
+ * K/256*144 for Q4_K):
+ *   Q8_0: 32 weights in 34 bytes, fp16 d then 32 int8 q;  w = d * q.
+ *   Q4_K: 256 weights in 144 bytes, fp16 d, fp16 dmin, 12 bytes of eight
+ *     6-bit scales sc_j and mins m_j (j < 4: sc = s[j] & 63, m = s[j+4] & 63;
+ *     j >= 4: sc = (s[j+4] & 15) | (s[j-4] >> 6) << 4,
+ *             m  = (s[j+4] >> 4) | (s[j] >> 6) << 4),
+ *     then 128 bytes of 4-bit quants: weights 64c..64c+31 are the low
+ *     nibbles of quant bytes 32c..32c+31 (j = 2c), weights 64c+32..64c+63
+ *     their high nibbles (j = 2c+1);  w = (d * sc_j) * q - dmin * m_j.
+ * Decoding runs in fp32 (only the Q4_K subtraction rounds: the products of
+ * these small integers and fp16 values are exact); the layer consumes the
+ * decoded weights rounded to bf16 (nearest even).
+ *
+ * Weight-only linear:
+ *     Y_mn = bf16_rne(fl32(sum_k X_mk * bf16(w_nk)) + bias_n)
+ * with fp32 tensor-core accumulation, as w8a8_linear_bf16.
+ *   X [M,K] bf16, Wraw [N rows of blocks], bias [N] fp32 or NULL, read.
+ *   Y [M,N] bf16, written.  fmt W8A8_GGUF_Q8_0 or W8A8_GGUF_Q4_K, else
+ *   W8A8_ERR_INVALID_ARG; N a multiple of 8 and K of 256, else
+ *   W8A8_ERR_UNSUPPORTED_SHAPE.
+ */
+W8A8_API w8a8_status w8a8_linear_gguf(const uint16_t *X, const uint8_t *Wraw, int fmt,
+                                      const float *bias, int M, int N, int K, uint16_t *Y,
+                                      void *stream);
+
+/* Test export: the decoded weights W [N,K] bf16, written. */
+W8A8_API w8a8_status w8a8_debug_gguf_dequant(const uint8_t *Wraw, int fmt, int N, int K,
+                                             uint16_t *W, void *stream);
+
+/* ------------------------------------------------------------------------
  * a3 fused with its neighbours in the DiT block.
  * ---------------------------------------------------------------------- */
 

@@ -247,6 +247,34 @@ w8a8_status w8a8_linear_bf16(const uint16_t *X, const uint16_t *W, const float *
     return from_cuda(w8a8::launch_gemm_bf16(X, W, bias, M, N, K, Y, err, as_stream(stream)));
 }
 
+static w8a8_status check_gguf(const void *Wraw, int fmt, int N, int K) {
+    if (fmt != W8A8_GGUF_Q8_0 && fmt != W8A8_GGUF_Q4_K) return W8A8_ERR_INVALID_ARG;
+    if (N <= 0 || (N % 8) != 0 || K <= 0 || (K % 256) != 0) return W8A8_ERR_UNSUPPORTED_SHAPE;
+    if (!Wraw) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(Wraw)) return W8A8_ERR_MISALIGNED;
+    return W8A8_OK;
+}
+
+w8a8_status w8a8_linear_gguf(const uint16_t *X, const uint8_t *Wraw, int fmt, const float *bias,
+                             int M, int N, int K, uint16_t *Y, void *stream) {
+    if (w8a8_status e = check_gguf(Wraw, fmt, N, K)) return e;
+    if (M < 0) return W8A8_ERR_UNSUPPORTED_SHAPE;
+    if (M == 0) return W8A8_OK;
+    if (!X || !Y) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(Y) || (bias && !aligned16(bias))) return W8A8_ERR_MISALIGNED;
+    unsigned int *err = device_error_word();
+    if (!err) return W8A8_ERR_CUDA;
+    return from_cuda(w8a8::launch_gemm_gguf(X, Wraw, fmt, bias, M, N, K, Y, err, as_stream(stream)));
+}
+
+w8a8_status w8a8_debug_gguf_dequant(const uint8_t *Wraw, int fmt, int N, int K, uint16_t *W,
+                                    void *stream) {
+    if (w8a8_status e = check_gguf(Wraw, fmt, N, K)) return e;
+    if (!W) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(W)) return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_gguf_dequant(Wraw, fmt, N, K, W, as_stream(stream)));
+}
+
 w8a8_status w8a8_layer_forward(const w8a8_layer *layer, const uint16_t *X, int M, int8_t *Xq_work,
                                float *x_scale_work, uint16_t *Y, void *stream) {
     if (!layer) return W8A8_ERR_INVALID_ARG;

@@ -65,6 +65,13 @@ cudaError_t launch_gemm_tc(const GemmBranch *br, int nb, int N, int K,
 cudaError_t launch_gemm_bf16(const uint16_t *X, const uint16_t *W, const float *bias, int M,
                              int N, int K, uint16_t *Y, unsigned int *err, cudaStream_t st);
 
+// GGUF weight-only linear (fmt 0 = Q8_0, 1 = Q4_K) on tcgen05 CTA pairs.
+cudaError_t launch_gemm_gguf(const uint16_t *X, const uint8_t *Wraw, int fmt, const float *bias, int M,
+                             int N, int K, uint16_t *Y, unsigned int *err, cudaStream_t st);
+// Test export: the decoded bf16 weights.
+cudaError_t launch_gguf_dequant(const uint8_t *Wraw, int fmt, int N, int K, uint16_t *W,
+                                cudaStream_t st);
+
 // Activation statistics: accumulate sums / absmax, then finalize.
 cudaError_t launch_act_stats_update(const uint16_t *X, int T, int K, const float *shift,
                                     double *sums, float *absmax, cudaStream_t st);

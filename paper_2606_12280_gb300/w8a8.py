@@ -46,7 +46,11 @@ SIGNATURES = {
     "w8a8_quant_act_dual": [_P, _I, _P],
     "w8a8_gelu_quant_act": [_P, _P, _I, _I, _P, _P, _P],
     "w8a8_debug_gelu": [_P, _I, _P, _P],
+    "w8a8_linear_gguf": [_P, _P, _I, _P, _I, _I, _I, _P, _P],
+    "w8a8_debug_gguf_dequant": [_P, _I, _I, _I, _P, _P],
 }
+
+GGUF_Q8_0, GGUF_Q4_K = 0, 1
 
 
 class W8A8Error(RuntimeError):
@@ -273,6 +277,28 @@ def gelu_quant_act(H, smooth=None, Xq=None, x_scale=None, stream=None):
         _ptr(H, torch.bfloat16, "H"), _ptr(smooth, torch.float32, "smooth"), M, K,
         _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"), _stream(stream)))
     return Xq, x_scale
+
+
+def linear_gguf(X, Wraw, fmt: int, N: int, bias=None, Y=None, stream=None):
+    """GGUF weight-only layer: Y = bf16(X dequant(W)^T + b); Wraw uint8 blocks
+    (Q8_0: fmt 0, Q4_K: fmt 1) of N rows."""
+    M, K = X.shape
+    if Y is None:
+        Y = torch.empty(M, N, dtype=torch.bfloat16, device=X.device)
+    _check("w8a8_linear_gguf", lib().w8a8_linear_gguf(
+        _ptr(X, torch.bfloat16, "X"), _ptr(Wraw, torch.uint8, "Wraw"), int(fmt),
+        _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(Y, torch.bfloat16, "Y"), _stream(stream)))
+    return Y
+
+
+def debug_gguf_dequant(Wraw, fmt: int, N: int, K: int, W=None, stream=None):
+    """The decoded weights [N, K] bf16."""
+    if W is None:
+        W = torch.empty(N, K, dtype=torch.bfloat16, device=Wraw.device)
+    _check("w8a8_debug_gguf_dequant", lib().w8a8_debug_gguf_dequant(
+        _ptr(Wraw, torch.uint8, "Wraw"), int(fmt), N, K, _ptr(W, torch.bfloat16, "W"),
+        _stream(stream)))
+    return W
 
 
 def debug_gelu(H, G=None, stream=None):

@@ -229,3 +229,17 @@ def test_fused_quant_validation(L):
     assert g(None, None, 4, 16, A, A, None) == INVALID
     assert g(A, U, 4, 16, A, A, None) == MISALIGNED
     assert g(None, None, 0, 16, None, None, None) == OK  # empty batch
+
+
+def test_gguf_validation(L):
+    f = L.w8a8_linear_gguf
+    assert f(A, A, 2, None, 4, 8, 256, A, None) == INVALID          # format
+    assert f(A, A, 1, None, 4, 8, 128, A, None) == SHAPE            # K % 256
+    assert f(A, A, 0, None, 4, 12, 256, A, None) == SHAPE           # N % 8
+    assert f(A, None, 1, None, 4, 8, 256, A, None) == INVALID
+    assert f(A, U, 1, None, 4, 8, 256, A, None) == MISALIGNED
+    assert f(A, A, 1, U, 4, 8, 256, A, None) == MISALIGNED          # bias
+    assert f(None, A, 1, None, 0, 8, 256, None, None) == OK        # empty batch
+    g = L.w8a8_debug_gguf_dequant
+    assert g(A, 1, 8, 256, None, None) == INVALID
+    assert g(A, 0, 8, 256, U, None) == MISALIGNED
