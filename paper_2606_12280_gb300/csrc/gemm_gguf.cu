@@ -11,11 +11,11 @@
 // CTA: warp 0 issues TMA loads of X tiles [128 x 64] straight into the
 // 128-byte-swizzled K-major layout and of raw weight blocks [128 rows x one
 // 256-weight span] into a raw ring; warp 1 allocates TMEM (both CTAs) and,
-// on the leader, issues one M=256 N=256 K=16 bf16 MMA per K step; warps 2-9
-// decode the raw blocks of each K=64 step into the swizzled bf16 B tile
-// (fp32 arithmetic as the decoder defines it, then round to bf16); warps
-// 10-13 drain the fp32 accumulator (two TMEM buffers), add the bias and write
-// bf16.  All waits are bounded in time.
+// on the leader, issues one M=256 N=256 K=16 bf16 MMA per K step; the
+// converter warps decode the raw blocks of each K=64 step into the swizzled
+// bf16 B tile (fp32 arithmetic as the decoder defines it, then round to
+// bf16); the last four warps drain the fp32 accumulator (two TMEM buffers),
+// add the bias and write bf16.  All waits are bounded in time.
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_fp16.h>
@@ -36,7 +36,13 @@ constexpr int SUBS = KR / BK;                  // MMA stages per raw span
 constexpr int S = 4;                           // bf16 stage ring
 constexpr int TILE_BYTES = CTA_M * BK * 2;     // 16 KB, A or B
 constexpr int STAGE = 2 * TILE_BYTES;          // A then B
-constexpr int NUM_CONV_WARPS = 8;
+#ifndef W8A8_GGUF_CONV_WARPS
+#define W8A8_GGUF_CONV_WARPS 16
+#endif
+constexpr int NUM_CONV_WARPS = W8A8_GGUF_CONV_WARPS;
+constexpr int CONV_TASKS = CTA_N * 4;          // per K=64 step: 128 rows x 4 chunk pairs
+constexpr int kTasksPerThread = CONV_TASKS / (32 * NUM_CONV_WARPS);
+static_assert(CONV_TASKS % (32 * NUM_CONV_WARPS) == 0, "whole tasks per converter thread");
 constexpr int NUM_EPI_WARPS = 4;
 constexpr int CONV_WARP0 = 2, EPI_WARP0 = CONV_WARP0 + NUM_CONV_WARPS;
 constexpr int THREADS = 32 * (EPI_WARP0 + NUM_EPI_WARPS);
@@ -92,20 +98,6 @@ struct Params {
     uint64_t wait_limit_ns;
 };
 
-__device__ __forceinline__ uint32_t bf16_rne_bits(float f) {
-    uint32_t u = __float_as_uint(f);
-    if ((u & 0x7fffffffu) > 0x7f800000u) return (u >> 16) | 0x40u;
-    u += 0x7fffu + ((u >> 16) & 1u);
-    return u >> 16;
-}
-
-// two fp32 -> one bf16x2 word (low = a), each rounded to nearest even
-__device__ __forceinline__ uint32_t pack_bf16(float a, float b) {
-    uint32_t r;
-    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(b), "f"(a));
-    return r;
-}
-
 __device__ __forceinline__ uint32_t ld_shared_u32(uint32_t a) {
     uint32_t v;
     asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
@@ -128,11 +120,6 @@ __device__ __forceinline__ float f16_bits_to_f32(uint32_t h) {
     return __half2float(__ushort_as_half(static_cast<unsigned short>(h)));
 }
 
-// Exact small integer -> fp32: 2^23 + v has v in its low mantissa bits.
-__device__ __forceinline__ float small_uint_to_f32(uint32_t v) {
-    return __uint_as_float(0x4B000000u | v) - 8388608.0f;
-}
-
 // The 6-bit scale and min of Q4_K sub-block j from the 12 scale bytes
 // (three little-endian words w0 = bytes 0-3, w1 = 4-7, w2 = 8-11).
 __device__ __forceinline__ void q4k_scale_min(uint32_t w0, uint32_t w1, uint32_t w2, int j,
@@ -148,70 +135,126 @@ __device__ __forceinline__ void q4k_scale_min(uint32_t w0, uint32_t w1, uint32_t
     }
 }
 
-// Decode 8 weights d1 * q - m1 (q the 4-bit values of 8 consecutive nibbles
-// selected by `shift` from the 8 quant bytes in v) into 4 bf16x2 words.
-__device__ __forceinline__ uint4 q4k_chunk(uint2 v, int shift, float d1, float m1) {
+// Packed fp32 pairs (each packed operation rounds like its scalar form).
+__device__ __forceinline__ uint64_t pk2(uint32_t a, uint32_t b) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "r"(a), "r"(b));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t pkf(float a) {
+    uint64_t r;
+    asm("mov.b64 %0, {%1, %1};" : "=l"(r) : "f"(a));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t add2(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t mul2(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+    uint64_t r;
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(r) : "l"(a), "l"(b), "l"(c));
+    return r;
+}
+
+// the pair as one bf16x2 word (low = first), each rounded to nearest even
+__device__ __forceinline__ uint32_t pack_bf16_pair(uint64_t v) {
+    uint32_t a, b, r;
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(a), "=r"(b) : "l"(v));
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "r"(b), "r"(a));
+    return r;
+}
+
+// fp32 bit patterns 2^23 + byte_i(x) for bytes i0 and i1 of x, as a pair:
+// one byte permute each (the byte lands in the low mantissa bits of 2^23).
+template <int I0, int I1>
+__device__ __forceinline__ uint64_t magic_pair(uint32_t x) {
+    return pk2(__byte_perm(x, 0x4B000000u, 0x7440 | I0), __byte_perm(x, 0x4B000000u, 0x7440 | I1));
+}
+
+// Decode 8 Q4_K weights d1 * q - m1 (q = the low (SHIFT 0) or high (SHIFT 4)
+// nibbles of the 8 quant bytes in v) into 4 bf16x2 words.  d1 * q is exact
+// (17 + 4 bits), so the fused multiply-add rounds once, as the decoder does.
+template <int SHIFT>
+__device__ __forceinline__ uint4 q4k_chunk(uint2 v, float d1, float m1) {
+    const uint32_t n0 = (v.x >> SHIFT) & 0x0f0f0f0fu, n1 = (v.y >> SHIFT) & 0x0f0f0f0fu;
+    const uint64_t bias = pkf(-8388608.0f), D = pkf(d1), Mn = pkf(-m1);
     uint32_t w[4];
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-        const uint32_t b = ((h ? v.y : v.x) >> shift) & 0x0f0f0f0fu;
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            const float q0 = small_uint_to_f32((b >> (16 * e)) & 15u);
-            const float q1 = small_uint_to_f32((b >> (16 * e + 8)) & 15u);
-            // d1 * q is exact (17 + 4 bits): one rounding, as in the decoder
-            w[2 * h + e] = pack_bf16(fmaf(d1, q0, -m1), fmaf(d1, q1, -m1));
-        }
-    }
+    w[0] = pack_bf16_pair(fma2(D, add2(magic_pair<0, 1>(n0), bias), Mn));
+    w[1] = pack_bf16_pair(fma2(D, add2(magic_pair<2, 3>(n0), bias), Mn));
+    w[2] = pack_bf16_pair(fma2(D, add2(magic_pair<0, 1>(n1), bias), Mn));
+    w[3] = pack_bf16_pair(fma2(D, add2(magic_pair<2, 3>(n1), bias), Mn));
     return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
-// Decode 8 int8 quants (bytes of lo, hi) times d into 4 bf16x2 words.
+// Decode 8 Q8_0 quants (bytes of lo, hi) times d into 4 bf16x2 words:
+// 2^23 + (q + 128) minus 2^23 + 128 is q exactly, d * q is exact.
 __device__ __forceinline__ uint4 q8_chunk(uint32_t lo, uint32_t hi, float d) {
+    const uint32_t a = lo ^ 0x80808080u, b = hi ^ 0x80808080u;
+    const uint64_t bias = pkf(-8388736.0f), D = pkf(d);
     uint32_t w[4];
-#pragma unroll
-    for (int h = 0; h < 2; ++h) {
-        const uint32_t b = (h ? hi : lo) ^ 0x80808080u;      // q + 128, as unsigned bytes
-#pragma unroll
-        for (int e = 0; e < 2; ++e) {
-            // 2^23 + (q + 128) minus 2^23 + 128: exact
-            const float q0 = __uint_as_float(0x4B000000u | ((b >> (16 * e)) & 0xffu)) - 8388736.0f;
-            const float q1 = __uint_as_float(0x4B000000u | ((b >> (16 * e + 8)) & 0xffu)) - 8388736.0f;
-            w[2 * h + e] = pack_bf16(__fmul_rn(d, q0), __fmul_rn(d, q1));   // exact products
-        }
-    }
+    w[0] = pack_bf16_pair(mul2(D, add2(magic_pair<0, 1>(a), bias)));
+    w[1] = pack_bf16_pair(mul2(D, add2(magic_pair<2, 3>(a), bias)));
+    w[2] = pack_bf16_pair(mul2(D, add2(magic_pair<0, 1>(b), bias)));
+    w[3] = pack_bf16_pair(mul2(D, add2(magic_pair<2, 3>(b), bias)));
     return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
-// One converter thread, one task: row `row` of the CTA's 128 weight rows,
-// output chunks c and c + 4 (16 bf16) of K=64 step u of the raw span.
+// Per-row constants of one 256-weight span, computed once per span and kept
+// in registers: Q4_K d * sc_j and dmin * m_j for the eight sub-blocks; Q8_0
+// the eight block scales d (in d1).
+struct Q4kRow {
+    float d1[8], m1[8];
+};
+
+__device__ __forceinline__ void q8_row_consts(uint32_t src, Q4kRow &r) {
+#pragma unroll
+    for (int b = 0; b < 8; ++b) r.d1[b] = f16_bits_to_f32(ld_shared_u16(src + 34 * b));
+}
+
+__device__ __forceinline__ void q4k_row_consts(uint32_t src, Q4kRow &r) {
+    const uint32_t dd = ld_shared_u32(src);
+    const float d = f16_bits_to_f32(dd & 0xffffu), dmin = f16_bits_to_f32(dd >> 16);
+    const uint32_t w0 = ld_shared_u32(src + 4), w1 = ld_shared_u32(src + 8), w2 = ld_shared_u32(src + 12);
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+        uint32_t sc, m;
+        q4k_scale_min(w0, w1, w2, j, sc, m);
+        r.d1[j] = __fmul_rn(d, static_cast<float>(sc));     // exact: 11 x 6 bits
+        r.m1[j] = __fmul_rn(dmin, static_cast<float>(m));
+    }
+}
+
+// One converter task: row `row` of the CTA's 128 weight rows, output chunks c
+// and c + 4 (16 bf16) of K=64 step u of the raw span.  Q4_K: chunk c holds
+// the low nibbles (sub-block 2u), chunk c + 4 the high nibbles (2u + 1) of
+// the same 8 quant bytes.  Q8_0: chunks c and c + 4 come from blocks 2u and
+// 2u + 1, whose 8 quant bytes start 2 bytes into their 34-byte block.
 template <int FMT>
-__device__ __forceinline__ void convert_task(uint32_t raw, uint32_t dst, int row, int c, int u) {
+__device__ __forceinline__ void convert_task(uint32_t raw, uint32_t dst, int row, int c, int u,
+                                             float d1a, float m1a, float d1b, float m1b) {
     const uint32_t src = raw + static_cast<uint32_t>(row) * Fmt<FMT>::ROW;
     uint4 lo, hi;
     if (FMT == 1) {
-        const uint32_t dd = ld_shared_u32(src);
-        const float d = f16_bits_to_f32(dd & 0xffffu), dmin = f16_bits_to_f32(dd >> 16);
-        const uint32_t w0 = ld_shared_u32(src + 4), w1 = ld_shared_u32(src + 8),
-                       w2 = ld_shared_u32(src + 12);
-        uint32_t s0, m0, s1, m1;
-        q4k_scale_min(w0, w1, w2, 2 * u, s0, m0);
-        q4k_scale_min(w0, w1, w2, 2 * u + 1, s1, m1);
         const uint2 v = ld_shared_v2(src + 16 + 32 * u + 8 * c);
-        lo = q4k_chunk(v, 0, __fmul_rn(d, static_cast<float>(s0)), __fmul_rn(dmin, static_cast<float>(m0)));
-        hi = q4k_chunk(v, 4, __fmul_rn(d, static_cast<float>(s1)), __fmul_rn(dmin, static_cast<float>(m1)));
+        lo = q4k_chunk<0>(v, d1a, m1a);
+        hi = q4k_chunk<4>(v, d1b, m1b);
     } else {
-        // blocks 2u (chunk c) and 2u + 1 (chunk c + 4) of the span; the 8 quant
-        // bytes of a chunk start 2 bytes into their 34-byte block
-        const uint32_t b0 = src + 34 * (2 * u), b1 = b0 + 34;
-        const float d0 = f16_bits_to_f32(ld_shared_u16(b0)), d1 = f16_bits_to_f32(ld_shared_u16(b1));
-        const uint32_t q0 = b0 + 2 + 8 * c, q1 = b1 + 2 + 8 * c;
-        const uint32_t a0 = ld_shared_u16(q0) | (ld_shared_u16(q0 + 2) << 16);
-        const uint32_t a1 = ld_shared_u16(q0 + 4) | (ld_shared_u16(q0 + 6) << 16);
-        const uint32_t c0 = ld_shared_u16(q1) | (ld_shared_u16(q1 + 2) << 16);
-        const uint32_t c1 = ld_shared_u16(q1 + 4) | (ld_shared_u16(q1 + 6) << 16);
-        lo = q8_chunk(a0, a1, d0);
-        hi = q8_chunk(c0, c1, d1);
+        // block 2u's quants start 2 mod 4 bytes into the row: three aligned
+        // words and two byte permutes; block 2u + 1's are 4-byte aligned
+        const uint32_t q0 = src + 34 * (2 * u) + 2 + 8 * c, q1 = q0 + 34;
+        const uint32_t x0 = ld_shared_u32(q0 - 2), x1 = ld_shared_u32(q0 + 2), x2 = ld_shared_u32(q0 + 6);
+        lo = q8_chunk(__byte_perm(x0, x1, 0x5432), __byte_perm(x1, x2, 0x5432), d1a);
+        hi = q8_chunk(ld_shared_u32(q1), ld_shared_u32(q1 + 4), d1b);
     }
     // 128-byte swizzle: 16-byte chunk k of row r at (k ^ (r & 7))
     const uint32_t rb = dst + static_cast<uint32_t>(row) * 128;
@@ -256,11 +299,9 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
                         }
                         uint32_t w[4];
 #pragma unroll
-                        for (int i = 0; i < 4; ++i) {
-                            const float y0 = __fadd_rn(__uint_as_float(v[8 * h + 2 * i]), b[2 * i]);
-                            const float y1 = __fadd_rn(__uint_as_float(v[8 * h + 2 * i + 1]), b[2 * i + 1]);
-                            w[i] = bf16_rne_bits(y0) | (bf16_rne_bits(y1) << 16);
-                        }
+                        for (int i = 0; i < 4; ++i)
+                            w[i] = pack_bf16_pair(add2(pk2(v[8 * h + 2 * i], v[8 * h + 2 * i + 1]),
+                                                       pk2(__float_as_uint(b[2 * i]), __float_as_uint(b[2 * i + 1]))));
                         *reinterpret_cast<uint4 *>(out + cc * 16 + 8 * h) = make_uint4(w[0], w[1], w[2], w[3]);
                     }
                 }
@@ -408,7 +449,7 @@ gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
     } else if (warp < EPI_WARP0) {
         // ------------------------------------------------------ converters
         const int cw = warp - CONV_WARP0;
-        const int tid = cw * 32 + lane;                 // 0 .. 255: 2 tasks each
+        const int tid = cw * 32 + lane;
         const uint32_t full0 = leader ? 0u : mapa_shared(sb + L::BAR_FULL, 0);
         uint32_t j = 0;
         bool ok = true;
@@ -420,7 +461,20 @@ gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                                                     ERR_CONVERTER)))
                 break;
             const uint32_t raw = sb + L::OFF_RAW + rs * L::RAW_SLOT;
-            for (int u = 0; u < SUBS; ++u, ++j) {
+            // this thread's tasks: a warp's 32 tasks are 8 consecutive rows
+            // (lane & 7) x the 4 chunk pairs (lane >> 3), so that every
+            // quarter-warp stores to 8 different 16-byte bank groups of the
+            // swizzled tile
+            Q4kRow rc[kTasksPerThread];
+#pragma unroll
+            for (int i = 0; i < kTasksPerThread; ++i) {
+                const int task = tid + 32 * NUM_CONV_WARPS * i;
+                const uint32_t rsrc = raw + static_cast<uint32_t>(8 * (task >> 5) + (task & 7)) * Fmt<FMT>::ROW;
+                if (FMT == 1) q4k_row_consts(rsrc, rc[i]);
+                else q8_row_consts(rsrc, rc[i]);
+            }
+#pragma unroll
+            for (int u = 0; u < SUBS; ++u) {
                 const uint32_t st = j % S;
                 if (!__all_sync(0xffffffffu, mbar_wait_cluster(sb + L::BAR_EMPTY + 8 * st,
                                                                ((j / S) & 1) ^ 1, wc, ERR_CONVERTER))) {
@@ -429,9 +483,10 @@ gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                 }
                 const uint32_t dst = sb + L::OFF_ST + st * STAGE + TILE_BYTES;
 #pragma unroll
-                for (int i = 0; i < 2; ++i) {
-                    const int task = tid + 256 * i;            // 512 tasks: 128 rows x 4
-                    convert_task<FMT>(raw, dst, task >> 2, task & 3, u);
+                for (int i = 0; i < kTasksPerThread; ++i) {
+                    const int task = tid + 32 * NUM_CONV_WARPS * i;
+                    convert_task<FMT>(raw, dst, 8 * (task >> 5) + (task & 7), (task >> 3) & 3, u,
+                                      rc[i].d1[2 * u], rc[i].m1[2 * u], rc[i].d1[2 * u + 1], rc[i].m1[2 * u + 1]);
                 }
                 fence_proxy_async_smem();
                 __syncwarp();
@@ -448,6 +503,7 @@ gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                     if (leader) mbar_arrive(sb + L::BAR_FULL + 8 * st);
                     else mbar_arrive_cluster_relaxed(full0 + 8 * st);
                 }
+                ++j;
             }
             if (!ok) break;
             if (lane == 0) mbar_arrive(sb + L::BAR_REMPTY + 8 * rs);
@@ -484,8 +540,9 @@ __global__ void gguf_dequant_kernel(const uint8_t *__restrict__ raw, int N, int 
             uint32_t sc, m;
             q4k_scale_min(w[1], w[2], w[3], 2 * u + (cc >= 4 ? 1 : 0), sc, m);
             const uint2 v = *reinterpret_cast<const uint2 *>(src + 16 + 32 * u + 8 * (cc & 3));
-            out = q4k_chunk(v, cc >= 4 ? 4 : 0, __fmul_rn(f16_bits_to_f32(dd & 0xffffu), static_cast<float>(sc)),
-                            __fmul_rn(f16_bits_to_f32(dd >> 16), static_cast<float>(m)));
+            const float d1 = __fmul_rn(f16_bits_to_f32(dd & 0xffffu), static_cast<float>(sc));
+            const float m1 = __fmul_rn(f16_bits_to_f32(dd >> 16), static_cast<float>(m));
+            out = cc >= 4 ? q4k_chunk<4>(v, d1, m1) : q4k_chunk<0>(v, d1, m1);
         } else {
             const uint8_t *blk = src + 34 * (2 * u + (cc >= 4 ? 1 : 0));
             const uint16_t *h = reinterpret_cast<const uint16_t *>(blk);
