@@ -32,12 +32,22 @@ using namespace tc;
 constexpr int PAIR_M = 256, CTA_M = 128, PAIR_N = 256, CTA_N = 128;
 constexpr int BK = 64;                         // bf16 per swizzle row = one MMA stage
 constexpr int KR = 256;                        // weights per raw span (one Q4_K block)
-constexpr int SUBS = KR / BK;                  // MMA stages per raw span
-constexpr int S = 4;                           // bf16 stage ring
-constexpr int TILE_BYTES = CTA_M * BK * 2;     // 16 KB, A or B
-constexpr int STAGE = 2 * TILE_BYTES;          // A then B
+#ifndef W8A8_GGUF_SUB
+#define W8A8_GGUF_SUB 2
+#endif
+#ifndef W8A8_GGUF_STAGES
+#define W8A8_GGUF_STAGES 2
+#endif
+constexpr int SUB = W8A8_GGUF_SUB;             // K=64 steps per pipeline stage
+constexpr int SUBS = KR / BK;                  // K=64 steps per raw span
+constexpr int STAGES_PER_SPAN = SUBS / SUB;
+constexpr int S = W8A8_GGUF_STAGES;            // bf16 stage ring
+constexpr int TILE_BYTES = CTA_M * BK * 2;     // 16 KB, A or B of one K=64 step
+constexpr int STEP_BYTES = 2 * TILE_BYTES;     // A then B
+constexpr int STAGE = SUB * STEP_BYTES;
+static_assert(SUBS % SUB == 0, "whole stages per raw span");
 #ifndef W8A8_GGUF_CONV_WARPS
-#define W8A8_GGUF_CONV_WARPS 16
+#define W8A8_GGUF_CONV_WARPS 8
 #endif
 constexpr int NUM_CONV_WARPS = W8A8_GGUF_CONV_WARPS;
 constexpr int CONV_TASKS = CTA_N * 4;          // per K=64 step: 128 rows x 4 chunk pairs
@@ -392,16 +402,18 @@ gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
             for (int qs = 0; ok && qs < total_spans; ++qs) {
                 const int t = pair + (qs / p.spans) * npairs;
                 const int arow = (t % p.m_tiles) * PAIR_M + static_cast<int>(rank) * CTA_M;
-                for (int u = 0; ok && u < SUBS; ++u, ++j) {
+                for (int g = 0; ok && g < STAGES_PER_SPAN; ++g, ++j) {
                     const uint32_t st = j % S;
                     if (!mbar_wait_cluster(sb + L::BAR_EMPTY + 8 * st, ((j / S) & 1) ^ 1, wc, ERR_PRODUCER)) {
                         ok = false;
                         break;
                     }
-                    mbar_arrive_expect_tx(sb + L::BAR_AFULL + 8 * st, TILE_BYTES);
-                    tma_load_2d(sb + L::OFF_ST + st * STAGE, &tmA, ((qs % p.spans) * SUBS + u) * BK, arow,
-                                sb + L::BAR_AFULL + 8 * st);
-                    if (u == 0 && qs + 1 < total_spans) ok = issue_raw(qs + 1);
+                    mbar_arrive_expect_tx(sb + L::BAR_AFULL + 8 * st, SUB * TILE_BYTES);
+#pragma unroll
+                    for (int v = 0; v < SUB; ++v)
+                        tma_load_2d(sb + L::OFF_ST + st * STAGE + v * STEP_BYTES, &tmA,
+                                    ((qs % p.spans) * SUBS + g * SUB + v) * BK, arow, sb + L::BAR_AFULL + 8 * st);
+                    if (g == 0 && qs + 1 < total_spans) ok = issue_raw(qs + 1);
                 }
             }
             // drain: every issued TMA has landed before the CTA may exit
@@ -425,7 +437,7 @@ gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                 }
                 tc_fence_after();
                 const uint32_t d = tmem + buf * PAIR_N;
-                const int nk = p.spans * SUBS;
+                const int nk = p.spans * STAGES_PER_SPAN;
                 for (int ks = 0; ks < nk; ++ks, ++j) {
                     const uint32_t st = j % S;
                     if (!mbar_wait_cluster(sb + L::BAR_FULL + 8 * st, (j / S) & 1, wc, ERR_MMA)) {
@@ -433,12 +445,15 @@ gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t a = sb + L::OFF_ST + st * STAGE;
-                    const uint32_t b = a + TILE_BYTES;
 #pragma unroll
-                    for (int kk = 0; kk < BK / 16; ++kk)
-                        mma_f16_ss_pair(d, smem_desc_sw128(a + kk * 32), smem_desc_sw128(b + kk * 32), idesc,
-                                        (ks > 0 || kk > 0) ? 1u : 0u);
+                    for (int v = 0; v < SUB; ++v) {
+                        const uint32_t a = sb + L::OFF_ST + st * STAGE + v * STEP_BYTES;
+                        const uint32_t b = a + TILE_BYTES;
+#pragma unroll
+                        for (int kk = 0; kk < BK / 16; ++kk)
+                            mma_f16_ss_pair(d, smem_desc_sw128(a + kk * 32), smem_desc_sw128(b + kk * 32), idesc,
+                                            (ks > 0 || v > 0 || kk > 0) ? 1u : 0u);
+                    }
                     mma_commit_pair_multicast(sb + L::BAR_EMPTY + 8 * st, 0x3);
                 }
                 if (ok) mma_commit_pair_multicast(sb + L::BAR_ACCFULL + 8 * buf, 0x3);
@@ -474,19 +489,24 @@ gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                 else q8_row_consts(rsrc, rc[i]);
             }
 #pragma unroll
-            for (int u = 0; u < SUBS; ++u) {
+            for (int g = 0; g < STAGES_PER_SPAN; ++g) {
                 const uint32_t st = j % S;
                 if (!__all_sync(0xffffffffu, mbar_wait_cluster(sb + L::BAR_EMPTY + 8 * st,
                                                                ((j / S) & 1) ^ 1, wc, ERR_CONVERTER))) {
                     ok = false;
                     break;
                 }
-                const uint32_t dst = sb + L::OFF_ST + st * STAGE + TILE_BYTES;
 #pragma unroll
-                for (int i = 0; i < kTasksPerThread; ++i) {
-                    const int task = tid + 32 * NUM_CONV_WARPS * i;
-                    convert_task<FMT>(raw, dst, 8 * (task >> 5) + (task & 7), (task >> 3) & 3, u,
-                                      rc[i].d1[2 * u], rc[i].m1[2 * u], rc[i].d1[2 * u + 1], rc[i].m1[2 * u + 1]);
+                for (int v = 0; v < SUB; ++v) {
+                    const int u = g * SUB + v;                 // K=64 step within the span
+                    const uint32_t dst = sb + L::OFF_ST + st * STAGE + v * STEP_BYTES + TILE_BYTES;
+#pragma unroll
+                    for (int i = 0; i < kTasksPerThread; ++i) {
+                        const int task = tid + 32 * NUM_CONV_WARPS * i;
+                        convert_task<FMT>(raw, dst, 8 * (task >> 5) + (task & 7), (task >> 3) & 3, u,
+                                          rc[i].d1[2 * u], rc[i].m1[2 * u], rc[i].d1[2 * u + 1],
+                                          rc[i].m1[2 * u + 1]);
+                    }
                 }
                 fence_proxy_async_smem();
                 __syncwarp();
