@@ -164,6 +164,37 @@ W8A8_API w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int
                                 int N, int K, int32_t *acc, void *stream);
 
 /* ------------------------------------------------------------------------
+ * The same layer with the activation codes in a 16-bit container.
+ * ---------------------------------------------------------------------- */
+
+/*
+ * a3 with the codes written as fp16 values: Xq16_mj is the fp16 bit pattern
+ * of the same integer code w8a8_quant_act writes as int8 (every integer in
+ * [-127, 127] is exactly an fp16 value), x_scale as w8a8_quant_act.  gelu
+ * nonzero: quantize GELU(X) as w8a8_gelu_quant_act does.  The GEMM below then
+ * takes A without converting it.  K <= 16384, else
+ * W8A8_ERR_UNSUPPORTED_SHAPE.  Writes 2MK + 4M bytes (one MK more than a3).
+ *   X [M,K] bf16, smooth [K] fp32 or NULL, read.
+ *   Xq16 [M,K] fp16 codes (uint16 bit patterns), x_scale [M] fp32, written.
+ */
+W8A8_API w8a8_status w8a8_quant_act_f16codes(const uint16_t *X, const float *smooth, int M,
+                                             int K, uint16_t *Xq16, float *x_scale, int gelu,
+                                             void *stream);
+
+/*
+ * a4 + a5 with the activation codes as fp16 values (from
+ * w8a8_quant_act_f16codes): the same exact INT32 product and epilogue as
+ * w8a8_linear, bitwise equal outputs; the codes go to the tensor cores
+ * without a conversion, which halves the shared-memory traffic of the
+ * operand staging.  Xq16 [M,K] fp16 codes, otherwise as w8a8_linear.
+ * Uses the CTA-pair engine whatever w8a8_set_gemm_engine says.
+ */
+W8A8_API w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale,
+                                          const int8_t *Wq, const float *w_scale,
+                                          const float *bias, int M, int N, int K, uint16_t *Y,
+                                          void *stream);
+
+/* ------------------------------------------------------------------------
  * GGUF weight-only layers (Sec. 3, "GGUF k-quants": the DiT serialized to
  * Q8_0, 8.5 bits per weight, and Q4_K, 4.5 bits, the paper's memory-Pareto
  * variant, which it ran with a Torch dequantization).

@@ -68,7 +68,7 @@ w8a8_status run_gemm(const w8a8::GemmBranch *br, int nb, int N, int K, bool out_
     if (g_engine == 1 || g_engine == 2) {
         unsigned int *err = device_error_word();
         if (!err) return W8A8_ERR_CUDA;
-        if (g_engine == 2) return from_cuda(w8a8::launch_gemm_tc2(br, nb, N, K, out_i32, err, st));
+        if (g_engine == 2) return from_cuda(w8a8::launch_gemm_tc2(br, nb, N, K, out_i32, false, err, st));
         return from_cuda(w8a8::launch_gemm_tc(br, nb, N, K, out_i32, err, st));
     }
     return from_cuda(w8a8::launch_gemm_mma(br, nb, N, K, out_i32, st));
@@ -196,6 +196,31 @@ w8a8_status w8a8_debug_gelu(const uint16_t *H, int n, float *G, void *stream) {
     if (!H || !G) return W8A8_ERR_INVALID_ARG;
     if (!aligned16(H) || !aligned16(G)) return W8A8_ERR_MISALIGNED;
     return from_cuda(w8a8::launch_debug_gelu(H, n, G, as_stream(stream)));
+}
+
+w8a8_status w8a8_quant_act_f16codes(const uint16_t *X, const float *smooth, int M, int K,
+                                    uint16_t *Xq16, float *x_scale, int gelu, void *stream) {
+    if (w8a8_status e = check_mk(M, K)) return e;
+    if (K > 16384) return W8A8_ERR_UNSUPPORTED_SHAPE;
+    if (M == 0) return W8A8_OK;
+    if (!X || !Xq16 || !x_scale) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(Xq16) || !aligned16(x_scale) || (smooth && !aligned16(smooth)))
+        return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_quant_act_f16codes(X, smooth, M, K, Xq16, x_scale, gelu != 0,
+                                                     as_stream(stream)));
+}
+
+w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale, const int8_t *Wq,
+                                 const float *w_scale, const float *bias, int M, int N, int K,
+                                 uint16_t *Y, void *stream) {
+    if (w8a8_status e = check_nk(N, K)) return e;
+    if (w8a8_status e = check_mk(M, K)) return e;
+    w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), x_scale, Wq, w_scale, bias, Y, M};
+    if (w8a8_status e = check_branch(b, true, N, K)) return e;
+    if (M == 0) return W8A8_OK;
+    unsigned int *err = device_error_word();
+    if (!err) return W8A8_ERR_CUDA;
+    return from_cuda(w8a8::launch_gemm_tc2(&b, 1, N, K, false, true, err, as_stream(stream)));
 }
 
 w8a8_status w8a8_quant_act_per_tensor(const uint16_t *X, const float *smooth, int M, int K,

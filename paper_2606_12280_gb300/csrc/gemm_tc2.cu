@@ -15,10 +15,13 @@
 // every SM stages and feeds half of B, which is what the shared-memory
 // bandwidth of the int8 -> fp16 staging needs.
 //
-// Per CTA: warp 0 TMA producer (int8 tiles, 6-stage ring), warp 1 TMEM
-// allocation (both CTAs) and MMA issue (leader only), warps 2-7 converters
-// (3-stage fp16 ring), warps 8-15 epilogue (TMEM -> int32 running sums ->
-// bf16 dequantized output).  Cross-CTA signalling: converters and epilogue
+// Per CTA: warp 0 TMA producer (int8 tiles), warp 1 TMEM allocation (both
+// CTAs) and MMA issue (leader only), warps 2-7 converters (int8 -> fp16 into
+// the swizzled fp16 ring), warps 8-15 epilogue (TMEM -> int32 running sums ->
+// bf16 dequantized output).  Pipeline stages carry SUB K=64 sub-blocks.  The
+// A16 variant takes the activation codes already as fp16 values: lane 1 of
+// warp 0 loads them by TMA straight into the fp16 ring and the converters
+// handle the weights only.  Cross-CTA signalling: converters and epilogue
 // warps arrive on the leader's barriers through cluster addresses; the leader
 // commits MMA completion to both CTAs' barriers by multicast.  All waits are
 // bounded in time.
@@ -50,12 +53,9 @@ constexpr int PAIR_M = 256, CTA_M = 128, PAIR_N = 256, CTA_N = 128, BK = 64;
 constexpr int SUB = W8A8_TC2_SUB;
 constexpr int KC_BLOCKS = 16;                        // K chunk = 1024 (exactness bound)
 constexpr int KC_STAGES = KC_BLOCKS / SUB;           // stages per K chunk
-constexpr int S8 = W8A8_TC2_S8, S16 = W8A8_TC2_S16;
-constexpr int SUB8_A = CTA_M * BK, SUB8_B = CTA_N * BK;
-constexpr int SUB8 = SUB8_A + SUB8_B;                // 16 KB int8 per sub-block
+constexpr int SUB8_A = CTA_M * BK, SUB8_B = CTA_N * BK;   // int8 bytes of A, B per sub-block
 constexpr int SUB16_A = CTA_M * BK * 2, SUB16_B = CTA_N * BK * 2;
 constexpr int SUB16 = SUB16_A + SUB16_B;             // 32 KB fp16 per sub-block
-constexpr int STAGE8 = SUB * SUB8;
 constexpr int STAGE16 = SUB * SUB16;
 static_assert(KC_BLOCKS % SUB == 0, "chunk of whole stages");
 constexpr int NUM_CONV_WARPS = 6;
@@ -63,31 +63,54 @@ constexpr int NUM_EPI_WARPS = 8;
 constexpr int THREADS = 512;
 constexpr int TMEM_COLS = 512;
 constexpr int SMEM_BARRIERS = 256;
-constexpr int SMEM_EPI = NUM_EPI_WARPS * 1024;
-constexpr int SMEM_TOTAL = 1024 + S16 * STAGE16 + S8 * STAGE8 + SMEM_BARRIERS + SMEM_EPI;
 constexpr int LAUNCH_REGS = 128;
 constexpr int REGS_LOW = 72, REGS_HIGH = 184;
 static_assert(256 * REGS_LOW + 256 * REGS_HIGH <= THREADS * LAUNCH_REGS, "register split");
 static_assert(KC_BLOCKS * BK * 127 * 127 < (1 << 24), "fp32 exactness bound");
-static_assert(1024 + S16 * STAGE16 + S8 * STAGE8 + 512 + 8192 <= 232448, "shared memory");
 
 constexpr unsigned ERR_PRODUCER = 1u, ERR_CONVERTER = 2u, ERR_MMA = 4u, ERR_EPILOGUE = 8u,
                    ERR_DRAIN = 16u, ERR_TMEM_PAIR = 64u;
 
-constexpr uint32_t OFF_ST16 = 0;
-constexpr uint32_t OFF_ST8 = OFF_ST16 + S16 * STAGE16;
-constexpr uint32_t OFF_BAR = OFF_ST8 + S8 * STAGE8;
-constexpr uint32_t BAR_FULL8 = OFF_BAR;
-constexpr uint32_t BAR_EMPTY8 = BAR_FULL8 + 8 * S8;
-constexpr uint32_t BAR_FULL16 = BAR_EMPTY8 + 8 * S8;
-constexpr uint32_t BAR_EMPTY16 = BAR_FULL16 + 8 * S16;
-constexpr uint32_t BAR_ACCFULL = BAR_EMPTY16 + 8 * S16;
-constexpr uint32_t BAR_ACCEMPTY = BAR_ACCFULL + 16;
-constexpr uint32_t BAR_DRAIN = BAR_ACCEMPTY + 16;
-constexpr uint32_t OFF_TMEM = BAR_DRAIN + 8;
-constexpr uint32_t OFF_ABORT = OFF_TMEM + 4;
-static_assert(OFF_ABORT + 4 - OFF_BAR <= SMEM_BARRIERS, "barrier area");
-constexpr uint32_t OFF_EPI = OFF_BAR + SMEM_BARRIERS;
+#ifndef W8A8_TC2_A16_S8
+#define W8A8_TC2_A16_S8 2
+#endif
+#ifndef W8A8_TC2_STAGE_EPI
+#define W8A8_TC2_STAGE_EPI 1
+#endif
+#ifndef W8A8_TC2_A16_S16
+#define W8A8_TC2_A16_S16 3
+#endif
+// Shared-memory layout of one variant: fp16 stages, then int8 stages, then
+// barriers, then (int8-A variant) the epilogue's staging of w_scale / bias.
+// The A16 variant's int8 stages carry B only, which leaves room for a third
+// fp16 stage; its epilogue reads w_scale and bias through L1 instead.
+template <bool A16> struct Lay {
+    static constexpr int NCONV = NUM_CONV_WARPS;              // converter warps 2 .. 7
+    static constexpr int S8 = A16 ? W8A8_TC2_A16_S8 : W8A8_TC2_S8;
+    static constexpr int S16 = A16 ? W8A8_TC2_A16_S16 : W8A8_TC2_S16;
+    static constexpr int SUB8 = A16 ? SUB8_B : SUB8_A + SUB8_B;     // int8 bytes per sub-block
+    static constexpr int B8 = A16 ? 0 : SUB8_A;                      // B's offset in it
+    static constexpr int STAGE8 = SUB * SUB8;
+    static constexpr bool STAGE_EPI = !A16 && W8A8_TC2_STAGE_EPI;
+    static constexpr int SMEM_EPI = STAGE_EPI ? NUM_EPI_WARPS * 1024 : 0;
+    static constexpr uint32_t OFF_ST16 = 0;
+    static constexpr uint32_t OFF_ST8 = OFF_ST16 + S16 * STAGE16;
+    static constexpr uint32_t OFF_BAR = OFF_ST8 + S8 * STAGE8;
+    static constexpr uint32_t BAR_FULL8 = OFF_BAR;
+    static constexpr uint32_t BAR_EMPTY8 = BAR_FULL8 + 8 * S8;
+    static constexpr uint32_t BAR_FULL16 = BAR_EMPTY8 + 8 * S8;
+    static constexpr uint32_t BAR_EMPTY16 = BAR_FULL16 + 8 * S16;
+    static constexpr uint32_t BAR_ACCFULL = BAR_EMPTY16 + 8 * S16;
+    static constexpr uint32_t BAR_ACCEMPTY = BAR_ACCFULL + 16;
+    static constexpr uint32_t BAR_DRAIN = BAR_ACCEMPTY + 16;
+    static constexpr uint32_t BAR_AFULL16 = BAR_DRAIN + 8;          // fp16-coded A landed
+    static constexpr uint32_t OFF_TMEM = BAR_AFULL16 + 8 * S16;
+    static constexpr uint32_t OFF_ABORT = OFF_TMEM + 4;
+    static constexpr uint32_t OFF_EPI = OFF_BAR + SMEM_BARRIERS;
+    static constexpr int SMEM_TOTAL = 1024 + OFF_EPI + SMEM_EPI;
+    static_assert(OFF_ABORT + 4 - OFF_BAR <= SMEM_BARRIERS, "barrier area");
+    static_assert(SMEM_TOTAL <= 232448, "shared memory");
+};
 
 struct BranchArgs {
     const float *x_scale;
@@ -144,10 +167,11 @@ __device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t
     asm("sub.f16x2 %0, %0, %1;" : "+r"(hi) : "r"(0x64806480u));
 }
 
-template <bool OUT_I32>
+template <bool OUT_I32, bool A16>
 __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint32_t tmem,
                                               const WaitCtx &wc, int warp, int lane, int NC,
                                               uint32_t rank, int pair, int npairs) {
+    using L = Lay<A16>;
     const int e = warp - 8;
     const int q = warp & 3;            // TMEM lane quarter this warp may access
     const int h = e >> 2;              // column half of the 256-wide tile
@@ -159,7 +183,7 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
         for (int i = 0; i < 128; ++i) run[i] = 0;
         for (int ci = 0; ci < NC; ++ci, ++c) {
             const uint32_t buf = c & 1;
-            if (!mbar_wait_cluster(sb + BAR_ACCFULL + 8 * buf, (c >> 1) & 1, wc, ERR_EPILOGUE)) {
+            if (!mbar_wait_cluster(sb + L::BAR_ACCFULL + 8 * buf, (c >> 1) & 1, wc, ERR_EPILOGUE)) {
                 ok = false;
                 break;
             }
@@ -176,8 +200,8 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
             tc_fence_before();
             __syncwarp();
             if (lane == 0) {
-                if (rank == 0) mbar_arrive(sb + BAR_ACCEMPTY + 8 * buf);
-                else mbar_arrive_cluster_relaxed(mapa_shared(sb + BAR_ACCEMPTY + 8 * buf, 0));
+                if (rank == 0) mbar_arrive(sb + L::BAR_ACCEMPTY + 8 * buf);
+                else mbar_arrive_cluster_relaxed(mapa_shared(sb + L::BAR_ACCEMPTY + 8 * buf, 0));
             }
         }
         if (!ok) break;
@@ -185,8 +209,8 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
         const BranchArgs &br = p.br[tl.branch];
         const int m = tl.m0 + static_cast<int>(rank) * CTA_M + q * 32 + lane;
         const int n_base = tl.n0 + h * 128;
-        const uint32_t epi = sb + OFF_EPI + e * 1024;
-        if (!OUT_I32) {
+        const uint32_t epi = sb + L::OFF_EPI + e * 1024;
+        if (!OUT_I32 && L::STAGE_EPI) {
             const int n = n_base + lane * 4;
             float4 w = make_float4(0.f, 0.f, 0.f, 0.f), b = w;
             if (n < p.N) {
@@ -218,12 +242,24 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
 #pragma unroll
                 for (int g = 0; g < 16; ++g) {
                     if (n_base + g * 8 < p.N) {
-                        const float4 w0 = ld_shared_f4(epi + g * 32);
-                        const float4 w1 = ld_shared_f4(epi + g * 32 + 16);
-                        float4 b0 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = b0;
-                        if (hb) {
-                            b0 = ld_shared_f4(epi + 512 + g * 32);
-                            b1 = ld_shared_f4(epi + 512 + g * 32 + 16);
+                        float4 w0, w1, b0 = make_float4(0.f, 0.f, 0.f, 0.f), b1 = b0;
+                        if (L::STAGE_EPI) {
+                            w0 = ld_shared_f4(epi + g * 32);
+                            w1 = ld_shared_f4(epi + g * 32 + 16);
+                            if (hb) {
+                                b0 = ld_shared_f4(epi + 512 + g * 32);
+                                b1 = ld_shared_f4(epi + 512 + g * 32 + 16);
+                            }
+                        } else {
+                            // every lane reads the same 8 columns: L1 broadcast
+                            const float4 *wp = reinterpret_cast<const float4 *>(br.w_scale + n_base + g * 8);
+                            w0 = __ldg(wp);
+                            w1 = __ldg(wp + 1);
+                            if (hb) {
+                                const float4 *bp = reinterpret_cast<const float4 *>(br.bias + n_base + g * 8);
+                                b0 = __ldg(bp);
+                                b1 = __ldg(bp + 1);
+                            }
                         }
                         const uint32_t y0 = epilogue_value(run[g * 8 + 0], sx, w0.x, b0.x, hb);
                         const uint32_t y1 = epilogue_value(run[g * 8 + 1], sx, w0.y, b0.y, hb);
@@ -243,11 +279,15 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
     }
 }
 
-template <bool OUT_I32>
+// A16: the activation codes arrive as fp16 values (exact: |q| <= 127), so
+// TMA puts A straight into the swizzled fp16 tile and only the weights are
+// converted; the int8 ring then carries B alone (in its B half).
+template <bool OUT_I32, bool A16>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
 gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant__ CUtensorMap tmB0,
                 const __grid_constant__ CUtensorMap tmA1, const __grid_constant__ CUtensorMap tmB1,
                 const Params p) {
+    using L = Lay<A16>;
     extern __shared__ uint8_t smem_raw[];
     const uint32_t sb = (smem_addr(smem_raw) + 1023u) & ~1023u;
     const int warp = threadIdx.x >> 5;
@@ -258,20 +298,21 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
     const int npairs = gridDim.x >> 1;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < S8; ++i) {
-            mbar_init(sb + BAR_FULL8 + 8 * i, 1);
-            mbar_init(sb + BAR_EMPTY8 + 8 * i, NUM_CONV_WARPS);
+        for (int i = 0; i < L::S8; ++i) {
+            mbar_init(sb + L::BAR_FULL8 + 8 * i, 1);
+            mbar_init(sb + L::BAR_EMPTY8 + 8 * i, L::NCONV);
         }
-        for (int i = 0; i < S16; ++i) {
-            mbar_init(sb + BAR_FULL16 + 8 * i, 2 * NUM_CONV_WARPS);
-            mbar_init(sb + BAR_EMPTY16 + 8 * i, 1);
+        for (int i = 0; i < L::S16; ++i) {
+            mbar_init(sb + L::BAR_FULL16 + 8 * i, 2 * L::NCONV);
+            mbar_init(sb + L::BAR_EMPTY16 + 8 * i, 1);
         }
         for (int i = 0; i < 2; ++i) {
-            mbar_init(sb + BAR_ACCFULL + 8 * i, 1);
-            mbar_init(sb + BAR_ACCEMPTY + 8 * i, 2 * NUM_EPI_WARPS);
+            mbar_init(sb + L::BAR_ACCFULL + 8 * i, 1);
+            mbar_init(sb + L::BAR_ACCEMPTY + 8 * i, 2 * NUM_EPI_WARPS);
         }
-        mbar_init(sb + BAR_DRAIN, 1);
-        st_shared_s32(sb + OFF_ABORT, 0);
+        for (int i = 0; i < L::S16; ++i) mbar_init(sb + L::BAR_AFULL16 + 8 * i, 1);
+        mbar_init(sb + L::BAR_DRAIN, 1);
+        st_shared_s32(sb + L::OFF_ABORT, 0);
         fence_barrier_init();
     }
     if (warp == 0 && lane == 0) {
@@ -281,24 +322,24 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
         tma_prefetch_desc(&tmB1);
     }
     if (warp == 1) {
-        tmem_alloc_pair(sb + OFF_TMEM, TMEM_COLS);
+        tmem_alloc_pair(sb + L::OFF_TMEM, TMEM_COLS);
         tmem_relinquish_pair();
     }
     tc_fence_before();
     cluster_sync();
     tc_fence_after();
-    const uint32_t tmem = static_cast<uint32_t>(ld_shared_s32(sb + OFF_TMEM));
-    const uint32_t peer_tmem = ld_shared_cluster_u32(mapa_shared(sb + OFF_TMEM, rank ^ 1u));
+    const uint32_t tmem = static_cast<uint32_t>(ld_shared_s32(sb + L::OFF_TMEM));
+    const uint32_t peer_tmem = ld_shared_cluster_u32(mapa_shared(sb + L::OFF_TMEM, rank ^ 1u));
     const bool run_ok = (tmem == peer_tmem);
     if (!run_ok && threadIdx.x == 0) atomicOr(p.err, ERR_TMEM_PAIR);
-    const WaitCtx wc{sb + OFF_ABORT, p.err, p.wait_limit_ns};
+    const WaitCtx wc{sb + L::OFF_ABORT, p.err, p.wait_limit_ns};
     const int KB = p.k_blocks;
     const int NS = (KB + SUB - 1) / SUB;                  // pipeline stages per tile
     const int NC = (KB + KC_BLOCKS - 1) / KC_BLOCKS;
 
     if (warp >= 8) {
         asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(REGS_HIGH));
-        if (run_ok) epilogue_role<OUT_I32>(p, sb, tmem, wc, warp, lane, NC, rank, pair, npairs);
+        if (run_ok) epilogue_role<OUT_I32, A16>(p, sb, tmem, wc, warp, lane, NC, rank, pair, npairs);
         tc_fence_before();
         __syncwarp();
         asm volatile("bar.sync 1, %0;" ::"n"(THREADS) : "memory");
@@ -308,6 +349,9 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
         if (!run_ok) {
         } else if (warp == 0) {
             // -------------------------------------------------- TMA producer
+            // lane 0: the int8 ring (A and B, or B alone for A16); lane 1
+            // (A16): A straight into the fp16 ring, as soon as the MMA frees a
+            // slot, so that A's copy latency never waits behind B's ring
             if (lane == 0) {
                 uint32_t j = 0;
                 bool ok = true;
@@ -318,23 +362,47 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                     const int arow = tl.m0 + static_cast<int>(rank) * CTA_M;
                     const int brow = tl.n0 + static_cast<int>(rank) * CTA_N;
                     for (int ks = 0; ks < NS; ++ks, ++j) {
-                        const uint32_t st = j % S8;
-                        if (!mbar_wait(sb + BAR_EMPTY8 + 8 * st, ((j / S8) & 1) ^ 1, wc, ERR_PRODUCER)) {
+                        const uint32_t st = j % L::S8;
+                        if (!mbar_wait(sb + L::BAR_EMPTY8 + 8 * st, ((j / L::S8) & 1) ^ 1, wc, ERR_PRODUCER)) {
                             ok = false;
                             break;
                         }
-                        const uint32_t fb = sb + BAR_FULL8 + 8 * st;
-                        mbar_arrive_expect_tx(fb, STAGE8);
+                        const uint32_t fb = sb + L::BAR_FULL8 + 8 * st;
+                        mbar_arrive_expect_tx(fb, L::STAGE8);
 #pragma unroll
                         for (int u = 0; u < SUB; ++u) {
-                            const uint32_t dst = sb + OFF_ST8 + st * STAGE8 + u * SUB8;
-                            tma_load_2d(dst, mA, (ks * SUB + u) * BK, arow, fb);
-                            tma_load_2d(dst + SUB8_A, mB, (ks * SUB + u) * BK, brow, fb);
+                            const uint32_t dst = sb + L::OFF_ST8 + st * L::STAGE8 + u * L::SUB8;
+                            if (!A16) tma_load_2d(dst, mA, (ks * SUB + u) * BK, arow, fb);
+                            tma_load_2d(dst + L::B8, mB, (ks * SUB + u) * BK, brow, fb);
                         }
                     }
                 }
-                for (uint32_t i = (j > S8 ? j - S8 : 0); i < j; ++i)
-                    mbar_wait(sb + BAR_FULL8 + 8 * (i % S8), (i / S8) & 1, wc, ERR_DRAIN, false);
+                for (uint32_t i = (j > L::S8 ? j - L::S8 : 0); i < j; ++i)
+                    mbar_wait(sb + L::BAR_FULL8 + 8 * (i % L::S8), (i / L::S8) & 1, wc, ERR_DRAIN, false);
+            } else if (A16 && lane == 1) {
+                uint32_t j = 0;
+                bool ok = true;
+                for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+                    const Tile tl = tile_coords(p, t);
+                    const CUtensorMap *mA = tl.branch ? &tmA1 : &tmA0;
+                    const int arow = tl.m0 + static_cast<int>(rank) * CTA_M;
+                    for (int ks = 0; ks < NS; ++ks, ++j) {
+                        const uint32_t s16 = j % L::S16;
+                        if (!mbar_wait_cluster(sb + L::BAR_EMPTY16 + 8 * s16, ((j / L::S16) & 1) ^ 1, wc,
+                                               ERR_PRODUCER)) {
+                            ok = false;
+                            break;
+                        }
+                        const uint32_t ab = sb + L::BAR_AFULL16 + 8 * s16;
+                        mbar_arrive_expect_tx(ab, SUB * SUB16_A);
+#pragma unroll
+                        for (int u = 0; u < SUB; ++u)
+                            tma_load_2d(sb + L::OFF_ST16 + s16 * STAGE16 + u * SUB16, mA, (ks * SUB + u) * BK,
+                                        arow, ab);
+                    }
+                }
+                for (uint32_t i = (j > L::S16 ? j - L::S16 : 0); i < j; ++i)
+                    mbar_wait(sb + L::BAR_AFULL16 + 8 * (i % L::S16), (i / L::S16) & 1, wc, ERR_DRAIN, false);
             }
         } else if (warp == 1) {
             // ------------------------------------------- MMA issue (leader)
@@ -345,7 +413,7 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                 for (int t = pair; ok && t < p.total_tiles; t += npairs) {
                     for (int ci = 0; ok && ci < NC; ++ci, ++c) {
                         const uint32_t buf = c & 1;
-                        if (!mbar_wait_cluster(sb + BAR_ACCEMPTY + 8 * buf, ((c >> 1) & 1) ^ 1, wc,
+                        if (!mbar_wait_cluster(sb + L::BAR_ACCEMPTY + 8 * buf, ((c >> 1) & 1) ^ 1, wc,
                                                ERR_MMA)) {
                             ok = false;
                             break;
@@ -355,15 +423,15 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                         const int ks0 = ci * KC_STAGES;
                         const int ks1 = min(NS, ks0 + KC_STAGES);
                         for (int ks = ks0; ks < ks1; ++ks, ++j) {
-                            const uint32_t st = j % S16;
-                            if (!mbar_wait_cluster(sb + BAR_FULL16 + 8 * st, (j / S16) & 1, wc, ERR_MMA)) {
+                            const uint32_t st = j % L::S16;
+                            if (!mbar_wait_cluster(sb + L::BAR_FULL16 + 8 * st, (j / L::S16) & 1, wc, ERR_MMA)) {
                                 ok = false;
                                 break;
                             }
                             tc_fence_after();
 #pragma unroll
                             for (int u = 0; u < SUB; ++u) {
-                                const uint32_t a = sb + OFF_ST16 + st * STAGE16 + u * SUB16;
+                                const uint32_t a = sb + L::OFF_ST16 + st * STAGE16 + u * SUB16;
                                 const uint32_t b = a + SUB16_A;
 #pragma unroll
                                 for (int kk = 0; kk < BK / 16; ++kk) {
@@ -372,13 +440,13 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                                                     (ks > ks0 || u > 0 || kk > 0) ? 1u : 0u);
                                 }
                             }
-                            mma_commit_pair_multicast(sb + BAR_EMPTY16 + 8 * st, 0x3);
+                            mma_commit_pair_multicast(sb + L::BAR_EMPTY16 + 8 * st, 0x3);
                         }
-                        if (ok) mma_commit_pair_multicast(sb + BAR_ACCFULL + 8 * buf, 0x3);
+                        if (ok) mma_commit_pair_multicast(sb + L::BAR_ACCFULL + 8 * buf, 0x3);
                     }
                 }
-                mma_commit_pair(sb + BAR_DRAIN);
-                mbar_wait_cluster(sb + BAR_DRAIN, 0, wc, ERR_DRAIN, false);
+                mma_commit_pair(sb + L::BAR_DRAIN);
+                mbar_wait_cluster(sb + L::BAR_DRAIN, 0, wc, ERR_DRAIN, false);
             }
         } else {
             // ---------------------------------------------------- converters
@@ -392,50 +460,73 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
             bool ok = true;
             for (int t = pair; ok && t < p.total_tiles; t += npairs) {
                 for (int ks = 0; ks < NS; ++ks, ++j) {
-                    const uint32_t s8 = j % S8, s16 = j % S16;
-                    if (!mbar_wait(sb + BAR_FULL8 + 8 * s8, (j / S8) & 1, wc, ERR_CONVERTER) ||
-                        !mbar_wait_cluster(sb + BAR_EMPTY16 + 8 * s16, ((j / S16) & 1) ^ 1, wc,
-                                           ERR_CONVERTER)) {
+                    const uint32_t s8 = j % L::S8, s16 = j % L::S16;
+                    // every lane waits; __all_sync keeps the warp's control flow
+                    // uniform if a wait gives up
+                    if (!__all_sync(0xffffffffu, mbar_wait(sb + L::BAR_FULL8 + 8 * s8, (j / L::S8) & 1, wc,
+                                                            ERR_CONVERTER) &&
+                                                     mbar_wait_cluster(sb + L::BAR_EMPTY16 + 8 * s16,
+                                                                       ((j / L::S16) & 1) ^ 1, wc,
+                                                                       ERR_CONVERTER))) {
                         ok = false;
                         break;
                     }
-                    const uint32_t src = sb + OFF_ST8 + s8 * STAGE8 + src_off;
-                    const uint32_t dst = sb + OFF_ST16 + s16 * STAGE16;
-                    // per sub-block, all of this warp's 8-row groups in flight at
+                    const uint32_t src = sb + L::OFF_ST8 + s8 * L::STAGE8 + src_off;
+                    const uint32_t dst = sb + L::OFF_ST16 + s16 * STAGE16;
+                    // all of this warp's 8-row groups of a sub-block in flight at
                     // once: every load is issued before the first conversion needs
                     // its data (group g of sub-block u sits at u * kG1 + g in both
                     // rings: a sub-block is CTA_M + CTA_N rows of 64 int8 bytes,
-                    // 128 fp16 bytes)
+                    // 128 fp16 bytes; the A16 variant converts only the B groups,
+                    // kG0 .. kG1 - 1, and keeps both sub-blocks' loads in flight)
                     constexpr int kG1 = (CTA_M + CTA_N) / 8;
-                    constexpr int kPer = (kG1 + NUM_CONV_WARPS - 1) / NUM_CONV_WARPS;
+                    constexpr int kG0 = A16 ? CTA_M / 8 : 0;
+                    constexpr int kPer = (kG1 - kG0 + L::NCONV - 1) / L::NCONV;
+                    constexpr int kAtOnce = A16 ? SUB : 1;
 #pragma unroll
-                    for (int u = 0; u < SUB; ++u) {
-                        uint4 v[kPer];
+                    for (int u0 = 0; u0 < SUB; u0 += kAtOnce) {
+                        uint4 v[kAtOnce][kPer];
 #pragma unroll
-                        for (int i = 0; i < kPer; ++i) {
-                            const int g = cw + i * NUM_CONV_WARPS;
-                            if (g < kG1) v[i] = ld_shared_v4(src + (u * kG1 + g) * 8 * BK);
-                        }
+                        for (int uu = 0; uu < kAtOnce; ++uu)
 #pragma unroll
-                        for (int i = 0; i < kPer; ++i) {
-                            const int g = cw + i * NUM_CONV_WARPS;
-                            if (g < kG1) {
-                                uint4 o0, o1;
-                                i8x4_to_f16x4(v[i].x, o0.x, o0.y);
-                                i8x4_to_f16x4(v[i].y, o0.z, o0.w);
-                                i8x4_to_f16x4(v[i].z, o1.x, o1.y);
-                                i8x4_to_f16x4(v[i].w, o1.z, o1.w);
-                                st_shared_v4(dst + (u * kG1 + g) * 1024 + dst_off0, o0);
-                                st_shared_v4(dst + (u * kG1 + g) * 1024 + dst_off1, o1);
+                            for (int i = 0; i < kPer; ++i) {
+                                const int g = kG0 + cw + i * L::NCONV;
+                                if (g < kG1) v[uu][i] = ld_shared_v4(src + (u0 + uu) * L::SUB8 + (g - kG0) * 8 * BK);
                             }
-                        }
+#pragma unroll
+                        for (int uu = 0; uu < kAtOnce; ++uu)
+#pragma unroll
+                            for (int i = 0; i < kPer; ++i) {
+                                const int g = kG0 + cw + i * L::NCONV;
+                                const int u = u0 + uu;
+                                if (g < kG1) {
+                                    uint4 o0, o1;
+                                    i8x4_to_f16x4(v[uu][i].x, o0.x, o0.y);
+                                    i8x4_to_f16x4(v[uu][i].y, o0.z, o0.w);
+                                    i8x4_to_f16x4(v[uu][i].z, o1.x, o1.y);
+                                    i8x4_to_f16x4(v[uu][i].w, o1.z, o1.w);
+                                    st_shared_v4(dst + (u * kG1 + g) * 1024 + dst_off0, o0);
+                                    st_shared_v4(dst + (u * kG1 + g) * 1024 + dst_off1, o1);
+                                }
+                            }
                     }
                     fence_proxy_async_smem();
                     __syncwarp();
+                    if (A16) {
+                        // this CTA's A tile must have landed too before the
+                        // leader may issue: converter warp 0 checks it
+                        bool a_ok = true;
+                        if (cw == 0 && lane == 0)
+                            a_ok = mbar_wait(sb + L::BAR_AFULL16 + 8 * s16, (j / L::S16) & 1, wc, ERR_CONVERTER);
+                        if (!__shfl_sync(0xffffffffu, a_ok ? 1 : 0, 0)) {
+                            ok = false;
+                            break;
+                        }
+                    }
                     if (lane == 0) {
-                        if (leader) mbar_arrive(sb + BAR_FULL16 + 8 * s16);
-                        else mbar_arrive_cluster_relaxed(mapa_shared(sb + BAR_FULL16 + 8 * s16, 0));
-                        mbar_arrive(sb + BAR_EMPTY8 + 8 * s8);
+                        if (leader) mbar_arrive(sb + L::BAR_FULL16 + 8 * s16);
+                        else mbar_arrive_cluster_relaxed(mapa_shared(sb + L::BAR_FULL16 + 8 * s16, 0));
+                        mbar_arrive(sb + L::BAR_EMPTY8 + 8 * s8);
                     }
                 }
             }
@@ -484,26 +575,42 @@ bool make_map(CUtensorMap *m, const int8_t *base, int rows, int K, int box_rows)
                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// fp16 row-major [rows, K] -> 2-D map with box [box_rows, 64 elements] landing
+// in the 128-byte swizzled layout, zero fill.
+bool make_map_f16(CUtensorMap *m, const void *base, int rows, int K, int box_rows) {
+    EncodeTiledFn enc = get_encode();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {static_cast<cuuint64_t>(K), static_cast<cuuint64_t>(rows)};
+    cuuint64_t strides[1] = {static_cast<cuuint64_t>(K) * 2};
+    cuuint32_t box[2] = {static_cast<cuuint32_t>(BK), static_cast<cuuint32_t>(box_rows)};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(m, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, 2, const_cast<void *>(base), dims, strides, box,
+               estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+               CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
 int g_sms = 0;
-int g_kernel_regs[2] = {-1, -1};
+int g_kernel_regs[4] = {-1, -1, -1, -1};
 
 }  // namespace
 
-cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K, bool out_i32,
+cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K, bool out_i32, bool a16,
                             unsigned int *err, cudaStream_t st) {
     if (g_sms == 0) {
         int dev = 0;
         cudaGetDevice(&dev);
         cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
     }
-    const int ki = out_i32 ? 1 : 0;
-    auto kern = out_i32 ? gemm_tc2_kernel<true> : gemm_tc2_kernel<false>;
+    const int ki = (out_i32 ? 1 : 0) + (a16 ? 2 : 0);
+    const int smem_total = a16 ? Lay<true>::SMEM_TOTAL : Lay<false>::SMEM_TOTAL;
+    auto kern = a16 ? (out_i32 ? gemm_tc2_kernel<true, true> : gemm_tc2_kernel<false, true>)
+                    : (out_i32 ? gemm_tc2_kernel<true, false> : gemm_tc2_kernel<false, false>);
     if (g_kernel_regs[ki] < 0) {
         cudaFuncAttributes fa;
         cudaError_t e = cudaFuncGetAttributes(&fa, kern);
         if (e != cudaSuccess) return e;
         g_kernel_regs[ki] = fa.numRegs;
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_TOTAL);
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_total);
         if (e != cudaSuccess) return e;
     }
     if (g_kernel_regs[ki] != LAUNCH_REGS) return cudaErrorInvalidConfiguration;
@@ -523,8 +630,9 @@ cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K, bool out
             a.M = b->M;
             a.m_tiles = (b->M + PAIR_M - 1) / PAIR_M;
             a.tiles = a.m_tiles * ((N + PAIR_N - 1) / PAIR_N);
-            if (!make_map(&maps[2 * i], b->Xq, b->M, K, CTA_M) ||
-                !make_map(&maps[2 * i + 1], b->Wq, N, K, CTA_N))
+            const bool okA = a16 ? make_map_f16(&maps[2 * i], b->Xq, b->M, K, CTA_M)
+                                 : make_map(&maps[2 * i], b->Xq, b->M, K, CTA_M);
+            if (!okA || !make_map(&maps[2 * i + 1], b->Wq, N, K, CTA_N))
                 return cudaErrorInvalidValue;
             if (first < 0) first = i;
         }
@@ -542,7 +650,7 @@ cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K, bool out
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
     const int pairs = p.total_tiles < g_sms / 2 ? p.total_tiles : g_sms / 2;
-    kern<<<2 * pairs, THREADS, SMEM_TOTAL, st>>>(maps[0], maps[1], maps[2], maps[3], p);
+    kern<<<2 * pairs, THREADS, smem_total, st>>>(maps[0], maps[1], maps[2], maps[3], p);
     return cudaGetLastError();
 }
 

@@ -53,9 +53,14 @@ cudaError_t launch_debug_gelu(const uint16_t *H, int n, float *G, cudaStream_t s
 cudaError_t launch_gemm_mma(const GemmBranch *br, int nb, int N, int K,
                             bool out_i32, cudaStream_t st);
 
-// tcgen05 GEMM on pairs of SMs (cta_group::2), same exact scheme.
+// tcgen05 GEMM on pairs of SMs (cta_group::2), same exact scheme.  a16: Xq
+// holds the codes as fp16 values (2 bytes each) and is not converted.
 cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K,
-                            bool out_i32, unsigned int *err, cudaStream_t st);
+                            bool out_i32, bool a16, unsigned int *err, cudaStream_t st);
+
+// a3 (optionally of GELU(X)) writing the codes as fp16 values, K <= 16384.
+cudaError_t launch_quant_act_f16codes(const uint16_t *X, const float *lambda, int M, int K,
+                                     uint16_t *Xq16, float *x_scale, bool gelu, cudaStream_t st);
 
 // tcgen05 GEMM (exact integer products on the fp16 tensor datapath).
 cudaError_t launch_gemm_tc(const GemmBranch *br, int nb, int N, int K,

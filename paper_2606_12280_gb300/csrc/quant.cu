@@ -399,7 +399,17 @@ struct ActParams {
     int teams0;
 };
 
-template <int U, int TW, int S, bool GELU>
+// two fp32 -> one f16x2 word (low = a), each rounded to nearest even (exact
+// for the integer codes |q| <= 127)
+__device__ __forceinline__ uint32_t pack_f16(float a, float b) {
+    uint32_t r;
+    asm("cvt.rn.f16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(b), "f"(a));
+    return r;
+}
+
+// OUT16: the codes are written as fp16 values (uint16 bit patterns, 2 bytes
+// each) instead of int8, for the GEMM that takes A without converting it.
+template <int U, int TW, int S, bool GELU, bool OUT16>
 __global__ void __launch_bounds__(TW > 8 ? 32 * TW : 256)
 act_quant_team_kernel(const __grid_constant__ ActParams p) {
     constexpr int kThreads = TW > 8 ? 32 * TW : 256;
@@ -486,10 +496,30 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
         // a and 127/a finite: |x' * inv| <= 127 (1 + 2^-23), no clamp needed
         const bool fast = (a <= 3.402823466e38f) && (inv <= 3.402823466e38f);
         uint2 *qr = reinterpret_cast<uint2 *>(b.Xq + (size_t)row * K);
+        uint4 *qr16 = reinterpret_cast<uint4 *>(b.Xq + 2 * (size_t)row * K);
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const int c = (u * TW + tw) * 32 + lane;
             if (c >= cpr) continue;
+            if (OUT16) {
+                uint32_t hw[4] = {0u, 0u, 0u, 0u};
+                if (zero_row) {
+                } else if (fast) {
+                    // rne(x' * inv) as an fp32 integer: the magic sum minus the
+                    // magic (both in [2^23, 2^24): exact)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        hw[q] = pack_f16(__fadd_rn(__fadd_rn(__fmul_rn(xs[u][q].x, inv), kRoundMagic), -kRoundMagic),
+                                         __fadd_rn(__fadd_rn(__fmul_rn(xs[u][q].y, inv), kRoundMagic), -kRoundMagic));
+                } else {
+#pragma unroll
+                    for (int q = 0; q < 4; ++q)
+                        hw[q] = pack_f16(static_cast<float>(quantize_rne_clamp(__fmul_rn(xs[u][q].x, inv))),
+                                         static_cast<float>(quantize_rne_clamp(__fmul_rn(xs[u][q].y, inv))));
+                }
+                qr16[c] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
+                continue;
+            }
             uint32_t word[2] = {0u, 0u};
             if (zero_row) {
             } else if (fast) {
@@ -513,14 +543,14 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
     asm volatile("cp.async.wait_group 0;" ::: "memory");
 }
 
-template <int U, int TW, bool GELU>
+template <int U, int TW, bool GELU, bool OUT16>
 cudaError_t launch_act_quant_team(ActParams p, cudaStream_t st) {
     constexpr int S = 4;
     constexpr int kThreads = TW > 8 ? 32 * TW : 256;
     constexpr int kTeams = kThreads / (32 * TW);
     constexpr size_t smem = (size_t)(kThreads / 32) * S * U * 32 * 16;
     static int per_sm = 0;
-    auto kern = act_quant_team_kernel<U, TW, S, GELU>;
+    auto kern = act_quant_team_kernel<U, TW, S, GELU, OUT16>;
     if (per_sm == 0) {
         if (smem > 48 * 1024) {
             cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -547,17 +577,17 @@ cudaError_t launch_act_quant_team(ActParams p, cudaStream_t st) {
     return cudaGetLastError();
 }
 
-template <bool GELU>
+template <bool GELU, bool OUT16 = false>
 cudaError_t launch_act_quant_teams(const ActParams &p, cudaStream_t st) {
     // team of TW warps per row, U chunks of 8 values per lane: K <= 256 U TW
     const int K = p.K;
-    if (K <= 256) return launch_act_quant_team<1, 1, GELU>(p, st);
-    if (K <= 512) return launch_act_quant_team<2, 1, GELU>(p, st);
-    if (K <= 1024) return launch_act_quant_team<2, 2, GELU>(p, st);
-    if (K <= 2048) return launch_act_quant_team<2, 4, GELU>(p, st);
-    if (K <= 4096) return launch_act_quant_team<2, 8, GELU>(p, st);
-    if (K <= 8192) return launch_act_quant_team<2, 16, GELU>(p, st);
-    return launch_act_quant_team<4, 16, GELU>(p, st);
+    if (K <= 256) return launch_act_quant_team<1, 1, GELU, OUT16>(p, st);
+    if (K <= 512) return launch_act_quant_team<2, 1, GELU, OUT16>(p, st);
+    if (K <= 1024) return launch_act_quant_team<2, 2, GELU, OUT16>(p, st);
+    if (K <= 2048) return launch_act_quant_team<2, 4, GELU, OUT16>(p, st);
+    if (K <= 4096) return launch_act_quant_team<2, 8, GELU, OUT16>(p, st);
+    if (K <= 8192) return launch_act_quant_team<2, 16, GELU, OUT16>(p, st);
+    return launch_act_quant_team<4, 16, GELU, OUT16>(p, st);
 }
 
 // ----------------------------------------------------------- column absmax
@@ -653,6 +683,14 @@ cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M, int 
         return launch_act_quant_teams<false>(p, st);
     }
     return launch_row_quant<uint16_t, true>(X, lambda, M, K, Xq, x_scale, st);
+}
+
+cudaError_t launch_quant_act_f16codes(const uint16_t *X, const float *lambda, int M, int K,
+                                     uint16_t *Xq16, float *x_scale, bool gelu, cudaStream_t st) {
+    ActParams p{};
+    p.br[0] = ActBranch{X, lambda, reinterpret_cast<int8_t *>(Xq16), x_scale, M};
+    p.K = K;
+    return gelu ? launch_act_quant_teams<true, true>(p, st) : launch_act_quant_teams<false, true>(p, st);
 }
 
 cudaError_t launch_quant_act_dual(const QuantActBranch *br, int K, cudaStream_t st) {

@@ -48,6 +48,8 @@ SIGNATURES = {
     "w8a8_debug_gelu": [_P, _I, _P, _P],
     "w8a8_linear_gguf": [_P, _P, _I, _P, _I, _I, _I, _P, _P],
     "w8a8_debug_gguf_dequant": [_P, _I, _I, _I, _P, _P],
+    "w8a8_quant_act_f16codes": [_P, _P, _I, _I, _P, _P, _I, _P],
+    "w8a8_linear_f16codes": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P],
 }
 
 GGUF_Q8_0, GGUF_Q4_K = 0, 1
@@ -277,6 +279,33 @@ def gelu_quant_act(H, smooth=None, Xq=None, x_scale=None, stream=None):
         _ptr(H, torch.bfloat16, "H"), _ptr(smooth, torch.float32, "smooth"), M, K,
         _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"), _stream(stream)))
     return Xq, x_scale
+
+
+def quant_act_f16codes(X, smooth=None, Xq16=None, x_scale=None, gelu=False, stream=None):
+    """a3 with the codes as fp16 values: returns (Xq16 [M,K] float16, sx [M])."""
+    M, K = X.shape
+    if Xq16 is None:
+        Xq16 = torch.empty(M, K, dtype=torch.float16, device=X.device)
+    if x_scale is None:
+        x_scale = torch.empty(M, dtype=torch.float32, device=X.device)
+    _check("w8a8_quant_act_f16codes", lib().w8a8_quant_act_f16codes(
+        _ptr(X, torch.bfloat16, "X"), _ptr(smooth, torch.float32, "smooth"), M, K,
+        _ptr(Xq16, torch.float16, "Xq16"), _ptr(x_scale, torch.float32, "x_scale"),
+        1 if gelu else 0, _stream(stream)))
+    return Xq16, x_scale
+
+
+def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, stream=None):
+    """a4 + a5 with fp16-coded activations: Y = bf16((Xq Wq^T) * sx * sw + b)."""
+    M, K = Xq16.shape
+    N = Wq.shape[0]
+    if Y is None:
+        Y = torch.empty(M, N, dtype=torch.bfloat16, device=Xq16.device)
+    _check("w8a8_linear_f16codes", lib().w8a8_linear_f16codes(
+        _ptr(Xq16, torch.float16, "Xq16"), _ptr(x_scale, torch.float32, "x_scale"),
+        _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
+        _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(Y, torch.bfloat16, "Y"), _stream(stream)))
+    return Y
 
 
 def linear_gguf(X, Wraw, fmt: int, N: int, bias=None, Y=None, stream=None):

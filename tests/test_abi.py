@@ -243,3 +243,17 @@ def test_gguf_validation(L):
     g = L.w8a8_debug_gguf_dequant
     assert g(A, 1, 8, 256, None, None) == INVALID
     assert g(A, 0, 8, 256, U, None) == MISALIGNED
+
+
+def test_f16codes_validation(L):
+    f = L.w8a8_quant_act_f16codes
+    assert f(A, None, 4, 16400, A, A, 0, None) == SHAPE         # K beyond 16384
+    assert f(A, None, 4, 24, A, A, 0, None) == SHAPE
+    assert f(None, None, 4, 16, A, A, 0, None) == INVALID
+    assert f(A, None, 4, 16, U, A, 0, None) == MISALIGNED
+    assert f(None, None, 0, 16, None, None, 0, None) == OK
+    g = L.w8a8_linear_f16codes
+    assert g(A, A, A, A, None, 4, 12, 16, A, None) == SHAPE
+    assert g(None, A, A, A, None, 4, 8, 16, A, None) == INVALID
+    assert g(A, A, U, A, None, 4, 8, 16, A, None) == MISALIGNED
+    assert g(A, A, A, A, None, 0, 8, 16, A, None) == OK

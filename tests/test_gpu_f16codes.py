@@ -1,0 +1,111 @@
+"""GPU parity of the layer with activation codes in a 16-bit container.
+
+`w8a8_quant_act_f16codes` writes the same integer codes as `w8a8_quant_act`
+as fp16 values; `w8a8_linear_f16codes` computes the same exact INT32 product
+and epilogue from them.  Bar: codes and scales bit-exact against the oracle,
+outputs bit-exact against the oracle and bitwise equal to the int8-container
+path.
+"""
+
+import numpy as np
+import pytest
+import torch
+
+from paper_2606_12280_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+DEV = "cuda"
+
+
+@pytest.fixture(scope="module")
+def w8():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    from paper_2606_12280_gb300 import w8a8
+    w8a8.lib()
+    return w8a8
+
+
+def bf(a):
+    return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(DEV)
+
+
+def t(a):
+    return torch.from_numpy(np.ascontiguousarray(a)).to(DEV)
+
+
+def u16(x):
+    return x.contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+
+
+def codes(Xq16):
+    q = Xq16.float().cpu().numpy()
+    assert np.all(q == np.rint(q)) and np.all(np.abs(q) <= 127)
+    return q.astype(np.int8)
+
+
+@pytest.mark.parametrize("M,K", [(1, 16), (300, 528), (257, 4096), (64, 16384)])
+def test_quant_act_f16codes_exact(w8, oracle_mod, M, K):
+    X = wl.random_bf16((M, K), seed=M + K, scale=2.0)
+    X[0, :] = 0                                         # an all-zero token
+    lam = wl.random_uniform_f32((K,), seed=K, lo=0.25, hi=4.0)
+    q16, sx = w8.quant_act_f16codes(bf(X), t(lam))
+    wq, wsx = oracle_mod.quant_act(X, lam)
+    np.testing.assert_array_equal(codes(q16), wq)
+    np.testing.assert_array_equal(sx.cpu().numpy(), wsx)
+    q8, sx8 = w8.quant_act(bf(X), t(lam))
+    assert torch.equal(q16.to(torch.int8), q8) and torch.equal(sx, sx8)
+
+
+def test_quant_act_f16codes_gelu_matches_int8_gelu(w8):
+    H = wl.ffn_preactivation(129, 16384, seed=5)
+    lam = wl.random_uniform_f32((16384,), seed=6, lo=0.25, hi=4.0)
+    q16, sx = w8.quant_act_f16codes(bf(H), t(lam), gelu=True)
+    q8, sx8 = w8.gelu_quant_act(bf(H), t(lam))
+    assert torch.equal(q16.to(torch.int8), q8) and torch.equal(sx, sx8)
+
+
+@pytest.mark.parametrize("M,N,K", [(1, 8, 16), (300, 264, 528), (513, 520, 1040), (64, 256, 16384)])
+@pytest.mark.parametrize("with_bias", [True, False])
+def test_linear_f16codes_exact(w8, oracle_mod, M, N, K, with_bias):
+    c = wl.make_case(M, K, N, seed=M + N + K)
+    s = oracle_mod.channel_absmax(c.X_cal)
+    lam = oracle_mod.smooth_scales(s, c.W[0], c.alpha)
+    Wq, sw = oracle_mod.quantize_weights(c.W[0], lam)
+    b = c.bias[0] if with_bias else None
+    q16, sx = w8.quant_act_f16codes(bf(c.X[0]), t(lam))
+    Y = w8.linear_f16codes(q16, sx, t(Wq), t(sw), t(b) if with_bias else None)
+    Xq, wsx = oracle_mod.quant_act(c.X[0], lam)
+    np.testing.assert_array_equal(u16(Y), oracle_mod.linear(Xq, wsx, Wq, sw, b))
+    Y8 = w8.linear(q16.to(torch.int8), sx, t(Wq), t(sw), t(b) if with_bias else None)
+    assert torch.equal(Y, Y8)
+
+
+def test_linear_f16codes_extremes(w8, oracle_mod):
+    # all codes +-127 at the longest K the int32 chunks see in practice
+    M, N, K = 256, 256, 16384
+    rng = np.random.default_rng(7)
+    Xq = np.where(rng.random((M, K)) < 0.5, -127, 127).astype(np.int8)
+    Wq = np.where(rng.random((N, K)) < 0.5, -127, 127).astype(np.int8)
+    Xq[0] = 127
+    Wq[0] = 127
+    sx = np.full(M, 1e-3, np.float32)
+    sw = np.full(N, 1e-3, np.float32)
+    q16 = torch.from_numpy(Xq.astype(np.float16)).to(DEV)
+    Y = w8.linear_f16codes(q16, t(sx), t(Wq), t(sw))
+    np.testing.assert_array_equal(u16(Y), oracle_mod.linear(Xq, sx, Wq, sw, None))
+
+
+@pytest.mark.slow
+def test_linear_f16codes_qkv_sampled_rows(w8, oracle_mod):
+    case = wl.workload_cases("qkv_m4608_k4096_n12288")[0]
+    s = oracle_mod.channel_absmax(case.X_cal)
+    lam = oracle_mod.smooth_scales(s, case.W[0], case.alpha)
+    Wq, sw = oracle_mod.quantize_weights(case.W[0], lam)
+    q16, sx = w8.quant_act_f16codes(bf(case.X[0]), t(lam))
+    Y = u16(w8.linear_f16codes(q16, sx, t(Wq), t(sw), t(case.bias[0])))
+    Xq, wsx = oracle_mod.quant_act(case.X[0], lam)
+    np.testing.assert_array_equal(codes(q16), Xq)
+    for r in [0, 1, 255, 256, 2047, 4095, 4350, 4607]:
+        np.testing.assert_array_equal(Y[r:r + 1], oracle_mod.linear(Xq, wsx, Wq, sw, case.bias[0],
+                                                                     rows=(r, r + 1)))
