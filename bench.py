@@ -205,7 +205,7 @@ METRIC = "W8A8 linear INT8 TOPS (act-quant + INT8 GEMM + fused dequant epilogue)
 # from the ncu capture summarised in profiles/gemm_tc2_qkv_m4608_k4096_n12288.md;
 # valid only for the kernel version profiled there (removed whenever that
 # kernel changes, until the capture is repeated).
-GEMM_TRAFFIC_BYTES = {(2, "qkv_m4608_k4096_n12288"): 147.85e6}
+GEMM_TRAFFIC_BYTES = {(2, "qkv_m4608_k4096_n12288"): 147.97e6}
 
 
 # --------------------------------------------------------------------- ours
