@@ -56,7 +56,6 @@ constexpr int KC_STAGES = KC_BLOCKS / SUB;           // stages per K chunk
 constexpr int SUB8_A = CTA_M * BK, SUB8_B = CTA_N * BK;   // int8 bytes of A, B per sub-block
 constexpr int SUB16_A = CTA_M * BK * 2, SUB16_B = CTA_N * BK * 2;
 constexpr int SUB16 = SUB16_A + SUB16_B;             // 32 KB fp16 per sub-block
-constexpr int STAGE16 = SUB * SUB16;
 static_assert(KC_BLOCKS % SUB == 0, "chunk of whole stages");
 constexpr int NUM_CONV_WARPS = 6;
 constexpr int NUM_EPI_WARPS = 8;
@@ -80,10 +79,15 @@ constexpr unsigned ERR_PRODUCER = 1u, ERR_CONVERTER = 2u, ERR_MMA = 4u, ERR_EPIL
 #ifndef W8A8_TC2_A16_S16
 #define W8A8_TC2_A16_S16 3
 #endif
+#ifndef W8A8_TC2_A16_SA
+#define W8A8_TC2_A16_SA 3
+#endif
 // Shared-memory layout of one variant: fp16 stages, then int8 stages, then
-// barriers, then (int8-A variant) the epilogue's staging of w_scale / bias.
-// The A16 variant's int8 stages carry B only, which leaves room for a third
-// fp16 stage; its epilogue reads w_scale and bias through L1 instead.
+// (A16) the A ring, then barriers, then (int8-A variant) the epilogue's
+// staging of w_scale / bias.  In the A16 variant the fp16 and int8 stages
+// carry B only and A has its own, deeper ring (TMA straight from the fp16
+// codes), so that the A copy latency has SA - 1 stages of slack; its epilogue
+// reads w_scale and bias through L1.
 template <bool A16> struct Lay {
     static constexpr int NCONV = NUM_CONV_WARPS;              // converter warps 2 .. 7
     static constexpr int S8 = A16 ? W8A8_TC2_A16_S8 : W8A8_TC2_S8;
@@ -91,11 +95,17 @@ template <bool A16> struct Lay {
     static constexpr int SUB8 = A16 ? SUB8_B : SUB8_A + SUB8_B;     // int8 bytes per sub-block
     static constexpr int B8 = A16 ? 0 : SUB8_A;                      // B's offset in it
     static constexpr int STAGE8 = SUB * SUB8;
+    static constexpr int SUB16S = A16 ? SUB16_B : SUB16;            // fp16 bytes per sub-block
+    static constexpr int STAGE16S = SUB * SUB16S;
+    static constexpr int SA = A16 ? W8A8_TC2_A16_SA : 0;            // A ring stages
+    static constexpr int SAm = SA > 0 ? SA : 1;                      // modulus (int8-A: unused)
+    static constexpr int STAGEA = SUB * SUB16_A;
     static constexpr bool STAGE_EPI = !A16 && W8A8_TC2_STAGE_EPI;
     static constexpr int SMEM_EPI = STAGE_EPI ? NUM_EPI_WARPS * 1024 : 0;
     static constexpr uint32_t OFF_ST16 = 0;
-    static constexpr uint32_t OFF_ST8 = OFF_ST16 + S16 * STAGE16;
-    static constexpr uint32_t OFF_BAR = OFF_ST8 + S8 * STAGE8;
+    static constexpr uint32_t OFF_ST8 = OFF_ST16 + S16 * STAGE16S;
+    static constexpr uint32_t OFF_A = OFF_ST8 + S8 * STAGE8;
+    static constexpr uint32_t OFF_BAR = OFF_A + SA * STAGEA;
     static constexpr uint32_t BAR_FULL8 = OFF_BAR;
     static constexpr uint32_t BAR_EMPTY8 = BAR_FULL8 + 8 * S8;
     static constexpr uint32_t BAR_FULL16 = BAR_EMPTY8 + 8 * S8;
@@ -103,8 +113,17 @@ template <bool A16> struct Lay {
     static constexpr uint32_t BAR_ACCFULL = BAR_EMPTY16 + 8 * S16;
     static constexpr uint32_t BAR_ACCEMPTY = BAR_ACCFULL + 16;
     static constexpr uint32_t BAR_DRAIN = BAR_ACCEMPTY + 16;
-    static constexpr uint32_t BAR_AFULL16 = BAR_DRAIN + 8;          // fp16-coded A landed
-    static constexpr uint32_t OFF_TMEM = BAR_AFULL16 + 8 * S16;
+    static constexpr uint32_t BAR_AFULL = BAR_DRAIN + 8;            // A16: A slot landed
+    static constexpr uint32_t BAR_AEMPTY = BAR_AFULL + 8 * SA;      // A16: MMA done with A slot
+    static constexpr uint32_t OFF_TMEM = BAR_AEMPTY + 8 * SA;
+    // operand addresses of sub-block u of stage (fp16 slot s16, A slot sa)
+    static __device__ __forceinline__ uint32_t a_addr(uint32_t sb, uint32_t s16, uint32_t sa, int u) {
+        return A16 ? sb + OFF_A + sa * STAGEA + u * SUB16_A : sb + OFF_ST16 + s16 * STAGE16S + u * SUB16;
+    }
+    static __device__ __forceinline__ uint32_t b_addr(uint32_t sb, uint32_t s16, int u) {
+        return A16 ? sb + OFF_ST16 + s16 * STAGE16S + u * SUB16_B
+                   : sb + OFF_ST16 + s16 * STAGE16S + u * SUB16 + SUB16_A;
+    }
     static constexpr uint32_t OFF_ABORT = OFF_TMEM + 4;
     static constexpr uint32_t OFF_EPI = OFF_BAR + SMEM_BARRIERS;
     static constexpr int SMEM_TOTAL = 1024 + OFF_EPI + SMEM_EPI;
@@ -310,7 +329,10 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
             mbar_init(sb + L::BAR_ACCFULL + 8 * i, 1);
             mbar_init(sb + L::BAR_ACCEMPTY + 8 * i, 2 * NUM_EPI_WARPS);
         }
-        for (int i = 0; i < L::S16; ++i) mbar_init(sb + L::BAR_AFULL16 + 8 * i, 1);
+        for (int i = 0; i < L::SA; ++i) {
+            mbar_init(sb + L::BAR_AFULL + 8 * i, 1);
+            mbar_init(sb + L::BAR_AEMPTY + 8 * i, 1);
+        }
         mbar_init(sb + L::BAR_DRAIN, 1);
         st_shared_s32(sb + L::OFF_ABORT, 0);
         fence_barrier_init();
@@ -387,22 +409,21 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                     const CUtensorMap *mA = tl.branch ? &tmA1 : &tmA0;
                     const int arow = tl.m0 + static_cast<int>(rank) * CTA_M;
                     for (int ks = 0; ks < NS; ++ks, ++j) {
-                        const uint32_t s16 = j % L::S16;
-                        if (!mbar_wait_cluster(sb + L::BAR_EMPTY16 + 8 * s16, ((j / L::S16) & 1) ^ 1, wc,
+                        const uint32_t sa = j % L::SAm;
+                        if (!mbar_wait_cluster(sb + L::BAR_AEMPTY + 8 * sa, ((j / L::SAm) & 1) ^ 1, wc,
                                                ERR_PRODUCER)) {
                             ok = false;
                             break;
                         }
-                        const uint32_t ab = sb + L::BAR_AFULL16 + 8 * s16;
-                        mbar_arrive_expect_tx(ab, SUB * SUB16_A);
+                        const uint32_t ab = sb + L::BAR_AFULL + 8 * sa;
+                        mbar_arrive_expect_tx(ab, L::STAGEA);
 #pragma unroll
                         for (int u = 0; u < SUB; ++u)
-                            tma_load_2d(sb + L::OFF_ST16 + s16 * STAGE16 + u * SUB16, mA, (ks * SUB + u) * BK,
-                                        arow, ab);
+                            tma_load_2d(L::a_addr(sb, 0, sa, u), mA, (ks * SUB + u) * BK, arow, ab);
                     }
                 }
-                for (uint32_t i = (j > L::S16 ? j - L::S16 : 0); i < j; ++i)
-                    mbar_wait(sb + L::BAR_AFULL16 + 8 * (i % L::S16), (i / L::S16) & 1, wc, ERR_DRAIN, false);
+                for (uint32_t i = (j > L::SA ? j - L::SA : 0); i < j; ++i)
+                    mbar_wait(sb + L::BAR_AFULL + 8 * (i % L::SAm), (i / L::SAm) & 1, wc, ERR_DRAIN, false);
             }
         } else if (warp == 1) {
             // ------------------------------------------- MMA issue (leader)
@@ -429,10 +450,11 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                                 break;
                             }
                             tc_fence_after();
+                            const uint32_t sa = A16 ? j % L::SAm : 0;
 #pragma unroll
                             for (int u = 0; u < SUB; ++u) {
-                                const uint32_t a = sb + L::OFF_ST16 + st * STAGE16 + u * SUB16;
-                                const uint32_t b = a + SUB16_A;
+                                const uint32_t a = L::a_addr(sb, st, sa, u);
+                                const uint32_t b = L::b_addr(sb, st, u);
 #pragma unroll
                                 for (int kk = 0; kk < BK / 16; ++kk) {
                                     mma_f16_ss_pair(d, smem_desc_sw128(a + kk * 32),
@@ -441,6 +463,7 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                                 }
                             }
                             mma_commit_pair_multicast(sb + L::BAR_EMPTY16 + 8 * st, 0x3);
+                            if (A16) mma_commit_pair_multicast(sb + L::BAR_AEMPTY + 8 * sa, 0x3);
                         }
                         if (ok) mma_commit_pair_multicast(sb + L::BAR_ACCFULL + 8 * buf, 0x3);
                     }
@@ -472,7 +495,7 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                         break;
                     }
                     const uint32_t src = sb + L::OFF_ST8 + s8 * L::STAGE8 + src_off;
-                    const uint32_t dst = sb + L::OFF_ST16 + s16 * STAGE16;
+                    const uint32_t dst = sb + L::OFF_ST16 + s16 * L::STAGE16S;
                     // all of this warp's 8-row groups of a sub-block in flight at
                     // once: every load is issued before the first conversion needs
                     // its data (group g of sub-block u sits at u * kG1 + g in both
@@ -505,8 +528,11 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                                     i8x4_to_f16x4(v[uu][i].y, o0.z, o0.w);
                                     i8x4_to_f16x4(v[uu][i].z, o1.x, o1.y);
                                     i8x4_to_f16x4(v[uu][i].w, o1.z, o1.w);
-                                    st_shared_v4(dst + (u * kG1 + g) * 1024 + dst_off0, o0);
-                                    st_shared_v4(dst + (u * kG1 + g) * 1024 + dst_off1, o1);
+                                    // A16: the fp16 stage holds B alone
+                                    const uint32_t gd = dst + (A16 ? u * SUB16_B + (g - kG0) * 1024
+                                                                   : (u * kG1 + g) * 1024);
+                                    st_shared_v4(gd + dst_off0, o0);
+                                    st_shared_v4(gd + dst_off1, o1);
                                 }
                             }
                     }
@@ -517,7 +543,8 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
                         // leader may issue: converter warp 0 checks it
                         bool a_ok = true;
                         if (cw == 0 && lane == 0)
-                            a_ok = mbar_wait(sb + L::BAR_AFULL16 + 8 * s16, (j / L::S16) & 1, wc, ERR_CONVERTER);
+                            a_ok = mbar_wait(sb + L::BAR_AFULL + 8 * (j % L::SAm), (j / L::SAm) & 1, wc,
+                                             ERR_CONVERTER);
                         if (!__shfl_sync(0xffffffffu, a_ok ? 1 : 0, 0)) {
                             ok = false;
                             break;
