@@ -343,6 +343,31 @@ W8A8_API w8a8_status w8a8_act_stats_finalize(const double *sums, const float *ab
                                              const float *shift, long long count, int K,
                                              float *chan, float *tensor, void *stream);
 
+/* Largest K of w8a8_act_stats_noalloc (its static scratch holds 36 bytes per
+ * input channel: 1.125 MB). */
+#define W8A8_NOALLOC_STATS_MAX_K 32768
+
+/*
+ * No counterpart in the paper: the statistics of ONE batch without caller
+ * accumulators, for callers that want max-abs / mean / std / kurtosis of a
+ * single activation tensor and no allocation.  Same arithmetic as
+ * w8a8_act_stats_update then w8a8_act_stats_finalize with count = T; the
+ * power sums and max-abs live in a file-scope static device scratch of the
+ * library (36 bytes x W8A8_NOALLOC_STATS_MAX_K), which every call clears
+ * (cudaMemsetAsync) before use.  The library allocates nothing.
+ *   - K <= W8A8_NOALLOC_STATS_MAX_K, else W8A8_ERR_UNSUPPORTED_SHAPE; T >= 1,
+ *     else W8A8_ERR_INVALID_ARG.
+ *   - Calls that overlap in time (different streams, host threads or graphs
+ *     in flight at once) share the scratch and race: order them.
+ *   - The first call on a device looks the scratch address up
+ *     (cudaGetSymbolAddress); make one call before capturing a stream into a
+ *     CUDA graph, the later ones are capturable.
+ *   X [T,K] bf16, shift [K] fp32 or NULL, read.  chan [4,K], tensor [4] fp32,
+ *   written, as w8a8_act_stats_finalize.
+ */
+W8A8_API w8a8_status w8a8_act_stats_noalloc(const uint16_t *X, int T, int K, const float *shift,
+                                            float *chan, float *tensor, void *stream);
+
 /*
  * Protected layer (Sec. 3, "Activation-fragility profiling and protection":
  * the most fragile layers keep bf16 weights and no activation quantization):

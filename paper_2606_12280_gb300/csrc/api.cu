@@ -259,6 +259,16 @@ w8a8_status w8a8_act_stats_finalize(const double *sums, const float *absmax, con
                                                      as_stream(stream)));
 }
 
+w8a8_status w8a8_act_stats_noalloc(const uint16_t *X, int T, int K, const float *shift, float *chan,
+                                   float *tensor, void *stream) {
+    if (K <= 0 || (K % 16) != 0 || K > W8A8_NOALLOC_STATS_MAX_K) return W8A8_ERR_UNSUPPORTED_SHAPE;
+    if (T < 0) return W8A8_ERR_UNSUPPORTED_SHAPE;
+    if (T == 0 || !X || !chan || !tensor) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(X) || !aligned16(chan) || !aligned16(tensor) || (shift && !aligned16(shift)))
+        return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_act_stats_noalloc(X, T, K, shift, chan, tensor, as_stream(stream)));
+}
+
 w8a8_status w8a8_linear_bf16(const uint16_t *X, const uint16_t *W, const float *bias, int M,
                              int N, int K, uint16_t *Y, void *stream) {
     if (w8a8_status e = check_nk(N, K)) return e;

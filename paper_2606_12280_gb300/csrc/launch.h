@@ -84,6 +84,11 @@ cudaError_t launch_act_stats_finalize(const double *sums, const float *absmax, c
                                       long long count, int K, float *chan, float *tensor,
                                       cudaStream_t st);
 
+// One-shot statistics of one batch into chan / tensor, with the sums in the
+// library's static device scratch (K <= W8A8_NOALLOC_STATS_MAX_K).
+cudaError_t launch_act_stats_noalloc(const uint16_t *X, int T, int K, const float *shift, float *chan,
+                                     float *tensor, cudaStream_t st);
+
 // Per-tensor activation quantization (two passes: tensor max, then codes).
 cudaError_t launch_quant_act_per_tensor(const uint16_t *X, const float *lambda, int M, int K,
                                         int8_t *Xq, float *x_scale, float *amax, cudaStream_t st);

@@ -450,6 +450,26 @@ struct SlabCache {
     int gx = -1, rows = -1, gy = 0;
 };
 
+// One-shot statistics without caller accumulators: a file-scope scratch of
+// power sums (4 x max K doubles) then max-abs (max K floats), cleared at the
+// start of every call.  Calls that overlap in time share it.
+constexpr int kNoAllocMaxK = W8A8_NOALLOC_STATS_MAX_K;
+static __device__ __align__(256) unsigned char g_stats_scratch[kNoAllocMaxK * (4 * sizeof(double) + sizeof(float))];
+
+// Device address of the scratch on the current device, looked up once per
+// device (the lookup is not a stream operation: do it before any capture).
+void *stats_scratch_address() {
+    constexpr int kMaxDevices = 64;
+    static void *cache[kMaxDevices] = {};
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
+    if (cache[dev]) return cache[dev];
+    void *p = nullptr;
+    if (cudaGetSymbolAddress(&p, g_stats_scratch) != cudaSuccess) return nullptr;
+    cache[dev] = p;
+    return p;
+}
+
 }  // namespace
 
 cudaError_t launch_act_stats_update(const uint16_t *X, int T, int K, const float *shift,
@@ -497,6 +517,25 @@ cudaError_t launch_quant_act_per_tensor(const uint16_t *X, const float *lambda, 
     tensor_quant_kernel<<<dim3(gx, (M + rps2 - 1) / rps2), 32 * kQWarps, 0, st>>>(
         X, lambda, M, K, rps2, amax, Xq, x_scale);
     return cudaGetLastError();
+}
+
+}  // namespace w8a8
+
+namespace w8a8 {
+
+cudaError_t launch_act_stats_noalloc(const uint16_t *X, int T, int K, const float *shift, float *chan,
+                                     float *tensor, cudaStream_t st) {
+    void *base = stats_scratch_address();
+    if (!base) return cudaErrorInvalidSymbol;
+    double *sums = static_cast<double *>(base);
+    float *absmax = reinterpret_cast<float *>(sums + 4 * static_cast<size_t>(kNoAllocMaxK));
+    cudaError_t e = cudaMemsetAsync(sums, 0, sizeof(double) * 4 * static_cast<size_t>(K), st);
+    if (e != cudaSuccess) return e;
+    e = cudaMemsetAsync(absmax, 0, sizeof(float) * static_cast<size_t>(K), st);
+    if (e != cudaSuccess) return e;
+    e = launch_act_stats_update(X, T, K, shift, sums, absmax, st);
+    if (e != cudaSuccess) return e;
+    return launch_act_stats_finalize(sums, absmax, shift, T, K, chan, tensor, st);
 }
 
 }  // namespace w8a8

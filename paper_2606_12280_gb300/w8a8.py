@@ -50,7 +50,10 @@ SIGNATURES = {
     "w8a8_debug_gguf_dequant": [_P, _I, _I, _I, _P, _P],
     "w8a8_quant_act_f16codes": [_P, _P, _I, _I, _P, _P, _I, _P],
     "w8a8_linear_f16codes": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P],
+    "w8a8_act_stats_noalloc": [_P, _I, _I, _P, _P, _P, _P],
 }
+
+NOALLOC_STATS_MAX_K = 32768
 
 GGUF_Q8_0, GGUF_Q4_K = 0, 1
 
@@ -376,6 +379,20 @@ def act_stats_finalize(sums, absmax, count: int, shift=None, chan=None, tensor=N
         _ptr(sums, torch.float64, "sums"), _ptr(absmax, torch.float32, "absmax"),
         _ptr(shift, torch.float32, "shift"), int(count), K, _ptr(chan, torch.float32, "chan"),
         _ptr(tensor, torch.float32, "tensor"), _stream(stream)))
+    return chan, tensor
+
+
+def act_stats_noalloc(X, shift=None, chan=None, tensor=None, stream=None):
+    """Statistics of one batch X [T,K] bf16 with the library's static scratch:
+    (chan [4,K], tensor [4]) fp32.  Overlapping calls race (shared scratch)."""
+    T, K = X.shape
+    if chan is None:
+        chan = torch.empty(4, K, dtype=torch.float32, device=X.device)
+    if tensor is None:
+        tensor = torch.empty(4, dtype=torch.float32, device=X.device)
+    _check("w8a8_act_stats_noalloc", lib().w8a8_act_stats_noalloc(
+        _ptr(X, torch.bfloat16, "X"), T, K, _ptr(shift, torch.float32, "shift"),
+        _ptr(chan, torch.float32, "chan"), _ptr(tensor, torch.float32, "tensor"), _stream(stream)))
     return chan, tensor
 
 

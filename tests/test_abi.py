@@ -257,3 +257,12 @@ def test_f16codes_validation(L):
     assert g(None, A, A, A, None, 4, 8, 16, A, None) == INVALID
     assert g(A, A, U, A, None, 4, 8, 16, A, None) == MISALIGNED
     assert g(A, A, A, A, None, 0, 8, 16, A, None) == OK
+
+
+def test_noalloc_stats_validation(L):
+    f = L.w8a8_act_stats_noalloc
+    assert f(A, 4, 32768 + 16, None, A, A, None) == SHAPE       # beyond the static scratch
+    assert f(A, 4, 24, None, A, A, None) == SHAPE
+    assert f(A, 0, 16, None, A, A, None) == INVALID            # no tokens
+    assert f(None, 4, 16, None, A, A, None) == INVALID
+    assert f(A, 4, 16, None, U, A, None) == MISALIGNED
