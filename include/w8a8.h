@@ -184,15 +184,45 @@ W8A8_API w8a8_status w8a8_quant_act_f16codes(const uint16_t *X, const float *smo
 /*
  * a4 + a5 with the activation codes as fp16 values (from
  * w8a8_quant_act_f16codes): the same exact INT32 product and epilogue as
- * w8a8_linear, bitwise equal outputs; the codes go to the tensor cores
- * without a conversion, which halves the shared-memory traffic of the
- * operand staging.  Xq16 [M,K] fp16 codes, otherwise as w8a8_linear.
+ * w8a8_linear, bitwise equal outputs.  The codes go to the tensor cores by
+ * TMA without a conversion and the int8 weights are converted into tensor
+ * memory, so no converted operand passes through shared memory.
+ *   Xq16 [M,K] fp16 codes (|code| <= 128), otherwise as w8a8_linear.
+ *   chunk_plan: NULL, or the plan that w8a8_chunk_plan wrote for this Wq
+ *     (same N, K); with it the integer sums are drained from the fp32
+ *     accumulator only where the weights require it (see w8a8_chunk_plan).
+ *     A plan of other weights voids the exactness guarantee.
  * Uses the CTA-pair engine whatever w8a8_set_gemm_engine says.
  */
 W8A8_API w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale,
                                           const int8_t *Wq, const float *w_scale,
-                                          const float *bias, int M, int N, int K, uint16_t *Y,
-                                          void *stream);
+                                          const float *bias, int M, int N, int K,
+                                          const uint32_t *chunk_plan, uint16_t *Y, void *stream);
+
+/*
+ * Test export of the product above alone: acc = Xq16 Wq^T as int32 [M,N],
+ * written.  Same shape rules and plan.
+ */
+W8A8_API w8a8_status w8a8_debug_gemm_f16codes_i32(const uint16_t *Xq16, const int8_t *Wq, int M,
+                                                  int N, int K, const uint32_t *chunk_plan,
+                                                  int32_t *acc, void *stream);
+
+/*
+ * Drain plan of an int8 weight matrix for w8a8_linear_f16codes (no
+ * counterpart in the paper: a property of the exact-integer scheme on fp32
+ * accumulators).  The GEMM accumulates integer products in fp32 tensor
+ * memory, exact while every partial sum stays within 2^24; with codes
+ * |a| <= 128 a partial sum over a K range is at most 128 * sum |w_k| over
+ * it, so a run of K chunks (1024 each) can accumulate without a drain while
+ * every weight row of a 256-row block has sum |w_k| <= 2^17 over the run.
+ * The plan records, per 256-row block, after which chunks the run ends (the
+ * worst case, |w| = 127 everywhere, ends it after every chunk).  Computed
+ * once per weight matrix; its layout is internal to the library.
+ *   w8a8_chunk_plan_size: the number of uint32 words of the plan (>= 1).
+ *   Wq [N,K] int8, read;  plan [w8a8_chunk_plan_size(N, K)] uint32, written.
+ */
+W8A8_API long long w8a8_chunk_plan_size(int N, int K);
+W8A8_API w8a8_status w8a8_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, void *stream);
 
 /* ------------------------------------------------------------------------
  * GGUF weight-only layers (Sec. 3, "GGUF k-quants": the DiT serialized to

@@ -212,15 +212,41 @@ w8a8_status w8a8_quant_act_f16codes(const uint16_t *X, const float *smooth, int 
 
 w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale, const int8_t *Wq,
                                  const float *w_scale, const float *bias, int M, int N, int K,
-                                 uint16_t *Y, void *stream) {
+                                 const uint32_t *chunk_plan, uint16_t *Y, void *stream) {
     if (w8a8_status e = check_nk(N, K)) return e;
     if (w8a8_status e = check_mk(M, K)) return e;
     w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), x_scale, Wq, w_scale, bias, Y, M};
     if (w8a8_status e = check_branch(b, true, N, K)) return e;
+    if (chunk_plan && !aligned16(chunk_plan)) return W8A8_ERR_MISALIGNED;
     if (M == 0) return W8A8_OK;
     unsigned int *err = device_error_word();
     if (!err) return W8A8_ERR_CUDA;
-    return from_cuda(w8a8::launch_gemm_tc2(&b, 1, N, K, false, true, err, as_stream(stream)));
+    return from_cuda(w8a8::launch_gemm_ts(&b, 1, N, K, false, chunk_plan, err, as_stream(stream)));
+}
+
+w8a8_status w8a8_debug_gemm_f16codes_i32(const uint16_t *Xq16, const int8_t *Wq, int M, int N, int K,
+                                         const uint32_t *chunk_plan, int32_t *acc, void *stream) {
+    if (w8a8_status e = check_nk(N, K)) return e;
+    if (w8a8_status e = check_mk(M, K)) return e;
+    w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), nullptr, Wq, nullptr, nullptr, acc, M};
+    if (w8a8_status e = check_branch(b, false, N, K)) return e;
+    if (chunk_plan && !aligned16(chunk_plan)) return W8A8_ERR_MISALIGNED;
+    if (M == 0) return W8A8_OK;
+    unsigned int *err = device_error_word();
+    if (!err) return W8A8_ERR_CUDA;
+    return from_cuda(w8a8::launch_gemm_ts(&b, 1, N, K, true, chunk_plan, err, as_stream(stream)));
+}
+
+long long w8a8_chunk_plan_size(int N, int K) {
+    if (N <= 0 || K <= 0) return 1;
+    return static_cast<long long>((N + 255) / 256) * w8a8::chunk_plan_words(K);
+}
+
+w8a8_status w8a8_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, void *stream) {
+    if (w8a8_status e = check_nk(N, K)) return e;
+    if (!Wq || !plan) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(Wq) || !aligned16(plan)) return W8A8_ERR_MISALIGNED;
+    return from_cuda(w8a8::launch_chunk_plan(Wq, N, K, plan, as_stream(stream)));
 }
 
 w8a8_status w8a8_quant_act_per_tensor(const uint16_t *X, const float *smooth, int M, int K,

@@ -1,0 +1,708 @@
+// gemm_ts.cu -- the W8A8 linear (a4 + a5, dual-branch a6) on pairs of SMs with
+// the weights in tensor memory: tcgen05.mma.cta_group::2 in its "TS" form
+// (A operand in TMEM, B operand in shared memory).
+//
+// Same exact-integer scheme as gemm_tc2.cu: int8 values are fp16 values,
+// products are exact in fp32, and partial sums of at most 1024 products stay
+// below 2^24, so K advances in chunks of 1024 that are drained from TMEM into
+// int32 running sums.  What changes is where each operand lives.  The
+// activation codes arrive as fp16 values (the fp16-code variant of a3 writes
+// them), so TMA puts them straight into the 128-byte swizzled B operand; the
+// int8 weights are the A operand: TMA stages them in an int8 ring, the
+// converter warps turn each CTA's 128 weight rows into fp16 in registers and
+// write them into TMEM with tcgen05.st, and the MMA reads A from there.  Per SM
+// and K=128 stage, shared memory then carries 16 KB of int8 weights (one TMA
+// write, one converter read) and 32 KB of activations (one TMA write, one
+// tensor-core read): no fp16 store of a converted operand and no tensor-core
+// read of one.
+//
+// A cluster of two CTAs computes a 256 (output features) x 256 (tokens) tile
+// of Y^T: CTA r holds weight rows f0 + 128r .. +127 in its TMEM lanes and the
+// tokens t0 + 128r .. +127 in its shared memory; the leader issues M=256 N=256
+// K=16 MMAs (eight per stage: N=256 keeps each instruction long enough for one
+// issuing thread to keep the tensor pipe fed) and each CTA's TMEM receives its
+// 128 feature rows x 256 tokens of the fp32 accumulator.  TMEM per CTA: one
+// 256-column accumulator + four 64-column weight slots of K=128 = 512 columns.
+// With a single accumulator the MMA waits at every K chunk until the
+// epilogue has drained it; the drain is short (TMEM -> registers) and the
+// stores of a finished tile overlap the next tile's first chunk.
+//
+// Per CTA: warp 0 TMA producer of the int8 weight ring, warp 2 TMA producer of
+// the fp16 activation ring (both CTAs load against the leader's barrier, so
+// the leader learns directly that both halves of B have landed), warp 1 TMEM
+// allocation (both CTAs) and MMA issue (leader only), warps 4-7 converters
+// (warp w owns TMEM lanes 32(w%4) .. +31, one weight row per thread), warps
+// 8-15 epilogue (TMEM -> int32 running sums -> bf16 dequantized output, one
+// output feature per thread).  Cross-CTA signalling: converters and epilogue
+// warps arrive on the leader's barriers through cluster addresses; the leader
+// commits MMA completion to both CTAs' barriers by multicast.  All waits are
+// bounded in time.
+#include <cstdint>
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include "common.cuh"
+#include "launch.h"
+#include "tc_ptx.cuh"
+
+namespace w8a8 {
+namespace {
+
+using namespace tc;
+
+#ifndef W8A8_TS_S8
+#define W8A8_TS_S8 4
+#endif
+constexpr int PAIR_F = 256, CTA_F = 128;             // output features per pair / CTA (MMA M)
+constexpr int PAIR_T = 256, CTA_T = 128;             // tokens per pair / CTA (MMA N)
+constexpr int BK = 64;                               // K per sub-block (one swizzle atom row)
+constexpr int SUB = 2;                               // sub-blocks per stage
+constexpr int KC_BLOCKS = 16;                        // K chunk = 1024 (exactness bound)
+static_assert(KC_BLOCKS * BK * 127 * 127 < (1 << 24), "fp32 exactness bound");
+static_assert(KC_BLOCKS % SUB == 0, "chunk of whole stages");
+constexpr int KC_STAGES = KC_BLOCKS / SUB;
+// One slot index for the stage's weights in TMEM and its activations in
+// shared memory, so that one barrier says "both landed" and one MMA commit
+// frees both.
+constexpr int SA = 4;                                // slots: TMEM weights + smem activations
+constexpr int SX = SA;
+constexpr int S8 = W8A8_TS_S8;                       // weight ring (int8, smem)
+constexpr int SUBX = CTA_T * BK * 2;                 // 16 KB: one sub-block of activations
+constexpr int SUBW = CTA_F * BK;                     // 8 KB: one sub-block of weights
+constexpr int STAGE_X = SUB * SUBX;
+constexpr int STAGE_W = SUB * SUBW;
+constexpr uint32_t ACC_COLS = PAIR_T;                // fp32 columns of the accumulator
+constexpr uint32_t A_COL0 = ACC_COLS;                // first weight-slot column
+constexpr uint32_t A_SLOT_COLS = SUB * BK / 2;       // fp16 pairs per row of a slot
+constexpr int TMEM_COLS = 512;
+static_assert(A_COL0 + SA * A_SLOT_COLS <= TMEM_COLS, "tensor memory");
+constexpr int NUM_CONV_WARPS = 4;
+constexpr int NUM_EPI_WARPS = 8;
+constexpr int THREADS = 512;
+constexpr int LAUNCH_REGS = 128;
+constexpr int REGS_LOW = 72, REGS_HIGH = 184;
+static_assert(256 * REGS_LOW + 256 * REGS_HIGH <= THREADS * LAUNCH_REGS, "register split");
+constexpr int RUN = PAIR_T / 2;                      // running sums per epilogue thread
+
+constexpr unsigned ERR_PRODUCER = 1u, ERR_CONVERTER = 2u, ERR_MMA = 4u, ERR_EPILOGUE = 8u,
+                   ERR_DRAIN = 16u, ERR_TMEM_PAIR = 64u;
+
+constexpr uint32_t OFF_X = 0;
+constexpr uint32_t OFF_W = OFF_X + SX * STAGE_X;
+constexpr uint32_t OFF_BAR = OFF_W + S8 * STAGE_W;
+constexpr uint32_t BAR_FULL8 = OFF_BAR;                     // weight stage landed (tx)
+constexpr uint32_t BAR_EMPTY8 = BAR_FULL8 + 8 * S8;          // converters read it
+// leader's: this slot's weights written by all converter warps of both CTAs
+// (arrivals) and both CTAs' activations landed (transaction bytes, armed by
+// the leader's activation producer, which also counts as one arrival)
+constexpr uint32_t BAR_SFULL = BAR_EMPTY8 + 8 * S8;
+constexpr uint32_t BAR_SEMPTY = BAR_SFULL + 8 * SA;          // MMA done with the slot (commit)
+constexpr uint32_t BAR_ACCFULL = BAR_SEMPTY + 8 * SA;        // chunk accumulated
+constexpr uint32_t BAR_ACCEMPTY = BAR_ACCFULL + 8;           // leader: chunk drained
+constexpr uint32_t BAR_DRAIN = BAR_ACCEMPTY + 8;
+constexpr uint32_t OFF_TMEM = BAR_DRAIN + 8;
+constexpr uint32_t OFF_ABORT = OFF_TMEM + 4;
+constexpr uint32_t SMEM_BARRIERS = 512;
+static_assert(OFF_ABORT + 4 - OFF_BAR <= SMEM_BARRIERS, "barrier area");
+// per epilogue warp: the activation scales of its 128 tokens
+constexpr uint32_t OFF_EPI = OFF_BAR + SMEM_BARRIERS;
+constexpr uint32_t EPI_BYTES = (PAIR_T / 2) * 4;
+constexpr int SMEM_TOTAL = 1024 + OFF_EPI + NUM_EPI_WARPS * EPI_BYTES;
+static_assert(SMEM_TOTAL <= 232448, "shared memory");
+static_assert(SUBX % 1024 == 0 && SUBW % 1024 == 0, "swizzle atoms stay aligned");
+
+struct BranchArgs {
+    const float *x_scale;
+    const float *w_scale;
+    const float *bias;
+    void *out;
+    int M;           // tokens
+    int t_tiles;     // token tiles of 256
+    int tiles;       // t_tiles * feature tiles
+};
+
+struct Params {
+    BranchArgs br[2];
+    int N, K;
+    int total_tiles;
+    int k_blocks;
+    // optional drain plan (see plan_drains): per 256-row weight block,
+    // plan_words words of bits, bit c set = drain after K chunk c; null =
+    // drain after every chunk
+    const uint32_t *plan;
+    int plan_words;
+    unsigned int *err;
+    uint64_t wait_limit_ns;
+};
+
+struct Tile {
+    int branch, t0, f0;
+};
+
+__device__ __forceinline__ Tile tile_coords(const Params &p, int t) {
+    Tile r;
+    r.branch = t >= p.br[0].tiles ? 1 : 0;
+    const int local = t - (r.branch ? p.br[0].tiles : 0);
+    const int tt = p.br[r.branch].t_tiles;
+    r.t0 = (local % tt) * PAIR_T;
+    r.f0 = (local / tt) * PAIR_F;
+    return r;
+}
+
+// int8 x4 -> two fp16x2 words, exact (bytes + 128 in the mantissa of 1024.0,
+// minus 1152).
+// Does the accumulation stop (the epilogue drains TMEM) after K chunk ci of a
+// tile of weight block fb?  Always after the tile's last chunk.
+__device__ __forceinline__ bool plan_drains(const Params &p, int fb, int ci, int NC) {
+    if (ci == NC - 1 || p.plan == nullptr) return true;
+    return (__ldg(p.plan + (size_t)fb * p.plan_words + (ci >> 5)) >> (ci & 31)) & 1u;
+}
+
+__device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
+    const uint32_t u = w ^ 0x80808080u;
+    asm("prmt.b32 %0, %1, %2, 0x4140;" : "=r"(lo) : "r"(u), "r"(0x64646464u));
+    asm("prmt.b32 %0, %1, %2, 0x4342;" : "=r"(hi) : "r"(u), "r"(0x64646464u));
+    asm("sub.f16x2 %0, %0, %1;" : "+r"(lo) : "r"(0x64806480u));
+    asm("sub.f16x2 %0, %0, %1;" : "+r"(hi) : "r"(0x64806480u));
+}
+
+__device__ __forceinline__ void arrive_leader(uint32_t bar, uint32_t rank) {
+    if (rank == 0) mbar_arrive(bar);
+    else mbar_arrive_cluster_relaxed(mapa_shared(bar, 0));
+}
+
+template <bool OUT_I32>
+__device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint32_t tmem,
+                                              const WaitCtx &wc, int warp, int lane, int NC,
+                                              uint32_t rank, int pair, int npairs) {
+    const int q = warp & 3;            // TMEM lane quarter this warp may access
+    const int h = (warp - 8) >> 2;     // token half of the 256-wide tile
+    uint32_t c = 0;                    // drains so far
+    bool ok = true;
+    for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+        const int fb = tile_coords(p, t).f0 / PAIR_F;
+        int32_t run[RUN];
+#pragma unroll
+        for (int i = 0; i < RUN; ++i) run[i] = 0;
+        for (int ci = 0; ci < NC; ++ci) {
+            if (!plan_drains(p, fb, ci, NC)) continue;
+            if (!mbar_wait_cluster(sb + BAR_ACCFULL, c & 1, wc, ERR_EPILOGUE)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) + h * (PAIR_T / 2);
+            // two loads in flight per wait: the MMA is stopped until every
+            // epilogue warp has drained its part
+#pragma unroll
+            for (int jj = 0; jj < RUN / 16; jj += 2) {
+                uint32_t v[2][16];
+#pragma unroll
+                for (int g = 0; g < 2; ++g) tmem_ld_32x32b_x16(base + (jj + g) * 16, v[g]);
+                tmem_ld_wait();
+                // the values are exact integers.  Below 2^22 in magnitude (in
+                // practice always) v + 1.5 * 2^23 holds v in its low mantissa
+                // bits, exactly: one add instead of a conversion instruction,
+                // which runs at a fraction of the add rate and would stall the
+                // MMA for the whole drain.  OR-ing the magnitudes' bit patterns
+                // bounds them all; the exact conversion is the (warp-uniform)
+                // fallback.
+                uint32_t any = 0;
+#pragma unroll
+                for (int g = 0; g < 2; ++g)
+#pragma unroll
+                    for (int i = 0; i < 16; ++i) any |= v[g][i] & 0x7fffffffu;
+                if (__any_sync(0xffffffffu, any >= 0x4A800000u)) {
+#pragma unroll
+                    for (int g = 0; g < 2; ++g)
+#pragma unroll
+                        for (int i = 0; i < 16; ++i)
+                            run[(jj + g) * 16 + i] += __float2int_rn(__uint_as_float(v[g][i]));
+                } else {
+#pragma unroll
+                    for (int g = 0; g < 2; ++g)
+#pragma unroll
+                        for (int i = 0; i < 16; ++i)
+                            run[(jj + g) * 16 + i] += static_cast<int32_t>(
+                                __float_as_uint(__fadd_rn(__uint_as_float(v[g][i]), 12582912.0f)) - 0x4B400000u);
+                }
+            }
+            tc_fence_before();
+            __syncwarp();
+            if (lane == 0) arrive_leader(sb + BAR_ACCEMPTY, rank);
+            ++c;
+        }
+        if (!ok) break;
+        const Tile tl = tile_coords(p, t);
+        const BranchArgs &br = p.br[tl.branch];
+        const int f = tl.f0 + static_cast<int>(rank) * CTA_F + q * 32 + lane;   // output feature
+        const int tok0 = tl.t0 + h * (PAIR_T / 2);
+        const int ntok = min(RUN, br.M - tok0);
+        const bool fok = f < p.N;
+        if (ntok > 0) {             // uniform across the warp (one token range)
+            if (OUT_I32 && fok) {
+                int32_t *out = static_cast<int32_t *>(br.out) + (size_t)tok0 * p.N + f;
+#pragma unroll
+                for (int i = 0; i < RUN; ++i)
+                    if (i < ntok) out[(size_t)i * p.N] = run[i];
+            } else if (!OUT_I32) {
+                const float sw = fok ? __ldg(br.w_scale + f) : 0.0f;
+                const bool hb = br.bias != nullptr;
+                const float b = (hb && fok) ? __ldg(br.bias + f) : 0.0f;
+                // the warp's 128 token scales go through shared memory once
+                // (one 16-byte load per lane), then every lane reads them as
+                // broadcasts: a global load per token inside the store loop
+                // would wait a full memory latency per token
+                const uint32_t epi = sb + OFF_EPI + (warp - 8) * EPI_BYTES;
+                {
+                    const float *sxp = br.x_scale + tok0;
+                    float4 s4;
+                    if (4 * lane + 3 < ntok) {
+                        s4 = __ldg(reinterpret_cast<const float4 *>(sxp) + lane);
+                    } else {
+                        s4.x = 4 * lane < ntok ? __ldg(sxp + 4 * lane) : 0.0f;
+                        s4.y = 4 * lane + 1 < ntok ? __ldg(sxp + 4 * lane + 1) : 0.0f;
+                        s4.z = 4 * lane + 2 < ntok ? __ldg(sxp + 4 * lane + 2) : 0.0f;
+                        s4.w = 0.0f;
+                    }
+                    st_shared_v4(epi + 16 * lane, make_uint4(__float_as_uint(s4.x), __float_as_uint(s4.y),
+                                                             __float_as_uint(s4.z), __float_as_uint(s4.w)));
+                    __syncwarp();
+                }
+                // lanes 2i and 2i+1 (features f, f+1) swap one value per pair
+                // of tokens, so that each stores one 32-bit word: the even
+                // lane both features of the first token, the odd lane both of
+                // the second (N even: the word is 4-byte aligned)
+                const bool odd = lane & 1;
+                const int fw = f & ~1;
+                uint16_t *out = static_cast<uint16_t *>(br.out) + (size_t)tok0 * p.N + fw;
+                const bool paired = (p.N & 1) == 0;
+#pragma unroll
+                for (int i = 0; i < RUN; i += 4) {
+                    const uint4 s4 = ld_shared_v4(epi + 4 * i);
+                    const float sxv[4] = {__uint_as_float(s4.x), __uint_as_float(s4.y), __uint_as_float(s4.z),
+                                          __uint_as_float(s4.w)};
+#pragma unroll
+                    for (int u = 0; u < 4; u += 2) {
+                        const uint32_t y0 = epilogue_value(run[i + u], sxv[u], sw, b, hb);
+                        const uint32_t y1 = epilogue_value(run[i + u + 1], sxv[u + 1], sw, b, hb);
+                        const uint32_t other = __shfl_xor_sync(0xffffffffu, odd ? y0 : y1, 1);
+                        const int tk = i + u + (odd ? 1 : 0);
+                        if (paired) {
+                            const uint32_t word = odd ? (other | (y1 << 16)) : (y0 | (other << 16));
+                            if (tk < ntok && fok)
+                                *reinterpret_cast<uint32_t *>(out + (size_t)tk * p.N) = word;
+                        } else {
+                            uint16_t *o = out + (f - fw);
+                            if (fok && i + u < ntok) o[(size_t)(i + u) * p.N] = static_cast<uint16_t>(y0);
+                            if (fok && i + u + 1 < ntok)
+                                o[(size_t)(i + u + 1) * p.N] = static_cast<uint16_t>(y1);
+                        }
+                    }
+                }
+            }
+        }
+        __syncwarp();
+    }
+}
+
+template <bool OUT_I32>
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
+gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__ CUtensorMap tmW0,
+               const __grid_constant__ CUtensorMap tmX1, const __grid_constant__ CUtensorMap tmW1,
+               const Params p) {
+    extern __shared__ uint8_t smem_raw[];
+    const uint32_t sb = (smem_addr(smem_raw) + 1023u) & ~1023u;
+    const int warp = threadIdx.x >> 5;
+    const int lane = threadIdx.x & 31;
+    const uint32_t rank = cluster_ctarank();
+    const bool leader = rank == 0;
+    const int pair = blockIdx.x >> 1;
+    const int npairs = gridDim.x >> 1;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < S8; ++i) {
+            mbar_init(sb + BAR_FULL8 + 8 * i, 1);
+            mbar_init(sb + BAR_EMPTY8 + 8 * i, NUM_CONV_WARPS);
+        }
+        for (int i = 0; i < SA; ++i) {
+            mbar_init(sb + BAR_SFULL + 8 * i, 2 * NUM_CONV_WARPS + 1);
+            mbar_init(sb + BAR_SEMPTY + 8 * i, 1);
+        }
+        mbar_init(sb + BAR_ACCFULL, 1);
+        mbar_init(sb + BAR_ACCEMPTY, 2 * NUM_EPI_WARPS);
+        mbar_init(sb + BAR_DRAIN, 1);
+        st_shared_s32(sb + OFF_ABORT, 0);
+        fence_barrier_init();
+    }
+    if (warp == 0 && lane == 0) {
+        tma_prefetch_desc(&tmX0);
+        tma_prefetch_desc(&tmW0);
+        tma_prefetch_desc(&tmX1);
+        tma_prefetch_desc(&tmW1);
+    }
+    if (warp == 1) {
+        tmem_alloc_pair(sb + OFF_TMEM, TMEM_COLS);
+        tmem_relinquish_pair();
+    }
+    tc_fence_before();
+    cluster_sync();
+    tc_fence_after();
+    const uint32_t tmem = static_cast<uint32_t>(ld_shared_s32(sb + OFF_TMEM));
+    const uint32_t peer_tmem = ld_shared_cluster_u32(mapa_shared(sb + OFF_TMEM, rank ^ 1u));
+    const bool run_ok = (tmem == peer_tmem);
+    if (!run_ok && threadIdx.x == 0) atomicOr(p.err, ERR_TMEM_PAIR);
+    const WaitCtx wc{sb + OFF_ABORT, p.err, p.wait_limit_ns};
+    const int KB = p.k_blocks;                            // K=64 sub-blocks per tile
+    const int NS = (KB + SUB - 1) / SUB;                  // stages per tile
+    const int NC = (KB + KC_BLOCKS - 1) / KC_BLOCKS;      // chunks per tile
+
+    if (warp >= 8) {
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(REGS_HIGH));
+        if (run_ok) epilogue_role<OUT_I32>(p, sb, tmem, wc, warp, lane, NC, rank, pair, npairs);
+    } else {
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(REGS_LOW));
+        if (!run_ok) {
+        } else if (warp == 0) {
+            // ------------------------------------------ TMA producer: weights
+            if (lane == 0) {
+                uint32_t j = 0;
+                bool ok = true;
+                for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+                    const Tile tl = tile_coords(p, t);
+                    const CUtensorMap *mW = tl.branch ? &tmW1 : &tmW0;
+                    const int frow = tl.f0 + static_cast<int>(rank) * CTA_F;
+                    for (int ks = 0; ks < NS; ++ks, ++j) {
+                        const uint32_t s = j % S8;
+                        if (!mbar_wait(sb + BAR_EMPTY8 + 8 * s, ((j / S8) & 1) ^ 1, wc, ERR_PRODUCER)) {
+                            ok = false;
+                            break;
+                        }
+                        const uint32_t fb = sb + BAR_FULL8 + 8 * s;
+                        const int nsub = min(SUB, KB - ks * SUB);     // the last stage may be half
+                        mbar_arrive_expect_tx(fb, nsub * SUBW);
+                        for (int u = 0; u < nsub; ++u)
+                            tma_load_2d(sb + OFF_W + s * STAGE_W + u * SUBW, mW, (ks * SUB + u) * BK, frow, fb);
+                    }
+                }
+                for (uint32_t i = (j > S8 ? j - S8 : 0); i < j; ++i)
+                    mbar_wait(sb + BAR_FULL8 + 8 * (i % S8), (i / S8) & 1, wc, ERR_DRAIN, false);
+            }
+        } else if (warp == 2) {
+            // -------------------------------------- TMA producer: activations
+            // fp16 activation codes of this CTA's 128 tokens, straight into
+            // the swizzled B operand; completion lands on the leader's
+            // barrier, which the leader armed for both CTAs' bytes.  (Every
+            // load has landed before the kernel ends: the MMA waits for each.)
+            if (lane == 0) {
+                uint32_t j = 0;
+                bool ok = true;
+                for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+                    const Tile tl = tile_coords(p, t);
+                    const CUtensorMap *mX = tl.branch ? &tmX1 : &tmX0;
+                    const int trow = tl.t0 + static_cast<int>(rank) * CTA_T;
+                    for (int ks = 0; ks < NS; ++ks, ++j) {
+                        const uint32_t s = j % SX;
+                        if (!mbar_wait_cluster(sb + BAR_SEMPTY + 8 * s, ((j / SX) & 1) ^ 1, wc, ERR_PRODUCER)) {
+                            ok = false;
+                            break;
+                        }
+                        const uint32_t fb = mapa_shared(sb + BAR_SFULL + 8 * s, 0);
+                        const int nsub = min(SUB, KB - ks * SUB);
+                        if (leader) mbar_arrive_expect_tx(sb + BAR_SFULL + 8 * s, 2 * nsub * SUBX);
+                        for (int u = 0; u < nsub; ++u)
+                            tma_load_2d_pair(sb + OFF_X + s * STAGE_X + u * SUBX, mX, (ks * SUB + u) * BK, trow, fb);
+                    }
+                }
+            }
+        } else if (warp == 1) {
+            // ------------------------------------------- MMA issue (leader)
+            if (lane == 0 && leader) {
+                constexpr uint32_t idesc = idesc_f16_f32(PAIR_F, PAIR_T);
+                uint32_t j = 0, c = 0;         // stages, drains so far
+                bool ok = true;
+                for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+                    const int fb = tile_coords(p, t).f0 / PAIR_F;
+                    bool fresh = true;         // the next MMA starts a new accumulation
+                    for (int ci = 0; ok && ci < NC; ++ci) {
+                        if (fresh) {
+                            // the epilogue has drained the previous accumulation
+                            if (!mbar_wait_cluster(sb + BAR_ACCEMPTY, (c & 1) ^ 1, wc, ERR_MMA)) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after();
+                        }
+                        const int ks0 = ci * KC_STAGES;
+                        const int ks1 = min(NS, ks0 + KC_STAGES);
+                        for (int ks = ks0; ks < ks1; ++ks, ++j) {
+                            const uint32_t sa = j % SA, sx = sa;
+                            if (!mbar_wait_cluster(sb + BAR_SFULL + 8 * sa, (j / SA) & 1, wc, ERR_MMA)) {
+                                ok = false;
+                                break;
+                            }
+                            tc_fence_after();
+                            const uint32_t a = tmem + A_COL0 + sa * A_SLOT_COLS;
+                            const uint32_t b = sb + OFF_X + sx * STAGE_X;
+#pragma unroll
+                            for (int u = 0; u < SUB; ++u) {
+                                if (ks * SUB + u >= KB) break;
+#pragma unroll
+                                for (int kk = 0; kk < BK / 16; ++kk)
+                                    mma_f16_ts_pair(tmem, a + u * (BK / 2) + kk * 8,
+                                                    smem_desc_sw128(b + u * SUBX + kk * 32), idesc,
+                                                    (!fresh || ks > ks0 || u > 0 || kk > 0) ? 1u : 0u);
+                            }
+                            mma_commit_pair_multicast(sb + BAR_SEMPTY + 8 * sa, 0x3);
+                        }
+                        fresh = plan_drains(p, fb, ci, NC);
+                        if (ok && fresh) {
+                            mma_commit_pair_multicast(sb + BAR_ACCFULL, 0x3);
+                            ++c;
+                        }
+                    }
+                }
+                mma_commit_pair(sb + BAR_DRAIN);
+                mbar_wait_cluster(sb + BAR_DRAIN, 0, wc, ERR_DRAIN, false);
+            }
+        } else if (warp >= 4) {
+            // ---------------------------------------------------- converters
+            // thread = weight row r of this CTA = TMEM lane r; each K=64
+            // sub-block of the row is 64 bytes in four 16-byte chunks, chunk
+            // c at c ^ ((r >> 1) & 3) (the 64-byte swizzle, which spreads 8
+            // consecutive rows over all banks)
+            const uint32_t r = static_cast<uint32_t>((warp & 3) * 32 + lane);
+            const uint32_t src_row = r * BK;
+            const uint32_t sw = (r >> 1) & 3;
+            const uint32_t a_lane = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + A_COL0;
+            uint32_t j = 0;
+            bool ok = true;
+            for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+                for (int ks = 0; ks < NS; ++ks, ++j) {
+                    const uint32_t s8 = j % S8, sa = j % SA;
+                    // every lane waits; __all_sync keeps the warp's control flow
+                    // uniform if a wait gives up
+                    if (!__all_sync(0xffffffffu, mbar_wait(sb + BAR_FULL8 + 8 * s8, (j / S8) & 1, wc,
+                                                            ERR_CONVERTER))) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t src = sb + OFF_W + s8 * STAGE_W + src_row;
+                    uint4 v[4];
+#pragma unroll
+                    for (int cc = 0; cc < 4; ++cc) v[cc] = ld_shared_v4(src + ((cc ^ sw) << 4));
+                    if (!__all_sync(0xffffffffu, mbar_wait_cluster(sb + BAR_SEMPTY + 8 * sa, ((j / SA) & 1) ^ 1,
+                                                                    wc, ERR_CONVERTER))) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    // convert sub-block u (its codes in v) and write it into
+                    // the slot's columns 32u .. 32u + 31
+                    auto convert_store = [&](int u) {
+                        uint32_t w[32];
+#pragma unroll
+                        for (int cc = 0; cc < 4; ++cc) {
+                            i8x4_to_f16x4(v[cc].x, w[8 * cc + 0], w[8 * cc + 1]);
+                            i8x4_to_f16x4(v[cc].y, w[8 * cc + 2], w[8 * cc + 3]);
+                            i8x4_to_f16x4(v[cc].z, w[8 * cc + 4], w[8 * cc + 5]);
+                            i8x4_to_f16x4(v[cc].w, w[8 * cc + 6], w[8 * cc + 7]);
+                        }
+                        tmem_st_32x32b_x32(a_lane + sa * A_SLOT_COLS + u * (BK / 2), w);
+                    };
+                    static_assert(SUB == 2, "two sub-blocks per stage");
+                    convert_store(0);
+                    if (ks * SUB + 1 < KB) {            // the last stage may be half
+                        // loaded once sub-block 0's codes are out of the way
+#pragma unroll
+                        for (int cc = 0; cc < 4; ++cc) v[cc] = ld_shared_v4(src + SUBW + ((cc ^ sw) << 4));
+                        convert_store(1);
+                    }
+                    // the stage's bytes are all in registers (and in TMEM) now
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive(sb + BAR_EMPTY8 + 8 * s8);
+                    tmem_st_wait();
+                    tc_fence_before();
+                    __syncwarp();
+                    if (lane == 0) arrive_leader(sb + BAR_SFULL + 8 * sa, rank);
+                }
+            }
+        }
+    }
+    tc_fence_before();
+    __syncwarp();
+    asm volatile("bar.sync 1, %0;" ::"n"(THREADS) : "memory");
+    cluster_sync();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc_pair(tmem, TMEM_COLS);
+    }
+}
+
+// ------------------------------------------------------------ drain plan
+//
+// The fixed chunk of 1024 products is the worst case (every |a|, |w| at its
+// maximum).  A tighter bound holds per weight row: every partial sum that
+// the tensor core forms over a K range is at most sum |a_k| |w_k| <=
+// 128 * sum |w_k| over that range (|a| <= 128 for an int8 code), so runs of
+// chunks whose weight rows all have sum |w_k| <= 2^17 keep every partial sum
+// within 2^24, exact in fp32, and need no drain in between.  The plan is
+// built once per weight matrix: per block of 256 rows (one tile of the GEMM),
+// chunks are merged greedily while the largest row's sum over the merged run
+// stays within the bound.
+constexpr uint32_t kPlanL1Limit = 1u << 17;
+constexpr int KC = KC_BLOCKS * BK;                   // K per chunk
+
+__global__ void __launch_bounds__(PAIR_F)
+chunk_plan_kernel(const int8_t *__restrict__ Wq, int N, int K, int NC, int words, uint32_t *__restrict__ plan) {
+    __shared__ uint32_t red[PAIR_F / 32];
+    const int fb = blockIdx.x;
+    const int r = fb * PAIR_F + threadIdx.x;
+    uint32_t *row_plan = plan + (size_t)fb * words;
+    if (threadIdx.x == 0)
+        for (int w = 0; w < words; ++w) row_plan[w] = 0u;
+    uint32_t cur = 0;                                 // this row's sum |w| since the last drain
+    for (int c = 0; c < NC; ++c) {
+        uint32_t l1 = 0;
+        if (r < N) {
+            const int k1 = min(K, (c + 1) * KC);
+            const uint4 *src = reinterpret_cast<const uint4 *>(Wq + (size_t)r * K);
+            for (int k = c * KC; k < k1; k += 16) {
+                const uint4 v = __ldg(src + k / 16);
+                l1 = __dp4a(__vabsdiffs4(v.x, 0u), 0x01010101u, l1);
+                l1 = __dp4a(__vabsdiffs4(v.y, 0u), 0x01010101u, l1);
+                l1 = __dp4a(__vabsdiffs4(v.z, 0u), 0x01010101u, l1);
+                l1 = __dp4a(__vabsdiffs4(v.w, 0u), 0x01010101u, l1);
+            }
+        }
+        const uint32_t cand = cur + l1;
+        const uint32_t wm = __reduce_max_sync(0xffffffffu, cand);
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = wm;
+        __syncthreads();
+        uint32_t m = 0;
+#pragma unroll
+        for (int w = 0; w < PAIR_F / 32; ++w) m = max(m, red[w]);
+        __syncthreads();
+        if (m > kPlanL1Limit) {                       // chunk c starts a new run
+            if (threadIdx.x == 0) row_plan[(c - 1) >> 5] |= 1u << ((c - 1) & 31);
+            cur = l1;
+        } else {
+            cur = cand;
+        }
+    }
+    if (threadIdx.x == 0) row_plan[(NC - 1) >> 5] |= 1u << ((NC - 1) & 31);
+}
+
+// ------------------------------------------------------------------ host
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
+                                  const cuuint64_t *, const cuuint64_t *, const cuuint32_t *,
+                                  const cuuint32_t *, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encode() {
+    static EncodeTiledFn fn = nullptr;
+    if (!fn) {
+        void *ptr = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
+                                             cudaEnableDefault, &q) == cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            fn = reinterpret_cast<EncodeTiledFn>(ptr);
+    }
+    return fn;
+}
+
+// row-major [rows, inner] -> 2-D map with box [box_rows, box_inner], zero fill
+bool make_map(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint64_t inner, uint64_t rows,
+              uint64_t row_bytes, uint32_t box_inner, uint32_t box_rows, CUtensorMapSwizzle sw) {
+    EncodeTiledFn enc = get_encode();
+    if (!enc) return false;
+    cuuint64_t dims[2] = {inner, rows};
+    cuuint64_t strides[1] = {row_bytes};
+    cuuint32_t box[2] = {box_inner, box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return enc(m, dt, 2, const_cast<void *>(base), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+               sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int g_sms = 0;
+int g_kernel_regs[2] = {-1, -1};
+
+}  // namespace
+
+int chunk_plan_words(int K) {
+    const int NC = (K + KC - 1) / KC;
+    return (NC + 31) / 32;
+}
+
+cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cudaStream_t st) {
+    const int NC = (K + KC - 1) / KC;
+    chunk_plan_kernel<<<(N + PAIR_F - 1) / PAIR_F, PAIR_F, 0, st>>>(Wq, N, K, NC, chunk_plan_words(K), plan);
+    return cudaGetLastError();
+}
+
+cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, const uint32_t *plan,
+                           unsigned int *err, cudaStream_t st) {
+    if (g_sms == 0) {
+        int dev = 0;
+        cudaGetDevice(&dev);
+        cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
+    }
+    const int ki = out_i32 ? 1 : 0;
+    auto kern = out_i32 ? gemm_ts_kernel<true> : gemm_ts_kernel<false>;
+    if (g_kernel_regs[ki] < 0) {
+        cudaFuncAttributes fa;
+        cudaError_t e = cudaFuncGetAttributes(&fa, kern);
+        if (e != cudaSuccess) return e;
+        g_kernel_regs[ki] = fa.numRegs;
+        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_TOTAL);
+        if (e != cudaSuccess) return e;
+    }
+    // the register split above assumes the launch gets exactly this many
+    if (g_kernel_regs[ki] != LAUNCH_REGS) return cudaErrorInvalidConfiguration;
+
+    Params p{};
+    CUtensorMap maps[4];
+    int first = -1;
+    const int f_tiles = (N + PAIR_F - 1) / PAIR_F;
+    for (int i = 0; i < 2; ++i) {
+        const GemmBranch *b = (i < nb) ? &br[i] : nullptr;
+        BranchArgs &a = p.br[i];
+        a = BranchArgs{nullptr, nullptr, nullptr, nullptr, 0, 0, 0};
+        if (b && b->M > 0) {
+            a.x_scale = b->x_scale;
+            a.w_scale = b->w_scale;
+            a.bias = b->bias;
+            a.out = b->out;
+            a.M = b->M;
+            a.t_tiles = (b->M + PAIR_T - 1) / PAIR_T;
+            a.tiles = a.t_tiles * f_tiles;
+            if (!make_map(&maps[2 * i], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, b->Xq, K, b->M, 2ull * K, BK, CTA_T,
+                          CU_TENSOR_MAP_SWIZZLE_128B) ||
+                !make_map(&maps[2 * i + 1], CU_TENSOR_MAP_DATA_TYPE_UINT8, b->Wq, K, N, K, BK, CTA_F,
+                          CU_TENSOR_MAP_SWIZZLE_64B))
+                return cudaErrorInvalidValue;
+            if (first < 0) first = i;
+        }
+    }
+    if (first < 0) return cudaSuccess;
+    for (int i = 0; i < 2; ++i)
+        if (p.br[i].M == 0) {
+            maps[2 * i] = maps[2 * first];
+            maps[2 * i + 1] = maps[2 * first + 1];
+        }
+    p.N = N;
+    p.K = K;
+    p.total_tiles = p.br[0].tiles + p.br[1].tiles;
+    p.k_blocks = (K + BK - 1) / BK;
+    p.plan = plan;
+    p.plan_words = chunk_plan_words(K);
+    p.err = err;
+    p.wait_limit_ns = 2000000000ull;
+    const int pairs = p.total_tiles < g_sms / 2 ? p.total_tiles : g_sms / 2;
+    kern<<<2 * pairs, THREADS, SMEM_TOTAL, st>>>(maps[0], maps[1], maps[2], maps[3], p);
+    return cudaGetLastError();
+}
+
+}  // namespace w8a8

@@ -58,6 +58,15 @@ cudaError_t launch_gemm_mma(const GemmBranch *br, int nb, int N, int K,
 cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K,
                             bool out_i32, bool a16, unsigned int *err, cudaStream_t st);
 
+// tcgen05 GEMM on CTA pairs with the weights in tensor memory: Xq holds the
+// activation codes as fp16 values (2 bytes each), Wq the int8 weights.  plan
+// (optional, from launch_chunk_plan on the same Wq) lets runs of K chunks
+// accumulate without a drain where the weights bound the partial sums.
+cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, const uint32_t *plan,
+                           unsigned int *err, cudaStream_t st);
+int chunk_plan_words(int K);    // per block of 256 weight rows
+cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cudaStream_t st);
+
 // a3 (optionally of GELU(X)) writing the codes as fp16 values, K <= 16384.
 cudaError_t launch_quant_act_f16codes(const uint16_t *X, const float *lambda, int M, int K,
                                      uint16_t *Xq16, float *x_scale, bool gelu, cudaStream_t st);

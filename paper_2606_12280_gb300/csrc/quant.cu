@@ -552,11 +552,11 @@ cudaError_t launch_act_quant_team(ActParams p, cudaStream_t st) {
     static int per_sm = 0;
     auto kern = act_quant_team_kernel<U, TW, S, GELU, OUT16>;
     if (per_sm == 0) {
-        if (smem > 48 * 1024) {
-            cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                                 (int)smem);
-            if (e != cudaSuccess) return e;
-        }
+        // always opted in: the static reduction array counts against the
+        // 48 KB default too
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                             (int)smem);
+        if (e != cudaSuccess) return e;
         cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem);
         if (per_sm < 1) per_sm = 1;
     }

@@ -49,7 +49,10 @@ SIGNATURES = {
     "w8a8_linear_gguf": [_P, _P, _I, _P, _I, _I, _I, _P, _P],
     "w8a8_debug_gguf_dequant": [_P, _I, _I, _I, _P, _P],
     "w8a8_quant_act_f16codes": [_P, _P, _I, _I, _P, _P, _I, _P],
-    "w8a8_linear_f16codes": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P],
+    "w8a8_linear_f16codes": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P],
+    "w8a8_debug_gemm_f16codes_i32": [_P, _P, _I, _I, _I, _P, _P, _P],
+    "w8a8_chunk_plan_size": [_I, _I],
+    "w8a8_chunk_plan": [_P, _I, _I, _P, _P],
     "w8a8_act_stats_noalloc": [_P, _I, _I, _P, _P, _P, _P],
 }
 
@@ -100,6 +103,7 @@ def lib() -> ctypes.CDLL:
                 fn.argtypes = args
                 fn.restype = ctypes.c_int
             L.w8a8_status_string.restype = ctypes.c_char_p
+            L.w8a8_chunk_plan_size.restype = ctypes.c_longlong
             _lib = L
     return _lib
 
@@ -298,8 +302,9 @@ def quant_act_f16codes(X, smooth=None, Xq16=None, x_scale=None, gelu=False, stre
     return Xq16, x_scale
 
 
-def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, stream=None):
-    """a4 + a5 with fp16-coded activations: Y = bf16((Xq Wq^T) * sx * sw + b)."""
+def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, stream=None):
+    """a4 + a5 with fp16-coded activations: Y = bf16((Xq Wq^T) * sx * sw + b).
+    plan: None or ``chunk_plan(Wq)``."""
     M, K = Xq16.shape
     N = Wq.shape[0]
     if Y is None:
@@ -307,8 +312,37 @@ def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, stream=None):
     _check("w8a8_linear_f16codes", lib().w8a8_linear_f16codes(
         _ptr(Xq16, torch.float16, "Xq16"), _ptr(x_scale, torch.float32, "x_scale"),
         _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
-        _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(Y, torch.bfloat16, "Y"), _stream(stream)))
+        _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(plan, torch.int32, "plan"),
+        _ptr(Y, torch.bfloat16, "Y"), _stream(stream)))
     return Y
+
+
+def debug_gemm_f16codes_i32(Xq16, Wq, plan=None, acc=None, stream=None):
+    """Exact int32 acc = Xq16 Wq^T (test export of the fp16-code GEMM)."""
+    M, K = Xq16.shape
+    N = Wq.shape[0]
+    if acc is None:
+        acc = torch.empty(M, N, dtype=torch.int32, device=Xq16.device)
+    _check("w8a8_debug_gemm_f16codes_i32", lib().w8a8_debug_gemm_f16codes_i32(
+        _ptr(Xq16, torch.float16, "Xq16"), _ptr(Wq, torch.int8, "Wq"), M, N, K,
+        _ptr(plan, torch.int32, "plan"), _ptr(acc, torch.int32, "acc"), _stream(stream)))
+    return acc
+
+
+def chunk_plan_size(N: int, K: int) -> int:
+    """Words of the drain plan of an [N, K] int8 weight."""
+    return int(lib().w8a8_chunk_plan_size(int(N), int(K)))
+
+
+def chunk_plan(Wq, plan=None, stream=None):
+    """Drain plan of the int8 weights Wq [N, K] for ``linear_f16codes`` (an
+    int32 tensor holding the library's uint32 words)."""
+    N, K = Wq.shape
+    if plan is None:
+        plan = torch.empty(chunk_plan_size(N, K), dtype=torch.int32, device=Wq.device)
+    _check("w8a8_chunk_plan", lib().w8a8_chunk_plan(
+        _ptr(Wq, torch.int8, "Wq"), N, K, _ptr(plan, torch.int32, "plan"), _stream(stream)))
+    return plan
 
 
 def linear_gguf(X, Wraw, fmt: int, N: int, bias=None, Y=None, stream=None):

@@ -67,14 +67,16 @@ def test_quant_act_f16codes_gelu_matches_int8_gelu(w8):
 
 @pytest.mark.parametrize("M,N,K", [(1, 8, 16), (300, 264, 528), (513, 520, 1040), (64, 256, 16384)])
 @pytest.mark.parametrize("with_bias", [True, False])
-def test_linear_f16codes_exact(w8, oracle_mod, M, N, K, with_bias):
+@pytest.mark.parametrize("with_plan", [True, False])
+def test_linear_f16codes_exact(w8, oracle_mod, M, N, K, with_bias, with_plan):
     c = wl.make_case(M, K, N, seed=M + N + K)
     s = oracle_mod.channel_absmax(c.X_cal)
     lam = oracle_mod.smooth_scales(s, c.W[0], c.alpha)
     Wq, sw = oracle_mod.quantize_weights(c.W[0], lam)
     b = c.bias[0] if with_bias else None
     q16, sx = w8.quant_act_f16codes(bf(c.X[0]), t(lam))
-    Y = w8.linear_f16codes(q16, sx, t(Wq), t(sw), t(b) if with_bias else None)
+    plan = w8.chunk_plan(t(Wq)) if with_plan else None
+    Y = w8.linear_f16codes(q16, sx, t(Wq), t(sw), t(b) if with_bias else None, plan=plan)
     Xq, wsx = oracle_mod.quant_act(c.X[0], lam)
     np.testing.assert_array_equal(u16(Y), oracle_mod.linear(Xq, wsx, Wq, sw, b))
     Y8 = w8.linear(q16.to(torch.int8), sx, t(Wq), t(sw), t(b) if with_bias else None)
@@ -103,9 +105,95 @@ def test_linear_f16codes_qkv_sampled_rows(w8, oracle_mod):
     lam = oracle_mod.smooth_scales(s, case.W[0], case.alpha)
     Wq, sw = oracle_mod.quantize_weights(case.W[0], lam)
     q16, sx = w8.quant_act_f16codes(bf(case.X[0]), t(lam))
-    Y = u16(w8.linear_f16codes(q16, sx, t(Wq), t(sw), t(case.bias[0])))
+    Y = u16(w8.linear_f16codes(q16, sx, t(Wq), t(sw), t(case.bias[0]), plan=w8.chunk_plan(t(Wq))))
     Xq, wsx = oracle_mod.quant_act(case.X[0], lam)
     np.testing.assert_array_equal(codes(q16), Xq)
     for r in [0, 1, 255, 256, 2047, 4095, 4350, 4607]:
         np.testing.assert_array_equal(Y[r:r + 1], oracle_mod.linear(Xq, wsx, Wq, sw, case.bias[0],
                                                                      rows=(r, r + 1)))
+
+
+# ------------------------------------------------------------------ drain plan
+
+def plan_reference(Wq, limit=1 << 17, kc=1024, rows=256):
+    """The drain plan restated: per block of `rows` weight rows, a run of K
+    chunks ends before chunk c when some row's sum |w| over the run including
+    c would exceed `limit` (then 128 * limit = 2^24 bounds every partial sum of
+    codes |a| <= 128); the last chunk always ends a run.  Bit c of a block's
+    words = a run ends after chunk c."""
+    N, K = Wq.shape
+    nc = -(-K // kc)
+    words = -(-nc // 32)
+    nb = -(-N // rows)
+    a = np.abs(Wq.astype(np.int64))
+    l1 = np.stack([a[:, c * kc:(c + 1) * kc].sum(1) for c in range(nc)], 1)
+    plan = np.zeros((nb, words), np.uint32)
+    for b in range(nb):
+        blk = l1[b * rows:(b + 1) * rows]
+        cur = np.zeros(blk.shape[0], np.int64)
+        for c in range(nc):
+            cand = cur + blk[:, c]
+            if cand.max() > limit:
+                plan[b, (c - 1) // 32] |= np.uint32(1 << ((c - 1) % 32))
+                cur = blk[:, c].copy()
+            else:
+                cur = cand
+        plan[b, (nc - 1) // 32] |= np.uint32(1 << ((nc - 1) % 32))
+    return plan.reshape(-1)
+
+
+def gauss_codes(shape, seed, sigma):
+    rng = np.random.default_rng(seed)
+    return np.clip(np.rint(rng.normal(0, sigma, shape)), -127, 127).astype(np.int8)
+
+
+def plan_cases():
+    rng = np.random.default_rng(11)
+    small = gauss_codes((520, 3 * 1024 + 320), 1, 20.0)             # runs merge
+    uni = rng.integers(-127, 128, (296, 5 * 1024), dtype=np.int8)    # pairs of chunks
+    full = np.full((256, 4096), 127, np.int8)                       # a drain after every chunk
+    mixed = np.concatenate([gauss_codes((256, 8192), 2, 12.0), np.full((200, 8192), -127, np.int8)])
+    many = gauss_codes((296, 40 * 1024), 3, 8.0)                    # two plan words per block
+    return {"small": small, "uniform": uni, "full": full, "mixed": mixed, "many": many}
+
+
+@pytest.mark.parametrize("name", ["small", "uniform", "full", "mixed", "many"])
+def test_chunk_plan_matches_reference(w8, name):
+    Wq = plan_cases()[name]
+    plan = w8.chunk_plan(t(Wq)).cpu().numpy().view(np.uint32)
+    assert plan.size == w8.chunk_plan_size(*Wq.shape)
+    np.testing.assert_array_equal(plan, plan_reference(Wq))
+
+
+def test_chunk_plan_reference_needs_drains_where_fp32_would_round():
+    # (host check of the plan's premise) the all-max block: a single fp32 run
+    # over two chunks of positive products passes 2^24 and rounds, so the
+    # plan must end a run after every chunk there
+    Wq = plan_cases()["full"]
+    assert np.all(plan_reference(Wq) == np.uint32(0b1111))
+    prod = np.full(2048, 127 * 127, np.float32)
+    prod[1::3] = 127 * 125
+    acc = np.float32(0)
+    for v in prod:
+        acc = np.float32(acc + v)
+    assert int(acc) != int(prod.astype(np.int64).sum())
+
+
+@pytest.mark.parametrize("name", ["small", "uniform", "full", "mixed"])
+@pytest.mark.parametrize("with_plan", [True, False])
+def test_gemm_f16codes_i32_exact(w8, name, with_plan):
+    Wq = plan_cases()[name]
+    N, K = Wq.shape
+    M = 300
+    rng = np.random.default_rng(N + K)
+    Xq = rng.integers(-127, 128, (M, K), dtype=np.int8)
+    if name in ("full", "mixed"):
+        # products of one sign and near the maximum: partial sums near 2^24
+        Xq = np.where(rng.random((M, K)) < 0.3, 125, 127).astype(np.int8)
+        if name == "mixed":
+            Xq[:150] = -Xq[:150]
+    q16 = torch.from_numpy(Xq.astype(np.float16)).to(DEV)
+    plan = w8.chunk_plan(t(Wq)) if with_plan else None
+    acc = w8.debug_gemm_f16codes_i32(q16, t(Wq), plan=plan).cpu().numpy()
+    want = Xq.astype(np.int64) @ Wq.astype(np.int64).T
+    np.testing.assert_array_equal(acc, want)
