@@ -166,6 +166,21 @@ __device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t
     asm("sub.f16x2 %0, %0, %1;" : "+r"(hi) : "r"(0x64806480u));
 }
 
+// The int32 value of an fp32 integer v, |v| <= 2^24, without a conversion
+// instruction (those run at a fraction of the add rate, and the MMA waits for
+// the drain): t = v + 1.5 * 2^25 lies in [2^25, 2^26], where fp32 values are
+// 4 apart, so t's bit pattern counts v rounded to a multiple of 4, t - 1.5 *
+// 2^25 is that multiple exactly, and the rest (|lo| <= 2, exact) is read in
+// the low mantissa bits of lo + 1.5 * 2^23.  The bit count stays linear at
+// t = 2^26 (the mantissa carries into the exponent).
+__device__ __forceinline__ int32_t exact_int(uint32_t vb) {
+    const float v = __uint_as_float(vb);
+    const float t = __fadd_rn(v, 50331648.0f);
+    const float lo = __fadd_rn(v, -__fadd_rn(t, -50331648.0f));
+    const uint32_t hi4 = (__float_as_uint(t) - 0x4C400000u) << 2;
+    return static_cast<int32_t>(hi4 + (__float_as_uint(__fadd_rn(lo, 12582912.0f)) - 0x4B400000u));
+}
+
 __device__ __forceinline__ void arrive_leader(uint32_t bar, uint32_t rank) {
     if (rank == 0) mbar_arrive(bar);
     else mbar_arrive_cluster_relaxed(mapa_shared(bar, 0));
@@ -193,39 +208,18 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
             tc_fence_after();
             const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) + h * (PAIR_T / 2);
             // two loads in flight per wait: the MMA is stopped until every
-            // epilogue warp has drained its part
+            // epilogue warp has drained its part, so the values are read with
+            // adds instead of conversion instructions (exact_int)
 #pragma unroll
             for (int jj = 0; jj < RUN / 16; jj += 2) {
                 uint32_t v[2][16];
 #pragma unroll
                 for (int g = 0; g < 2; ++g) tmem_ld_32x32b_x16(base + (jj + g) * 16, v[g]);
                 tmem_ld_wait();
-                // the values are exact integers.  Below 2^22 in magnitude (in
-                // practice always) v + 1.5 * 2^23 holds v in its low mantissa
-                // bits, exactly: one add instead of a conversion instruction,
-                // which runs at a fraction of the add rate and would stall the
-                // MMA for the whole drain.  OR-ing the magnitudes' bit patterns
-                // bounds them all; the exact conversion is the (warp-uniform)
-                // fallback.
-                uint32_t any = 0;
 #pragma unroll
                 for (int g = 0; g < 2; ++g)
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) any |= v[g][i] & 0x7fffffffu;
-                if (__any_sync(0xffffffffu, any >= 0x4A800000u)) {
-#pragma unroll
-                    for (int g = 0; g < 2; ++g)
-#pragma unroll
-                        for (int i = 0; i < 16; ++i)
-                            run[(jj + g) * 16 + i] += __float2int_rn(__uint_as_float(v[g][i]));
-                } else {
-#pragma unroll
-                    for (int g = 0; g < 2; ++g)
-#pragma unroll
-                        for (int i = 0; i < 16; ++i)
-                            run[(jj + g) * 16 + i] += static_cast<int32_t>(
-                                __float_as_uint(__fadd_rn(__uint_as_float(v[g][i]), 12582912.0f)) - 0x4B400000u);
-                }
+                    for (int i = 0; i < 16; ++i) run[(jj + g) * 16 + i] += exact_int(v[g][i]);
             }
             tc_fence_before();
             __syncwarp();
