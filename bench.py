@@ -201,11 +201,12 @@ def run_reference(args):
 
 METRIC = "W8A8 linear INT8 TOPS (act-quant + INT8 GEMM + fused dequant epilogue)"
 
-# DRAM bytes (read + write) of one GEMM launch, keyed by (engine, workload),
-# from the ncu capture summarised in profiles/gemm_tc2_qkv_m4608_k4096_n12288.md;
-# valid only for the kernel version profiled there (removed whenever that
-# kernel changes, until the capture is repeated).
-GEMM_TRAFFIC_BYTES = {(2, "qkv_m4608_k4096_n12288"): 147.97e6}
+# DRAM bytes (read + write) of one GEMM launch, keyed by (kernel, workload),
+# from the ncu captures summarised under profiles/ (gemm_tc2_*.md for the
+# int8-code engine, gemm_ts_*.md for the fp16-code one); valid only for the
+# kernel version profiled there (removed whenever that kernel changes, until
+# the capture is repeated).
+GEMM_TRAFFIC_BYTES = {("tc2", "qkv_m4608_k4096_n12288"): 147.97e6}
 
 
 # --------------------------------------------------------------------- ours
@@ -239,7 +240,8 @@ def run_ours(args):
     bias = torch.from_numpy(case.bias[0]).to(dev)
 
     # offline: calibration statistic, smoothing vector, weight quantization
-    e = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    # and the weights' drain plan
+    e = [torch.cuda.Event(enable_timing=True) for _ in range(5)]
     e[0].record()
     s = w8a8.channel_absmax(X_cal)
     e[1].record()
@@ -247,29 +249,48 @@ def run_ours(args):
     e[2].record()
     Wq, sw = w8a8.quantize_weights(W, lam)
     e[3].record()
+    plan = w8a8.chunk_plan(Wq)
+    e[4].record()
     torch.cuda.synchronize()
     offline = {"channel_absmax": e[0].elapsed_time(e[1]), "smooth_scales": e[1].elapsed_time(e[2]),
-               "quantize_weights": e[2].elapsed_time(e[3])}
+               "quantize_weights": e[2].elapsed_time(e[3]), "chunk_plan": e[3].elapsed_time(e[4])}
+
+    # the activation codes' container: fp16 values (the default: the GEMM
+    # takes them without conversion) or int8
+    f16 = args.codes == "f16"
+    code_bytes = 2 if f16 else 1
 
     # rotate input sets so the bytes touched between two uses of one set
     # exceed L2 (no flush needed): each set holds its own X and Wq copy
-    set_bytes = 2 * M * K + M * K + N * K + 2 * M * N
+    set_bytes = 2 * M * K + code_bytes * M * K + N * K + 2 * M * N
     n_sets = max(2, math.ceil(2 * L2_BYTES / set_bytes))
     X0 = bf(case.X[0])
     Xs = [X0] + [X0.clone() for _ in range(n_sets - 1)]
     Wqs = [Wq] + [Wq.clone() for _ in range(n_sets - 1)]
-    Xqs = [torch.empty(M, K, dtype=torch.int8, device=dev) for _ in range(n_sets)]
+    Xqs = [torch.empty(M, K, dtype=torch.float16 if f16 else torch.int8, device=dev) for _ in range(n_sets)]
     sxs = [torch.empty(M, dtype=torch.float32, device=dev) for _ in range(n_sets)]
     Ys = [torch.empty(M, N, dtype=torch.bfloat16, device=dev) for _ in range(n_sets)]
+
+    def quant(j, st):
+        if f16:
+            w8a8.quant_act_f16codes(Xs[j], lam, Xq16=Xqs[j], x_scale=sxs[j], stream=st)
+        else:
+            w8a8.quant_act(Xs[j], lam, Xq=Xqs[j], x_scale=sxs[j], stream=st)
+
+    def gemm(j, st):
+        if f16:
+            w8a8.linear_f16codes(Xqs[j], sxs[j], Wqs[j], sw, bias, Y=Ys[j], plan=plan, stream=st)
+        else:
+            w8a8.linear(Xqs[j], sxs[j], Wqs[j], sw, bias, Y=Ys[j], stream=st)
 
     def step(i, ev=None):
         j = i % n_sets
         if ev is not None:
             ev[0].record(stream)
-        w8a8.quant_act(Xs[j], lam, Xq=Xqs[j], x_scale=sxs[j], stream=stream)
+        quant(j, stream)
         if ev is not None:
             ev[1].record(stream)
-        w8a8.linear(Xqs[j], sxs[j], Wqs[j], sw, bias, Y=Ys[j], stream=stream)
+        gemm(j, stream)
         if ev is not None:
             ev[2].record(stream)
 
@@ -317,7 +338,8 @@ def run_ours(args):
     e2e_steps = max(4, min(args.steps, 10))
     depth = 2
     Y_hosts = [torch.empty(M, N, dtype=torch.bfloat16).pin_memory() for _ in range(depth)]
-    runner = StreamedLinear(M, K, N, lam, Wq, sw, bias, depth=depth, device=dev)
+    runner = StreamedLinear(M, K, N, lam, Wq, sw, bias, depth=depth, device=dev,
+                            plan=plan if f16 else None, codes=args.codes)
     runner.run([X_host] * depth, Y_hosts)
     runner.synchronize()
     torch.cuda.synchronize()
@@ -337,7 +359,8 @@ def run_ours(args):
 
     def e2e_serial_step():
         Xd.copy_(X_host, non_blocking=True)
-        Y = w8a8.quantized_linear_forward(Xd, lam, Wq, sw, bias, stream=stream)
+        Y = w8a8.quantized_linear_forward(Xd, lam, Wq, sw, bias, plan=plan if f16 else None,
+                                          codes=args.codes, stream=stream)
         Y_host.copy_(Y, non_blocking=True)
 
     for _ in range(2):
@@ -372,10 +395,26 @@ def run_ours(args):
         torch.cuda.synchronize()
         return a0.elapsed_time(a1) / reps
 
-    quant_iso = isolated(lambda i, st: w8a8.quant_act(Xs[i % n_sets], lam, Xq=Xqs[i % n_sets],
-                                                      x_scale=sxs[i % n_sets], stream=st), 40)
-    gemm_iso = isolated(lambda i, st: w8a8.linear(Xqs[i % n_sets], sxs[i % n_sets], Wqs[i % n_sets],
-                                                  sw, bias, Y=Ys[i % n_sets], stream=st), 10)
+    quant_iso = isolated(lambda i, st: quant(i % n_sets, st), 40)
+    gemm_iso = isolated(lambda i, st: gemm(i % n_sets, st), 10)
+
+    # the other container of the codes, alone in graphs on the same
+    # workload: a3 and the GEMM of the int8-code path (the codes as the
+    # paper stores them) when the step runs fp16 codes, and the other way
+    # round
+    Xq_o = [torch.empty(M, K, dtype=torch.int8 if f16 else torch.float16, device=dev) for _ in range(2)]
+    if f16:
+        other_quant = isolated(lambda i, st: w8a8.quant_act(Xs[i % n_sets], lam, Xq=Xq_o[i % 2],
+                                                            x_scale=sxs[i % n_sets], stream=st), 40)
+        other_gemm = isolated(lambda i, st: w8a8.linear(Xq_o[i % 2], sxs[i % n_sets], Wqs[i % n_sets], sw,
+                                                        bias, Y=Ys[i % n_sets], stream=st), 10)
+    else:
+        other_quant = isolated(lambda i, st: w8a8.quant_act_f16codes(Xs[i % n_sets], lam, Xq16=Xq_o[i % 2],
+                                                                     x_scale=sxs[i % n_sets], stream=st), 40)
+        other_gemm = isolated(lambda i, st: w8a8.linear_f16codes(Xq_o[i % 2], sxs[i % n_sets],
+                                                                 Wqs[i % n_sets], sw, bias, Y=Ys[i % n_sets],
+                                                                 plan=plan, stream=st), 10)
+    del Xq_o
 
     # the pieces around the layer, each alone in a CUDA graph on the same
     # workload: the protected bf16 linear, the statistics pass of fragility
@@ -389,9 +428,11 @@ def run_ours(args):
     stats_iso = isolated(lambda i, st: w8a8.act_stats_update(Xs[i % n_sets], st_sums, st_max,
                                                              stream=st), 40)
     amax = torch.empty(1, dtype=torch.float32, device=dev)
-    pt_iso = isolated(lambda i, st: w8a8.quant_act_per_tensor(Xs[i % n_sets], lam, Xq=Xqs[i % n_sets],
+    Xq8 = [torch.empty(M, K, dtype=torch.int8, device=dev) for _ in range(2)]
+    pt_iso = isolated(lambda i, st: w8a8.quant_act_per_tensor(Xs[i % n_sets], lam, Xq=Xq8[i % 2],
                                                               x_scale=sxs[i % n_sets], amax=amax,
                                                               stream=st), 40)
+    del Xq8
     # a3 fused with its neighbours: both branches of the dual-branch workload
     # (4608 x 4096 each) in one launch against two launches, and GELU folded
     # into the quantization of the FFN down-projection input (4608 x 16384)
@@ -431,9 +472,11 @@ def run_ours(args):
     quant_avg = sum(quant_ms) / len(quant_ms)
     gemm_tflops = ops_step / (gemm_avg * 1e-3) / 1e12
     engine = w8a8.get_gemm_engine()
+    engine_name = "ts" if f16 else {2: "tc2", 1: "tc", 0: "mma"}[engine]
     peak_t = peaks["bf16_tflops"]
-    quant_bytes = 3.0 * M * K + 4.0 * M + 4.0 * K
+    quant_bytes = (2.0 + code_bytes) * M * K + 4.0 * M + 4.0 * K
     quant_gbs = quant_bytes / (quant_iso * 1e-3) / 1e9
+    other_bytes = (2.0 + 3 - code_bytes) * M * K + 4.0 * M + 4.0 * K
 
     line = None
     if rank == 0:
@@ -450,19 +493,32 @@ def run_ours(args):
             "config": {"workload": args.workload, "M": M, "K": K, "N": N, "alpha": case.alpha,
                        "l2": f"{n_sets} rotating input sets of {set_bytes / 2**20:.0f} MiB "
                              f"(> L2 between reuses), no flush",
-                       "gemm_engine": {2: "tcgen05 cta pair", 1: "tcgen05", 0: "mma.sync"}[engine]},
+                       "codes": f"{args.codes} container of the int8 activation codes",
+                       "gemm_engine": {"ts": "tcgen05 cta pair, weights in TMEM, drain plan",
+                                       "tc2": "tcgen05 cta pair", "tc": "tcgen05",
+                                       "mma": "mma.sync"}[engine_name]},
             "roofline": {"bound": "tensor", "achieved": gemm_tflops, "peak": peak_t,
                          "unit": "TFLOP/s", "frac": gemm_tflops / peak_t,
-                         "traffic": GEMM_TRAFFIC_BYTES.get((engine, args.workload)),
+                         "traffic": GEMM_TRAFFIC_BYTES.get((engine_name, args.workload)),
                          "traffic_unit": "bytes per launch (ncu dram read + write)",
-                         "algorithmic_bytes": float(M * K + N * K + 2 * M * N + 4 * (M + 2 * N)),
-                         "kernel": "w8a8_linear (a4+a5)",
+                         "algorithmic_bytes": float(code_bytes * M * K + N * K + 2 * M * N
+                                                    + 4 * (M + 2 * N)),
+                         "kernel": "w8a8_linear_f16codes (a4+a5)" if f16 else "w8a8_linear (a4+a5)",
                          "peak_source": f"{peak_kind} bf16 dense burst (the fp16/bf16 tensor "
                                         f"datapath the exact-integer GEMM runs on)"},
             "act_quant": {"bound": "hbm", "achieved": quant_gbs, "peak": peaks["hbm_gbs"],
                           "unit": "GB/s", "frac": quant_gbs / peaks["hbm_gbs"],
                           "ms_isolated": quant_iso, "ms_in_step": quant_avg, "bytes": quant_bytes,
-                          "kernel": "w8a8_quant_act (a3)"},
+                          "kernel": "w8a8_quant_act_f16codes (a3)" if f16 else "w8a8_quant_act (a3)"},
+            "other_codes": {
+                "codes": "int8" if f16 else "f16",
+                "step_ms_isolated": other_quant + other_gemm,
+                "value": ops_step / ((other_quant + other_gemm) * 1e-3) / 1e12,
+                "gemm_tflops": ops_step / (other_gemm * 1e-3) / 1e12,
+                "act_quant_gbs": other_bytes / (other_quant * 1e-3) / 1e9,
+                "kernels": "w8a8_quant_act + w8a8_linear" if f16
+                           else "w8a8_quant_act_f16codes + w8a8_linear_f16codes",
+                "unit": "TOPS (value), TFLOP/s, GB/s; sum of the two kernels each alone in a graph"},
             "protect": {
                 "linear_bf16": {"bound": "tensor", "achieved": ops_step / (bf16_iso * 1e-3) / 1e12,
                                 "peak": peak_t, "unit": "TFLOP/s",
@@ -524,7 +580,10 @@ def main(argv=None):
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="qkv_m4608_k4096_n12288")
-    p.add_argument("--engine", type=int, default=None, help="1 tcgen05, 0 mma.sync")
+    p.add_argument("--engine", type=int, default=None,
+                   help="int8 codes: 2 tcgen05 pairs (default), 1 tcgen05, 0 mma.sync")
+    p.add_argument("--codes", choices=["f16", "int8"], default="f16",
+                   help="container of the activation codes between a3 and the GEMM")
     p.add_argument("--no-cpu-baseline", action="store_true")
     p.add_argument("--cpu-seconds", type=float, default=10.0)
     args = p.parse_args(argv)

@@ -24,13 +24,19 @@ class StreamedLinear:
     outputs."""
 
     def __init__(self, M: int, K: int, N: int, smooth, Wq, w_scale, bias=None, depth: int = 2,
-                 device=None):
+                 device=None, plan=None, codes: str = "f16"):
+        """codes: "f16" (a3 writes the codes as fp16 values and the GEMM takes
+        them unconverted; plan = ``w8a8.chunk_plan(Wq)`` or None) or "int8"."""
+        if codes not in ("f16", "int8"):
+            raise ValueError("codes must be 'f16' or 'int8'")
         self.M, self.K, self.N = M, K, N
         self.smooth, self.Wq, self.w_scale, self.bias = smooth, Wq, w_scale, bias
+        self.plan, self.f16 = plan, codes == "f16"
         dev = device if device is not None else Wq.device
         self.depth = depth
         self.X = [torch.empty(M, K, dtype=torch.bfloat16, device=dev) for _ in range(depth)]
-        self.Xq = [torch.empty(M, K, dtype=torch.int8, device=dev) for _ in range(depth)]
+        self.Xq = [torch.empty(M, K, dtype=torch.float16 if self.f16 else torch.int8, device=dev)
+                   for _ in range(depth)]
         self.sx = [torch.empty(M, dtype=torch.float32, device=dev) for _ in range(depth)]
         self.Y = [torch.empty(M, N, dtype=torch.bfloat16, device=dev) for _ in range(depth)]
         self.up = torch.cuda.Stream(device=dev)
@@ -60,10 +66,19 @@ class StreamedLinear:
                 self.comp.wait_event(self.x_ready[s])
                 if self.started[s]:
                     self.comp.wait_event(self.y_free[s])
-                w8a8.quant_act(self.X[s], self.smooth, Xq=self.Xq[s], x_scale=self.sx[s], stream=self.comp)
+                if self.f16:
+                    w8a8.quant_act_f16codes(self.X[s], self.smooth, Xq16=self.Xq[s], x_scale=self.sx[s],
+                                            stream=self.comp)
+                else:
+                    w8a8.quant_act(self.X[s], self.smooth, Xq=self.Xq[s], x_scale=self.sx[s],
+                                   stream=self.comp)
                 self.x_free[s].record(self.comp)
-                w8a8.linear(self.Xq[s], self.sx[s], self.Wq, self.w_scale, self.bias, Y=self.Y[s],
-                            stream=self.comp)
+                if self.f16:
+                    w8a8.linear_f16codes(self.Xq[s], self.sx[s], self.Wq, self.w_scale, self.bias,
+                                         Y=self.Y[s], plan=self.plan, stream=self.comp)
+                else:
+                    w8a8.linear(self.Xq[s], self.sx[s], self.Wq, self.w_scale, self.bias, Y=self.Y[s],
+                                stream=self.comp)
                 self.y_ready[s].record(self.comp)
             with torch.cuda.stream(self.down):
                 self.down.wait_event(self.y_ready[s])

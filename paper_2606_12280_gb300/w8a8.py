@@ -475,7 +475,15 @@ def select_protected(scores, n_protect: int):
     return [int(f) for f in flags]
 
 
-def quantized_linear_forward(X, smooth, Wq, w_scale, bias=None, stream=None):
-    """The per-call hot path of one quantized linear: a3 then a4+a5."""
+def quantized_linear_forward(X, smooth, Wq, w_scale, bias=None, plan=None, codes="f16", stream=None):
+    """The per-call hot path of one quantized linear: a3 then a4+a5.  codes:
+    "f16" (the codes as fp16 values, the faster GEMM; K <= 16384, else the
+    int8 container is used) or "int8"; plan: ``chunk_plan(Wq)`` or None (used
+    with fp16 codes)."""
+    if codes not in ("f16", "int8"):
+        raise ValueError("codes must be 'f16' or 'int8'")
+    if codes == "f16" and X.shape[1] <= 16384:
+        Xq16, sx = quant_act_f16codes(X, smooth, stream=stream)
+        return linear_f16codes(Xq16, sx, Wq, w_scale, bias, plan=plan, stream=stream)
     Xq, sx = quant_act(X, smooth, stream=stream)
     return linear(Xq, sx, Wq, w_scale, bias, stream=stream)

@@ -10,7 +10,8 @@ from paper_2606_12280_gb300 import workloads as wl
 pytestmark = pytest.mark.gpu
 
 
-def test_streamed_matches_direct():
+@pytest.mark.parametrize("codes", ["f16", "int8"])
+def test_streamed_matches_direct(codes):
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     from paper_2606_12280_gb300 import w8a8
@@ -26,10 +27,14 @@ def test_streamed_matches_direct():
     batches = [torch.from_numpy(wl.random_bf16((M, K), seed=100 + i, scale=1.0 + i).view(np.int16))
                .view(torch.bfloat16).pin_memory() for i in range(5)]
     outs = [torch.empty(M, N, dtype=torch.bfloat16).pin_memory() for _ in range(5)]
-    r = StreamedLinear(M, K, N, lam, Wq, sw, bias, depth=2)
+    plan = w8a8.chunk_plan(Wq) if codes == "f16" else None
+    r = StreamedLinear(M, K, N, lam, Wq, sw, bias, depth=2, plan=plan, codes=codes)
     r.run(batches, outs)
     r.synchronize()
     for xh, yh in zip(batches, outs):
-        want = w8a8.quantized_linear_forward(xh.to(dev), lam, Wq, sw, bias)
+        want = w8a8.quantized_linear_forward(xh.to(dev), lam, Wq, sw, bias, plan=plan, codes=codes)
+        other = w8a8.quantized_linear_forward(xh.to(dev), lam, Wq, sw, bias,
+                                              codes="int8" if codes == "f16" else "f16")
         torch.cuda.synchronize()
         assert torch.equal(yh, want.cpu())
+        assert torch.equal(want, other)
