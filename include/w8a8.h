@@ -176,10 +176,13 @@ W8A8_API w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int
  * W8A8_ERR_UNSUPPORTED_SHAPE.  Writes 2MK + 4M bytes (one MK more than a3).
  *   X [M,K] bf16, smooth [K] fp32 or NULL, read.
  *   Xq16 [M,K] fp16 codes (uint16 bit patterns), x_scale [M] fp32, written.
+ *   x_sumsq [M] uint32 or NULL: if given, sum_j Xq_mj^2 per token, written
+ *     (exact; no counterpart in the paper: w8a8_linear_f16codes uses it to
+ *     bound its partial sums).
  */
 W8A8_API w8a8_status w8a8_quant_act_f16codes(const uint16_t *X, const float *smooth, int M,
-                                             int K, uint16_t *Xq16, float *x_scale, int gelu,
-                                             void *stream);
+                                             int K, uint16_t *Xq16, float *x_scale,
+                                             uint32_t *x_sumsq, int gelu, void *stream);
 
 /*
  * a4 + a5 with the activation codes as fp16 values (from
@@ -192,20 +195,28 @@ W8A8_API w8a8_status w8a8_quant_act_f16codes(const uint16_t *X, const float *smo
  *     (same N, K); with it the integer sums are drained from the fp32
  *     accumulator only where the weights require it (see w8a8_chunk_plan).
  *     A plan of other weights voids the exactness guarantee.
+ *   x_sumsq: NULL, or the per-token sums of squared codes that
+ *     w8a8_quant_act_f16codes wrote with these Xq16 (used with a plan): an
+ *     output tile (256 tokens x 256 features) whose largest token sum times
+ *     its largest weight-row sum of squares is at most 2^48 has every partial
+ *     sum within 2^24 (Cauchy-Schwarz) and is accumulated without a drain.
+ *     Sums of other codes void the exactness guarantee.
  * Uses the CTA-pair engine whatever w8a8_set_gemm_engine says.
  */
 W8A8_API w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale,
                                           const int8_t *Wq, const float *w_scale,
                                           const float *bias, int M, int N, int K,
-                                          const uint32_t *chunk_plan, uint16_t *Y, void *stream);
+                                          const uint32_t *chunk_plan, const uint32_t *x_sumsq,
+                                          uint16_t *Y, void *stream);
 
 /*
  * Test export of the product above alone: acc = Xq16 Wq^T as int32 [M,N],
- * written.  Same shape rules and plan.
+ * written.  Same shape rules, plan and token sums.
  */
 W8A8_API w8a8_status w8a8_debug_gemm_f16codes_i32(const uint16_t *Xq16, const int8_t *Wq, int M,
                                                   int N, int K, const uint32_t *chunk_plan,
-                                                  int32_t *acc, void *stream);
+                                                  const uint32_t *x_sumsq, int32_t *acc,
+                                                  void *stream);
 
 /*
  * Drain plan of an int8 weight matrix for w8a8_linear_f16codes (no
@@ -216,8 +227,9 @@ W8A8_API w8a8_status w8a8_debug_gemm_f16codes_i32(const uint16_t *Xq16, const in
  * it, so a run of K chunks (1024 each) can accumulate without a drain while
  * every weight row of a 256-row block has sum |w_k| <= 2^17 over the run.
  * The plan records, per 256-row block, after which chunks the run ends (the
- * worst case, |w| = 127 everywhere, ends it after every chunk).  Computed
- * once per weight matrix; its layout is internal to the library.
+ * worst case, |w| = 127 everywhere, ends it after every chunk), and the
+ * block's largest row sum of squares (for the x_sumsq bound).  Computed once
+ * per weight matrix; its layout is internal to the library.
  *   w8a8_chunk_plan_size: the number of uint32 words of the plan (>= 1).
  *   Wq [N,K] int8, read;  plan [w8a8_chunk_plan_size(N, K)] uint32, written.
  */

@@ -199,25 +199,28 @@ w8a8_status w8a8_debug_gelu(const uint16_t *H, int n, float *G, void *stream) {
 }
 
 w8a8_status w8a8_quant_act_f16codes(const uint16_t *X, const float *smooth, int M, int K,
-                                    uint16_t *Xq16, float *x_scale, int gelu, void *stream) {
+                                    uint16_t *Xq16, float *x_scale, uint32_t *x_sumsq, int gelu,
+                                    void *stream) {
     if (w8a8_status e = check_mk(M, K)) return e;
     if (K > 16384) return W8A8_ERR_UNSUPPORTED_SHAPE;
     if (M == 0) return W8A8_OK;
     if (!X || !Xq16 || !x_scale) return W8A8_ERR_INVALID_ARG;
-    if (!aligned16(X) || !aligned16(Xq16) || !aligned16(x_scale) || (smooth && !aligned16(smooth)))
+    if (!aligned16(X) || !aligned16(Xq16) || !aligned16(x_scale) || (smooth && !aligned16(smooth)) ||
+        (x_sumsq && !aligned16(x_sumsq)))
         return W8A8_ERR_MISALIGNED;
-    return from_cuda(w8a8::launch_quant_act_f16codes(X, smooth, M, K, Xq16, x_scale, gelu != 0,
+    return from_cuda(w8a8::launch_quant_act_f16codes(X, smooth, M, K, Xq16, x_scale, x_sumsq, gelu != 0,
                                                      as_stream(stream)));
 }
 
 w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale, const int8_t *Wq,
                                  const float *w_scale, const float *bias, int M, int N, int K,
-                                 const uint32_t *chunk_plan, uint16_t *Y, void *stream) {
+                                 const uint32_t *chunk_plan, const uint32_t *x_sumsq, uint16_t *Y,
+                                 void *stream) {
     if (w8a8_status e = check_nk(N, K)) return e;
     if (w8a8_status e = check_mk(M, K)) return e;
-    w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), x_scale, Wq, w_scale, bias, Y, M};
+    w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), x_scale, Wq, w_scale, bias, Y, M, x_sumsq};
     if (w8a8_status e = check_branch(b, true, N, K)) return e;
-    if (chunk_plan && !aligned16(chunk_plan)) return W8A8_ERR_MISALIGNED;
+    if ((chunk_plan && !aligned16(chunk_plan)) || (x_sumsq && !aligned16(x_sumsq))) return W8A8_ERR_MISALIGNED;
     if (M == 0) return W8A8_OK;
     unsigned int *err = device_error_word();
     if (!err) return W8A8_ERR_CUDA;
@@ -225,12 +228,13 @@ w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale, con
 }
 
 w8a8_status w8a8_debug_gemm_f16codes_i32(const uint16_t *Xq16, const int8_t *Wq, int M, int N, int K,
-                                         const uint32_t *chunk_plan, int32_t *acc, void *stream) {
+                                         const uint32_t *chunk_plan, const uint32_t *x_sumsq, int32_t *acc,
+                                         void *stream) {
     if (w8a8_status e = check_nk(N, K)) return e;
     if (w8a8_status e = check_mk(M, K)) return e;
-    w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), nullptr, Wq, nullptr, nullptr, acc, M};
+    w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), nullptr, Wq, nullptr, nullptr, acc, M, x_sumsq};
     if (w8a8_status e = check_branch(b, false, N, K)) return e;
-    if (chunk_plan && !aligned16(chunk_plan)) return W8A8_ERR_MISALIGNED;
+    if ((chunk_plan && !aligned16(chunk_plan)) || (x_sumsq && !aligned16(x_sumsq))) return W8A8_ERR_MISALIGNED;
     if (M == 0) return W8A8_OK;
     unsigned int *err = device_error_word();
     if (!err) return W8A8_ERR_CUDA;

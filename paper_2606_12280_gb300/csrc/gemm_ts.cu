@@ -100,7 +100,9 @@ constexpr uint32_t BAR_SEMPTY = BAR_SFULL + 8 * SA;          // MMA done with th
 constexpr uint32_t BAR_ACCFULL = BAR_SEMPTY + 8 * SA;        // chunk accumulated
 constexpr uint32_t BAR_ACCEMPTY = BAR_ACCFULL + 8;           // leader: chunk drained
 constexpr uint32_t BAR_DRAIN = BAR_ACCEMPTY + 8;
-constexpr uint32_t OFF_TMEM = BAR_DRAIN + 8;
+constexpr uint32_t BAR_TFLAG = BAR_DRAIN + 8;              // a tile's single-run flag published
+constexpr uint32_t OFF_TFLAG = BAR_TFLAG + 16;             // the flags (two tiles in flight)
+constexpr uint32_t OFF_TMEM = OFF_TFLAG + 8;
 constexpr uint32_t OFF_ABORT = OFF_TMEM + 4;
 constexpr uint32_t SMEM_BARRIERS = 512;
 static_assert(OFF_ABORT + 4 - OFF_BAR <= SMEM_BARRIERS, "barrier area");
@@ -116,6 +118,7 @@ struct BranchArgs {
     const float *w_scale;
     const float *bias;
     void *out;
+    const uint32_t *x_sumsq;   // per token sum of squared codes, or null
     int M;           // tokens
     int t_tiles;     // token tiles of 256
     int tiles;       // t_tiles * feature tiles
@@ -130,7 +133,10 @@ struct Params {
     // plan_words words of bits, bit c set = drain after K chunk c; null =
     // drain after every chunk
     const uint32_t *plan;
-    int plan_words;
+    int plan_words;            // per block: the drain bits, then the block's max sum of squares
+    // plan and every branch's x_sumsq given: tiles whose activation and weight
+    // norms bound every partial sum run without an intermediate drain
+    int single_ok;
     unsigned int *err;
     uint64_t wait_limit_ns;
 };
@@ -158,6 +164,23 @@ __device__ __forceinline__ bool plan_drains(const Params &p, int fb, int ci, int
     return (__ldg(p.plan + (size_t)fb * p.plan_words + (ci >> 5)) >> (ci & 31)) & 1u;
 }
 
+// Can tile t run without an intermediate drain?  Every partial sum P over a
+// subset S of K obeys |P| <= ||a_S|| ||w_S|| <= ||a|| ||w|| (Cauchy-Schwarz),
+// so max_t ||a_t||^2 * max_f ||w_f||^2 <= 2^48 over the tile's 256 tokens and
+// 256 weight rows keeps every one within 2^24, exact in fp32.  Warp-wide: all
+// lanes take part.
+__device__ __forceinline__ bool tile_single_run(const Params &p, int t, int lane) {
+    const Tile tl = tile_coords(p, t);
+    const BranchArgs &br = p.br[tl.branch];
+    uint32_t m = 0;
+#pragma unroll
+    for (int i = lane; i < PAIR_T; i += 32)
+        if (tl.t0 + i < br.M) m = max(m, __ldg(br.x_sumsq + tl.t0 + i));
+    m = __reduce_max_sync(0xffffffffu, m);
+    const uint32_t wm = __ldg(p.plan + (size_t)(tl.f0 / PAIR_F) * p.plan_words + p.plan_words - 1);
+    return static_cast<uint64_t>(m) * wm <= (1ull << 48);
+}
+
 __device__ __forceinline__ void i8x4_to_f16x4(uint32_t w, uint32_t &lo, uint32_t &hi) {
     const uint32_t u = w ^ 0x80808080u;
     asm("prmt.b32 %0, %1, %2, 0x4140;" : "=r"(lo) : "r"(u), "r"(0x64646464u));
@@ -181,6 +204,23 @@ __device__ __forceinline__ int32_t exact_int(uint32_t vb) {
     return static_cast<int32_t>(hi4 + (__float_as_uint(__fadd_rn(lo, 12582912.0f)) - 0x4B400000u));
 }
 
+// exact_int of two values at once with packed fp32 adds (same steps).
+__device__ __forceinline__ void exact_int2(uint32_t v0, uint32_t v1, int32_t &r0, int32_t &r1) {
+    uint64_t v, t, h, lo, m;
+    asm("mov.b64 %0, {%1, %2};" : "=l"(v) : "r"(v0), "r"(v1));
+    const uint64_t C = 0x4C4000004C400000ull, NC = 0xCC400000CC400000ull, M = 0x4B4000004B400000ull,
+                   NEG1 = 0xBF800000BF800000ull;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(t) : "l"(v), "l"(C));
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(h) : "l"(t), "l"(NC));
+    asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(lo) : "l"(h), "l"(NEG1), "l"(v));
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(m) : "l"(lo), "l"(M));
+    uint32_t t0, t1, m0, m1;
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(t0), "=r"(t1) : "l"(t));
+    asm("mov.b64 {%0, %1}, %2;" : "=r"(m0), "=r"(m1) : "l"(m));
+    r0 = static_cast<int32_t>(((t0 - 0x4C400000u) << 2) + (m0 - 0x4B400000u));
+    r1 = static_cast<int32_t>(((t1 - 0x4C400000u) << 2) + (m1 - 0x4B400000u));
+}
+
 __device__ __forceinline__ void arrive_leader(uint32_t bar, uint32_t rank) {
     if (rank == 0) mbar_arrive(bar);
     else mbar_arrive_cluster_relaxed(mapa_shared(bar, 0));
@@ -194,13 +234,27 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
     const int h = (warp - 8) >> 2;     // token half of the 256-wide tile
     uint32_t c = 0;                    // drains so far
     bool ok = true;
-    for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+    // single-run tiles: every warp decides for itself (the same inputs give
+    // the same answer in both CTAs); warp 8 of the leader publishes the
+    // answer for the MMA thread, one tile ahead, so it never waits for it
+    const bool use_single = p.single_ok != 0;
+    const bool publisher = use_single && rank == 0 && warp == 8;
+    auto publish = [&](int n, bool v) {
+        if (publisher && lane == 0) {
+            st_shared_s32(sb + OFF_TFLAG + 4 * (n & 1), v ? 1 : 0);
+            mbar_arrive(sb + BAR_TFLAG + 8 * (n & 1));
+        }
+    };
+    bool single = use_single && pair < p.total_tiles && tile_single_run(p, pair, lane);
+    if (pair < p.total_tiles) publish(0, single);
+    int n = 0;                         // tiles so far
+    for (int t = pair; ok && t < p.total_tiles; t += npairs, ++n) {
         const int fb = tile_coords(p, t).f0 / PAIR_F;
         int32_t run[RUN];
 #pragma unroll
         for (int i = 0; i < RUN; ++i) run[i] = 0;
         for (int ci = 0; ci < NC; ++ci) {
-            if (!plan_drains(p, fb, ci, NC)) continue;
+            if (ci != NC - 1 && (single || !plan_drains(p, fb, ci, NC))) continue;
             if (!mbar_wait_cluster(sb + BAR_ACCFULL, c & 1, wc, ERR_EPILOGUE)) {
                 ok = false;
                 break;
@@ -208,18 +262,39 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
             tc_fence_after();
             const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) + h * (PAIR_T / 2);
             // two loads in flight per wait: the MMA is stopped until every
-            // epilogue warp has drained its part, so the values are read with
+            // epilogue warp has drained its part.  A tile's only run is kept
+            // as fp32 (its values are the exact integers, and (float)acc is
+            // all the epilogue needs); otherwise the values are read with
             // adds instead of conversion instructions (exact_int)
+            if (single) {
 #pragma unroll
-            for (int jj = 0; jj < RUN / 16; jj += 2) {
-                uint32_t v[2][16];
+                for (int jj = 0; jj < RUN / 16; jj += 4) {
+                    uint32_t v[4][16];
 #pragma unroll
-                for (int g = 0; g < 2; ++g) tmem_ld_32x32b_x16(base + (jj + g) * 16, v[g]);
-                tmem_ld_wait();
+                    for (int g = 0; g < 4; ++g) tmem_ld_32x32b_x16(base + (jj + g) * 16, v[g]);
+                    tmem_ld_wait();
 #pragma unroll
-                for (int g = 0; g < 2; ++g)
+                    for (int g = 0; g < 4; ++g)
 #pragma unroll
-                    for (int i = 0; i < 16; ++i) run[(jj + g) * 16 + i] += exact_int(v[g][i]);
+                        for (int i = 0; i < 16; ++i) run[(jj + g) * 16 + i] = static_cast<int32_t>(v[g][i]);
+                }
+            } else {
+#pragma unroll
+                for (int jj = 0; jj < RUN / 16; jj += 2) {
+                    uint32_t v[2][16];
+#pragma unroll
+                    for (int g = 0; g < 2; ++g) tmem_ld_32x32b_x16(base + (jj + g) * 16, v[g]);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int g = 0; g < 2; ++g)
+#pragma unroll
+                        for (int i = 0; i < 16; i += 2) {
+                            int32_t r0, r1;
+                            exact_int2(v[g][i], v[g][i + 1], r0, r1);
+                            run[(jj + g) * 16 + i] += r0;
+                            run[(jj + g) * 16 + i + 1] += r1;
+                        }
+                }
             }
             tc_fence_before();
             __syncwarp();
@@ -227,6 +302,24 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
             ++c;
         }
         if (!ok) break;
+        // the next tile's decision, before this tile's stores
+        const bool raw = single;
+        if (use_single) {
+            const int tn = t + npairs;
+            single = tn < p.total_tiles && tile_single_run(p, tn, lane);
+            if (tn < p.total_tiles) publish(n + 1, single);
+        }
+        // one representation for the stores: int32 for the int32 export,
+        // fp32 (the exact value, |acc| <= 2^24 or rounded as (float)acc)
+        // for the dequantized output
+#pragma unroll
+        for (int i = 0; i < RUN; ++i) {
+            if (OUT_I32) {
+                if (raw) run[i] = exact_int(static_cast<uint32_t>(run[i]));
+            } else if (!raw) {
+                run[i] = static_cast<int32_t>(__float_as_uint(__int2float_rn(run[i])));
+            }
+        }
         const Tile tl = tile_coords(p, t);
         const BranchArgs &br = p.br[tl.branch];
         const int f = tl.f0 + static_cast<int>(rank) * CTA_F + q * 32 + lane;   // output feature
@@ -278,8 +371,10 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
                                           __uint_as_float(s4.w)};
 #pragma unroll
                     for (int u = 0; u < 4; u += 2) {
-                        const uint32_t y0 = epilogue_value(run[i + u], sxv[u], sw, b, hb);
-                        const uint32_t y1 = epilogue_value(run[i + u + 1], sxv[u + 1], sw, b, hb);
+                        const uint32_t y0 = epilogue_value_f(__uint_as_float(static_cast<uint32_t>(run[i + u])),
+                                                             sxv[u], sw, b, hb);
+                        const uint32_t y1 = epilogue_value_f(__uint_as_float(static_cast<uint32_t>(run[i + u + 1])),
+                                                             sxv[u + 1], sw, b, hb);
                         const uint32_t other = __shfl_xor_sync(0xffffffffu, odd ? y0 : y1, 1);
                         const int tk = i + u + (odd ? 1 : 0);
                         if (paired) {
@@ -326,6 +421,8 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
         mbar_init(sb + BAR_ACCFULL, 1);
         mbar_init(sb + BAR_ACCEMPTY, 2 * NUM_EPI_WARPS);
         mbar_init(sb + BAR_DRAIN, 1);
+        mbar_init(sb + BAR_TFLAG, 1);
+        mbar_init(sb + BAR_TFLAG + 8, 1);
         st_shared_s32(sb + OFF_ABORT, 0);
         fence_barrier_init();
     }
@@ -413,10 +510,18 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
             // ------------------------------------------- MMA issue (leader)
             if (lane == 0 && leader) {
                 constexpr uint32_t idesc = idesc_f16_f32(PAIR_F, PAIR_T);
+                // the descriptor's start-address field is addr >> 4 in its
+                // low 14 bits: offsets within the ring add without a carry
+                const uint64_t b_desc0 = smem_desc_sw128(sb + OFF_X);
+                static_assert(OFF_X + SX * STAGE_X <= (1u << 18), "descriptor start field");
+                const uint32_t a_base = tmem + A_COL0;
                 uint32_t j = 0, c = 0;         // stages, drains so far
                 bool ok = true;
-                for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+                const bool use_single = p.single_ok != 0;
+                int n = 0;                     // tiles so far
+                for (int t = pair; ok && t < p.total_tiles; t += npairs, ++n) {
                     const int fb = tile_coords(p, t).f0 / PAIR_F;
+                    bool single = false;       // the tile is one run (published by the epilogue)
                     bool fresh = true;         // the next MMA starts a new accumulation
                     for (int ci = 0; ok && ci < NC; ++ci) {
                         if (fresh) {
@@ -429,27 +534,41 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
                         }
                         const int ks0 = ci * KC_STAGES;
                         const int ks1 = min(NS, ks0 + KC_STAGES);
+                        // one thread issues every MMA, at ~100 clk per
+                        // instruction against 128 clk of tensor work each,
+                        // so the per-stage bookkeeping is kept to a minimum:
+                        // slot addresses and descriptors are offsets of
+                        // values computed once, the accumulate flag is
+                        // computed once per stage
+                        static_assert(SA == 4 && SUB == 2, "slot arithmetic below");
                         for (int ks = ks0; ks < ks1; ++ks, ++j) {
-                            const uint32_t sa = j % SA, sx = sa;
-                            if (!mbar_wait_cluster(sb + BAR_SFULL + 8 * sa, (j / SA) & 1, wc, ERR_MMA)) {
+                            const uint32_t sa = j & 3u;
+                            if (!mbar_wait_cluster(sb + BAR_SFULL + 8 * sa, (j >> 2) & 1, wc, ERR_MMA)) {
                                 ok = false;
                                 break;
                             }
                             tc_fence_after();
-                            const uint32_t a = tmem + A_COL0 + sa * A_SLOT_COLS;
-                            const uint32_t b = sb + OFF_X + sx * STAGE_X;
+                            const uint32_t a = a_base + sa * A_SLOT_COLS;
+                            const uint64_t bd = b_desc0 + sa * (STAGE_X >> 4);
+                            const uint32_t acc = (!fresh || ks > ks0) ? 1u : 0u;
 #pragma unroll
-                            for (int u = 0; u < SUB; ++u) {
-                                if (ks * SUB + u >= KB) break;
+                            for (int kk = 0; kk < BK / 16; ++kk)
+                                mma_f16_ts_pair(tmem, a + kk * 8, bd + kk * 2, idesc, kk > 0 ? 1u : acc);
+                            if (ks * SUB + 1 < KB) {
 #pragma unroll
                                 for (int kk = 0; kk < BK / 16; ++kk)
-                                    mma_f16_ts_pair(tmem, a + u * (BK / 2) + kk * 8,
-                                                    smem_desc_sw128(b + u * SUBX + kk * 32), idesc,
-                                                    (!fresh || ks > ks0 || u > 0 || kk > 0) ? 1u : 0u);
+                                    mma_f16_ts_pair(tmem, a + BK / 2 + kk * 8, bd + (SUBX >> 4) + kk * 2, idesc, 1u);
                             }
                             mma_commit_pair_multicast(sb + BAR_SEMPTY + 8 * sa, 0x3);
                         }
-                        fresh = plan_drains(p, fb, ci, NC);
+                        if (use_single && ci == 0 && ok) {
+                            if (!mbar_wait(sb + BAR_TFLAG + 8 * (n & 1), (n >> 1) & 1, wc, ERR_MMA)) {
+                                ok = false;
+                                break;
+                            }
+                            single = ld_shared_s32(sb + OFF_TFLAG + 4 * (n & 1)) != 0;
+                        }
+                        fresh = ci == NC - 1 || (!single && plan_drains(p, fb, ci, NC));
                         if (ok && fresh) {
                             mma_commit_pair_multicast(sb + BAR_ACCFULL, 0x3);
                             ++c;
@@ -543,7 +662,9 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
 // within 2^24, exact in fp32, and need no drain in between.  The plan is
 // built once per weight matrix: per block of 256 rows (one tile of the GEMM),
 // chunks are merged greedily while the largest row's sum over the merged run
-// stays within the bound.
+// stays within the bound.  A block's last word holds the largest sum of
+// squares of its rows, for the bound that uses the activations too (see
+// tile_single_run).
 constexpr uint32_t kPlanL1Limit = 1u << 17;
 constexpr int KC = KC_BLOCKS * BK;                   // K per chunk
 
@@ -552,10 +673,11 @@ chunk_plan_kernel(const int8_t *__restrict__ Wq, int N, int K, int NC, int words
     __shared__ uint32_t red[PAIR_F / 32];
     const int fb = blockIdx.x;
     const int r = fb * PAIR_F + threadIdx.x;
-    uint32_t *row_plan = plan + (size_t)fb * words;
+    uint32_t *row_plan = plan + (size_t)fb * (words + 1);
     if (threadIdx.x == 0)
         for (int w = 0; w < words; ++w) row_plan[w] = 0u;
     uint32_t cur = 0;                                 // this row's sum |w| since the last drain
+    uint32_t sq = 0;                                  // this row's sum of squares (< 2^32: K * 127^2)
     for (int c = 0; c < NC; ++c) {
         uint32_t l1 = 0;
         if (r < N) {
@@ -563,10 +685,13 @@ chunk_plan_kernel(const int8_t *__restrict__ Wq, int N, int K, int NC, int words
             const uint4 *src = reinterpret_cast<const uint4 *>(Wq + (size_t)r * K);
             for (int k = c * KC; k < k1; k += 16) {
                 const uint4 v = __ldg(src + k / 16);
-                l1 = __dp4a(__vabsdiffs4(v.x, 0u), 0x01010101u, l1);
-                l1 = __dp4a(__vabsdiffs4(v.y, 0u), 0x01010101u, l1);
-                l1 = __dp4a(__vabsdiffs4(v.z, 0u), 0x01010101u, l1);
-                l1 = __dp4a(__vabsdiffs4(v.w, 0u), 0x01010101u, l1);
+                const uint32_t w4[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                    const uint32_t a4 = __vabsdiffs4(w4[e], 0u);
+                    l1 = __dp4a(a4, 0x01010101u, l1);
+                    sq = __dp4a(a4, a4, sq);
+                }
             }
         }
         const uint32_t cand = cur + l1;
@@ -584,7 +709,16 @@ chunk_plan_kernel(const int8_t *__restrict__ Wq, int N, int K, int NC, int words
             cur = cand;
         }
     }
-    if (threadIdx.x == 0) row_plan[(NC - 1) >> 5] |= 1u << ((NC - 1) & 31);
+    const uint32_t wm = __reduce_max_sync(0xffffffffu, sq);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = wm;
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        uint32_t m = 0;
+#pragma unroll
+        for (int w = 0; w < PAIR_F / 32; ++w) m = max(m, red[w]);
+        row_plan[words] = m;
+        row_plan[(NC - 1) >> 5] |= 1u << ((NC - 1) & 31);
+    }
 }
 
 // ------------------------------------------------------------------ host
@@ -625,14 +759,16 @@ int g_kernel_regs[2] = {-1, -1};
 
 }  // namespace
 
-int chunk_plan_words(int K) {
+int chunk_plan_bits_words(int K) {
     const int NC = (K + KC - 1) / KC;
     return (NC + 31) / 32;
 }
 
+int chunk_plan_words(int K) { return chunk_plan_bits_words(K) + 1; }
+
 cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cudaStream_t st) {
     const int NC = (K + KC - 1) / KC;
-    chunk_plan_kernel<<<(N + PAIR_F - 1) / PAIR_F, PAIR_F, 0, st>>>(Wq, N, K, NC, chunk_plan_words(K), plan);
+    chunk_plan_kernel<<<(N + PAIR_F - 1) / PAIR_F, PAIR_F, 0, st>>>(Wq, N, K, NC, chunk_plan_bits_words(K), plan);
     return cudaGetLastError();
 }
 
@@ -663,12 +799,13 @@ cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_
     for (int i = 0; i < 2; ++i) {
         const GemmBranch *b = (i < nb) ? &br[i] : nullptr;
         BranchArgs &a = p.br[i];
-        a = BranchArgs{nullptr, nullptr, nullptr, nullptr, 0, 0, 0};
+        a = BranchArgs{nullptr, nullptr, nullptr, nullptr, nullptr, 0, 0, 0};
         if (b && b->M > 0) {
             a.x_scale = b->x_scale;
             a.w_scale = b->w_scale;
             a.bias = b->bias;
             a.out = b->out;
+            a.x_sumsq = b->x_sumsq;
             a.M = b->M;
             a.t_tiles = (b->M + PAIR_T - 1) / PAIR_T;
             a.tiles = a.t_tiles * f_tiles;
@@ -692,6 +829,9 @@ cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_
     p.k_blocks = (K + BK - 1) / BK;
     p.plan = plan;
     p.plan_words = chunk_plan_words(K);
+    p.single_ok = plan != nullptr;
+    for (int i = 0; i < 2; ++i)
+        if (p.br[i].M > 0 && p.br[i].x_sumsq == nullptr) p.single_ok = 0;
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
     const int pairs = p.total_tiles < g_sms / 2 ? p.total_tiles : g_sms / 2;

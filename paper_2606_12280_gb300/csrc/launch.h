@@ -15,6 +15,7 @@ struct GemmBranch {
     const float *bias;
     void *out;        // uint16_t* bf16 Y, or int32_t* acc for the debug export
     int M;
+    const uint32_t *x_sumsq;   // fp16-code GEMM: per token sum of squared codes, or null
 };
 
 cudaError_t launch_channel_absmax(const uint16_t *X, int T, int K, float *s,
@@ -69,7 +70,8 @@ cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cu
 
 // a3 (optionally of GELU(X)) writing the codes as fp16 values, K <= 16384.
 cudaError_t launch_quant_act_f16codes(const uint16_t *X, const float *lambda, int M, int K,
-                                     uint16_t *Xq16, float *x_scale, bool gelu, cudaStream_t st);
+                                     uint16_t *Xq16, float *x_scale, uint32_t *sumsq, bool gelu,
+                                     cudaStream_t st);
 
 // tcgen05 GEMM (exact integer products on the fp16 tensor datapath).
 cudaError_t launch_gemm_tc(const GemmBranch *br, int nb, int N, int K,

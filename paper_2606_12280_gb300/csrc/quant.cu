@@ -388,6 +388,7 @@ struct ActBranch {
     int8_t *Xq;
     float *x_scale;
     int M;
+    uint32_t *sumsq;      // fp16-code variant, optional: sum of the row's squared codes
 };
 
 // One launch covers up to two independent row sets (the conditional and
@@ -416,6 +417,7 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
     constexpr int kTeams = kThreads / (32 * TW);
     extern __shared__ __align__(16) uint4 ring_s[];
     __shared__ float red[2][kThreads / 32];
+    __shared__ uint32_t sred[2][kThreads / 32];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int team = warp / TW, tw = warp % TW;
     const int K = p.K;
@@ -459,7 +461,11 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
         }
     }
 
-    int parity = 0;
+    // OUT16: the squared codes of a row are summed (exactly, in int32: at most
+    // 16384 * 127^2 < 2^31) for the GEMM's bound on its partial sums; the
+    // team's per-warp sums of row k are combined after row k + 1's barrier
+    const bool want_ss = OUT16 && b.sumsq != nullptr;
+    int parity = 0, prev_row = -1;
     for (int k = 0;; ++k, parity ^= 1) {
         const int row = first + k * teams;                  // uniform across the team
         if (row >= M) break;
@@ -489,6 +495,12 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
             asm volatile("bar.sync %0, %1;" ::"r"(1 + team), "r"(TW * 32) : "memory");
 #pragma unroll
             for (int w = 0; w < TW; ++w) a = fmaxf(a, red[parity][team * TW + w]);
+            if (want_ss && prev_row >= 0 && tw == 0 && lane == 0) {
+                uint32_t t = 0;
+#pragma unroll
+                for (int w = 0; w < TW; ++w) t += sred[parity ^ 1][team * TW + w];
+                b.sumsq[prev_row] = t;
+            }
         }
         const bool zero_row = (a == 0.0f);
         const float inv = zero_row ? 0.0f : __fdiv_rn(127.0f, a);
@@ -497,6 +509,7 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
         const bool fast = (a <= 3.402823466e38f) && (inv <= 3.402823466e38f);
         uint2 *qr = reinterpret_cast<uint2 *>(b.Xq + (size_t)row * K);
         uint4 *qr16 = reinterpret_cast<uint4 *>(b.Xq + 2 * (size_t)row * K);
+        uint32_t ss = 0;
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const int c = (u * TW + tw) * 32 + lane;
@@ -506,16 +519,27 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
                 if (zero_row) {
                 } else if (fast) {
                     // rne(x' * inv) as an fp32 integer: the magic sum minus the
-                    // magic (both in [2^23, 2^24): exact)
+                    // magic (both in [2^23, 2^24): exact); the magic sum's bit
+                    // pattern minus the magic's is the integer code
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        hw[q] = pack_f16(__fadd_rn(__fadd_rn(__fmul_rn(xs[u][q].x, inv), kRoundMagic), -kRoundMagic),
-                                         __fadd_rn(__fadd_rn(__fmul_rn(xs[u][q].y, inv), kRoundMagic), -kRoundMagic));
+                    for (int q = 0; q < 4; ++q) {
+                        const float r0 = __fadd_rn(__fmul_rn(xs[u][q].x, inv), kRoundMagic);
+                        const float r1 = __fadd_rn(__fmul_rn(xs[u][q].y, inv), kRoundMagic);
+                        hw[q] = pack_f16(__fadd_rn(r0, -kRoundMagic), __fadd_rn(r1, -kRoundMagic));
+                        if (want_ss) {
+                            const int q0 = static_cast<int>(__float_as_uint(r0) - 0x4B400000u);
+                            const int q1 = static_cast<int>(__float_as_uint(r1) - 0x4B400000u);
+                            ss += static_cast<uint32_t>(q0 * q0 + q1 * q1);
+                        }
+                    }
                 } else {
 #pragma unroll
-                    for (int q = 0; q < 4; ++q)
-                        hw[q] = pack_f16(static_cast<float>(quantize_rne_clamp(__fmul_rn(xs[u][q].x, inv))),
-                                         static_cast<float>(quantize_rne_clamp(__fmul_rn(xs[u][q].y, inv))));
+                    for (int q = 0; q < 4; ++q) {
+                        const int q0 = quantize_rne_clamp(__fmul_rn(xs[u][q].x, inv));
+                        const int q1 = quantize_rne_clamp(__fmul_rn(xs[u][q].y, inv));
+                        hw[q] = pack_f16(static_cast<float>(q0), static_cast<float>(q1));
+                        ss += static_cast<uint32_t>(q0 * q0 + q1 * q1);
+                    }
                 }
                 qr16[c] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
                 continue;
@@ -538,6 +562,25 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
                 }
             }
             qr[c] = make_uint2(word[0], word[1]);
+        }
+        if (want_ss) {
+            ss = __reduce_add_sync(0xffffffffu, ss);
+            if (TW > 1) {
+                if (lane == 0) sred[parity][warp] = ss;
+            } else if (lane == 0) {
+                b.sumsq[row] = ss;
+            }
+            prev_row = row;
+        }
+    }
+    if (TW > 1 && want_ss && prev_row >= 0) {
+        // the last row's sums: one more team barrier
+        asm volatile("bar.sync %0, %1;" ::"r"(1 + team), "r"(TW * 32) : "memory");
+        if (tw == 0 && lane == 0) {
+            uint32_t t = 0;
+#pragma unroll
+            for (int w = 0; w < TW; ++w) t += sred[parity ^ 1][team * TW + w];
+            b.sumsq[prev_row] = t;
         }
     }
     asm volatile("cp.async.wait_group 0;" ::: "memory");
@@ -686,9 +729,10 @@ cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M, int 
 }
 
 cudaError_t launch_quant_act_f16codes(const uint16_t *X, const float *lambda, int M, int K,
-                                     uint16_t *Xq16, float *x_scale, bool gelu, cudaStream_t st) {
+                                     uint16_t *Xq16, float *x_scale, uint32_t *sumsq, bool gelu,
+                                     cudaStream_t st) {
     ActParams p{};
-    p.br[0] = ActBranch{X, lambda, reinterpret_cast<int8_t *>(Xq16), x_scale, M};
+    p.br[0] = ActBranch{X, lambda, reinterpret_cast<int8_t *>(Xq16), x_scale, M, sumsq};
     p.K = K;
     return gelu ? launch_act_quant_teams<true, true>(p, st) : launch_act_quant_teams<false, true>(p, st);
 }
@@ -697,7 +741,7 @@ cudaError_t launch_quant_act_dual(const QuantActBranch *br, int K, cudaStream_t 
     if (K <= 16384) {
         ActParams p{};
         for (int i = 0; i < 2; ++i)
-            p.br[i] = ActBranch{br[i].X, br[i].lambda, br[i].Xq, br[i].x_scale, br[i].M};
+            p.br[i] = ActBranch{br[i].X, br[i].lambda, br[i].Xq, br[i].x_scale, br[i].M, nullptr};
         p.K = K;
         return launch_act_quant_teams<false>(p, st);
     }

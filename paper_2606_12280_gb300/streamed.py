@@ -38,6 +38,7 @@ class StreamedLinear:
         self.Xq = [torch.empty(M, K, dtype=torch.float16 if self.f16 else torch.int8, device=dev)
                    for _ in range(depth)]
         self.sx = [torch.empty(M, dtype=torch.float32, device=dev) for _ in range(depth)]
+        self.ss = [torch.empty(M, dtype=torch.int32, device=dev) for _ in range(depth)] if self.f16 else None
         self.Y = [torch.empty(M, N, dtype=torch.bfloat16, device=dev) for _ in range(depth)]
         self.up = torch.cuda.Stream(device=dev)
         self.comp = torch.cuda.Stream(device=dev)
@@ -68,14 +69,16 @@ class StreamedLinear:
                     self.comp.wait_event(self.y_free[s])
                 if self.f16:
                     w8a8.quant_act_f16codes(self.X[s], self.smooth, Xq16=self.Xq[s], x_scale=self.sx[s],
-                                            stream=self.comp)
+                                            sumsq=self.ss[s], stream=self.comp)
                 else:
                     w8a8.quant_act(self.X[s], self.smooth, Xq=self.Xq[s], x_scale=self.sx[s],
                                    stream=self.comp)
                 self.x_free[s].record(self.comp)
                 if self.f16:
                     w8a8.linear_f16codes(self.Xq[s], self.sx[s], self.Wq, self.w_scale, self.bias,
-                                         Y=self.Y[s], plan=self.plan, stream=self.comp)
+                                         Y=self.Y[s], plan=self.plan,
+                                         x_sumsq=self.ss[s] if self.plan is not None else None,
+                                         stream=self.comp)
                 else:
                     w8a8.linear(self.Xq[s], self.sx[s], self.Wq, self.w_scale, self.bias, Y=self.Y[s],
                                 stream=self.comp)

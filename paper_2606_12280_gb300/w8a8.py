@@ -48,9 +48,9 @@ SIGNATURES = {
     "w8a8_debug_gelu": [_P, _I, _P, _P],
     "w8a8_linear_gguf": [_P, _P, _I, _P, _I, _I, _I, _P, _P],
     "w8a8_debug_gguf_dequant": [_P, _I, _I, _I, _P, _P],
-    "w8a8_quant_act_f16codes": [_P, _P, _I, _I, _P, _P, _I, _P],
-    "w8a8_linear_f16codes": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P],
-    "w8a8_debug_gemm_f16codes_i32": [_P, _P, _I, _I, _I, _P, _P, _P],
+    "w8a8_quant_act_f16codes": [_P, _P, _I, _I, _P, _P, _P, _I, _P],
+    "w8a8_linear_f16codes": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P],
+    "w8a8_debug_gemm_f16codes_i32": [_P, _P, _I, _I, _I, _P, _P, _P, _P],
     "w8a8_chunk_plan_size": [_I, _I],
     "w8a8_chunk_plan": [_P, _I, _I, _P, _P],
     "w8a8_act_stats_noalloc": [_P, _I, _I, _P, _P, _P, _P],
@@ -288,8 +288,10 @@ def gelu_quant_act(H, smooth=None, Xq=None, x_scale=None, stream=None):
     return Xq, x_scale
 
 
-def quant_act_f16codes(X, smooth=None, Xq16=None, x_scale=None, gelu=False, stream=None):
-    """a3 with the codes as fp16 values: returns (Xq16 [M,K] float16, sx [M])."""
+def quant_act_f16codes(X, smooth=None, Xq16=None, x_scale=None, gelu=False, sumsq=None, stream=None):
+    """a3 with the codes as fp16 values: returns (Xq16 [M,K] float16, sx [M]).
+    sumsq: None, or an int32 [M] tensor that receives sum_j Xq_mj^2 per token
+    (uint32 values; for ``linear_f16codes(..., x_sumsq=)``)."""
     M, K = X.shape
     if Xq16 is None:
         Xq16 = torch.empty(M, K, dtype=torch.float16, device=X.device)
@@ -298,13 +300,14 @@ def quant_act_f16codes(X, smooth=None, Xq16=None, x_scale=None, gelu=False, stre
     _check("w8a8_quant_act_f16codes", lib().w8a8_quant_act_f16codes(
         _ptr(X, torch.bfloat16, "X"), _ptr(smooth, torch.float32, "smooth"), M, K,
         _ptr(Xq16, torch.float16, "Xq16"), _ptr(x_scale, torch.float32, "x_scale"),
-        1 if gelu else 0, _stream(stream)))
+        _ptr(sumsq, torch.int32, "sumsq"), 1 if gelu else 0, _stream(stream)))
     return Xq16, x_scale
 
 
-def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, stream=None):
+def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, x_sumsq=None, stream=None):
     """a4 + a5 with fp16-coded activations: Y = bf16((Xq Wq^T) * sx * sw + b).
-    plan: None or ``chunk_plan(Wq)``."""
+    plan: None or ``chunk_plan(Wq)``; x_sumsq: None or the token sums that
+    ``quant_act_f16codes(..., sumsq=)`` wrote for these codes."""
     M, K = Xq16.shape
     N = Wq.shape[0]
     if Y is None:
@@ -313,11 +316,11 @@ def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, st
         _ptr(Xq16, torch.float16, "Xq16"), _ptr(x_scale, torch.float32, "x_scale"),
         _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
         _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(plan, torch.int32, "plan"),
-        _ptr(Y, torch.bfloat16, "Y"), _stream(stream)))
+        _ptr(x_sumsq, torch.int32, "x_sumsq"), _ptr(Y, torch.bfloat16, "Y"), _stream(stream)))
     return Y
 
 
-def debug_gemm_f16codes_i32(Xq16, Wq, plan=None, acc=None, stream=None):
+def debug_gemm_f16codes_i32(Xq16, Wq, plan=None, x_sumsq=None, acc=None, stream=None):
     """Exact int32 acc = Xq16 Wq^T (test export of the fp16-code GEMM)."""
     M, K = Xq16.shape
     N = Wq.shape[0]
@@ -325,7 +328,8 @@ def debug_gemm_f16codes_i32(Xq16, Wq, plan=None, acc=None, stream=None):
         acc = torch.empty(M, N, dtype=torch.int32, device=Xq16.device)
     _check("w8a8_debug_gemm_f16codes_i32", lib().w8a8_debug_gemm_f16codes_i32(
         _ptr(Xq16, torch.float16, "Xq16"), _ptr(Wq, torch.int8, "Wq"), M, N, K,
-        _ptr(plan, torch.int32, "plan"), _ptr(acc, torch.int32, "acc"), _stream(stream)))
+        _ptr(plan, torch.int32, "plan"), _ptr(x_sumsq, torch.int32, "x_sumsq"),
+        _ptr(acc, torch.int32, "acc"), _stream(stream)))
     return acc
 
 
@@ -483,7 +487,8 @@ def quantized_linear_forward(X, smooth, Wq, w_scale, bias=None, plan=None, codes
     if codes not in ("f16", "int8"):
         raise ValueError("codes must be 'f16' or 'int8'")
     if codes == "f16" and X.shape[1] <= 16384:
-        Xq16, sx = quant_act_f16codes(X, smooth, stream=stream)
-        return linear_f16codes(Xq16, sx, Wq, w_scale, bias, plan=plan, stream=stream)
+        ss = torch.empty(X.shape[0], dtype=torch.int32, device=X.device) if plan is not None else None
+        Xq16, sx = quant_act_f16codes(X, smooth, sumsq=ss, stream=stream)
+        return linear_f16codes(Xq16, sx, Wq, w_scale, bias, plan=plan, x_sumsq=ss, stream=stream)
     Xq, sx = quant_act(X, smooth, stream=stream)
     return linear(Xq, sx, Wq, w_scale, bias, stream=stream)

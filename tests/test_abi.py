@@ -247,32 +247,36 @@ def test_gguf_validation(L):
 
 def test_f16codes_validation(L):
     f = L.w8a8_quant_act_f16codes
-    assert f(A, None, 4, 16400, A, A, 0, None) == SHAPE         # K beyond 16384
-    assert f(A, None, 4, 24, A, A, 0, None) == SHAPE
-    assert f(None, None, 4, 16, A, A, 0, None) == INVALID
-    assert f(A, None, 4, 16, U, A, 0, None) == MISALIGNED
-    assert f(None, None, 0, 16, None, None, 0, None) == OK
+    assert f(A, None, 4, 16400, A, A, None, 0, None) == SHAPE         # K beyond 16384
+    assert f(A, None, 4, 24, A, A, None, 0, None) == SHAPE
+    assert f(None, None, 4, 16, A, A, None, 0, None) == INVALID
+    assert f(A, None, 4, 16, U, A, None, 0, None) == MISALIGNED
+    assert f(A, None, 4, 16, A, A, U, 0, None) == MISALIGNED          # sumsq
+    assert f(None, None, 0, 16, None, None, None, 0, None) == OK
     g = L.w8a8_linear_f16codes
-    assert g(A, A, A, A, None, 4, 12, 16, None, A, None) == SHAPE
-    assert g(None, A, A, A, None, 4, 8, 16, None, A, None) == INVALID
-    assert g(A, A, U, A, None, 4, 8, 16, None, A, None) == MISALIGNED
-    assert g(A, A, A, A, None, 4, 8, 16, U, A, None) == MISALIGNED      # plan
-    assert g(A, A, A, A, None, 0, 8, 16, None, A, None) == OK
+    assert g(A, A, A, A, None, 4, 12, 16, None, None, A, None) == SHAPE
+    assert g(None, A, A, A, None, 4, 8, 16, None, None, A, None) == INVALID
+    assert g(A, A, U, A, None, 4, 8, 16, None, None, A, None) == MISALIGNED
+    assert g(A, A, A, A, None, 4, 8, 16, U, None, A, None) == MISALIGNED      # plan
+    assert g(A, A, A, A, None, 4, 8, 16, A, U, A, None) == MISALIGNED         # token sums
+    assert g(A, A, A, A, None, 0, 8, 16, None, None, A, None) == OK
     d = L.w8a8_debug_gemm_f16codes_i32
-    assert d(A, A, 4, 12, 16, None, A, None) == SHAPE
-    assert d(None, A, 4, 8, 16, None, A, None) == INVALID
-    assert d(A, U, 4, 8, 16, None, A, None) == MISALIGNED
-    assert d(A, A, 0, 8, 16, None, A, None) == OK
+    assert d(A, A, 4, 12, 16, None, None, A, None) == SHAPE
+    assert d(None, A, 4, 8, 16, None, None, A, None) == INVALID
+    assert d(A, U, 4, 8, 16, None, None, A, None) == MISALIGNED
+    assert d(A, A, 4, 8, 16, None, U, A, None) == MISALIGNED
+    assert d(A, A, 0, 8, 16, None, None, A, None) == OK
 
 
 def test_chunk_plan_validation(L):
     size = L.w8a8_chunk_plan_size
     # one word per 256-row block up to 32 chunks of 1024
-    assert size(256, 4096) == 1
-    assert size(257, 4096) == 2
-    assert size(12288, 4096) == 48
-    assert size(256, 32 * 1024) == 1
-    assert size(256, 32 * 1024 + 16) == 2
+    # per 256-row block: one word per 32 chunks of 1024, plus one
+    assert size(256, 4096) == 2
+    assert size(257, 4096) == 4
+    assert size(12288, 4096) == 96
+    assert size(256, 32 * 1024) == 2
+    assert size(256, 32 * 1024 + 16) == 3
     assert size(0, 16) == 1
     f = L.w8a8_chunk_plan
     assert f(A, 12, 16, A, None) == SHAPE

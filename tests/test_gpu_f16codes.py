@@ -120,14 +120,16 @@ def plan_reference(Wq, limit=1 << 17, kc=1024, rows=256):
     chunks ends before chunk c when some row's sum |w| over the run including
     c would exceed `limit` (then 128 * limit = 2^24 bounds every partial sum of
     codes |a| <= 128); the last chunk always ends a run.  Bit c of a block's
-    words = a run ends after chunk c."""
+    words = a run ends after chunk c; the block's last word = the largest
+    sum of squares of its rows."""
     N, K = Wq.shape
     nc = -(-K // kc)
     words = -(-nc // 32)
     nb = -(-N // rows)
     a = np.abs(Wq.astype(np.int64))
     l1 = np.stack([a[:, c * kc:(c + 1) * kc].sum(1) for c in range(nc)], 1)
-    plan = np.zeros((nb, words), np.uint32)
+    plan = np.zeros((nb, words + 1), np.uint32)
+    sq = (Wq.astype(np.int64) ** 2).sum(1)
     for b in range(nb):
         blk = l1[b * rows:(b + 1) * rows]
         cur = np.zeros(blk.shape[0], np.int64)
@@ -139,6 +141,7 @@ def plan_reference(Wq, limit=1 << 17, kc=1024, rows=256):
             else:
                 cur = cand
         plan[b, (nc - 1) // 32] |= np.uint32(1 << ((nc - 1) % 32))
+        plan[b, words] = np.uint32(sq[b * rows:(b + 1) * rows].max())
     return plan.reshape(-1)
 
 
@@ -170,7 +173,7 @@ def test_chunk_plan_reference_needs_drains_where_fp32_would_round():
     # over two chunks of positive products passes 2^24 and rounds, so the
     # plan must end a run after every chunk there
     Wq = plan_cases()["full"]
-    assert np.all(plan_reference(Wq) == np.uint32(0b1111))
+    assert plan_reference(Wq)[0] == np.uint32(0b1111)
     prod = np.full(2048, 127 * 127, np.float32)
     prod[1::3] = 127 * 125
     acc = np.float32(0)
@@ -197,3 +200,70 @@ def test_gemm_f16codes_i32_exact(w8, name, with_plan):
     acc = w8.debug_gemm_f16codes_i32(q16, t(Wq), plan=plan).cpu().numpy()
     want = Xq.astype(np.int64) @ Wq.astype(np.int64).T
     np.testing.assert_array_equal(acc, want)
+
+
+# ------------------------------------------------------- token sums of squares
+
+@pytest.mark.parametrize("M,K,gelu", [(1, 16, False), (300, 528, False), (257, 4096, False),
+                                      (64, 16384, False), (129, 4096, True)])
+def test_quant_act_f16codes_sumsq_exact(w8, M, K, gelu):
+    X = wl.random_bf16((M, K), seed=M + 3 * K, scale=2.0)
+    X[0, :] = 0                                         # an all-zero token
+    lam = wl.random_uniform_f32((K,), seed=K + 1, lo=0.25, hi=4.0)
+    ss = torch.empty(M, dtype=torch.int32, device=DEV)
+    q16, sx = w8.quant_act_f16codes(bf(X), t(lam), gelu=gelu, sumsq=ss)
+    q = codes(q16).astype(np.int64)
+    np.testing.assert_array_equal(ss.cpu().numpy().view(np.uint32), (q * q).sum(1).astype(np.uint32))
+    q16b, sxb = w8.quant_act_f16codes(bf(X), t(lam), gelu=gelu)
+    assert torch.equal(q16, q16b) and torch.equal(sx, sxb)
+
+
+def sumsq_cases():
+    rng = np.random.default_rng(23)
+    # 1: Gaussian codes and weights: every tile one run (bound holds)
+    W1 = gauss_codes((520, 4096), 5, 30.0)
+    X1 = gauss_codes((600, 4096), 6, 30.0)
+    # 2: near-max codes in the second token block: those tiles fall back to
+    # the plan (the bound fails), the first block's tiles run as one
+    W2 = gauss_codes((264, 8192), 7, 40.0)
+    X2 = gauss_codes((520, 8192), 8, 20.0)
+    X2[256:] = np.where(rng.random((264, 8192)) < 0.5, -127, 127)
+    # 3: worst case everywhere
+    W3 = np.full((256, 3072), 127, np.int8)
+    X3 = np.where(rng.random((300, 3072)) < 0.3, 125, 127).astype(np.int8)
+    return {"single": (X1, W1), "mixed": (X2, W2), "worst": (X3, W3)}
+
+
+@pytest.mark.parametrize("name", ["single", "mixed", "worst"])
+def test_gemm_f16codes_i32_exact_with_sumsq(w8, name):
+    Xq, Wq = sumsq_cases()[name]
+    q16 = torch.from_numpy(Xq.astype(np.float16)).to(DEV)
+    ss = torch.from_numpy(((Xq.astype(np.int64) ** 2).sum(1)).astype(np.uint32).view(np.int32)).to(DEV)
+    plan = w8.chunk_plan(t(Wq))
+    acc = w8.debug_gemm_f16codes_i32(q16, t(Wq), plan=plan, x_sumsq=ss).cpu().numpy()
+    np.testing.assert_array_equal(acc, Xq.astype(np.int64) @ Wq.astype(np.int64).T)
+
+
+def test_single_run_bound_premise():
+    # (host check) the cases above exercise both sides of the bound
+    X1, W1 = sumsq_cases()["single"]
+    a = (X1.astype(np.int64) ** 2).sum(1).max()
+    w = (W1.astype(np.int64) ** 2).sum(1).max()
+    assert a * w <= 2 ** 48
+    X2, W2 = sumsq_cases()["mixed"]
+    w = (W2.astype(np.int64) ** 2).sum(1).max()
+    assert (X2[:256].astype(np.int64) ** 2).sum(1).max() * w <= 2 ** 48
+    assert (X2[256:].astype(np.int64) ** 2).sum(1).max() * w > 2 ** 48
+
+
+@pytest.mark.parametrize("M,N,K", [(300, 264, 528), (513, 520, 4096)])
+def test_linear_f16codes_exact_with_sumsq(w8, oracle_mod, M, N, K):
+    c = wl.make_case(M, K, N, seed=M + N + 2 * K)
+    s = oracle_mod.channel_absmax(c.X_cal)
+    lam = oracle_mod.smooth_scales(s, c.W[0], c.alpha)
+    Wq, sw = oracle_mod.quantize_weights(c.W[0], lam)
+    ss = torch.empty(M, dtype=torch.int32, device=DEV)
+    q16, sx = w8.quant_act_f16codes(bf(c.X[0]), t(lam), sumsq=ss)
+    Y = w8.linear_f16codes(q16, sx, t(Wq), t(sw), t(c.bias[0]), plan=w8.chunk_plan(t(Wq)), x_sumsq=ss)
+    Xq, wsx = oracle_mod.quant_act(c.X[0], lam)
+    np.testing.assert_array_equal(u16(Y), oracle_mod.linear(Xq, wsx, Wq, sw, c.bias[0]))
