@@ -218,6 +218,44 @@ W8A8_API w8a8_status w8a8_debug_gemm_f16codes_i32(const uint16_t *Xq16, const in
                                                   const uint32_t *x_sumsq, int32_t *acc,
                                                   void *stream);
 
+/* One branch of the dual-branch layer with fp16 codes (a6 on this path). */
+typedef struct {
+    const uint16_t *X;     /* [M,K] bf16 */
+    const float *smooth;   /* [K] fp32 (this branch's lambda) or NULL */
+    int M;                 /* tokens of this branch, >= 0 */
+    uint16_t *Xq16;        /* [M,K] fp16 codes, written */
+    float *x_scale;        /* [M] fp32, written */
+    uint32_t *x_sumsq;     /* [M] uint32 or NULL, written */
+} w8a8_act_branch16;
+
+typedef struct {
+    const uint16_t *Xq16;        /* [M,K] fp16 codes */
+    const float *x_scale;        /* [M] fp32 */
+    const int8_t *Wq;            /* [N,K] int8 */
+    const float *w_scale;        /* [N] fp32 */
+    const float *bias;           /* [N] fp32 or NULL */
+    uint16_t *Y;                 /* [M,N] bf16, written */
+    int M;                       /* tokens of this branch, >= 0 */
+    const uint32_t *chunk_plan;  /* this branch's weights' plan or NULL */
+    const uint32_t *x_sumsq;     /* this branch's token sums or NULL */
+} w8a8_branch16;
+
+/*
+ * a3 of both separate-weight branches (Sec. 1 and 3: the conditional br[0]
+ * and unconditional br[1] backbones) with fp16 codes, in one launch, as
+ * w8a8_quant_act_dual does for int8 codes; each branch as
+ * w8a8_quant_act_f16codes.  K <= 16384.
+ */
+W8A8_API w8a8_status w8a8_quant_act_dual_f16codes(const w8a8_act_branch16 *br, int K, void *stream);
+
+/*
+ * a4 + a5 of both branches in one grouped launch (a6) with fp16 codes: the
+ * tile space covers both branches, each tile with its own branch's operands,
+ * plan and token sums; results as two w8a8_linear_f16codes calls, bitwise.
+ * The branches share N and K.
+ */
+W8A8_API w8a8_status w8a8_linear_dual_f16codes(const w8a8_branch16 *br, int N, int K, void *stream);
+
 /*
  * Drain plan of an int8 weight matrix for w8a8_linear_f16codes (no
  * counterpart in the paper: a property of the exact-integer scheme on fp32

@@ -180,6 +180,42 @@ w8a8_status w8a8_quant_act_dual(const w8a8_act_branch *br, int K, void *stream) 
     return from_cuda(w8a8::launch_quant_act_dual(b, K, as_stream(stream)));
 }
 
+w8a8_status w8a8_quant_act_dual_f16codes(const w8a8_act_branch16 *br, int K, void *stream) {
+    if (!br) return W8A8_ERR_INVALID_ARG;
+    if (K > 16384) return W8A8_ERR_UNSUPPORTED_SHAPE;
+    w8a8::QuantActBranch16 b[2];
+    for (int i = 0; i < 2; ++i) {
+        if (w8a8_status e = check_mk(br[i].M, K)) return e;
+        b[i] = w8a8::QuantActBranch16{br[i].X, br[i].smooth, br[i].M, br[i].Xq16, br[i].x_scale, br[i].x_sumsq};
+        if (br[i].M == 0) continue;
+        if (!br[i].X || !br[i].Xq16 || !br[i].x_scale) return W8A8_ERR_INVALID_ARG;
+        if (!aligned16(br[i].X) || !aligned16(br[i].Xq16) || !aligned16(br[i].x_scale) ||
+            (br[i].smooth && !aligned16(br[i].smooth)) || (br[i].x_sumsq && !aligned16(br[i].x_sumsq)))
+            return W8A8_ERR_MISALIGNED;
+    }
+    if (br[0].M == 0 && br[1].M == 0) return W8A8_OK;
+    return from_cuda(w8a8::launch_quant_act_dual_f16codes(b, K, as_stream(stream)));
+}
+
+w8a8_status w8a8_linear_dual_f16codes(const w8a8_branch16 *br, int N, int K, void *stream) {
+    if (!br) return W8A8_ERR_INVALID_ARG;
+    if (w8a8_status e = check_nk(N, K)) return e;
+    w8a8::GemmBranch b[2];
+    for (int i = 0; i < 2; ++i) {
+        b[i] = w8a8::GemmBranch{reinterpret_cast<const int8_t *>(br[i].Xq16), br[i].x_scale, br[i].Wq,
+                                br[i].w_scale, br[i].bias, br[i].Y, br[i].M, br[i].x_sumsq, br[i].chunk_plan};
+        if (w8a8_status e = check_mk(br[i].M, K)) return e;
+        if (w8a8_status e = check_branch(b[i], true, N, K)) return e;
+        if (br[i].M > 0 && ((br[i].chunk_plan && !aligned16(br[i].chunk_plan)) ||
+                            (br[i].x_sumsq && !aligned16(br[i].x_sumsq))))
+            return W8A8_ERR_MISALIGNED;
+    }
+    if (b[0].M == 0 && b[1].M == 0) return W8A8_OK;
+    unsigned int *err = device_error_word();
+    if (!err) return W8A8_ERR_CUDA;
+    return from_cuda(w8a8::launch_gemm_ts(b, 2, N, K, false, err, as_stream(stream)));
+}
+
 w8a8_status w8a8_gelu_quant_act(const uint16_t *H, const float *smooth, int M, int K, int8_t *Xq,
                                 float *x_scale, void *stream) {
     if (w8a8_status e = check_mk(M, K)) return e;
@@ -218,13 +254,14 @@ w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale, con
                                  void *stream) {
     if (w8a8_status e = check_nk(N, K)) return e;
     if (w8a8_status e = check_mk(M, K)) return e;
-    w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), x_scale, Wq, w_scale, bias, Y, M, x_sumsq};
+    w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), x_scale, Wq, w_scale, bias, Y, M, x_sumsq,
+                       chunk_plan};
     if (w8a8_status e = check_branch(b, true, N, K)) return e;
     if ((chunk_plan && !aligned16(chunk_plan)) || (x_sumsq && !aligned16(x_sumsq))) return W8A8_ERR_MISALIGNED;
     if (M == 0) return W8A8_OK;
     unsigned int *err = device_error_word();
     if (!err) return W8A8_ERR_CUDA;
-    return from_cuda(w8a8::launch_gemm_ts(&b, 1, N, K, false, chunk_plan, err, as_stream(stream)));
+    return from_cuda(w8a8::launch_gemm_ts(&b, 1, N, K, false, err, as_stream(stream)));
 }
 
 w8a8_status w8a8_debug_gemm_f16codes_i32(const uint16_t *Xq16, const int8_t *Wq, int M, int N, int K,
@@ -232,13 +269,14 @@ w8a8_status w8a8_debug_gemm_f16codes_i32(const uint16_t *Xq16, const int8_t *Wq,
                                          void *stream) {
     if (w8a8_status e = check_nk(N, K)) return e;
     if (w8a8_status e = check_mk(M, K)) return e;
-    w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), nullptr, Wq, nullptr, nullptr, acc, M, x_sumsq};
+    w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), nullptr, Wq, nullptr, nullptr, acc, M, x_sumsq,
+                       chunk_plan};
     if (w8a8_status e = check_branch(b, false, N, K)) return e;
     if ((chunk_plan && !aligned16(chunk_plan)) || (x_sumsq && !aligned16(x_sumsq))) return W8A8_ERR_MISALIGNED;
     if (M == 0) return W8A8_OK;
     unsigned int *err = device_error_word();
     if (!err) return W8A8_ERR_CUDA;
-    return from_cuda(w8a8::launch_gemm_ts(&b, 1, N, K, true, chunk_plan, err, as_stream(stream)));
+    return from_cuda(w8a8::launch_gemm_ts(&b, 1, N, K, true, err, as_stream(stream)));
 }
 
 long long w8a8_chunk_plan_size(int N, int K) {

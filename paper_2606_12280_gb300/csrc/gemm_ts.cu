@@ -119,6 +119,7 @@ struct BranchArgs {
     const float *bias;
     void *out;
     const uint32_t *x_sumsq;   // per token sum of squared codes, or null
+    const uint32_t *plan;      // the weights' drain plan (see plan_drains), or null
     int M;           // tokens
     int t_tiles;     // token tiles of 256
     int tiles;       // t_tiles * feature tiles
@@ -129,12 +130,11 @@ struct Params {
     int N, K;
     int total_tiles;
     int k_blocks;
-    // optional drain plan (see plan_drains): per 256-row weight block,
-    // plan_words words of bits, bit c set = drain after K chunk c; null =
-    // drain after every chunk
-    const uint32_t *plan;
-    int plan_words;            // per block: the drain bits, then the block's max sum of squares
-    // plan and every branch's x_sumsq given: tiles whose activation and weight
+    // per 256-row weight block of a branch's plan: plan_words words, the
+    // drain bits (bit c set = drain after K chunk c), then the block's max
+    // sum of squares
+    int plan_words;
+    // every branch has a plan and x_sumsq: tiles whose activation and weight
     // norms bound every partial sum run without an intermediate drain
     int single_ok;
     unsigned int *err;
@@ -159,9 +159,9 @@ __device__ __forceinline__ Tile tile_coords(const Params &p, int t) {
 // minus 1152).
 // Does the accumulation stop (the epilogue drains TMEM) after K chunk ci of a
 // tile of weight block fb?  Always after the tile's last chunk.
-__device__ __forceinline__ bool plan_drains(const Params &p, int fb, int ci, int NC) {
-    if (ci == NC - 1 || p.plan == nullptr) return true;
-    return (__ldg(p.plan + (size_t)fb * p.plan_words + (ci >> 5)) >> (ci & 31)) & 1u;
+__device__ __forceinline__ bool plan_drains(const Params &p, const uint32_t *plan, int fb, int ci, int NC) {
+    if (ci == NC - 1 || plan == nullptr) return true;
+    return (__ldg(plan + (size_t)fb * p.plan_words + (ci >> 5)) >> (ci & 31)) & 1u;
 }
 
 // Can tile t run without an intermediate drain?  Every partial sum P over a
@@ -177,7 +177,7 @@ __device__ __forceinline__ bool tile_single_run(const Params &p, int t, int lane
     for (int i = lane; i < PAIR_T; i += 32)
         if (tl.t0 + i < br.M) m = max(m, __ldg(br.x_sumsq + tl.t0 + i));
     m = __reduce_max_sync(0xffffffffu, m);
-    const uint32_t wm = __ldg(p.plan + (size_t)(tl.f0 / PAIR_F) * p.plan_words + p.plan_words - 1);
+    const uint32_t wm = __ldg(br.plan + (size_t)(tl.f0 / PAIR_F) * p.plan_words + p.plan_words - 1);
     return static_cast<uint64_t>(m) * wm <= (1ull << 48);
 }
 
@@ -249,12 +249,14 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
     if (pair < p.total_tiles) publish(0, single);
     int n = 0;                         // tiles so far
     for (int t = pair; ok && t < p.total_tiles; t += npairs, ++n) {
-        const int fb = tile_coords(p, t).f0 / PAIR_F;
+        const Tile tc = tile_coords(p, t);
+        const int fb = tc.f0 / PAIR_F;
+        const uint32_t *plan = p.br[tc.branch].plan;
         int32_t run[RUN];
 #pragma unroll
         for (int i = 0; i < RUN; ++i) run[i] = 0;
         for (int ci = 0; ci < NC; ++ci) {
-            if (ci != NC - 1 && (single || !plan_drains(p, fb, ci, NC))) continue;
+            if (ci != NC - 1 && (single || !plan_drains(p, plan, fb, ci, NC))) continue;
             if (!mbar_wait_cluster(sb + BAR_ACCFULL, c & 1, wc, ERR_EPILOGUE)) {
                 ok = false;
                 break;
@@ -520,7 +522,9 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
                 const bool use_single = p.single_ok != 0;
                 int n = 0;                     // tiles so far
                 for (int t = pair; ok && t < p.total_tiles; t += npairs, ++n) {
-                    const int fb = tile_coords(p, t).f0 / PAIR_F;
+                    const Tile tc = tile_coords(p, t);
+                    const int fb = tc.f0 / PAIR_F;
+                    const uint32_t *plan = p.br[tc.branch].plan;
                     bool single = false;       // the tile is one run (published by the epilogue)
                     bool fresh = true;         // the next MMA starts a new accumulation
                     for (int ci = 0; ok && ci < NC; ++ci) {
@@ -568,7 +572,7 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
                             }
                             single = ld_shared_s32(sb + OFF_TFLAG + 4 * (n & 1)) != 0;
                         }
-                        fresh = ci == NC - 1 || (!single && plan_drains(p, fb, ci, NC));
+                        fresh = ci == NC - 1 || (!single && plan_drains(p, plan, fb, ci, NC));
                         if (ok && fresh) {
                             mma_commit_pair_multicast(sb + BAR_ACCFULL, 0x3);
                             ++c;
@@ -772,8 +776,8 @@ cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cu
     return cudaGetLastError();
 }
 
-cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, const uint32_t *plan,
-                           unsigned int *err, cudaStream_t st) {
+cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, unsigned int *err,
+                           cudaStream_t st) {
     if (g_sms == 0) {
         int dev = 0;
         cudaGetDevice(&dev);
@@ -799,13 +803,14 @@ cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_
     for (int i = 0; i < 2; ++i) {
         const GemmBranch *b = (i < nb) ? &br[i] : nullptr;
         BranchArgs &a = p.br[i];
-        a = BranchArgs{nullptr, nullptr, nullptr, nullptr, nullptr, 0, 0, 0};
+        a = BranchArgs{nullptr, nullptr, nullptr, nullptr, nullptr, nullptr, 0, 0, 0};
         if (b && b->M > 0) {
             a.x_scale = b->x_scale;
             a.w_scale = b->w_scale;
             a.bias = b->bias;
             a.out = b->out;
             a.x_sumsq = b->x_sumsq;
+            a.plan = b->plan;
             a.M = b->M;
             a.t_tiles = (b->M + PAIR_T - 1) / PAIR_T;
             a.tiles = a.t_tiles * f_tiles;
@@ -827,11 +832,10 @@ cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_
     p.K = K;
     p.total_tiles = p.br[0].tiles + p.br[1].tiles;
     p.k_blocks = (K + BK - 1) / BK;
-    p.plan = plan;
     p.plan_words = chunk_plan_words(K);
-    p.single_ok = plan != nullptr;
+    p.single_ok = 1;
     for (int i = 0; i < 2; ++i)
-        if (p.br[i].M > 0 && p.br[i].x_sumsq == nullptr) p.single_ok = 0;
+        if (p.br[i].M > 0 && (p.br[i].x_sumsq == nullptr || p.br[i].plan == nullptr)) p.single_ok = 0;
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
     const int pairs = p.total_tiles < g_sms / 2 ? p.total_tiles : g_sms / 2;

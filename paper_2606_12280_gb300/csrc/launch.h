@@ -16,6 +16,7 @@ struct GemmBranch {
     void *out;        // uint16_t* bf16 Y, or int32_t* acc for the debug export
     int M;
     const uint32_t *x_sumsq;   // fp16-code GEMM: per token sum of squared codes, or null
+    const uint32_t *plan;      // fp16-code GEMM: the weights' drain plan, or null
 };
 
 cudaError_t launch_channel_absmax(const uint16_t *X, int T, int K, float *s,
@@ -41,6 +42,17 @@ struct QuantActBranch {
 // a3 for both branches in one launch (two launches for K > 16384).
 cudaError_t launch_quant_act_dual(const QuantActBranch *br, int K, cudaStream_t st);
 
+// a3 with fp16 codes for both branches in one launch, K <= 16384.
+struct QuantActBranch16 {
+    const uint16_t *X;
+    const float *lambda;
+    int M;
+    uint16_t *Xq16;
+    float *x_scale;
+    uint32_t *sumsq;
+};
+cudaError_t launch_quant_act_dual_f16codes(const QuantActBranch16 *br, int K, cudaStream_t st);
+
 // a3 of GELU(H): the GELU evaluated in fp32 and quantized without rounding
 // to bf16 in between.
 cudaError_t launch_gelu_quant_act(const uint16_t *H, const float *lambda, int M, int K, int8_t *Xq,
@@ -60,11 +72,11 @@ cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K,
                             bool out_i32, bool a16, unsigned int *err, cudaStream_t st);
 
 // tcgen05 GEMM on CTA pairs with the weights in tensor memory: Xq holds the
-// activation codes as fp16 values (2 bytes each), Wq the int8 weights.  plan
-// (optional, from launch_chunk_plan on the same Wq) lets runs of K chunks
-// accumulate without a drain where the weights bound the partial sums.
-cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, const uint32_t *plan,
-                           unsigned int *err, cudaStream_t st);
+// activation codes as fp16 values (2 bytes each), Wq the int8 weights.  A
+// branch's plan (from launch_chunk_plan on its Wq) and x_sumsq (from a3) let
+// the accumulation skip drains where they bound the partial sums.
+cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, unsigned int *err,
+                           cudaStream_t st);
 int chunk_plan_words(int K);    // per block of 256 weight rows
 cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cudaStream_t st);
 

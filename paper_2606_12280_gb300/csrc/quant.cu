@@ -737,6 +737,15 @@ cudaError_t launch_quant_act_f16codes(const uint16_t *X, const float *lambda, in
     return gelu ? launch_act_quant_teams<true, true>(p, st) : launch_act_quant_teams<false, true>(p, st);
 }
 
+cudaError_t launch_quant_act_dual_f16codes(const QuantActBranch16 *br, int K, cudaStream_t st) {
+    ActParams p{};
+    for (int i = 0; i < 2; ++i)
+        p.br[i] = ActBranch{br[i].X, br[i].lambda, reinterpret_cast<int8_t *>(br[i].Xq16), br[i].x_scale,
+                            br[i].M, br[i].sumsq};
+    p.K = K;
+    return launch_act_quant_teams<false, true>(p, st);
+}
+
 cudaError_t launch_quant_act_dual(const QuantActBranch *br, int K, cudaStream_t st) {
     if (K <= 16384) {
         ActParams p{};

@@ -52,6 +52,8 @@ SIGNATURES = {
     "w8a8_linear_f16codes": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P],
     "w8a8_debug_gemm_f16codes_i32": [_P, _P, _I, _I, _I, _P, _P, _P, _P],
     "w8a8_chunk_plan_size": [_I, _I],
+    "w8a8_quant_act_dual_f16codes": [_P, _I, _P],
+    "w8a8_linear_dual_f16codes": [_P, _I, _I, _P],
     "w8a8_chunk_plan": [_P, _I, _I, _P, _P],
     "w8a8_act_stats_noalloc": [_P, _I, _I, _P, _P, _P, _P],
 }
@@ -76,6 +78,17 @@ class Branch(ctypes.Structure):
 class ActBranch(ctypes.Structure):
     """Mirror of ``w8a8_act_branch``."""
     _fields_ = [("X", _P), ("smooth", _P), ("M", _I), ("Xq", _P), ("x_scale", _P)]
+
+
+class ActBranch16(ctypes.Structure):
+    """Mirror of ``w8a8_act_branch16``."""
+    _fields_ = [("X", _P), ("smooth", _P), ("M", _I), ("Xq16", _P), ("x_scale", _P), ("x_sumsq", _P)]
+
+
+class Branch16(ctypes.Structure):
+    """Mirror of ``w8a8_branch16``."""
+    _fields_ = [("Xq16", _P), ("x_scale", _P), ("Wq", _P), ("w_scale", _P), ("bias", _P), ("Y", _P),
+                ("M", _I), ("chunk_plan", _P), ("x_sumsq", _P)]
 
 
 class Layer(ctypes.Structure):
@@ -273,6 +286,56 @@ def quant_act_dual(branches, out=None, stream=None):
         res.append((Xq, sx))
     _check("w8a8_quant_act_dual", lib().w8a8_quant_act_dual(arr, K, _stream(stream)))
     return res
+
+
+def quant_act_dual_f16codes(branches, out=None, stream=None):
+    """a3 with fp16 codes for two branches in one launch: branches = [(X,
+    smooth), (X, smooth)]; returns [(Xq16, sx, sumsq), ...] (written into
+    `out` when given; sumsq int32 [M] holding the uint32 token sums)."""
+    if len(branches) != 2:
+        raise ValueError("quant_act_dual_f16codes takes exactly two branches")
+    K = branches[0][0].shape[1]
+    arr = (ActBranch16 * 2)()
+    res = []
+    for i, (X, sm) in enumerate(branches):
+        if X.shape[1] != K:
+            raise ValueError("branches must share K")
+        M = X.shape[0]
+        if out is not None:
+            Xq16, sx, ss = out[i]
+        else:
+            Xq16 = torch.empty(M, K, dtype=torch.float16, device=X.device)
+            sx = torch.empty(M, dtype=torch.float32, device=X.device)
+            ss = torch.empty(M, dtype=torch.int32, device=X.device)
+        arr[i] = ActBranch16(_ptr(X, torch.bfloat16, "X"), _ptr(sm, torch.float32, "smooth"), M,
+                             _ptr(Xq16, torch.float16, "Xq16"), _ptr(sx, torch.float32, "x_scale"),
+                             _ptr(ss, torch.int32, "sumsq"))
+        res.append((Xq16, sx, ss))
+    _check("w8a8_quant_act_dual_f16codes", lib().w8a8_quant_act_dual_f16codes(arr, K, _stream(stream)))
+    return res
+
+
+def linear_dual_f16codes(branches, Ys=None, stream=None):
+    """One grouped launch over two branches with fp16 codes.  branches: two
+    tuples (Xq16, x_scale, Wq, w_scale, bias, plan, x_sumsq) (plan and x_sumsq
+    may be None); returns [Y_cond, Y_uncond]."""
+    if len(branches) != 2:
+        raise ValueError("linear_dual_f16codes takes exactly two branches")
+    N, K = branches[0][2].shape
+    arr = (Branch16 * 2)()
+    out = []
+    for i, (Xq16, sx, Wq, sw, b, plan, ss) in enumerate(branches):
+        if tuple(Wq.shape) != (N, K) or Xq16.shape[1] != K:
+            raise ValueError("branches must share N and K")
+        Y = Ys[i] if Ys is not None else torch.empty(Xq16.shape[0], N, dtype=torch.bfloat16,
+                                                     device=Xq16.device)
+        arr[i] = Branch16(_ptr(Xq16, torch.float16, "Xq16"), _ptr(sx, torch.float32, "x_scale"),
+                          _ptr(Wq, torch.int8, "Wq"), _ptr(sw, torch.float32, "w_scale"),
+                          _ptr(b, torch.float32, "bias"), _ptr(Y, torch.bfloat16, "Y"), Xq16.shape[0],
+                          _ptr(plan, torch.int32, "plan"), _ptr(ss, torch.int32, "x_sumsq"))
+        out.append(Y)
+    _check("w8a8_linear_dual_f16codes", lib().w8a8_linear_dual_f16codes(arr, N, K, _stream(stream)))
+    return out
 
 
 def gelu_quant_act(H, smooth=None, Xq=None, x_scale=None, stream=None):

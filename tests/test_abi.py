@@ -292,3 +292,36 @@ def test_noalloc_stats_validation(L):
     assert f(A, 0, 16, None, A, A, None) == INVALID            # no tokens
     assert f(None, 4, 16, None, A, A, None) == INVALID
     assert f(A, 4, 16, None, U, A, None) == MISALIGNED
+
+
+def test_dual_f16codes_validation(L):
+    from paper_2606_12280_gb300.w8a8 import ActBranch16, Branch16
+    qa = (ActBranch16 * 2)()
+    for i in range(2):
+        qa[i] = ActBranch16(A, None, 4, A, A, None)
+    f = L.w8a8_quant_act_dual_f16codes
+    assert f(None, 16, None) == INVALID
+    assert f(qa, 24, None) == SHAPE
+    assert f(qa, 16400, None) == SHAPE                   # K beyond 16384
+    qa[1].x_sumsq = U
+    assert f(qa, 16, None) == MISALIGNED
+    qa[1].x_sumsq = None
+    qa[1].Xq16 = None
+    assert f(qa, 16, None) == INVALID
+    qa[0] = ActBranch16(None, None, 0, None, None, None)
+    qa[1] = ActBranch16(None, None, 0, None, None, None)
+    assert f(qa, 16, None) == OK                         # both branches empty
+    ga = (Branch16 * 2)()
+    for i in range(2):
+        ga[i] = Branch16(A, A, A, A, None, A, 4, None, None)
+    g = L.w8a8_linear_dual_f16codes
+    assert g(None, 8, 16, None) == INVALID
+    assert g(ga, 12, 16, None) == SHAPE
+    ga[1].chunk_plan = U
+    assert g(ga, 8, 16, None) == MISALIGNED
+    ga[1].chunk_plan = None
+    ga[1].Wq = None
+    assert g(ga, 8, 16, None) == INVALID
+    ga[0] = Branch16(None, None, None, None, None, None, 0, None, None)
+    ga[1] = Branch16(None, None, None, None, None, None, 0, None, None)
+    assert g(ga, 8, 16, None) == OK                      # both branches empty

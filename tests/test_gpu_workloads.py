@@ -2,7 +2,10 @@
 bench.py uses: the whole layer (calibration statistic, smoothing vector,
 weight quantization, activation quantization, INT8 GEMM with fused epilogue,
 the dual-branch launch where the workload has two branches) runs on the GPU
-through the C ABI and is compared with the CPU oracle.
+through the C ABI and is compared with the CPU oracle.  The fp16-code path
+(the benchmarked one: codes as fp16 values with their token sums of squares,
+the weights' drain plan, single or dual-branch launches) runs beside it and
+must give the same codes and bitwise the same outputs.
 
 lambda, Wq, w_scale, Xq and x_scale are compared in full (bit-exact); the bf16
 output is compared on sampled rows (first, last and seeded random rows), which
@@ -75,8 +78,29 @@ def run_case(w8, oracle_mod, case, info=False):
         Ys = w8.linear_dual(branches)
     else:
         Ys = [w8.linear(*branches[0])]
+    # the fp16-code path on the same layer
+    lams = [w8.smooth_scales(s, torch.from_numpy(case.W[i]).to(DEV), case.alpha) for i in range(nb)]
+    plans = [w8.chunk_plan(branches[i][2]) for i in range(nb)]
+    if nb == 2:
+        q = w8.quant_act_dual_f16codes([(bf(case.X[i]), lams[i]) for i in range(2)])
+        Y16 = w8.linear_dual_f16codes([(q[i][0], q[i][1], branches[i][2], branches[i][3], branches[i][4],
+                                        plans[i], q[i][2]) for i in range(2)])
+    else:
+        ss = torch.empty(M, dtype=torch.int32, device=DEV)
+        q16, sx16 = w8.quant_act_f16codes(bf(case.X[0]), lams[0], sumsq=ss)
+        q = [(q16, sx16, ss)]
+        Y16 = [w8.linear_f16codes(q16, sx16, branches[0][2], branches[0][3], branches[0][4],
+                                  plan=plans[0], x_sumsq=ss)]
     torch.cuda.synchronize()
     assert w8.device_status() == 0
+    for i in range(nb):
+        Xq_ref = refs[i][0]
+        assert torch.equal(q[i][0].to(torch.int8), branches[i][0])
+        assert torch.equal(q[i][1], branches[i][1])
+        np.testing.assert_array_equal(q[i][2].cpu().numpy().view(np.uint32),
+                                      (Xq_ref.astype(np.int64) ** 2).sum(1).astype(np.uint32))
+        assert torch.equal(Y16[i], Ys[i]), f"branch {i}: fp16-code path differs"
+    del Y16, q
     rows = sample_rows(M)
     for i in range(nb):
         got = u16(Ys[i])[rows]
