@@ -267,3 +267,35 @@ def test_linear_f16codes_exact_with_sumsq(w8, oracle_mod, M, N, K):
     Y = w8.linear_f16codes(q16, sx, t(Wq), t(sw), t(c.bias[0]), plan=w8.chunk_plan(t(Wq)), x_sumsq=ss)
     Xq, wsx = oracle_mod.quant_act(c.X[0], lam)
     np.testing.assert_array_equal(u16(Y), oracle_mod.linear(Xq, wsx, Wq, sw, c.bias[0]))
+
+
+# ------------------------------------------------------------- dual branches
+
+@pytest.mark.parametrize("M0,M1", [(300, 130), (0, 257), (513, 0), (256, 256)])
+def test_dual_f16codes_equals_singles(w8, oracle_mod, M0, M1):
+    N, K = 520, 1040
+    cs = [wl.make_case(max(M, 1), K, N, seed=M + 7 * b) for b, M in enumerate((M0, M1))]
+    branches_q, branches_g, singles = [], [], []
+    for b, (c, M) in enumerate(zip(cs, (M0, M1))):
+        s = oracle_mod.channel_absmax(c.X_cal)
+        lam = oracle_mod.smooth_scales(s, c.W[0], c.alpha)
+        Wq, sw = oracle_mod.quantize_weights(c.W[0], lam)
+        X = c.X[0][:M]
+        branches_q.append((bf(X) if M else torch.empty(0, K, dtype=torch.bfloat16, device=DEV), t(lam)))
+        branches_g.append((t(Wq), t(sw), t(c.bias[0]), w8.chunk_plan(t(Wq))))
+        singles.append((X, lam, Wq, sw, c.bias[0]))
+    q = w8.quant_act_dual_f16codes(branches_q)
+    Ys = w8.linear_dual_f16codes([(q[b][0], q[b][1], *branches_g[b][:3], branches_g[b][3], q[b][2])
+                                  for b in range(2)])
+    for b, (X, lam, Wq, sw, bias) in enumerate(singles):
+        M = X.shape[0]
+        if M == 0:
+            assert Ys[b].shape[0] == 0
+            continue
+        ss = torch.empty(M, dtype=torch.int32, device=DEV)
+        q16, sx = w8.quant_act_f16codes(bf(X), t(lam), sumsq=ss)
+        assert torch.equal(q16, q[b][0]) and torch.equal(sx, q[b][1]) and torch.equal(ss, q[b][2])
+        Y1 = w8.linear_f16codes(q16, sx, t(Wq), t(sw), t(bias), plan=branches_g[b][3], x_sumsq=ss)
+        assert torch.equal(Y1, Ys[b])
+        Xq, wsx = oracle_mod.quant_act(X, lam)
+        np.testing.assert_array_equal(u16(Ys[b]), oracle_mod.linear(Xq, wsx, Wq, sw, bias))
