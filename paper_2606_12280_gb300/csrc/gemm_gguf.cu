@@ -5,17 +5,23 @@
 // Sec. 3, "GGUF k-quants": the DiT serialized to Q8_0 (8.5 bits per weight)
 // and Q4_K (4.5 bits, the paper's memory-Pareto choice), which it ran with a
 // Torch dequantization (Sec. 5).  Here the weights stay in their GGUF blocks
-// in HBM and are decoded tile by tile in shared memory, next to the MMA.
+// in HBM and are decoded next to the MMA, straight into tensor memory: the
+// decoded weights are the MMA's A operand in TMEM ("TS" form), the
+// activations its B operand in shared memory, loaded by TMA unconverted, so
+// no decoded operand passes through shared memory (the same placement as
+// gemm_ts.cu).
 //
-// A cluster of two CTAs (one per SM) computes a 256 x 256 output tile.  Per
-// CTA: warp 0 issues TMA loads of X tiles [128 x 64] straight into the
-// 128-byte-swizzled K-major layout and of raw weight blocks [128 rows x one
-// 256-weight span] into a raw ring; warp 1 allocates TMEM (both CTAs) and,
-// on the leader, issues one M=256 N=256 K=16 bf16 MMA per K step; the
-// converter warps decode the raw blocks of each K=64 step into the swizzled
-// bf16 B tile (fp32 arithmetic as the decoder defines it, then round to
-// bf16); the last four warps drain the fp32 accumulator (two TMEM buffers),
-// add the bias and write bf16.  All waits are bounded in time.
+// A cluster of two CTAs computes a 256 (output features) x 256 (tokens) tile
+// of Y^T: CTA r decodes weight rows f0 + 128r .. +127 into its TMEM lanes
+// (one row per converter thread) and holds tokens t0 + 128r .. +127 in its
+// shared memory; the leader issues M=256 N=256 K=16 bf16 MMAs, eight per
+// stage of K=128.  TMEM per CTA: one 256-column fp32 accumulator and four
+// 64-column weight slots.  Per CTA: warp 0 TMA of the raw weight blocks (one
+// 256-weight span per ring slot), warp 2 TMA of the activations (both CTAs
+// against the leader's barrier), warp 1 TMEM allocation and MMA issue
+// (leader), warps 4-7 decode (warp w owns TMEM lanes 32(w%4) .. +31), warps
+// 8-15 drain the accumulator once per tile, add the bias and write bf16.
+// All waits are bounded in time.
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_fp16.h>
@@ -29,34 +35,27 @@ namespace {
 
 using namespace tc;
 
-constexpr int PAIR_M = 256, CTA_M = 128, PAIR_N = 256, CTA_N = 128;
-constexpr int BK = 64;                         // bf16 per swizzle row = one MMA stage
+constexpr int PAIR_F = 256, CTA_F = 128;      // output features per pair / CTA (MMA M)
+constexpr int PAIR_T = 256, CTA_T = 128;      // tokens per pair / CTA (MMA N)
+constexpr int BK = 64;                         // bf16 per swizzle row = one K=64 sub-block
 constexpr int KR = 256;                        // weights per raw span (one Q4_K block)
-#ifndef W8A8_GGUF_SUB
-#define W8A8_GGUF_SUB 2
-#endif
-#ifndef W8A8_GGUF_STAGES
-#define W8A8_GGUF_STAGES 2
-#endif
-constexpr int SUB = W8A8_GGUF_SUB;             // K=64 steps per pipeline stage
-constexpr int SUBS = KR / BK;                  // K=64 steps per raw span
-constexpr int STAGES_PER_SPAN = SUBS / SUB;
-constexpr int S = W8A8_GGUF_STAGES;            // bf16 stage ring
-constexpr int TILE_BYTES = CTA_M * BK * 2;     // 16 KB, A or B of one K=64 step
-constexpr int STEP_BYTES = 2 * TILE_BYTES;     // A then B
-constexpr int STAGE = SUB * STEP_BYTES;
-static_assert(SUBS % SUB == 0, "whole stages per raw span");
-#ifndef W8A8_GGUF_CONV_WARPS
-#define W8A8_GGUF_CONV_WARPS 8
-#endif
-constexpr int NUM_CONV_WARPS = W8A8_GGUF_CONV_WARPS;
-constexpr int CONV_TASKS = CTA_N * 4;          // per K=64 step: 128 rows x 4 chunk pairs
-constexpr int kTasksPerThread = CONV_TASKS / (32 * NUM_CONV_WARPS);
-static_assert(CONV_TASKS % (32 * NUM_CONV_WARPS) == 0, "whole tasks per converter thread");
-constexpr int NUM_EPI_WARPS = 4;
-constexpr int CONV_WARP0 = 2, EPI_WARP0 = CONV_WARP0 + NUM_CONV_WARPS;
-constexpr int THREADS = 32 * (EPI_WARP0 + NUM_EPI_WARPS);
+constexpr int SUB = 2;                         // sub-blocks per stage (K=128)
+constexpr int STAGES_PER_SPAN = KR / (SUB * BK);
+constexpr int SA = 4;                          // slots: TMEM weights + smem activations
+constexpr int SUBX = CTA_T * BK * 2;           // 16 KB of activations per sub-block
+constexpr int STAGE_X = SUB * SUBX;
+constexpr uint32_t ACC_COLS = PAIR_T;
+constexpr uint32_t A_COL0 = ACC_COLS;
+constexpr uint32_t A_SLOT_COLS = SUB * BK / 2; // bf16 pairs per row of a slot
+constexpr int NUM_CONV_WARPS = 4;
+constexpr int NUM_EPI_WARPS = 8;
+constexpr int THREADS = 512;
+constexpr int LAUNCH_REGS = 128;
+constexpr int REGS_LOW = 72, REGS_HIGH = 184;
+static_assert(256 * REGS_LOW + 256 * REGS_HIGH <= THREADS * LAUNCH_REGS, "register split");
+constexpr int RUN = PAIR_T / 2;                // accumulator columns per epilogue thread
 constexpr int TMEM_COLS = 512;
+static_assert(A_COL0 + SA * A_SLOT_COLS <= TMEM_COLS, "tensor memory");
 constexpr int SMEM_BARRIERS = 256;
 
 constexpr unsigned ERR_PRODUCER = 1u, ERR_CONVERTER = 2u, ERR_MMA = 4u, ERR_EPILOGUE = 8u,
@@ -74,24 +73,24 @@ template <> struct Fmt<1> {                    // Q4_K: fp16 d, fp16 dmin, 12 B 
 };
 
 template <int FMT> struct Layout {
-    static constexpr int RAW_SLOT = CTA_N * Fmt<FMT>::ROW;
+    static constexpr int RAW_SLOT = CTA_F * Fmt<FMT>::ROW;
     static constexpr int SR = Fmt<FMT>::SR;
-    static constexpr uint32_t OFF_ST = 0;
-    static constexpr uint32_t OFF_RAW = S * STAGE;
+    static constexpr uint32_t OFF_X = 0;
+    static constexpr uint32_t OFF_RAW = OFF_X + SA * STAGE_X;
     static constexpr uint32_t OFF_BAR = OFF_RAW + SR * RAW_SLOT;
     static constexpr uint32_t BAR_RFULL = OFF_BAR;
     static constexpr uint32_t BAR_REMPTY = BAR_RFULL + 8 * SR;
-    static constexpr uint32_t BAR_AFULL = BAR_REMPTY + 8 * SR;
-    static constexpr uint32_t BAR_FULL = BAR_AFULL + 8 * S;
-    static constexpr uint32_t BAR_EMPTY = BAR_FULL + 8 * S;
-    static constexpr uint32_t BAR_ACCFULL = BAR_EMPTY + 8 * S;
-    static constexpr uint32_t BAR_ACCEMPTY = BAR_ACCFULL + 16;
-    static constexpr uint32_t BAR_DRAIN = BAR_ACCEMPTY + 16;
+    static constexpr uint32_t BAR_SFULL = BAR_REMPTY + 8 * SR;     // leader: slot written and landed
+    static constexpr uint32_t BAR_SEMPTY = BAR_SFULL + 8 * SA;     // MMA done with the slot
+    static constexpr uint32_t BAR_ACCFULL = BAR_SEMPTY + 8 * SA;
+    static constexpr uint32_t BAR_ACCEMPTY = BAR_ACCFULL + 8;
+    static constexpr uint32_t BAR_DRAIN = BAR_ACCEMPTY + 8;
     static constexpr uint32_t OFF_TMEM = BAR_DRAIN + 8;
     static constexpr uint32_t OFF_ABORT = OFF_TMEM + 4;
     static constexpr int SMEM_TOTAL = 1024 + OFF_BAR + SMEM_BARRIERS;
     static_assert(OFF_ABORT + 4 - OFF_BAR <= SMEM_BARRIERS, "barrier area");
     static_assert(SMEM_TOTAL <= 232448, "shared memory");
+    static_assert(RAW_SLOT % 16 == 0 && STAGE_X % 1024 == 0, "TMA destinations aligned");
 };
 
 __host__ __device__ constexpr uint32_t idesc_bf16_f32(int M, int N) {
@@ -103,28 +102,10 @@ struct Params {
     const float *bias;
     uint16_t *Y;
     int M, N, K;
-    int m_tiles, total_tiles, spans;           // spans = K / 256 per tile
+    int t_tiles, total_tiles, spans;           // spans = K / 256 per tile
     unsigned int *err;
     uint64_t wait_limit_ns;
 };
-
-__device__ __forceinline__ uint32_t ld_shared_u32(uint32_t a) {
-    uint32_t v;
-    asm volatile("ld.shared.u32 %0, [%1];" : "=r"(v) : "r"(a));
-    return v;
-}
-
-__device__ __forceinline__ uint2 ld_shared_v2(uint32_t a) {
-    uint2 v;
-    asm volatile("ld.shared.v2.u32 {%0,%1}, [%2];" : "=r"(v.x), "=r"(v.y) : "r"(a));
-    return v;
-}
-
-__device__ __forceinline__ uint32_t ld_shared_u16(uint32_t a) {
-    uint16_t v;
-    asm volatile("ld.shared.u16 %0, [%1];" : "=h"(v) : "r"(a));
-    return v;
-}
 
 __device__ __forceinline__ float f16_bits_to_f32(uint32_t h) {
     return __half2float(__ushort_as_half(static_cast<unsigned short>(h)));
@@ -219,57 +200,98 @@ __device__ __forceinline__ uint4 q8_chunk(uint32_t lo, uint32_t hi, float d) {
     return make_uint4(w[0], w[1], w[2], w[3]);
 }
 
-// Per-row constants of one 256-weight span, computed once per span and kept
-// in registers: Q4_K d * sc_j and dmin * m_j for the eight sub-blocks; Q8_0
-// the eight block scales d (in d1).
-struct Q4kRow {
-    float d1[8], m1[8];
-};
-
-__device__ __forceinline__ void q8_row_consts(uint32_t src, Q4kRow &r) {
+// Decode stage H (weights 128H .. 128H + 127 of the 256-weight span) of one
+// weight row (`row`: its raw bytes in shared memory) into 64 bf16x2 columns
+// of TMEM at `tcol` (this warp's lanes), two tcgen05.st of 32 columns.
+//
+// Q8_0: blocks 4H .. 4H + 3, two at a time: the 68 bytes of blocks b0, b0 + 1
+// start 4-byte aligned (34 b0 = 136H + 68k) and are read as five 16-byte loads
+// (conflict-free across a warp's rows at the 272-byte stride); block b0's
+// quants start 2 bytes into it (byte permutes), block b0 + 1's are aligned.
+template <int H>
+__device__ __forceinline__ void q8_stage(uint32_t row, uint32_t tcol) {
 #pragma unroll
-    for (int b = 0; b < 8; ++b) r.d1[b] = f16_bits_to_f32(ld_shared_u16(src + 34 * b));
+    for (int k = 0; k < 2; ++k) {
+        const int s0 = 136 * H + 68 * k;
+        const int a0 = s0 & ~15;
+        const int w0 = (s0 - a0) / 4;
+        uint32_t W[20];
+#pragma unroll
+        for (int i = 0; i < 5; ++i) {
+            const uint4 v = ld_shared_v4(row + a0 + 16 * i);
+            W[4 * i] = v.x;
+            W[4 * i + 1] = v.y;
+            W[4 * i + 2] = v.z;
+            W[4 * i + 3] = v.w;
+        }
+        const float da = f16_bits_to_f32(W[w0] & 0xffffu);
+        const float db = f16_bits_to_f32(W[w0 + 8] >> 16);
+        uint32_t out[32];
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const uint4 o = q8_chunk(__byte_perm(W[w0 + 2 * c], W[w0 + 2 * c + 1], 0x5432),
+                                     __byte_perm(W[w0 + 2 * c + 1], W[w0 + 2 * c + 2], 0x5432), da);
+            out[4 * c] = o.x;
+            out[4 * c + 1] = o.y;
+            out[4 * c + 2] = o.z;
+            out[4 * c + 3] = o.w;
+        }
+#pragma unroll
+        for (int c = 0; c < 4; ++c) {
+            const uint4 o = q8_chunk(W[w0 + 9 + 2 * c], W[w0 + 10 + 2 * c], db);
+            out[16 + 4 * c] = o.x;
+            out[16 + 4 * c + 1] = o.y;
+            out[16 + 4 * c + 2] = o.z;
+            out[16 + 4 * c + 3] = o.w;
+        }
+        tmem_st_32x32b_x32(tcol + 32 * k, out);
+    }
 }
 
-__device__ __forceinline__ void q4k_row_consts(uint32_t src, Q4kRow &r) {
-    const uint32_t dd = ld_shared_u32(src);
-    const float d = f16_bits_to_f32(dd & 0xffffu), dmin = f16_bits_to_f32(dd >> 16);
-    const uint32_t w0 = ld_shared_u32(src + 4), w1 = ld_shared_u32(src + 8), w2 = ld_shared_u32(src + 12);
+// Q4_K: the block header (d, dmin, 12 scale bytes), then chunks c = 2H and
+// 2H + 1 of 32 quant bytes: low nibbles are weights 64c .. 64c + 31
+// (sub-block 2c), high nibbles 64c + 32 .. 64c + 63 (sub-block 2c + 1).
+template <int H>
+__device__ __forceinline__ void q4k_stage(uint32_t row, uint32_t tcol) {
+    const uint4 hd = ld_shared_v4(row);
+    const float d = f16_bits_to_f32(hd.x & 0xffffu), dmin = f16_bits_to_f32(hd.x >> 16);
 #pragma unroll
-    for (int j = 0; j < 8; ++j) {
+    for (int k = 0; k < 2; ++k) {
+        const int c = 2 * H + k;
+        const uint4 qa = ld_shared_v4(row + 16 + 32 * c), qb = ld_shared_v4(row + 32 + 32 * c);
         uint32_t sc, m;
-        q4k_scale_min(w0, w1, w2, j, sc, m);
-        r.d1[j] = __fmul_rn(d, static_cast<float>(sc));     // exact: 11 x 6 bits
-        r.m1[j] = __fmul_rn(dmin, static_cast<float>(m));
+        q4k_scale_min(hd.y, hd.z, hd.w, 2 * c, sc, m);
+        const float d1a = __fmul_rn(d, static_cast<float>(sc)), m1a = __fmul_rn(dmin, static_cast<float>(m));
+        q4k_scale_min(hd.y, hd.z, hd.w, 2 * c + 1, sc, m);
+        const float d1b = __fmul_rn(d, static_cast<float>(sc)), m1b = __fmul_rn(dmin, static_cast<float>(m));
+        const uint2 v[4] = {make_uint2(qa.x, qa.y), make_uint2(qa.z, qa.w), make_uint2(qb.x, qb.y),
+                            make_uint2(qb.z, qb.w)};
+        uint32_t out[32];
+#pragma unroll
+        for (int e = 0; e < 4; ++e) {
+            const uint4 lo = q4k_chunk<0>(v[e], d1a, m1a);
+            const uint4 hi = q4k_chunk<4>(v[e], d1b, m1b);
+            out[4 * e] = lo.x;
+            out[4 * e + 1] = lo.y;
+            out[4 * e + 2] = lo.z;
+            out[4 * e + 3] = lo.w;
+            out[16 + 4 * e] = hi.x;
+            out[16 + 4 * e + 1] = hi.y;
+            out[16 + 4 * e + 2] = hi.z;
+            out[16 + 4 * e + 3] = hi.w;
+        }
+        tmem_st_32x32b_x32(tcol + 32 * k, out);
     }
 }
 
-// One converter task: row `row` of the CTA's 128 weight rows, output chunks c
-// and c + 4 (16 bf16) of K=64 step u of the raw span.  Q4_K: chunk c holds
-// the low nibbles (sub-block 2u), chunk c + 4 the high nibbles (2u + 1) of
-// the same 8 quant bytes.  Q8_0: chunks c and c + 4 come from blocks 2u and
-// 2u + 1, whose 8 quant bytes start 2 bytes into their 34-byte block.
-template <int FMT>
-__device__ __forceinline__ void convert_task(uint32_t raw, uint32_t dst, int row, int c, int u,
-                                             float d1a, float m1a, float d1b, float m1b) {
-    const uint32_t src = raw + static_cast<uint32_t>(row) * Fmt<FMT>::ROW;
-    uint4 lo, hi;
-    if (FMT == 1) {
-        const uint2 v = ld_shared_v2(src + 16 + 32 * u + 8 * c);
-        lo = q4k_chunk<0>(v, d1a, m1a);
-        hi = q4k_chunk<4>(v, d1b, m1b);
-    } else {
-        // block 2u's quants start 2 mod 4 bytes into the row: three aligned
-        // words and two byte permutes; block 2u + 1's are 4-byte aligned
-        const uint32_t q0 = src + 34 * (2 * u) + 2 + 8 * c, q1 = q0 + 34;
-        const uint32_t x0 = ld_shared_u32(q0 - 2), x1 = ld_shared_u32(q0 + 2), x2 = ld_shared_u32(q0 + 6);
-        lo = q8_chunk(__byte_perm(x0, x1, 0x5432), __byte_perm(x1, x2, 0x5432), d1a);
-        hi = q8_chunk(ld_shared_u32(q1), ld_shared_u32(q1 + 4), d1b);
-    }
-    // 128-byte swizzle: 16-byte chunk k of row r at (k ^ (r & 7))
-    const uint32_t rb = dst + static_cast<uint32_t>(row) * 128;
-    st_shared_v4(rb + ((static_cast<uint32_t>(c) ^ (row & 7)) << 4), lo);
-    st_shared_v4(rb + ((static_cast<uint32_t>(c + 4) ^ (row & 7)) << 4), hi);
+__device__ __forceinline__ void arrive_leader(uint32_t bar, uint32_t rank) {
+    if (rank == 0) mbar_arrive(bar);
+    else mbar_arrive_cluster_relaxed(mapa_shared(bar, 0));
+}
+
+__device__ __forceinline__ void tile_coords(const Params &p, int t, int &t0, int &f0) {
+    t0 = (t % p.t_tiles) * PAIR_T;
+    f0 = (t / p.t_tiles) * PAIR_F;
 }
 
 template <int FMT>
@@ -278,57 +300,59 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
                                               uint32_t rank, int pair, int npairs) {
     using L = Layout<FMT>;
     const int q = warp & 3;                          // TMEM lane quarter of this warp
+    const int h = (warp - 8) >> 2;                   // token half of the tile
     uint32_t c = 0;
     for (int t = pair; t < p.total_tiles; t += npairs, ++c) {
-        const uint32_t buf = c & 1;
-        if (!mbar_wait_cluster(sb + L::BAR_ACCFULL + 8 * buf, (c >> 1) & 1, wc, ERR_EPILOGUE)) break;
+        if (!mbar_wait_cluster(sb + L::BAR_ACCFULL, c & 1, wc, ERR_EPILOGUE)) break;
         tc_fence_after();
-        const int m0 = (t % p.m_tiles) * PAIR_M;
-        const int n0 = (t / p.m_tiles) * PAIR_N;
-        const int m = m0 + static_cast<int>(rank) * CTA_M + q * 32 + lane;
-        const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * PAIR_N;
-        uint16_t *out = p.Y + (size_t)m * p.N + n0;
-#pragma unroll 1
-        for (int cc = 0; cc < PAIR_N / 16; ++cc) {
-            uint32_t v[16];
-            tmem_ld_32x32b_x16(base + cc * 16, v);
+        const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) + h * RUN;
+        uint32_t acc[RUN];
+#pragma unroll
+        for (int jj = 0; jj < RUN / 16; jj += 4) {
+            uint32_t v[4][16];
+#pragma unroll
+            for (int g = 0; g < 4; ++g) tmem_ld_32x32b_x16(base + (jj + g) * 16, v[g]);
             tmem_ld_wait();
-            const int n = n0 + cc * 16;
-            if (m < p.M) {
 #pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    if (n + 8 * h < p.N) {
-                        float b[8];
+            for (int g = 0; g < 4; ++g)
 #pragma unroll
-                        for (int i = 0; i < 8; ++i) b[i] = 0.0f;
-                        if (p.bias != nullptr) {
-                            const float4 b0 = __ldg(reinterpret_cast<const float4 *>(p.bias + n + 8 * h));
-                            const float4 b1 = __ldg(reinterpret_cast<const float4 *>(p.bias + n + 8 * h + 4));
-                            b[0] = b0.x; b[1] = b0.y; b[2] = b0.z; b[3] = b0.w;
-                            b[4] = b1.x; b[5] = b1.y; b[6] = b1.z; b[7] = b1.w;
-                        }
-                        uint32_t w[4];
-#pragma unroll
-                        for (int i = 0; i < 4; ++i)
-                            w[i] = pack_bf16_pair(add2(pk2(v[8 * h + 2 * i], v[8 * h + 2 * i + 1]),
-                                                       pk2(__float_as_uint(b[2 * i]), __float_as_uint(b[2 * i + 1]))));
-                        *reinterpret_cast<uint4 *>(out + cc * 16 + 8 * h) = make_uint4(w[0], w[1], w[2], w[3]);
-                    }
-                }
-            }
+                for (int i = 0; i < 16; ++i) acc[(jj + g) * 16 + i] = v[g][i];
         }
         tc_fence_before();
         __syncwarp();
-        if (lane == 0) {
-            if (rank == 0) mbar_arrive(sb + L::BAR_ACCEMPTY + 8 * buf);
-            else mbar_arrive_cluster_relaxed(mapa_shared(sb + L::BAR_ACCEMPTY + 8 * buf, 0));
+        if (lane == 0) arrive_leader(sb + L::BAR_ACCEMPTY, rank);
+        int t0, f0;
+        tile_coords(p, t, t0, f0);
+        const int f = f0 + static_cast<int>(rank) * CTA_F + q * 32 + lane;    // output feature
+        const int tok0 = t0 + h * RUN;
+        const int ntok = min(RUN, p.M - tok0);
+        const bool fok = f < p.N;
+        if (ntok > 0) {                              // uniform across the warp
+            const float b = (p.bias != nullptr && fok) ? __ldg(p.bias + f) : 0.0f;
+            // lanes 2i, 2i + 1 (features f, f + 1) swap one value per pair of
+            // tokens, so that each stores one 32-bit word (N % 8 == 0)
+            const bool odd = lane & 1;
+            uint16_t *out = p.Y + (size_t)tok0 * p.N + (f & ~1);
+#pragma unroll
+            for (int i = 0; i < RUN; i += 2) {
+                const uint32_t y = pack_bf16_pair(add2(pk2(acc[i], acc[i + 1]),
+                                                       pk2(__float_as_uint(b), __float_as_uint(b))));
+                // y: low = token i, high = token i + 1 of this feature
+                const uint32_t other = __shfl_xor_sync(0xffffffffu, odd ? (y & 0xffffu) : (y >> 16), 1);
+                const uint32_t word = odd ? (other | (y & 0xffff0000u)) : ((y & 0xffffu) | (other << 16));
+                const int tk = i + (odd ? 1 : 0);
+                if (tk < ntok && fok)
+                    asm volatile("st.global.cs.u32 [%0], %1;" ::"l"(out + (size_t)tk * p.N), "r"(word)
+                                 : "memory");
+            }
         }
+        __syncwarp();
     }
 }
 
 template <int FMT>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
-gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmW,
+gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant__ CUtensorMap tmW,
                  const Params p) {
     using L = Layout<FMT>;
     constexpr int SR = L::SR;
@@ -346,21 +370,18 @@ gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
             mbar_init(sb + L::BAR_RFULL + 8 * i, 1);
             mbar_init(sb + L::BAR_REMPTY + 8 * i, NUM_CONV_WARPS);
         }
-        for (int i = 0; i < S; ++i) {
-            mbar_init(sb + L::BAR_AFULL + 8 * i, 1);
-            mbar_init(sb + L::BAR_FULL + 8 * i, 2 * NUM_CONV_WARPS);
-            mbar_init(sb + L::BAR_EMPTY + 8 * i, 1);
+        for (int i = 0; i < SA; ++i) {
+            mbar_init(sb + L::BAR_SFULL + 8 * i, 2 * NUM_CONV_WARPS + 1);
+            mbar_init(sb + L::BAR_SEMPTY + 8 * i, 1);
         }
-        for (int i = 0; i < 2; ++i) {
-            mbar_init(sb + L::BAR_ACCFULL + 8 * i, 1);
-            mbar_init(sb + L::BAR_ACCEMPTY + 8 * i, 2 * NUM_EPI_WARPS);
-        }
+        mbar_init(sb + L::BAR_ACCFULL, 1);
+        mbar_init(sb + L::BAR_ACCEMPTY, 2 * NUM_EPI_WARPS);
         mbar_init(sb + L::BAR_DRAIN, 1);
         st_shared_s32(sb + L::OFF_ABORT, 0);
         fence_barrier_init();
     }
     if (warp == 0 && lane == 0) {
-        tma_prefetch_desc(&tmA);
+        tma_prefetch_desc(&tmX);
         tma_prefetch_desc(&tmW);
     }
     if (warp == 1) {
@@ -375,167 +396,153 @@ gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
     const bool run_ok = (tmem == peer_tmem);
     if (!run_ok && threadIdx.x == 0) atomicOr(p.err, ERR_TMEM_PAIR);
     const WaitCtx wc{sb + L::OFF_ABORT, p.err, p.wait_limit_ns};
-    // spans are numbered q = 0, 1, ... over this pair's tiles in order; span q
-    // is span (q % spans) of tile pair + (q / spans) * npairs
-    const int my_tiles = p.total_tiles > pair ? (p.total_tiles - pair + npairs - 1) / npairs : 0;
-    const int total_spans = my_tiles * p.spans;
+    const int NS = p.spans * STAGES_PER_SPAN;          // stages per tile
 
-    if (!run_ok) {
-    } else if (warp == 0) {
-        // ---------------------------------------------------- TMA producer
-        if (lane == 0) {
-            int raw_issued = 0;
-            auto issue_raw = [&](int qs) -> bool {
-                const int t = pair + (qs / p.spans) * npairs;
-                const int brow = (t / p.m_tiles) * PAIR_N + static_cast<int>(rank) * CTA_N;
-                const uint32_t rs = qs % SR;
-                if (!mbar_wait(sb + L::BAR_REMPTY + 8 * rs, ((qs / SR) & 1) ^ 1, wc, ERR_PRODUCER))
-                    return false;
-                mbar_arrive_expect_tx(sb + L::BAR_RFULL + 8 * rs, L::RAW_SLOT);
-                const int x = FMT == 1 ? (qs % p.spans) * Fmt<FMT>::ROW : (qs % p.spans) * (Fmt<FMT>::ROW / 2);
-                tma_load_2d(sb + L::OFF_RAW + rs * L::RAW_SLOT, &tmW, x, brow, sb + L::BAR_RFULL + 8 * rs);
-                ++raw_issued;
-                return true;
-            };
-            bool ok = total_spans == 0 || issue_raw(0);
-            uint32_t j = 0;
-            for (int qs = 0; ok && qs < total_spans; ++qs) {
-                const int t = pair + (qs / p.spans) * npairs;
-                const int arow = (t % p.m_tiles) * PAIR_M + static_cast<int>(rank) * CTA_M;
-                for (int g = 0; ok && g < STAGES_PER_SPAN; ++g, ++j) {
-                    const uint32_t st = j % S;
-                    if (!mbar_wait_cluster(sb + L::BAR_EMPTY + 8 * st, ((j / S) & 1) ^ 1, wc, ERR_PRODUCER)) {
-                        ok = false;
-                        break;
+    if (warp >= 8) {
+        asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(REGS_HIGH));
+        if (run_ok) epilogue_role<FMT>(p, sb, tmem, wc, warp, lane, rank, pair, npairs);
+    } else {
+        asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(REGS_LOW));
+        if (!run_ok) {
+        } else if (warp == 0) {
+            // ------------------------------- TMA producer: raw weight blocks
+            if (lane == 0) {
+                uint32_t qs = 0;                       // spans so far
+                bool ok = true;
+                for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+                    int t0, f0;
+                    tile_coords(p, t, t0, f0);
+                    const int frow = f0 + static_cast<int>(rank) * CTA_F;
+                    for (int sp = 0; sp < p.spans; ++sp, ++qs) {
+                        const uint32_t rs = qs % SR;
+                        if (!mbar_wait(sb + L::BAR_REMPTY + 8 * rs, ((qs / SR) & 1) ^ 1, wc, ERR_PRODUCER)) {
+                            ok = false;
+                            break;
+                        }
+                        mbar_arrive_expect_tx(sb + L::BAR_RFULL + 8 * rs, L::RAW_SLOT);
+                        const int x = FMT == 1 ? sp * Fmt<FMT>::ROW : sp * (Fmt<FMT>::ROW / 2);
+                        tma_load_2d(sb + L::OFF_RAW + rs * L::RAW_SLOT, &tmW, x, frow, sb + L::BAR_RFULL + 8 * rs);
                     }
-                    mbar_arrive_expect_tx(sb + L::BAR_AFULL + 8 * st, SUB * TILE_BYTES);
+                }
+                for (uint32_t i = (qs > SR ? qs - SR : 0); i < qs; ++i)
+                    mbar_wait(sb + L::BAR_RFULL + 8 * (i % SR), (i / SR) & 1, wc, ERR_DRAIN, false);
+            }
+        } else if (warp == 2) {
+            // ------------------------------- TMA producer: activations (bf16)
+            // both CTAs load against the leader's barrier, which the leader
+            // armed for both CTAs' bytes (every load has landed before the
+            // kernel ends: the MMA waits for each)
+            if (lane == 0) {
+                uint32_t j = 0;
+                bool ok = true;
+                for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+                    int t0, f0;
+                    tile_coords(p, t, t0, f0);
+                    const int trow = t0 + static_cast<int>(rank) * CTA_T;
+                    for (int ks = 0; ks < NS; ++ks, ++j) {
+                        const uint32_t s = j % SA;
+                        if (!mbar_wait_cluster(sb + L::BAR_SEMPTY + 8 * s, ((j / SA) & 1) ^ 1, wc, ERR_PRODUCER)) {
+                            ok = false;
+                            break;
+                        }
+                        const uint32_t fb = mapa_shared(sb + L::BAR_SFULL + 8 * s, 0);
+                        if (leader) mbar_arrive_expect_tx(sb + L::BAR_SFULL + 8 * s, 2 * STAGE_X);
 #pragma unroll
-                    for (int v = 0; v < SUB; ++v)
-                        tma_load_2d(sb + L::OFF_ST + st * STAGE + v * STEP_BYTES, &tmA,
-                                    ((qs % p.spans) * SUBS + g * SUB + v) * BK, arow, sb + L::BAR_AFULL + 8 * st);
-                    if (g == 0 && qs + 1 < total_spans) ok = issue_raw(qs + 1);
+                        for (int u = 0; u < SUB; ++u)
+                            tma_load_2d_pair(sb + L::OFF_X + s * STAGE_X + u * SUBX, &tmX, (ks * SUB + u) * BK, trow, fb);
+                    }
                 }
             }
-            // drain: every issued TMA has landed before the CTA may exit
-            const uint32_t nraw = static_cast<uint32_t>(raw_issued);
-            for (uint32_t i = (j > S ? j - S : 0); i < j; ++i)
-                mbar_wait(sb + L::BAR_AFULL + 8 * (i % S), (i / S) & 1, wc, ERR_DRAIN, false);
-            for (uint32_t i = (nraw > SR ? nraw - SR : 0); i < nraw; ++i)
-                mbar_wait(sb + L::BAR_RFULL + 8 * (i % SR), (i / SR) & 1, wc, ERR_DRAIN, false);
-        }
-    } else if (warp == 1) {
-        // ---------------------------------------------- MMA issue (leader)
-        if (lane == 0 && leader) {
-            constexpr uint32_t idesc = idesc_bf16_f32(PAIR_M, PAIR_N);
-            uint32_t j = 0, c = 0;
-            bool ok = true;
-            for (int t = pair; ok && t < p.total_tiles; t += npairs, ++c) {
-                const uint32_t buf = c & 1;
-                if (!mbar_wait_cluster(sb + L::BAR_ACCEMPTY + 8 * buf, ((c >> 1) & 1) ^ 1, wc, ERR_MMA)) {
-                    ok = false;
-                    break;
-                }
-                tc_fence_after();
-                const uint32_t d = tmem + buf * PAIR_N;
-                const int nk = p.spans * STAGES_PER_SPAN;
-                for (int ks = 0; ks < nk; ++ks, ++j) {
-                    const uint32_t st = j % S;
-                    if (!mbar_wait_cluster(sb + L::BAR_FULL + 8 * st, (j / S) & 1, wc, ERR_MMA)) {
+        } else if (warp == 1) {
+            // ---------------------------------------- MMA issue (leader)
+            if (lane == 0 && leader) {
+                constexpr uint32_t idesc = idesc_bf16_f32(PAIR_F, PAIR_T);
+                const uint64_t b_desc0 = smem_desc_sw128(sb + L::OFF_X);
+                const uint32_t a_base = tmem + A_COL0;
+                uint32_t j = 0, c = 0;
+                bool ok = true;
+                for (int t = pair; ok && t < p.total_tiles; t += npairs, ++c) {
+                    if (!mbar_wait_cluster(sb + L::BAR_ACCEMPTY, (c & 1) ^ 1, wc, ERR_MMA)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
+                    for (int ks = 0; ks < NS; ++ks, ++j) {
+                        const uint32_t sa = j % SA;
+                        if (!mbar_wait_cluster(sb + L::BAR_SFULL + 8 * sa, (j / SA) & 1, wc, ERR_MMA)) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t a = a_base + sa * A_SLOT_COLS;
+                        const uint64_t bd = b_desc0 + sa * (STAGE_X >> 4);
 #pragma unroll
-                    for (int v = 0; v < SUB; ++v) {
-                        const uint32_t a = sb + L::OFF_ST + st * STAGE + v * STEP_BYTES;
-                        const uint32_t b = a + TILE_BYTES;
+                        for (int u = 0; u < SUB; ++u)
 #pragma unroll
-                        for (int kk = 0; kk < BK / 16; ++kk)
-                            mma_f16_ss_pair(d, smem_desc_sw128(a + kk * 32), smem_desc_sw128(b + kk * 32), idesc,
-                                            (ks > 0 || v > 0 || kk > 0) ? 1u : 0u);
+                            for (int kk = 0; kk < BK / 16; ++kk)
+                                mma_f16_ts_pair(tmem, a + u * (BK / 2) + kk * 8, bd + u * (SUBX >> 4) + kk * 2, idesc,
+                                                (ks > 0 || u > 0 || kk > 0) ? 1u : 0u);
+                        mma_commit_pair_multicast(sb + L::BAR_SEMPTY + 8 * sa, 0x3);
                     }
-                    mma_commit_pair_multicast(sb + L::BAR_EMPTY + 8 * st, 0x3);
+                    if (ok) mma_commit_pair_multicast(sb + L::BAR_ACCFULL, 0x3);
                 }
-                if (ok) mma_commit_pair_multicast(sb + L::BAR_ACCFULL + 8 * buf, 0x3);
+                mma_commit_pair(sb + L::BAR_DRAIN);
+                mbar_wait_cluster(sb + L::BAR_DRAIN, 0, wc, ERR_DRAIN, false);
             }
-            mma_commit_pair(sb + L::BAR_DRAIN);
-            mbar_wait_cluster(sb + L::BAR_DRAIN, 0, wc, ERR_DRAIN, false);
-        }
-    } else if (warp < EPI_WARP0) {
-        // ------------------------------------------------------ converters
-        const int cw = warp - CONV_WARP0;
-        const int tid = cw * 32 + lane;
-        const uint32_t full0 = leader ? 0u : mapa_shared(sb + L::BAR_FULL, 0);
-        uint32_t j = 0;
-        bool ok = true;
-        for (int qs = 0; ok && qs < total_spans; ++qs) {
-            const uint32_t rs = qs % SR;
-            // every lane waits; __all_sync keeps the warp's control flow uniform
-            // if a wait gives up
-            if (!__all_sync(0xffffffffu, mbar_wait(sb + L::BAR_RFULL + 8 * rs, (qs / SR) & 1, wc,
-                                                    ERR_CONVERTER)))
-                break;
-            const uint32_t raw = sb + L::OFF_RAW + rs * L::RAW_SLOT;
-            // this thread's tasks: a warp's 32 tasks are 8 consecutive rows
-            // (lane & 7) x the 4 chunk pairs (lane >> 3), so that every
-            // quarter-warp stores to 8 different 16-byte bank groups of the
-            // swizzled tile
-            Q4kRow rc[kTasksPerThread];
+        } else if (warp >= 4) {
+            // ------------------------------------------------------ decoders
+            // thread = weight row r of this CTA = TMEM lane r
+            const uint32_t r = static_cast<uint32_t>((warp & 3) * 32 + lane);
+            const uint32_t a_lane = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + A_COL0;
+            uint32_t j = 0, qs = 0;
+            bool ok = true;
+            for (int t = pair; ok && t < p.total_tiles; t += npairs) {
+                for (int sp = 0; ok && sp < p.spans; ++sp, ++qs) {
+                    const uint32_t rs = qs % SR;
+                    // every lane waits; __all_sync keeps the warp's control flow
+                    // uniform if a wait gives up
+                    if (!__all_sync(0xffffffffu, mbar_wait(sb + L::BAR_RFULL + 8 * rs, (qs / SR) & 1, wc,
+                                                            ERR_CONVERTER))) {
+                        ok = false;
+                        break;
+                    }
+                    const uint32_t row = sb + L::OFF_RAW + rs * L::RAW_SLOT + r * Fmt<FMT>::ROW;
 #pragma unroll
-            for (int i = 0; i < kTasksPerThread; ++i) {
-                const int task = tid + 32 * NUM_CONV_WARPS * i;
-                const uint32_t rsrc = raw + static_cast<uint32_t>(8 * (task >> 5) + (task & 7)) * Fmt<FMT>::ROW;
-                if (FMT == 1) q4k_row_consts(rsrc, rc[i]);
-                else q8_row_consts(rsrc, rc[i]);
-            }
-#pragma unroll
-            for (int g = 0; g < STAGES_PER_SPAN; ++g) {
-                const uint32_t st = j % S;
-                if (!__all_sync(0xffffffffu, mbar_wait_cluster(sb + L::BAR_EMPTY + 8 * st,
-                                                               ((j / S) & 1) ^ 1, wc, ERR_CONVERTER))) {
-                    ok = false;
-                    break;
-                }
-#pragma unroll
-                for (int v = 0; v < SUB; ++v) {
-                    const int u = g * SUB + v;                 // K=64 step within the span
-                    const uint32_t dst = sb + L::OFF_ST + st * STAGE + v * STEP_BYTES + TILE_BYTES;
-#pragma unroll
-                    for (int i = 0; i < kTasksPerThread; ++i) {
-                        const int task = tid + 32 * NUM_CONV_WARPS * i;
-                        convert_task<FMT>(raw, dst, 8 * (task >> 5) + (task & 7), (task >> 3) & 3, u,
-                                          rc[i].d1[2 * u], rc[i].m1[2 * u], rc[i].d1[2 * u + 1],
-                                          rc[i].m1[2 * u + 1]);
+                    for (int hh = 0; hh < STAGES_PER_SPAN; ++hh, ++j) {
+                        const uint32_t sa = j % SA;
+                        if (!__all_sync(0xffffffffu, mbar_wait_cluster(sb + L::BAR_SEMPTY + 8 * sa,
+                                                                        ((j / SA) & 1) ^ 1, wc, ERR_CONVERTER))) {
+                            ok = false;
+                            break;
+                        }
+                        tc_fence_after();
+                        const uint32_t tcol = a_lane + sa * A_SLOT_COLS;
+                        if (FMT == 1) {
+                            if (hh == 0) q4k_stage<0>(row, tcol);
+                            else q4k_stage<1>(row, tcol);
+                        } else {
+                            if (hh == 0) q8_stage<0>(row, tcol);
+                            else q8_stage<1>(row, tcol);
+                        }
+                        if (hh == STAGES_PER_SPAN - 1) {
+                            // the span's bytes are all in registers (and TMEM)
+                            __syncwarp();
+                            if (lane == 0) mbar_arrive(sb + L::BAR_REMPTY + 8 * rs);
+                        }
+                        tmem_st_wait();
+                        tc_fence_before();
+                        __syncwarp();
+                        if (lane == 0) arrive_leader(sb + L::BAR_SFULL + 8 * sa, rank);
                     }
                 }
-                fence_proxy_async_smem();
-                __syncwarp();
-                // the A tile of this stage must have landed too before the
-                // leader may issue: converter warp 0 checks it
-                bool a_ok = true;
-                if (cw == 0 && lane == 0)
-                    a_ok = mbar_wait(sb + L::BAR_AFULL + 8 * st, (j / S) & 1, wc, ERR_CONVERTER);
-                if (!__shfl_sync(0xffffffffu, a_ok ? 1 : 0, 0)) {
-                    ok = false;
-                    break;
-                }
-                if (lane == 0) {
-                    if (leader) mbar_arrive(sb + L::BAR_FULL + 8 * st);
-                    else mbar_arrive_cluster_relaxed(full0 + 8 * st);
-                }
-                ++j;
             }
-            if (!ok) break;
-            if (lane == 0) mbar_arrive(sb + L::BAR_REMPTY + 8 * rs);
         }
-    } else {
-        epilogue_role<FMT>(p, sb, tmem, wc, warp, lane, rank, pair, npairs);
     }
     tc_fence_before();
     __syncwarp();
-    __syncthreads();
+    asm volatile("bar.sync 1, %0;" ::"n"(THREADS) : "memory");
     cluster_sync();
-    if (warp == 1 && run_ok) {
+    if (warp == 1) {
         tc_fence_after();
         tmem_dealloc_pair(tmem, TMEM_COLS);
     }
@@ -613,26 +620,31 @@ template <int FMT>
 cudaError_t launch_fmt(const uint16_t *X, const uint8_t *Wraw, const float *bias, int M, int N, int K,
                        uint16_t *Y, unsigned int *err, cudaStream_t st) {
     using L = Layout<FMT>;
-    static bool attr = false;
-    if (!attr) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_gguf_kernel<FMT>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, L::SMEM_TOTAL);
+    static int regs = -1;
+    if (regs < 0) {
+        cudaFuncAttributes fa;
+        cudaError_t e = cudaFuncGetAttributes(&fa, gemm_gguf_kernel<FMT>);
         if (e != cudaSuccess) return e;
-        attr = true;
+        regs = fa.numRegs;
+        e = cudaFuncSetAttribute(gemm_gguf_kernel<FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 L::SMEM_TOTAL);
+        if (e != cudaSuccess) return e;
     }
-    CUtensorMap mA, mW;
-    if (!make_map(&mA, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, X, static_cast<uint64_t>(K), M,
-                  static_cast<uint64_t>(K) * 2, BK, CTA_M, CU_TENSOR_MAP_SWIZZLE_128B))
+    // the register split above assumes the launch gets exactly this many
+    if (regs != LAUNCH_REGS) return cudaErrorInvalidConfiguration;
+    CUtensorMap mX, mW;
+    if (!make_map(&mX, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, X, static_cast<uint64_t>(K), M,
+                  static_cast<uint64_t>(K) * 2, BK, CTA_T, CU_TENSOR_MAP_SWIZZLE_128B))
         return cudaErrorInvalidValue;
     const uint64_t spans = static_cast<uint64_t>(K) / KR;
     const uint64_t row_bytes = spans * Fmt<FMT>::ROW;
     bool okw;
     if (FMT == 1)
         okw = make_map(&mW, CU_TENSOR_MAP_DATA_TYPE_UINT8, Wraw, row_bytes, N, row_bytes, Fmt<FMT>::ROW,
-                       CTA_N, CU_TENSOR_MAP_SWIZZLE_NONE);
+                       CTA_F, CU_TENSOR_MAP_SWIZZLE_NONE);
     else
         okw = make_map(&mW, CU_TENSOR_MAP_DATA_TYPE_UINT16, Wraw, row_bytes / 2, N, row_bytes,
-                       Fmt<FMT>::ROW / 2, CTA_N, CU_TENSOR_MAP_SWIZZLE_NONE);
+                       Fmt<FMT>::ROW / 2, CTA_F, CU_TENSOR_MAP_SWIZZLE_NONE);
     if (!okw) return cudaErrorInvalidValue;
     Params p{};
     p.bias = bias;
@@ -640,13 +652,13 @@ cudaError_t launch_fmt(const uint16_t *X, const uint8_t *Wraw, const float *bias
     p.M = M;
     p.N = N;
     p.K = K;
-    p.m_tiles = (M + PAIR_M - 1) / PAIR_M;
-    p.total_tiles = p.m_tiles * ((N + PAIR_N - 1) / PAIR_N);
+    p.t_tiles = (M + PAIR_T - 1) / PAIR_T;
+    p.total_tiles = p.t_tiles * ((N + PAIR_F - 1) / PAIR_F);
     p.spans = static_cast<int>(spans);
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
     const int pairs = p.total_tiles < g_sms / 2 ? p.total_tiles : g_sms / 2;
-    gemm_gguf_kernel<FMT><<<2 * pairs, THREADS, L::SMEM_TOTAL, st>>>(mA, mW, p);
+    gemm_gguf_kernel<FMT><<<2 * pairs, THREADS, L::SMEM_TOTAL, st>>>(mX, mW, p);
     return cudaGetLastError();
 }
 
