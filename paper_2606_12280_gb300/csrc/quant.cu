@@ -588,7 +588,12 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
 
 template <int U, int TW, bool GELU, bool OUT16>
 cudaError_t launch_act_quant_team(ActParams p, cudaStream_t st) {
-    constexpr int S = 4;
+    // ring depth, from timed sweeps on the workload shapes: every team has
+    // S - 1 rows in flight from its start and visits only a handful of rows
+    // (4608 rows on 608 teams for K = 4096), so a deeper ring only front-loads
+    // the reads; 2 slices suit the 256-thread teams writing fp16 codes, 3
+    // the int8 codes and the 16-warp teams of K > 8192
+    constexpr int S = GELU ? 4 : ((OUT16 && TW <= 8) ? 2 : 3);
     constexpr int kThreads = TW > 8 ? 32 * TW : 256;
     constexpr int kTeams = kThreads / (32 * TW);
     constexpr size_t smem = (size_t)(kThreads / 32) * S * U * 32 * 16;

@@ -271,7 +271,7 @@ def test_linear_f16codes_exact_with_sumsq(w8, oracle_mod, M, N, K):
 
 # ------------------------------------------------------------- dual branches
 
-@pytest.mark.parametrize("M0,M1", [(300, 130), (0, 257), (513, 0), (256, 256)])
+@pytest.mark.parametrize("M0,M1", [(300, 130), (0, 257), (513, 0), (256, 256), (2000, 800)])
 def test_dual_f16codes_equals_singles(w8, oracle_mod, M0, M1):
     N, K = 520, 1040
     cs = [wl.make_case(max(M, 1), K, N, seed=M + 7 * b) for b, M in enumerate((M0, M1))]
