@@ -97,6 +97,12 @@ __device__ __forceinline__ uint64_t fma_pk(uint64_t a, uint64_t b, uint64_t c) {
     return r;
 }
 
+__device__ __forceinline__ uint64_t add_pk(uint64_t a, uint64_t b) {
+    uint64_t r;
+    asm("add.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
+    return r;
+}
+
 __device__ __forceinline__ uint64_t mul_pk(uint64_t a, uint64_t b) {
     uint64_t r;
     asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
@@ -510,6 +516,10 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
         uint2 *qr = reinterpret_cast<uint2 *>(b.Xq + (size_t)row * K);
         uint4 *qr16 = reinterpret_cast<uint4 *>(b.Xq + 2 * (size_t)row * K);
         uint32_t ss = 0;
+        // fp16-code fast path: the lane's squared codes summed as fp32 pairs
+        // (integers below 2^24: at most 4U codes of 127^2 per component, so
+        // every sum is exact)
+        uint64_t ssq = 0;
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const int c = (u * TW + tw) * 32 + lane;
@@ -518,19 +528,20 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
                 uint32_t hw[4] = {0u, 0u, 0u, 0u};
                 if (zero_row) {
                 } else if (fast) {
-                    // rne(x' * inv) as an fp32 integer: the magic sum minus the
-                    // magic (both in [2^23, 2^24): exact); the magic sum's bit
-                    // pattern minus the magic's is the integer code
+                    // rne(x' * inv) as an fp32 integer: the product rounded
+                    // once (scalar multiplies, never fused), the magic sum
+                    // (in [2^23, 2^24], where one packed add rounds both
+                    // values to integers as the scalar add would), minus the
+                    // magic (exact)
+                    const uint64_t magic = pk(kRoundMagic, kRoundMagic);
+                    const uint64_t nmagic = pk(-kRoundMagic, -kRoundMagic);
 #pragma unroll
                     for (int q = 0; q < 4; ++q) {
-                        const float r0 = __fadd_rn(__fmul_rn(xs[u][q].x, inv), kRoundMagic);
-                        const float r1 = __fadd_rn(__fmul_rn(xs[u][q].y, inv), kRoundMagic);
-                        hw[q] = pack_f16(__fadd_rn(r0, -kRoundMagic), __fadd_rn(r1, -kRoundMagic));
-                        if (want_ss) {
-                            const int q0 = static_cast<int>(__float_as_uint(r0) - 0x4B400000u);
-                            const int q1 = static_cast<int>(__float_as_uint(r1) - 0x4B400000u);
-                            ss += static_cast<uint32_t>(q0 * q0 + q1 * q1);
-                        }
+                        const uint64_t c = add_pk(add_pk(pk(__fmul_rn(xs[u][q].x, inv),
+                                                            __fmul_rn(xs[u][q].y, inv)), magic), nmagic);
+                        const float2 cf = upk(c);
+                        hw[q] = pack_f16(cf.x, cf.y);
+                        if (want_ss) ssq = fma_pk(c, c, ssq);
                     }
                 } else {
 #pragma unroll
@@ -547,12 +558,18 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
             uint32_t word[2] = {0u, 0u};
             if (zero_row) {
             } else if (fast) {
+                // the products rounded once (scalar multiplies), their magic
+                // sums two at a time (one packed add, each value rounded to
+                // an integer as the scalar add would)
+                const uint64_t magic = pk(kRoundMagic, kRoundMagic);
 #pragma unroll
-                for (int h = 0; h < 2; ++h)
-                    word[h] = pack4_low_bytes(__fadd_rn(__fmul_rn(xs[u][2 * h].x, inv), kRoundMagic),
-                                              __fadd_rn(__fmul_rn(xs[u][2 * h].y, inv), kRoundMagic),
-                                              __fadd_rn(__fmul_rn(xs[u][2 * h + 1].x, inv), kRoundMagic),
-                                              __fadd_rn(__fmul_rn(xs[u][2 * h + 1].y, inv), kRoundMagic));
+                for (int h = 0; h < 2; ++h) {
+                    const float2 s0 = upk(add_pk(pk(__fmul_rn(xs[u][2 * h].x, inv),
+                                                    __fmul_rn(xs[u][2 * h].y, inv)), magic));
+                    const float2 s1 = upk(add_pk(pk(__fmul_rn(xs[u][2 * h + 1].x, inv),
+                                                    __fmul_rn(xs[u][2 * h + 1].y, inv)), magic));
+                    word[h] = pack4_low_bytes(s0.x, s0.y, s1.x, s1.y);
+                }
             } else {
 #pragma unroll
                 for (int e = 0; e < 8; ++e) {
@@ -564,6 +581,8 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
             qr[c] = make_uint2(word[0], word[1]);
         }
         if (want_ss) {
+            const float2 sf = upk(ssq);
+            ss += __float2uint_rn(__fadd_rn(sf.x, sf.y));
             ss = __reduce_add_sync(0xffffffffu, ss);
             if (TW > 1) {
                 if (lane == 0) sred[parity][warp] = ss;
