@@ -306,14 +306,44 @@ def run_ours(args):
 
     # the K timed steps run as one CUDA graph (captured after the warm-up,
     # replayed once untimed): two launches per step, no host launch cost in
-    # between; a second pass of K stream-launched steps with events around
-    # each kernel gives the per-kernel times for the roofline
-    graph = torch.cuda.CUDAGraph()
-    with torch.cuda.graph(graph):
-        for i in range(args.steps):
-            j = (args.warmup + i) % n_sets
-            quant(j, None)
-            gemm(j, None)
+    # between.  The steps are independent batches, so step i + 1's a3 runs on
+    # a second stream as soon as the GEMM that last read its input set is
+    # done, and overlaps step i's GEMM (whose last round of tiles leaves most
+    # SMs idle); each GEMM waits for its own a3.  The same K steps in one
+    # stream give `serial_value`.  A second pass of K stream-launched steps
+    # with events around each kernel gives the per-kernel times for the
+    # roofline.
+    side = torch.cuda.Stream(device=dev)
+
+    def capture(pipelined):
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g):
+            cs = torch.cuda.current_stream()
+            if not pipelined:
+                for i in range(args.steps):
+                    j = (args.warmup + i) % n_sets
+                    quant(j, cs)
+                    gemm(j, cs)
+                return g
+            side.wait_stream(cs)
+            gemm_done = []
+            for i in range(args.steps):
+                j = (args.warmup + i) % n_sets
+                with torch.cuda.stream(side):
+                    if i >= n_sets:
+                        side.wait_event(gemm_done[i - n_sets])
+                    quant(j, side)
+                    q_done = torch.cuda.Event()
+                    q_done.record(side)
+                cs.wait_event(q_done)
+                gemm(j, cs)
+                g_done = torch.cuda.Event()
+                g_done.record(cs)
+                gemm_done.append(g_done)
+            cs.wait_stream(side)
+        return g
+
+    graph = capture(True)
     graph.replay()
     torch.cuda.synchronize()
 
@@ -337,6 +367,15 @@ def run_ours(args):
     torch.cuda.synchronize()
     clk = clocks.stop()
     total_ms = t_start.elapsed_time(t_end)
+    graph_serial = capture(False)
+    graph_serial.replay()
+    torch.cuda.synchronize()
+    t_start.record(stream)
+    graph_serial.replay()
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    serial_ms = max_over_ranks(t_start.elapsed_time(t_end), ws, dev)
+    del graph_serial
     quant_ms = [ev[0].elapsed_time(ev[1]) for ev in evs]
     gemm_ms = [ev[1].elapsed_time(ev[2]) for ev in evs]
     if w8a8.device_status(stream) != 0:
@@ -533,13 +572,16 @@ def run_ours(args):
             "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": total_ms / args.steps, "higher_is_better": True,
+            "serial_value": all_ops / (serial_ms * 1e-3) / 1e12, "ms_per_step_serial": serial_ms / args.steps,
             "scaling": "weak", "vs_baseline": None, "dtype": "int8", "data": "synthetic",
             "config": {"workload": args.workload, "M": M, "K": K, "N": N, "alpha": case.alpha,
                        "l2": f"{n_sets} rotating input sets of {set_bytes / 2**20:.0f} MiB "
                              f"(> L2 between reuses), no flush",
-                       "timing": "the K steps replayed as one CUDA graph between two events; "
-                                 "per-kernel times (roofline, act_quant.ms_in_step) from a second "
-                                 "pass of K stream-launched steps with events around each kernel",
+                       "timing": "the K steps replayed as one CUDA graph between two events, "
+                                 "step i+1's a3 on a second stream overlapping step i's GEMM "
+                                 "(serial_value: the same steps in one stream); per-kernel times "
+                                 "(roofline, act_quant.ms_in_step) from a second pass of K "
+                                 "stream-launched steps with events around each kernel",
                        "codes": f"{args.codes} container of the int8 activation codes",
                        "gemm_engine": {"ts": "tcgen05 cta pair, weights in TMEM, drain plan + token sums",
                                        "tc2": "tcgen05 cta pair", "tc": "tcgen05",
