@@ -10,11 +10,11 @@
 // tile (B) with TMA straight into the 128-byte-swizzled K-major layout the
 // tensor core reads (no staging copy, no conversion), and the leader CTA
 // issues one M=256 N=256 K=16 bf16 MMA per K step over both CTAs' shared
-// memory.  Per CTA: warp 0 TMA producer, warp 1 TMEM allocation (both CTAs)
-// and MMA issue (leader only), warp 2 relays "stage landed" from its CTA's
-// local barrier to the leader's pair barrier, warps 4-7 drain the fp32
-// accumulator (double-buffered in TMEM, 2 x 256 columns), add the bias and
-// write bf16.  All waits are bounded in time.
+// memory.  Per CTA: warp 0 TMA producer (both CTAs' loads complete on the
+// leader's stage barrier, which the leader's producer arms for both CTAs'
+// bytes), warp 1 TMEM allocation (both CTAs) and MMA issue (leader only),
+// warps 4-7 drain the fp32 accumulator (double-buffered in TMEM, 2 x 256
+// columns), add the bias and write bf16.  All waits are bounded in time.
 #include <cstdint>
 #include <cuda.h>
 #include <cuda_runtime.h>
@@ -48,12 +48,11 @@ constexpr int SMEM_TOTAL = 1024 + S * STAGE + SMEM_BARRIERS;
 static_assert(SMEM_TOTAL <= 232448, "shared memory");
 
 constexpr unsigned ERR_PRODUCER = 1u, ERR_MMA = 4u, ERR_EPILOGUE = 8u, ERR_DRAIN = 16u,
-                   ERR_RELAY = 32u, ERR_TMEM_PAIR = 64u;
+                   ERR_TMEM_PAIR = 64u;
 
 constexpr uint32_t OFF_ST = 0;
 constexpr uint32_t OFF_BAR = OFF_ST + S * STAGE;
-constexpr uint32_t BAR_FULL = OFF_BAR;                // local: TMA bytes landed
-constexpr uint32_t BAR_PFULL = BAR_FULL + 8 * S;      // leader: both CTAs landed
+constexpr uint32_t BAR_PFULL = OFF_BAR;               // leader: both CTAs' bytes landed
 constexpr uint32_t BAR_EMPTY = BAR_PFULL + 8 * S;     // local: MMA done with the stage
 constexpr uint32_t BAR_ACCFULL = BAR_EMPTY + 8 * S;
 constexpr uint32_t BAR_ACCEMPTY = BAR_ACCFULL + 16;
@@ -161,8 +160,7 @@ gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < S; ++i) {
-            mbar_init(sb + BAR_FULL + 8 * i, 1);
-            mbar_init(sb + BAR_PFULL + 8 * i, 2);
+            mbar_init(sb + BAR_PFULL + 8 * i, 1);
             mbar_init(sb + BAR_EMPTY + 8 * i, 1);
         }
         for (int i = 0; i < 2; ++i) {
@@ -206,18 +204,19 @@ gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
                         ok = false;
                         break;
                     }
-                    const uint32_t fb = sb + BAR_FULL + 8 * st;
-                    mbar_arrive_expect_tx(fb, STAGE);
+                    // both CTAs' loads complete on the leader's barrier (the
+                    // MMA waits for every stage, so each load has landed
+                    // before the kernel ends)
+                    const uint32_t fb = mapa_shared(sb + BAR_PFULL + 8 * st, 0);
+                    if (leader) mbar_arrive_expect_tx(sb + BAR_PFULL + 8 * st, 2 * STAGE);
 #pragma unroll
                     for (int u = 0; u < SUB; ++u) {
                         const uint32_t dst = sb + OFF_ST + st * STAGE + u * SUB_BYTES;
-                        tma_load_2d(dst, &tmA, (ks * SUB + u) * BK, arow, fb);
-                        tma_load_2d(dst + BOX_A, &tmB, (ks * SUB + u) * BK, brow, fb);
+                        tma_load_2d_pair(dst, &tmA, (ks * SUB + u) * BK, arow, fb);
+                        tma_load_2d_pair(dst + BOX_A, &tmB, (ks * SUB + u) * BK, brow, fb);
                     }
                 }
             }
-            for (uint32_t i = (j > S ? j - S : 0); i < j; ++i)
-                mbar_wait(sb + BAR_FULL + 8 * (i % S), (i / S) & 1, wc, ERR_DRAIN, false);
         }
     } else if (warp == 1) {
         // --------------------------------------------- MMA issue (leader)
@@ -255,24 +254,6 @@ gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
             }
             mma_commit_pair(sb + BAR_DRAIN);
             mbar_wait_cluster(sb + BAR_DRAIN, 0, wc, ERR_DRAIN, false);
-        }
-    } else if (warp == 2) {
-        // ---------------------------- relay: this CTA's stage landed -> leader
-        if (lane == 0) {
-            const uint32_t pfull0 = leader ? 0u : mapa_shared(sb + BAR_PFULL, 0);
-            uint32_t j = 0;
-            bool ok = true;
-            for (int t = pair; ok && t < p.total_tiles; t += npairs) {
-                for (int ks = 0; ks < NS; ++ks, ++j) {
-                    const uint32_t st = j % S;
-                    if (!mbar_wait(sb + BAR_FULL + 8 * st, (j / S) & 1, wc, ERR_RELAY)) {
-                        ok = false;
-                        break;
-                    }
-                    if (leader) mbar_arrive(sb + BAR_PFULL + 8 * st);
-                    else mbar_arrive_cluster_relaxed(pfull0 + 8 * st);
-                }
-            }
         }
     } else if (warp >= 4) {
         epilogue_role(p, sb, tmem, wc, warp, lane, rank, pair, npairs);
