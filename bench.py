@@ -534,10 +534,46 @@ def run_ours(args):
     dual_q_iso = isolated(lambda i, st: w8a8.quant_act_dual_f16codes([(dual_in[b][0], dual_in[b][1])
                                                                       for b in range(2)],
                                                                      out=dq[i % 2], stream=st), 20)
-    dual_g_iso = isolated(lambda i, st: w8a8.linear_dual_f16codes(
-        [(dq[i % 2][b][0], dq[i % 2][b][1], dual_in[b][2], dual_in[b][3], dual_in[b][4], dual_in[b][5],
-          dq[i % 2][b][2]) for b in range(2)], Ys=dY[i % 2], stream=st), 10)
-    del dual_in, dq, dY
+    def dual_quant(i, st):
+        w8a8.quant_act_dual_f16codes([(dual_in[b][0], dual_in[b][1]) for b in range(2)], out=dq[i % 2],
+                                     stream=st)
+
+    def dual_gemm(i, st):
+        w8a8.linear_dual_f16codes([(dq[i % 2][b][0], dq[i % 2][b][1], dual_in[b][2], dual_in[b][3],
+                                    dual_in[b][4], dual_in[b][5], dq[i % 2][b][2]) for b in range(2)],
+                                  Ys=dY[i % 2], stream=st)
+
+    dual_g_iso = isolated(dual_gemm, 10)
+    # the dual steps pipelined like the headline step: step i+1's a3 on a
+    # second stream beside step i's grouped GEMM
+    dual_pipe_steps = 10
+    dual_graph = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(dual_graph):
+        cs = torch.cuda.current_stream()
+        side.wait_stream(cs)
+        done = []
+        for i in range(dual_pipe_steps):
+            with torch.cuda.stream(side):
+                if i >= 2:
+                    side.wait_event(done[i - 2])
+                dual_quant(i, side)
+                qd = torch.cuda.Event()
+                qd.record(side)
+            cs.wait_event(qd)
+            dual_gemm(i, cs)
+            gd = torch.cuda.Event()
+            gd.record(cs)
+            done.append(gd)
+        cs.wait_stream(side)
+    dual_graph.replay()
+    torch.cuda.synchronize()
+    a0, a1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a0.record(stream)
+    dual_graph.replay()
+    a1.record(stream)
+    torch.cuda.synchronize()
+    dual_pipe_ms = a0.elapsed_time(a1) / dual_pipe_steps
+    del dual_graph, dual_in, dq, dY
     # the GGUF weight-only layer on the same QKV shape (bf16 activations,
     # Q8_0 / Q4_K weight blocks decoded next to the MMA)
     gguf_iso = {}
@@ -643,7 +679,9 @@ def run_ours(args):
                                    "kernel": "w8a8_gelu_quant_act"},
             },
             "dual": {"workload": "2 x (M=4608, K=4096, N=4096), separate weights",
-                     "value": 2 * 2.0 * Md * Kd * Nd / ((dual_q_iso + dual_g_iso) * 1e-3) / 1e12,
+                     "value": 2 * 2.0 * Md * Kd * Nd / (dual_pipe_ms * 1e-3) / 1e12,
+                     "ms_per_step": dual_pipe_ms,
+                     "value_isolated_sum": 2 * 2.0 * Md * Kd * Nd / ((dual_q_iso + dual_g_iso) * 1e-3) / 1e12,
                      "unit": "TOPS", "ms_isolated": dual_q_iso + dual_g_iso, "a3_ms": dual_q_iso,
                      "gemm_ms": dual_g_iso,
                      "gemm_tflops": 2 * 2.0 * Md * Kd * Nd / (dual_g_iso * 1e-3) / 1e12,
