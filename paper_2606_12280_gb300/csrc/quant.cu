@@ -111,9 +111,17 @@ __device__ __forceinline__ uint64_t mul_pk(uint64_t a, uint64_t b) {
 
 __device__ __forceinline__ uint64_t splat(float c) { return pk(c, c); }
 
+// h Phi(-|h|) from P = log2 erfc(|h|/sqrt 2) - 1 (= log2 Phi(-|h|)), then
+// GELU(h) = h - h Phi(-|h|) for h >= 0 and h Phi(-|h|) for h < 0.
+__device__ __forceinline__ float2 gelu_tail(float2 h, uint64_t p) {
+    const float2 lg = upk(p);
+    const float2 q = upk(mul_pk(pk(h.x, h.y), pk(ex2_approx(lg.x), ex2_approx(lg.y))));   // h Phi(-|h|)
+    return make_float2(h.x >= 0.0f ? h.x - q.x : q.x, h.y >= 0.0f ? h.y - q.y : q.y);
+}
+
 // GELU of two values with packed fp32 instructions (each packed operation
-// rounds like its scalar form).
-__device__ __forceinline__ float2 gelu_erf2(float2 h) {
+// rounds like its scalar form), the degree-12 fit over |h| <= 8.
+__device__ __forceinline__ float2 gelu_erf2_long(float2 h) {
     const uint64_t u = fma_pk(pk(fminf(fabsf(h.x), 8.0f), fminf(fabsf(h.y), 8.0f)), splat(0.25f),
                               splat(-1.0f));
     uint64_t p = splat(-0.00130923442f);
@@ -129,12 +137,39 @@ __device__ __forceinline__ float2 gelu_erf2(float2 h) {
     p = fma_pk(p, u, splat(-11.0028801f));
     p = fma_pk(p, u, splat(-24.3850517f));
     p = fma_pk(p, u, splat(-14.9464674f));                  // C0 - 1: halves erfc
-    const float2 lg = upk(p);
-    const float2 q = upk(mul_pk(pk(h.x, h.y), pk(ex2_approx(lg.x), ex2_approx(lg.y))));   // h Phi(-|h|)
-    return make_float2(h.x >= 0.0f ? h.x - q.x : q.x, h.y >= 0.0f ? h.y - q.y : q.y);
+    return gelu_tail(h, p);
 }
 
-__device__ __forceinline__ float gelu_erf(float h) { return gelu_erf2(make_float2(h, 0.0f)).x; }
+// The degree-8 fit over |h| < 4 in v = |h|/2 - 1 (relative error of Phi
+// about 1e-6 in fp32, no worse than the long fit's there) at 8 instead of 12
+// multiply-adds.  Callers choose it for a whole warp's values at once, when
+// every one of them has |h| < 4 (most warps of Gaussian-like activations);
+// so a value's GELU may differ in the last bits with the company it keeps,
+// and a caller that evaluates a value twice uses gelu_erf (always the long
+// fit).
+__device__ __forceinline__ float2 gelu_erf2_short(float2 h) {
+    {
+        const uint64_t v = fma_pk(pk(fabsf(h.x), fabsf(h.y)), splat(0.5f), splat(-1.0f));
+        uint64_t p = splat(-0.000231636994f);
+        p = fma_pk(p, v, splat(-4.95363784e-05f));
+        p = fma_pk(p, v, splat(0.00274736318f));
+        p = fma_pk(p, v, splat(-0.0114125507f));
+        p = fma_pk(p, v, splat(0.0378777497f));
+        p = fma_pk(p, v, splat(-0.114114717f));
+        p = fma_pk(p, v, splat(-2.55564547f));
+        p = fma_pk(p, v, splat(-6.8476572f));
+        p = fma_pk(p, v, splat(-5.45798159f));               // S0 - 1: halves erfc
+        return gelu_tail(h, p);
+    }
+}
+
+// One pair with the fit chosen by a vote of the active lanes (test export).
+__device__ __forceinline__ float2 gelu_erf2_vote(float2 h) {
+    if (__all_sync(__activemask(), fmaxf(fabsf(h.x), fabsf(h.y)) < 4.0f)) return gelu_erf2_short(h);
+    return gelu_erf2_long(h);
+}
+
+__device__ __forceinline__ float gelu_erf(float h) { return gelu_erf2_long(make_float2(h, 0.0f)).x; }
 
 // ------------------------------------------------------------- row quant
 //
@@ -487,13 +522,36 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
                          : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(slot + u * 32 * 16));
             const uint32_t wd[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                float2 h = make_float2(__uint_as_float(wd[q] << 16), __uint_as_float(wd[q] & 0xffff0000u));
-                if (GELU) h = gelu_erf2(h);
-                xs[u][q] = mul2_rn(h, r[u][q]);
-            }
+            for (int q = 0; q < 4; ++q)
+                xs[u][q] = make_float2(__uint_as_float(wd[q] << 16), __uint_as_float(wd[q] & 0xffff0000u));
+        }
+        if (GELU) {
+            // one fit for all of the warp's values of this row: the short
+            // one when every |h| < 4
+            float hm = 0.0f;
 #pragma unroll
-            for (int q = 0; q < 4; ++q) a = fmaxf(a, fmaxf(fabsf(xs[u][q].x), fabsf(xs[u][q].y)));
+            for (int u = 0; u < U; ++u)
+#pragma unroll
+                for (int q = 0; q < 4; ++q) hm = fmaxf(hm, fmaxf(fabsf(xs[u][q].x), fabsf(xs[u][q].y)));
+            if (__all_sync(0xffffffffu, hm < 4.0f)) {
+#pragma unroll
+                for (int u = 0; u < U; ++u)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) xs[u][q] = gelu_erf2_short(xs[u][q]);
+            } else {
+#pragma unroll
+                for (int u = 0; u < U; ++u)
+#pragma unroll
+                    for (int q = 0; q < 4; ++q) xs[u][q] = gelu_erf2_long(xs[u][q]);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < U; ++u) {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                xs[u][q] = mul2_rn(xs[u][q], r[u][q]);
+                a = fmaxf(a, fmaxf(fabsf(xs[u][q].x), fabsf(xs[u][q].y)));
+            }
         }
         a = warp_max(a);
         if (TW > 1) {
@@ -790,7 +848,7 @@ cudaError_t launch_quant_act_dual(const QuantActBranch *br, int K, cudaStream_t 
 namespace {
 __global__ void gelu_values_kernel(const uint16_t *__restrict__ H, int n, float *__restrict__ G) {
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
-        G[i] = gelu_erf(bf16_bits_to_f32(H[i]));
+        G[i] = gelu_erf2_vote(make_float2(bf16_bits_to_f32(H[i]), 0.0f)).x;   // either fit, as the team kernel
 }
 }  // namespace
 
