@@ -82,14 +82,14 @@ __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
 // (2 kGroup + 4) * 2^-24 of sum |x - c|^p of its exact value.
 constexpr int kStatsWarps = 8;
 constexpr int kGroup = 64;
-constexpr int kUnroll = 8;
+constexpr int kUnroll = 16;
 static_assert(kGroup % kUnroll == 0, "whole unrolled batches per group");
 
 struct Acc4 {                   // one moment for the thread's 4 channels
     float2 a, b;
 };
 
-__global__ void __launch_bounds__(32 * kStatsWarps, 3)
+__global__ void __launch_bounds__(32 * kStatsWarps, 2)
 stats_update_kernel(const uint2 *__restrict__ X4, int T, int K, const float *__restrict__ shift,
                     int rows_per_slab, double *__restrict__ sums, float *__restrict__ absmax) {
     __shared__ double red_s[kStatsWarps][16][32];     // per-thread fp64 sums [p][e]
