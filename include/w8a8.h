@@ -36,7 +36,8 @@
  *     W8A8_ERR_UNSUPPORTED_SHAPE, W8A8_ERR_MISALIGNED (a pointer not 16-byte
  *     aligned) leave the stream untouched.  W8A8_ERR_CUDA reports a launch
  *     failure.  The library keeps one device-side error word (see
- *     w8a8_device_status); it holds no other state.
+ *     w8a8_device_status), the engine choice of w8a8_set_gemm_engine and
+ *     the fixed scratch of w8a8_act_stats_noalloc; it holds no other state.
  */
 #ifndef W8A8_H
 #define W8A8_H
