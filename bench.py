@@ -586,6 +586,47 @@ def run_ours(args):
     if w8a8.device_status(stream) != 0:
         raise RuntimeError("device error word set while timing the protection kernels")
 
+    # the token-count sweep of one DiT block: its four quantized linears (QKV
+    # 4096 -> 12288, out-projection 4096 -> 4096, FFN up 4096 -> 16384, FFN
+    # down 16384 -> 4096) for both branches at M in {1280, 4608, 16896}, each
+    # linear both branches' a3 in one launch and their GEMMs in one grouped
+    # launch on the fp16-code path; one block pass timed in a CUDA graph
+    block_sweep = {}
+    g = torch.Generator(device="cpu").manual_seed(4)
+    for Mb in (1280, 4608, 16896):
+        fns, ops_b = [], 0.0
+        for Kb, Nb in ((4096, 12288), (4096, 4096), (4096, 16384), (16384, 4096)):
+            idx = torch.randperm(Kb, generator=g)[:wl.n_outliers(Kb, 0.005)].to(dev)
+            br_in = []
+            for b in range(2):
+                Xb = torch.randn(Mb, Kb, device=dev)
+                Xb[:, idx] *= 20.0
+                Xb = Xb.to(torch.bfloat16)
+                Wb_ = torch.randn(Nb, Kb, device=dev) * 0.02
+                lam_b = w8a8.smooth_scales(w8a8.channel_absmax(Xb[:256].contiguous()), Wb_, 0.5)
+                Wq_b, sw_b = w8a8.quantize_weights(Wb_, lam_b)
+                del Wb_
+                codes = (torch.empty(Mb, Kb, dtype=torch.float16, device=dev),
+                         torch.empty(Mb, dtype=torch.float32, device=dev),
+                         torch.empty(Mb, dtype=torch.int32, device=dev))
+                br_in.append((Xb, lam_b, Wq_b, sw_b, torch.randn(Nb, device=dev) * 0.01, w8a8.chunk_plan(Wq_b),
+                              codes, torch.empty(Mb, Nb, dtype=torch.bfloat16, device=dev)))
+
+            def lin(st, br_in=br_in):
+                w8a8.quant_act_dual_f16codes([(bi[0], bi[1]) for bi in br_in], out=[bi[6] for bi in br_in],
+                                             stream=st)
+                w8a8.linear_dual_f16codes([(bi[6][0], bi[6][1], bi[2], bi[3], bi[4], bi[5], bi[6][2])
+                                           for bi in br_in], Ys=[bi[7] for bi in br_in], stream=st)
+
+            fns.append(lin)
+            ops_b += 2 * 2.0 * Mb * Kb * Nb
+        ms_b = isolated(lambda i, st: [f(st) for f in fns], 3)
+        block_sweep[f"m{Mb}"] = {"M": Mb, "ms_per_block": ms_b, "tops": ops_b / (ms_b * 1e-3) / 1e12,
+                                 "frac_of_bf16_peak": ops_b / (ms_b * 1e-3) / 1e12 / load_peaks()[0]["bf16_tflops"]}
+        del fns
+    if w8a8.device_status(stream) != 0:
+        raise RuntimeError("device error word set while timing the block sweep")
+
     peaks, peak_kind = load_peaks()
     gemm_avg = sum(gemm_ms) / len(gemm_ms)
     quant_avg = sum(quant_ms) / len(quant_ms)
@@ -692,6 +733,8 @@ def run_ours(args):
                             "ms_isolated": ms, "weight_bytes": nbytes,
                             "kernel": f"w8a8_linear_gguf ({name})"}
                      for name, (ms, nbytes) in gguf_iso.items()},
+            "block_sweep": {"workload": "one DiT block's four quantized linears (QKV, out, FFN up, FFN "
+                                        "down), both branches, a3 + GEMM each", "unit": "TOPS", **block_sweep},
             "gemm_ms": gemm_avg, "gemm_ms_isolated": gemm_iso, "offline_ms": offline,
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "TOPS", "h2d_bytes_per_step": 2 * M * K,
