@@ -131,9 +131,10 @@ class ClockSampler:
 
 # --------------------------------------------------------------- reference
 
-def cpu_oracle_sample(case, target_s: float = 10.0, max_rows: int | None = None):
+def cpu_oracle_sample(case, target_s: float = 10.0, max_rows: int | None = None, want_y: bool = False):
     """Time the CPU oracle (a3 + a4 + a5) on a bounded row sample of the
-    workload.  Returns (tops, seconds, rows, cores)."""
+    workload.  Returns (tops, seconds, rows, cores), and the oracle's output
+    rows (bf16 bit patterns) as a fifth item when want_y."""
     import oracle
     oracle.build()
     s = oracle.channel_absmax(case.X_cal)
@@ -143,10 +144,12 @@ def cpu_oracle_sample(case, target_s: float = 10.0, max_rows: int | None = None)
     N = Wq.shape[0]
     cores = oracle.num_threads()
 
+    out = {}
+
     def run(rows):
         t0 = time.perf_counter()
         Xq, sx = oracle.quant_act(case.X[0][:rows], lam)
-        oracle.linear(Xq, sx, Wq, sw, case.bias[0])
+        out["y"] = oracle.linear(Xq, sx, Wq, sw, case.bias[0])
         return time.perf_counter() - t0
 
     probe = min(M, 16)
@@ -155,6 +158,8 @@ def cpu_oracle_sample(case, target_s: float = 10.0, max_rows: int | None = None)
                    max(probe, probe * target_s / max(dt, 1e-6))))
     dt = run(rows)
     tops = 2.0 * rows * N * K / dt / 1e12
+    if want_y:
+        return tops, dt, rows, cores, out["y"]
     return tops, dt, rows, cores
 
 
@@ -643,9 +648,22 @@ def run_ours(args):
     if rank == 0:
         cpu = None
         if ws == 1 and not args.no_cpu_baseline:
-            tops_cpu, dt_cpu, rows, cores = cpu_oracle_sample(case, target_s=args.cpu_seconds)
+            tops_cpu, dt_cpu, rows, cores, y_cpu = cpu_oracle_sample(case, target_s=args.cpu_seconds,
+                                                                     want_y=True)
             cpu = {"value": tops_cpu, "unit": "TOPS", "cores": cores, "kind": "oracle",
                    "sample": f"{rows} of {M} tokens (a3+a4+a5), {dt_cpu:.1f} s of CPU work"}
+            # the benchmarked path's output for the same tokens, recomputed
+            # once, against the oracle's bit patterns
+            try:
+                quant(0, stream)
+                gemm(0, stream)
+                torch.cuda.synchronize()
+                y_gpu = Ys[0][:rows].contiguous().view(torch.int16).cpu().numpy().view(np.uint16)
+                diff = np.abs(y_gpu.astype(np.int32) - np.asarray(y_cpu).astype(np.int32))
+                cpu["parity"] = {"tokens": int(rows), "outputs": int(diff.size), "max_bf16_ulp": int(diff.max()),
+                                 "bit_identical": bool((diff == 0).all())}
+            except Exception as exc:  # reported, never fatal to the line
+                cpu["parity"] = {"error": repr(exc)[:200]}
         line = {
             "metric": METRIC, "value": value, "unit": "TOPS", "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup,
