@@ -143,11 +143,23 @@ def _ptr(t, dtype, name):
     return t.data_ptr()
 
 
+def _room(t, n, name):
+    """Refuse a tensor with fewer than n elements where the library reads or
+    writes n (the C ABI takes plain pointers and cannot check sizes)."""
+    if t is not None and t.numel() < n:
+        raise ValueError(f"{name} holds {t.numel()} elements, the call needs {n}")
+
+
+def _gguf_row_bytes(fmt: int, K: int) -> int:
+    return (K // 32) * 34 if int(fmt) == 0 else (K // 256) * 144
+
+
 def channel_absmax(X, s=None, stream=None):
     """s_j = max_t |X_tj| (calibration statistic).  X [T,K] bf16 -> s [K] fp32."""
     T, K = X.shape
     if s is None:
         s = torch.empty(K, dtype=torch.float32, device=X.device)
+    _room(s, K, "s")
     _check("w8a8_channel_absmax", lib().w8a8_channel_absmax(
         _ptr(X, torch.bfloat16, "X"), T, K, _ptr(s, torch.float32, "s"), _stream(stream)))
     return s
@@ -158,6 +170,8 @@ def smooth_scales(act_absmax, W, alpha: float, smooth=None, stream=None):
     N, K = W.shape
     if smooth is None:
         smooth = torch.empty(K, dtype=torch.float32, device=W.device)
+    _room(act_absmax, K, "act_absmax")
+    _room(smooth, K, "smooth")
     _check("w8a8_smooth_scales", lib().w8a8_smooth_scales(
         _ptr(act_absmax, torch.float32, "act_absmax"), _ptr(W, torch.float32, "W"), N, K,
         float(alpha), _ptr(smooth, torch.float32, "smooth"), _stream(stream)))
@@ -171,6 +185,9 @@ def quantize_weights(W, smooth=None, Wq=None, w_scale=None, stream=None):
         Wq = torch.empty(N, K, dtype=torch.int8, device=W.device)
     if w_scale is None:
         w_scale = torch.empty(N, dtype=torch.float32, device=W.device)
+    _room(smooth, K, "smooth")
+    _room(Wq, N * K, "Wq")
+    _room(w_scale, N, "w_scale")
     _check("w8a8_quantize_weights", lib().w8a8_quantize_weights(
         _ptr(W, torch.float32, "W"), _ptr(smooth, torch.float32, "smooth"), N, K,
         _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"), _stream(stream)))
@@ -184,6 +201,9 @@ def quant_act(X, smooth=None, Xq=None, x_scale=None, stream=None):
         Xq = torch.empty(M, K, dtype=torch.int8, device=X.device)
     if x_scale is None:
         x_scale = torch.empty(M, dtype=torch.float32, device=X.device)
+    _room(smooth, K, "smooth")
+    _room(Xq, M * K, "Xq")
+    _room(x_scale, M, "x_scale")
     _check("w8a8_quant_act", lib().w8a8_quant_act(
         _ptr(X, torch.bfloat16, "X"), _ptr(smooth, torch.float32, "smooth"), M, K,
         _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"), _stream(stream)))
@@ -198,6 +218,10 @@ def linear(Xq, x_scale, Wq, w_scale, bias=None, Y=None, stream=None):
         raise ValueError("Xq and Wq disagree on K")
     if Y is None:
         Y = torch.empty(M, N, dtype=torch.bfloat16, device=Xq.device)
+    _room(x_scale, M, "x_scale")
+    _room(w_scale, N, "w_scale")
+    _room(bias, N, "bias")
+    _room(Y, M * N, "Y")
     _check("w8a8_linear", lib().w8a8_linear(
         _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"),
         _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
@@ -219,6 +243,11 @@ def linear_dual(branches, Ys=None, stream=None):
             raise ValueError("branches must share N and K")
         Y = Ys[i] if Ys is not None else torch.empty(Xq.shape[0], N, dtype=torch.bfloat16,
                                                      device=Xq.device)
+        M = Xq.shape[0]
+        _room(sx, M, "x_scale")
+        _room(sw, N, "w_scale")
+        _room(b, N, "bias")
+        _room(Y, M * N, "Y")
         arr[i] = Branch(_ptr(Xq, torch.int8, "Xq"), _ptr(sx, torch.float32, "x_scale"),
                         _ptr(Wq, torch.int8, "Wq"), _ptr(sw, torch.float32, "w_scale"),
                         _ptr(b, torch.float32, "bias"), _ptr(Y, torch.bfloat16, "Y"),
@@ -234,6 +263,7 @@ def debug_gemm_i32(Xq, Wq, acc=None, stream=None):
     N = Wq.shape[0]
     if acc is None:
         acc = torch.empty(M, N, dtype=torch.int32, device=Xq.device)
+    _room(acc, M * N, "acc")
     _check("w8a8_debug_gemm_i32", lib().w8a8_debug_gemm_i32(
         _ptr(Xq, torch.int8, "Xq"), _ptr(Wq, torch.int8, "Wq"), M, N, K,
         _ptr(acc, torch.int32, "acc"), _stream(stream)))
@@ -281,6 +311,9 @@ def quant_act_dual(branches, out=None, stream=None):
         else:
             Xq = torch.empty(M, K, dtype=torch.int8, device=X.device)
             sx = torch.empty(M, dtype=torch.float32, device=X.device)
+        _room(sm, K, "smooth")
+        _room(Xq, M * K, "Xq")
+        _room(sx, M, "x_scale")
         arr[i] = ActBranch(_ptr(X, torch.bfloat16, "X"), _ptr(sm, torch.float32, "smooth"), M,
                            _ptr(Xq, torch.int8, "Xq"), _ptr(sx, torch.float32, "x_scale"))
         res.append((Xq, sx))
@@ -307,6 +340,10 @@ def quant_act_dual_f16codes(branches, out=None, stream=None):
             Xq16 = torch.empty(M, K, dtype=torch.float16, device=X.device)
             sx = torch.empty(M, dtype=torch.float32, device=X.device)
             ss = torch.empty(M, dtype=torch.int32, device=X.device)
+        _room(sm, K, "smooth")
+        _room(Xq16, M * K, "Xq16")
+        _room(sx, M, "x_scale")
+        _room(ss, M, "sumsq")
         arr[i] = ActBranch16(_ptr(X, torch.bfloat16, "X"), _ptr(sm, torch.float32, "smooth"), M,
                              _ptr(Xq16, torch.float16, "Xq16"), _ptr(sx, torch.float32, "x_scale"),
                              _ptr(ss, torch.int32, "sumsq"))
@@ -329,6 +366,14 @@ def linear_dual_f16codes(branches, Ys=None, stream=None):
             raise ValueError("branches must share N and K")
         Y = Ys[i] if Ys is not None else torch.empty(Xq16.shape[0], N, dtype=torch.bfloat16,
                                                      device=Xq16.device)
+        M = Xq16.shape[0]
+        _room(sx, M, "x_scale")
+        _room(sw, N, "w_scale")
+        _room(b, N, "bias")
+        if plan is not None:
+            _room(plan, chunk_plan_size(N, K), "plan")
+        _room(ss, M, "x_sumsq")
+        _room(Y, M * N, "Y")
         arr[i] = Branch16(_ptr(Xq16, torch.float16, "Xq16"), _ptr(sx, torch.float32, "x_scale"),
                           _ptr(Wq, torch.int8, "Wq"), _ptr(sw, torch.float32, "w_scale"),
                           _ptr(b, torch.float32, "bias"), _ptr(Y, torch.bfloat16, "Y"), Xq16.shape[0],
@@ -345,6 +390,9 @@ def gelu_quant_act(H, smooth=None, Xq=None, x_scale=None, stream=None):
         Xq = torch.empty(M, K, dtype=torch.int8, device=H.device)
     if x_scale is None:
         x_scale = torch.empty(M, dtype=torch.float32, device=H.device)
+    _room(smooth, K, "smooth")
+    _room(Xq, M * K, "Xq")
+    _room(x_scale, M, "x_scale")
     _check("w8a8_gelu_quant_act", lib().w8a8_gelu_quant_act(
         _ptr(H, torch.bfloat16, "H"), _ptr(smooth, torch.float32, "smooth"), M, K,
         _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"), _stream(stream)))
@@ -360,6 +408,10 @@ def quant_act_f16codes(X, smooth=None, Xq16=None, x_scale=None, gelu=False, sums
         Xq16 = torch.empty(M, K, dtype=torch.float16, device=X.device)
     if x_scale is None:
         x_scale = torch.empty(M, dtype=torch.float32, device=X.device)
+    _room(smooth, K, "smooth")
+    _room(Xq16, M * K, "Xq16")
+    _room(x_scale, M, "x_scale")
+    _room(sumsq, M, "sumsq")
     _check("w8a8_quant_act_f16codes", lib().w8a8_quant_act_f16codes(
         _ptr(X, torch.bfloat16, "X"), _ptr(smooth, torch.float32, "smooth"), M, K,
         _ptr(Xq16, torch.float16, "Xq16"), _ptr(x_scale, torch.float32, "x_scale"),
@@ -375,6 +427,13 @@ def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, x_
     N = Wq.shape[0]
     if Y is None:
         Y = torch.empty(M, N, dtype=torch.bfloat16, device=Xq16.device)
+    _room(x_scale, M, "x_scale")
+    _room(w_scale, N, "w_scale")
+    _room(bias, N, "bias")
+    if plan is not None:
+        _room(plan, chunk_plan_size(N, K), "plan")
+    _room(x_sumsq, M, "x_sumsq")
+    _room(Y, M * N, "Y")
     _check("w8a8_linear_f16codes", lib().w8a8_linear_f16codes(
         _ptr(Xq16, torch.float16, "Xq16"), _ptr(x_scale, torch.float32, "x_scale"),
         _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
@@ -389,6 +448,10 @@ def debug_gemm_f16codes_i32(Xq16, Wq, plan=None, x_sumsq=None, acc=None, stream=
     N = Wq.shape[0]
     if acc is None:
         acc = torch.empty(M, N, dtype=torch.int32, device=Xq16.device)
+    if plan is not None:
+        _room(plan, chunk_plan_size(N, K), "plan")
+    _room(x_sumsq, M, "x_sumsq")
+    _room(acc, M * N, "acc")
     _check("w8a8_debug_gemm_f16codes_i32", lib().w8a8_debug_gemm_f16codes_i32(
         _ptr(Xq16, torch.float16, "Xq16"), _ptr(Wq, torch.int8, "Wq"), M, N, K,
         _ptr(plan, torch.int32, "plan"), _ptr(x_sumsq, torch.int32, "x_sumsq"),
@@ -407,6 +470,7 @@ def chunk_plan(Wq, plan=None, stream=None):
     N, K = Wq.shape
     if plan is None:
         plan = torch.empty(chunk_plan_size(N, K), dtype=torch.int32, device=Wq.device)
+    _room(plan, chunk_plan_size(N, K), "plan")
     _check("w8a8_chunk_plan", lib().w8a8_chunk_plan(
         _ptr(Wq, torch.int8, "Wq"), N, K, _ptr(plan, torch.int32, "plan"), _stream(stream)))
     return plan
@@ -418,6 +482,10 @@ def linear_gguf(X, Wraw, fmt: int, N: int, bias=None, Y=None, stream=None):
     M, K = X.shape
     if Y is None:
         Y = torch.empty(M, N, dtype=torch.bfloat16, device=X.device)
+    if int(fmt) in (0, 1):
+        _room(Wraw, N * _gguf_row_bytes(fmt, K), "Wraw")
+    _room(bias, N, "bias")
+    _room(Y, M * N, "Y")
     _check("w8a8_linear_gguf", lib().w8a8_linear_gguf(
         _ptr(X, torch.bfloat16, "X"), _ptr(Wraw, torch.uint8, "Wraw"), int(fmt),
         _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(Y, torch.bfloat16, "Y"), _stream(stream)))
@@ -428,6 +496,9 @@ def debug_gguf_dequant(Wraw, fmt: int, N: int, K: int, W=None, stream=None):
     """The decoded weights [N, K] bf16."""
     if W is None:
         W = torch.empty(N, K, dtype=torch.bfloat16, device=Wraw.device)
+    if int(fmt) in (0, 1):
+        _room(Wraw, N * _gguf_row_bytes(fmt, K), "Wraw")
+    _room(W, N * K, "W")
     _check("w8a8_debug_gguf_dequant", lib().w8a8_debug_gguf_dequant(
         _ptr(Wraw, torch.uint8, "Wraw"), int(fmt), N, K, _ptr(W, torch.bfloat16, "W"),
         _stream(stream)))
@@ -439,6 +510,7 @@ def debug_gelu(H, G=None, stream=None):
     n = H.numel()
     if G is None:
         G = torch.empty(n, dtype=torch.float32, device=H.device)
+    _room(G, n, "G")
     _check("w8a8_debug_gelu", lib().w8a8_debug_gelu(
         _ptr(H, torch.bfloat16, "H"), n, _ptr(G, torch.float32, "G"), _stream(stream)))
     return G
@@ -453,6 +525,10 @@ def quant_act_per_tensor(X, smooth=None, Xq=None, x_scale=None, amax=None, strea
         x_scale = torch.empty(M, dtype=torch.float32, device=X.device)
     if amax is None:
         amax = torch.empty(1, dtype=torch.float32, device=X.device)
+    _room(smooth, K, "smooth")
+    _room(Xq, M * K, "Xq")
+    _room(x_scale, M, "x_scale")
+    _room(amax, 1, "amax")
     _check("w8a8_quant_act_per_tensor", lib().w8a8_quant_act_per_tensor(
         _ptr(X, torch.bfloat16, "X"), _ptr(smooth, torch.float32, "smooth"), M, K,
         _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"),
@@ -463,6 +539,9 @@ def quant_act_per_tensor(X, smooth=None, Xq=None, x_scale=None, amax=None, strea
 def act_stats_update(X, sums, absmax, shift=None, stream=None):
     """Accumulate the per-channel power sums [4,K] fp64 and absmax [K] of X [T,K] bf16."""
     T, K = X.shape
+    _room(shift, K, "shift")
+    _room(sums, 4 * K, "sums")
+    _room(absmax, K, "absmax")
     _check("w8a8_act_stats_update", lib().w8a8_act_stats_update(
         _ptr(X, torch.bfloat16, "X"), T, K, _ptr(shift, torch.float32, "shift"),
         _ptr(sums, torch.float64, "sums"), _ptr(absmax, torch.float32, "absmax"),
@@ -476,6 +555,10 @@ def act_stats_finalize(sums, absmax, count: int, shift=None, chan=None, tensor=N
         chan = torch.empty(4, K, dtype=torch.float32, device=absmax.device)
     if tensor is None:
         tensor = torch.empty(4, dtype=torch.float32, device=absmax.device)
+    _room(sums, 4 * K, "sums")
+    _room(shift, K, "shift")
+    _room(chan, 4 * K, "chan")
+    _room(tensor, 4, "tensor")
     _check("w8a8_act_stats_finalize", lib().w8a8_act_stats_finalize(
         _ptr(sums, torch.float64, "sums"), _ptr(absmax, torch.float32, "absmax"),
         _ptr(shift, torch.float32, "shift"), int(count), K, _ptr(chan, torch.float32, "chan"),
@@ -491,6 +574,9 @@ def act_stats_noalloc(X, shift=None, chan=None, tensor=None, stream=None):
         chan = torch.empty(4, K, dtype=torch.float32, device=X.device)
     if tensor is None:
         tensor = torch.empty(4, dtype=torch.float32, device=X.device)
+    _room(shift, K, "shift")
+    _room(chan, 4 * K, "chan")
+    _room(tensor, 4, "tensor")
     _check("w8a8_act_stats_noalloc", lib().w8a8_act_stats_noalloc(
         _ptr(X, torch.bfloat16, "X"), T, K, _ptr(shift, torch.float32, "shift"),
         _ptr(chan, torch.float32, "chan"), _ptr(tensor, torch.float32, "tensor"), _stream(stream)))
@@ -505,6 +591,8 @@ def linear_bf16(X, W, bias=None, Y=None, stream=None):
         raise ValueError("X and W disagree on K")
     if Y is None:
         Y = torch.empty(M, N, dtype=torch.bfloat16, device=X.device)
+    _room(bias, N, "bias")
+    _room(Y, M * N, "Y")
     _check("w8a8_linear_bf16", lib().w8a8_linear_bf16(
         _ptr(X, torch.bfloat16, "X"), _ptr(W, torch.bfloat16, "W"),
         _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(Y, torch.bfloat16, "Y"),
