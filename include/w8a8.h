@@ -17,6 +17,9 @@
  *   - Every pointer is a DEVICE pointer owned by the caller (for example the
  *     data_ptr() of a CUDA tensor).  The library allocates nothing and never
  *     frees anything.  Every base pointer must be 16-byte aligned.
+ *   - Every buffer must hold the elements that the call's shapes imply (for
+ *     example M * N for Y): the library receives plain pointers and cannot
+ *     check their extent.
  *   - Matrices are row-major and dense (row stride = number of columns).
  *     X [M,K] activations (tokens x input channels), W / Wq [N,K] weights
  *     (output channels x input channels, the nn.Linear layout), Y [M,N].
