@@ -39,8 +39,12 @@
  *     W8A8_ERR_UNSUPPORTED_SHAPE, W8A8_ERR_MISALIGNED (a pointer not 16-byte
  *     aligned) leave the stream untouched.  W8A8_ERR_CUDA reports a launch
  *     failure.  The library keeps one device-side error word (see
- *     w8a8_device_status), the engine choice of w8a8_set_gemm_engine and
- *     the fixed scratch of w8a8_act_stats_noalloc; it holds no other state.
+ *     w8a8_device_status) and the fixed scratch of w8a8_act_stats_noalloc;
+ *     it holds no other state (per-device kernel attributes are set once,
+ *     thread-safely), and calls on different streams or host threads do not
+ *     affect one another.
+ *   - Every pointer refers to memory of the CURRENT device (cudaSetDevice),
+ *     on which the call launches its work.
  */
 #ifndef W8A8_H
 #define W8A8_H
@@ -131,6 +135,9 @@ W8A8_API w8a8_status w8a8_quant_act(const uint16_t *X, const float *smooth, int 
  *     Y_mn   = bf16_rne(((float)acc_mn * x_scale_m) * w_scale_n + bias_n)
  *   Xq [M,K] int8, x_scale [M] fp32, Wq [N,K] int8, w_scale [N] fp32,
  *   bias [N] fp32 or NULL (no bias), all read.   Y [M,N] bf16, written.
+ * The product runs exactly on the fp16 tensor datapath (every int8 is an
+ * fp16 value, products are exact in fp32; partial sums of at most 1024
+ * products stay below 2^24 and are drained into int32).
  */
 W8A8_API w8a8_status w8a8_linear(const int8_t *Xq, const float *x_scale,
                         const int8_t *Wq, const float *w_scale,
@@ -166,6 +173,18 @@ W8A8_API w8a8_status w8a8_linear_dual(const w8a8_branch *br, int N, int K,
  */
 W8A8_API w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int M,
                                 int N, int K, int32_t *acc, void *stream);
+
+/*
+ * Test anchors (no counterpart in the paper): the same exact-integer product
+ * on the earlier int8-code GEMM engines, selected per call (nothing
+ * process-wide).  engine 2 = the engine of w8a8_linear (tcgen05 on pairs of
+ * SMs), 1 = tcgen05 on single SMs, 0 = warp-level mma.sync s8 (the legacy
+ * INT8 tensor path); other values give W8A8_ERR_INVALID_ARG.  nb = 1 or 2
+ * branches (br[0..nb-1]).  out_i32 nonzero: each branch's Y receives the
+ * int32 product [M,N] instead (x_scale, w_scale and bias unused).
+ */
+W8A8_API w8a8_status w8a8_debug_linear_engine(int engine, const w8a8_branch *br, int nb, int N, int K,
+                                              int out_i32, void *stream);
 
 /* ------------------------------------------------------------------------
  * The same layer with the activation codes in a 16-bit container.
@@ -205,7 +224,6 @@ W8A8_API w8a8_status w8a8_quant_act_f16codes(const uint16_t *X, const float *smo
  *     its largest weight-row sum of squares is at most 2^48 has every partial
  *     sum within 2^24 (Cauchy-Schwarz) and is accumulated without a drain.
  *     Sums of other codes void the exactness guarantee.
- * Uses the CTA-pair engine whatever w8a8_set_gemm_engine says.
  */
 W8A8_API w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale,
                                           const int8_t *Wq, const float *w_scale,
@@ -498,17 +516,6 @@ W8A8_API w8a8_status w8a8_layer_forward(const w8a8_layer *layer, const uint16_t 
  */
 W8A8_API w8a8_status w8a8_select_protected(const float *score, int L, int n_protect,
                                            int *protect_flags);
-
-/*
- * The GEMM engine that w8a8_linear, w8a8_linear_dual and w8a8_debug_gemm_i32
- * use: 2 = tcgen05 on pairs of SMs (cta_group::2, 256x256 tiles), 1 = tcgen05
- * on single SMs (128x256 tiles), both computing the exact integer product on
- * the fp16 tensor datapath; 0 = warp-level mma.sync s8 (legacy INT8 tensor
- * path).  The default is 2; w8a8_set_gemm_engine(-1) restores it; other
- * values give W8A8_ERR_INVALID_ARG.  The setting is process-wide.
- */
-W8A8_API w8a8_status w8a8_set_gemm_engine(int engine);
-W8A8_API int w8a8_get_gemm_engine(void);
 
 /*
  * Test hook for failure detection (no counterpart in the paper): enqueues one

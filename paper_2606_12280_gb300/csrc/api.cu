@@ -8,6 +8,7 @@
 #include <cuda_runtime.h>
 
 #include "../../include/w8a8.h"
+#include "host_once.h"
 #include "launch.h"
 
 namespace {
@@ -15,8 +16,6 @@ namespace {
 // The library's single device-side error word: kernels with bounded waits
 // record a nonzero code here instead of spinning forever.
 __device__ unsigned int g_w8a8_device_error = 0;
-
-int g_engine = 2;   // 2 = tcgen05 CTA pairs, 1 = tcgen05, 0 = mma.sync
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
@@ -35,17 +34,19 @@ w8a8_status from_cuda(cudaError_t e) { return e == cudaSuccess ? W8A8_OK : W8A8_
 
 cudaStream_t as_stream(void *s) { return static_cast<cudaStream_t>(s); }
 
-// Address of the error word on the current device, looked up once per device.
+// Address of the error word on the current device, looked up once per device
+// (under std::call_once: host threads may launch concurrently).
 unsigned int *device_error_word() {
-    constexpr int kMaxDevices = 64;
-    static unsigned int *cache[kMaxDevices] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess) return nullptr;
-    if (dev >= 0 && dev < kMaxDevices && cache[dev]) return cache[dev];
-    void *p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_w8a8_device_error) != cudaSuccess) return nullptr;
-    if (dev >= 0 && dev < kMaxDevices) cache[dev] = static_cast<unsigned int *>(p);
-    return static_cast<unsigned int *>(p);
+    static w8a8::PerDevice<unsigned int *> addr;
+    unsigned int *p = nullptr;
+    if (addr.get([](unsigned int *&v) {
+            void *q = nullptr;
+            cudaError_t e = cudaGetSymbolAddress(&q, g_w8a8_device_error);
+            v = static_cast<unsigned int *>(q);
+            return e;
+        }, &p) != cudaSuccess)
+        return nullptr;
+    return p;
 }
 
 // Validation shared by the single- and dual-branch linears.
@@ -63,14 +64,24 @@ w8a8_status check_branch(const w8a8::GemmBranch &b, bool need_scales, int N, int
     return W8A8_OK;
 }
 
+// a4 + a5 on int8 codes: the tcgen05 GEMM on CTA pairs (both operands
+// converted to fp16 in shared memory, two accumulators in tensor memory).
 w8a8_status run_gemm(const w8a8::GemmBranch *br, int nb, int N, int K, bool out_i32,
                      cudaStream_t st) {
-    if (g_engine == 1 || g_engine == 2) {
-        unsigned int *err = device_error_word();
-        if (!err) return W8A8_ERR_CUDA;
-        if (g_engine == 2) return from_cuda(w8a8::launch_gemm_tc2(br, nb, N, K, out_i32, false, err, st));
-        return from_cuda(w8a8::launch_gemm_tc(br, nb, N, K, out_i32, err, st));
-    }
+    unsigned int *err = device_error_word();
+    if (!err) return W8A8_ERR_CUDA;
+    return from_cuda(w8a8::launch_gemm_tc2(br, nb, N, K, out_i32, false, err, st));
+}
+
+// The same product on the earlier engines, kept as test anchors and never on
+// a product call: 1 = tcgen05 on single SMs, 0 = mma.sync s8; 2 is the
+// product engine.
+w8a8_status run_gemm_engine(int engine, const w8a8::GemmBranch *br, int nb, int N, int K, bool out_i32,
+                            cudaStream_t st) {
+    if (engine == 2) return run_gemm(br, nb, N, K, out_i32, st);
+    unsigned int *err = device_error_word();
+    if (!err) return W8A8_ERR_CUDA;
+    if (engine == 1) return from_cuda(w8a8::launch_gemm_tc(br, nb, N, K, out_i32, err, st));
     return from_cuda(w8a8::launch_gemm_mma(br, nb, N, K, out_i32, st));
 }
 
@@ -162,6 +173,20 @@ w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int M, int N
     if (w8a8_status e = check_branch(b, false, N, K)) return e;
     if (M == 0) return W8A8_OK;
     return run_gemm(&b, 1, N, K, true, as_stream(stream));
+}
+
+w8a8_status w8a8_debug_linear_engine(int engine, const w8a8_branch *br, int nb, int N, int K, int out_i32,
+                                     void *stream) {
+    if (engine < 0 || engine > 2 || !br || nb < 1 || nb > 2) return W8A8_ERR_INVALID_ARG;
+    if (w8a8_status e = check_nk(N, K)) return e;
+    w8a8::GemmBranch b[2];
+    for (int i = 0; i < nb; ++i) {
+        b[i] = w8a8::GemmBranch{br[i].Xq, br[i].x_scale, br[i].Wq, br[i].w_scale, br[i].bias, br[i].Y, br[i].M};
+        if (w8a8_status e = check_mk(br[i].M, K)) return e;
+        if (w8a8_status e = check_branch(b[i], out_i32 == 0, N, K)) return e;
+    }
+    if (b[0].M == 0 && (nb == 1 || b[1].M == 0)) return W8A8_OK;
+    return run_gemm_engine(engine, b, nb, N, K, out_i32 != 0, as_stream(stream));
 }
 
 w8a8_status w8a8_quant_act_dual(const w8a8_act_branch *br, int K, void *stream) {
@@ -330,8 +355,7 @@ w8a8_status w8a8_act_stats_finalize(const double *sums, const float *absmax, con
 w8a8_status w8a8_act_stats_noalloc(const uint16_t *X, int T, int K, const float *shift, float *chan,
                                    float *tensor, void *stream) {
     if (K <= 0 || (K % 16) != 0 || K > W8A8_NOALLOC_STATS_MAX_K) return W8A8_ERR_UNSUPPORTED_SHAPE;
-    if (T < 0) return W8A8_ERR_UNSUPPORTED_SHAPE;
-    if (T == 0 || !X || !chan || !tensor) return W8A8_ERR_INVALID_ARG;
+    if (T <= 0 || !X || !chan || !tensor) return W8A8_ERR_INVALID_ARG;
     if (!aligned16(X) || !aligned16(chan) || !aligned16(tensor) || (shift && !aligned16(shift)))
         return W8A8_ERR_MISALIGNED;
     return from_cuda(w8a8::launch_act_stats_noalloc(X, T, K, shift, chan, tensor, as_stream(stream)));
@@ -418,15 +442,6 @@ w8a8_status w8a8_select_protected(const float *score, int L, int n_protect, int 
     for (int i = 0; i < n_protect; ++i) protect_flags[order[static_cast<size_t>(i)]] = 1;
     return W8A8_OK;
 }
-
-w8a8_status w8a8_set_gemm_engine(int engine) {
-    if (engine == -1) engine = 2;
-    if (engine < 0 || engine > 2) return W8A8_ERR_INVALID_ARG;
-    g_engine = engine;
-    return W8A8_OK;
-}
-
-int w8a8_get_gemm_engine(void) { return g_engine; }
 
 w8a8_status w8a8_debug_wait_timeout(uint32_t limit_us, void *stream) {
     if (limit_us == 0 || limit_us > 2000000u) return W8A8_ERR_INVALID_ARG;

@@ -19,6 +19,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include "host_once.h"
 #include "launch.h"
 #include "tc_ptx.cuh"
 
@@ -276,15 +277,16 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 EncodeTiledFn get_encode() {
-    static EncodeTiledFn fn = nullptr;
-    if (!fn) {
+    // a function-local static: initialised once, thread-safe
+    static const EncodeTiledFn fn = [] {
         void *ptr = nullptr;
         cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
-                                             cudaEnableDefault, &q) == cudaSuccess &&
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    }
+            return reinterpret_cast<EncodeTiledFn>(ptr);
+        return static_cast<EncodeTiledFn>(nullptr);
+    }();
     return fn;
 }
 
@@ -302,24 +304,17 @@ bool make_map_bf16(CUtensorMap *m, const uint16_t *base, int rows, int K) {
                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int g_sms = 0;
-bool g_attr_set = false;
-
 }  // namespace
 
 cudaError_t launch_gemm_bf16(const uint16_t *X, const uint16_t *W, const float *bias, int M,
                              int N, int K, uint16_t *Y, unsigned int *err, cudaStream_t st) {
-    if (g_sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
-    }
-    if (!g_attr_set) {
-        cudaError_t e = cudaFuncSetAttribute(gemm_bf16_kernel,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_TOTAL);
-        if (e != cudaSuccess) return e;
-        g_attr_set = true;
-    }
+    const int sms = device_sms();
+    static PerDevice<int> attr;
+    int unused = 0;
+    cudaError_t e = attr.get([](int &) {
+        return cudaFuncSetAttribute(gemm_bf16_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_TOTAL);
+    }, &unused);
+    if (e != cudaSuccess) return e;
     CUtensorMap mA, mB;
     if (!make_map_bf16(&mA, X, M, K) || !make_map_bf16(&mB, W, N, K)) return cudaErrorInvalidValue;
     Params p{};
@@ -333,7 +328,7 @@ cudaError_t launch_gemm_bf16(const uint16_t *X, const uint16_t *W, const float *
     p.k_blocks = (K + BK - 1) / BK;
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
-    const int pairs = p.total_tiles < g_sms / 2 ? p.total_tiles : g_sms / 2;
+    const int pairs = p.total_tiles < sms / 2 ? p.total_tiles : sms / 2;
     gemm_bf16_kernel<<<2 * pairs, THREADS, SMEM_TOTAL, st>>>(mA, mB, p);
     return cudaGetLastError();
 }

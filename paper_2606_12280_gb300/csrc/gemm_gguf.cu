@@ -27,6 +27,7 @@
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 
+#include "host_once.h"
 #include "launch.h"
 #include "tc_ptx.cuh"
 
@@ -589,15 +590,16 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 EncodeTiledFn get_encode() {
-    static EncodeTiledFn fn = nullptr;
-    if (!fn) {
+    // a function-local static: initialised once, thread-safe
+    static const EncodeTiledFn fn = [] {
         void *ptr = nullptr;
         cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
-                                             cudaEnableDefault, &q) == cudaSuccess &&
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    }
+            return reinterpret_cast<EncodeTiledFn>(ptr);
+        return static_cast<EncodeTiledFn>(nullptr);
+    }();
     return fn;
 }
 
@@ -614,22 +616,21 @@ bool make_map(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint64_t
                CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int g_sms = 0;
-
 template <int FMT>
 cudaError_t launch_fmt(const uint16_t *X, const uint8_t *Wraw, const float *bias, int M, int N, int K,
                        uint16_t *Y, unsigned int *err, cudaStream_t st) {
     using L = Layout<FMT>;
-    static int regs = -1;
-    if (regs < 0) {
+    static PerDevice<int> setup;
+    int regs = -1;
+    cudaError_t e = setup.get([](int &v) {
         cudaFuncAttributes fa;
-        cudaError_t e = cudaFuncGetAttributes(&fa, gemm_gguf_kernel<FMT>);
-        if (e != cudaSuccess) return e;
-        regs = fa.numRegs;
-        e = cudaFuncSetAttribute(gemm_gguf_kernel<FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 L::SMEM_TOTAL);
-        if (e != cudaSuccess) return e;
-    }
+        cudaError_t r = cudaFuncGetAttributes(&fa, gemm_gguf_kernel<FMT>);
+        if (r != cudaSuccess) return r;
+        v = fa.numRegs;
+        return cudaFuncSetAttribute(gemm_gguf_kernel<FMT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    L::SMEM_TOTAL);
+    }, &regs);
+    if (e != cudaSuccess) return e;
     // the register split above assumes the launch gets exactly this many
     if (regs != LAUNCH_REGS) return cudaErrorInvalidConfiguration;
     CUtensorMap mX, mW;
@@ -657,7 +658,8 @@ cudaError_t launch_fmt(const uint16_t *X, const uint8_t *Wraw, const float *bias
     p.spans = static_cast<int>(spans);
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
-    const int pairs = p.total_tiles < g_sms / 2 ? p.total_tiles : g_sms / 2;
+    const int sms = device_sms();
+    const int pairs = p.total_tiles < sms / 2 ? p.total_tiles : sms / 2;
     gemm_gguf_kernel<FMT><<<2 * pairs, THREADS, L::SMEM_TOTAL, st>>>(mX, mW, p);
     return cudaGetLastError();
 }
@@ -666,11 +668,6 @@ cudaError_t launch_fmt(const uint16_t *X, const uint8_t *Wraw, const float *bias
 
 cudaError_t launch_gemm_gguf(const uint16_t *X, const uint8_t *Wraw, int fmt, const float *bias, int M,
                              int N, int K, uint16_t *Y, unsigned int *err, cudaStream_t st) {
-    if (g_sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
-    }
     return fmt == 1 ? launch_fmt<1>(X, Wraw, bias, M, N, K, Y, err, st)
                     : launch_fmt<0>(X, Wraw, bias, M, N, K, Y, err, st);
 }

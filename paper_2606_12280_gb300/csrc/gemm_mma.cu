@@ -12,6 +12,7 @@
 #include <cuda_runtime.h>
 
 #include "common.cuh"
+#include "host_once.h"
 #include "launch.h"
 
 namespace w8a8 {
@@ -179,13 +180,13 @@ cudaError_t launch_gemm_mma(const GemmBranch *br, int nb, int N, int K, bool out
     }
     if (maxM == 0) return cudaSuccess;
     dim3 grid((N + BN - 1) / BN, (maxM + BM - 1) / BM, nb);
-    static bool configured[2] = {false, false};
-    if (!configured[out_i32 ? 1 : 0]) {
-        cudaError_t e = cudaFuncSetAttribute(out_i32 ? gemm_mma_kernel<true> : gemm_mma_kernel<false>,
-                                             cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
-        if (e != cudaSuccess) return e;
-        configured[out_i32 ? 1 : 0] = true;
-    }
+    static PerDevice<int> attr[2];
+    int unused = 0;
+    cudaError_t e = attr[out_i32 ? 1 : 0].get([&](int &) {
+        return cudaFuncSetAttribute(out_i32 ? gemm_mma_kernel<true> : gemm_mma_kernel<false>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES);
+    }, &unused);
+    if (e != cudaSuccess) return e;
     if (out_i32) gemm_mma_kernel<true><<<grid, 256, SMEM_BYTES, st>>>(bs, N, K);
     else gemm_mma_kernel<false><<<grid, 256, SMEM_BYTES, st>>>(bs, N, K);
     return cudaGetLastError();

@@ -28,6 +28,7 @@
 #include <cuda_runtime.h>
 
 #include "common.cuh"
+#include "host_once.h"
 #include "launch.h"
 #include "tc_ptx.cuh"
 
@@ -413,15 +414,16 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 EncodeTiledFn get_encode() {
-    static EncodeTiledFn fn = nullptr;
-    if (!fn) {
+    // a function-local static: initialised once, thread-safe
+    static const EncodeTiledFn fn = [] {
         void *ptr = nullptr;
         cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
-                                             cudaEnableDefault, &q) == cudaSuccess &&
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    }
+            return reinterpret_cast<EncodeTiledFn>(ptr);
+        return static_cast<EncodeTiledFn>(nullptr);
+    }();
     return fn;
 }
 
@@ -438,31 +440,32 @@ bool make_map(CUtensorMap *m, const int8_t *base, int rows, int K, int box_rows)
                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int g_sms = 0;
-int g_kernel_regs[2] = {-1, -1};
+template <bool OUT_I32>
+cudaError_t prepare_tc_kernel() {
+    static PerDevice<int> setup;
+    int regs = -1;
+    cudaError_t e = setup.get([](int &v) {
+        cudaFuncAttributes fa;
+        cudaError_t r = cudaFuncGetAttributes(&fa, gemm_tc_kernel<OUT_I32>);
+        if (r != cudaSuccess) return r;
+        v = fa.numRegs;
+        return cudaFuncSetAttribute(gemm_tc_kernel<OUT_I32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    SMEM_TOTAL);
+    }, &regs);
+    if (e != cudaSuccess) return e;
+    // the warp-group register split relies on the launch holding exactly
+    // 512 x 128 registers
+    return regs == LAUNCH_REGS ? cudaSuccess : cudaErrorInvalidConfiguration;
+}
 
 }  // namespace
 
 cudaError_t launch_gemm_tc(const GemmBranch *br, int nb, int N, int K, bool out_i32,
                            unsigned int *err, cudaStream_t st) {
-    if (g_sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
-    }
-    const int ki = out_i32 ? 1 : 0;
+    const int sms = device_sms();
     auto kern = out_i32 ? gemm_tc_kernel<true> : gemm_tc_kernel<false>;
-    if (g_kernel_regs[ki] < 0) {
-        cudaFuncAttributes fa;
-        cudaError_t e = cudaFuncGetAttributes(&fa, kern);
-        if (e != cudaSuccess) return e;
-        g_kernel_regs[ki] = fa.numRegs;
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_TOTAL);
-        if (e != cudaSuccess) return e;
-    }
-    // the warp-group register split relies on the launch holding exactly
-    // 512 x 128 registers
-    if (g_kernel_regs[ki] != LAUNCH_REGS) return cudaErrorInvalidConfiguration;
+    cudaError_t e = out_i32 ? prepare_tc_kernel<true>() : prepare_tc_kernel<false>();
+    if (e != cudaSuccess) return e;
 
     Params p{};
     CUtensorMap maps[4];
@@ -498,7 +501,7 @@ cudaError_t launch_gemm_tc(const GemmBranch *br, int nb, int N, int K, bool out_
     p.k_blocks = (K + BK - 1) / BK;
     p.err = err;
     p.wait_limit_ns = 2000000000ull;       // 2 s per wait
-    const int grid = p.total_tiles < g_sms ? p.total_tiles : g_sms;
+    const int grid = p.total_tiles < sms ? p.total_tiles : sms;
     kern<<<grid, THREADS, SMEM_TOTAL, st>>>(maps[0], maps[1], maps[2], maps[3], p);
     return cudaGetLastError();
 }

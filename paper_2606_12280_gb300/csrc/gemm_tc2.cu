@@ -30,6 +30,7 @@
 #include <cuda_runtime.h>
 
 #include "common.cuh"
+#include "host_once.h"
 #include "launch.h"
 #include "tc_ptx.cuh"
 
@@ -577,15 +578,16 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 EncodeTiledFn get_encode() {
-    static EncodeTiledFn fn = nullptr;
-    if (!fn) {
+    // a function-local static: initialised once, thread-safe
+    static const EncodeTiledFn fn = [] {
         void *ptr = nullptr;
         cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
-                                             cudaEnableDefault, &q) == cudaSuccess &&
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    }
+            return reinterpret_cast<EncodeTiledFn>(ptr);
+        return static_cast<EncodeTiledFn>(nullptr);
+    }();
     return fn;
 }
 
@@ -616,31 +618,33 @@ bool make_map_f16(CUtensorMap *m, const void *base, int rows, int K, int box_row
                CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int g_sms = 0;
-int g_kernel_regs[4] = {-1, -1, -1, -1};
+template <bool OUT_I32, bool A16>
+cudaError_t prepare_tc2_kernel() {
+    static PerDevice<int> setup;
+    int regs = -1;
+    cudaError_t e = setup.get([](int &v) {
+        cudaFuncAttributes fa;
+        cudaError_t r = cudaFuncGetAttributes(&fa, gemm_tc2_kernel<OUT_I32, A16>);
+        if (r != cudaSuccess) return r;
+        v = fa.numRegs;
+        return cudaFuncSetAttribute(gemm_tc2_kernel<OUT_I32, A16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    Lay<A16>::SMEM_TOTAL);
+    }, &regs);
+    if (e != cudaSuccess) return e;
+    return regs == LAUNCH_REGS ? cudaSuccess : cudaErrorInvalidConfiguration;
+}
 
 }  // namespace
 
 cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K, bool out_i32, bool a16,
                             unsigned int *err, cudaStream_t st) {
-    if (g_sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
-    }
-    const int ki = (out_i32 ? 1 : 0) + (a16 ? 2 : 0);
+    const int sms = device_sms();
     const int smem_total = a16 ? Lay<true>::SMEM_TOTAL : Lay<false>::SMEM_TOTAL;
     auto kern = a16 ? (out_i32 ? gemm_tc2_kernel<true, true> : gemm_tc2_kernel<false, true>)
                     : (out_i32 ? gemm_tc2_kernel<true, false> : gemm_tc2_kernel<false, false>);
-    if (g_kernel_regs[ki] < 0) {
-        cudaFuncAttributes fa;
-        cudaError_t e = cudaFuncGetAttributes(&fa, kern);
-        if (e != cudaSuccess) return e;
-        g_kernel_regs[ki] = fa.numRegs;
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem_total);
-        if (e != cudaSuccess) return e;
-    }
-    if (g_kernel_regs[ki] != LAUNCH_REGS) return cudaErrorInvalidConfiguration;
+    cudaError_t e = a16 ? (out_i32 ? prepare_tc2_kernel<true, true>() : prepare_tc2_kernel<false, true>())
+                        : (out_i32 ? prepare_tc2_kernel<true, false>() : prepare_tc2_kernel<false, false>());
+    if (e != cudaSuccess) return e;
 
     Params p{};
     CUtensorMap maps[4];
@@ -676,7 +680,7 @@ cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K, bool out
     p.k_blocks = (K + BK - 1) / BK;
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
-    const int pairs = p.total_tiles < g_sms / 2 ? p.total_tiles : g_sms / 2;
+    const int pairs = p.total_tiles < sms / 2 ? p.total_tiles : sms / 2;
     kern<<<2 * pairs, THREADS, smem_total, st>>>(maps[0], maps[1], maps[2], maps[3], p);
     return cudaGetLastError();
 }

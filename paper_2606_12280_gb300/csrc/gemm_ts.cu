@@ -42,6 +42,7 @@
 #include <cuda_runtime.h>
 
 #include "common.cuh"
+#include "host_once.h"
 #include "launch.h"
 #include "tc_ptx.cuh"
 
@@ -737,15 +738,16 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
 EncodeTiledFn get_encode() {
-    static EncodeTiledFn fn = nullptr;
-    if (!fn) {
+    // a function-local static: initialised once, thread-safe
+    static const EncodeTiledFn fn = [] {
         void *ptr = nullptr;
         cudaDriverEntryPointQueryResult q;
-        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000,
-                                             cudaEnableDefault, &q) == cudaSuccess &&
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
             q == cudaDriverEntryPointSuccess)
-            fn = reinterpret_cast<EncodeTiledFn>(ptr);
-    }
+            return reinterpret_cast<EncodeTiledFn>(ptr);
+        return static_cast<EncodeTiledFn>(nullptr);
+    }();
     return fn;
 }
 
@@ -762,8 +764,24 @@ bool make_map(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint64_t
                sw, CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-int g_sms = 0;
-int g_kernel_regs[2] = {-1, -1};
+// Per variant and device: the dynamic shared memory limit set and the
+// registers ptxas gave the kernel (the register split assumes exactly
+// LAUNCH_REGS at launch).
+template <bool OUT_I32>
+cudaError_t prepare_ts_kernel() {
+    static PerDevice<int> regs;
+    int n = 0;
+    cudaError_t e = regs.get([](int &v) {
+        cudaFuncAttributes fa;
+        cudaError_t r = cudaFuncGetAttributes(&fa, gemm_ts_kernel<OUT_I32>);
+        if (r != cudaSuccess) return r;
+        v = fa.numRegs;
+        return cudaFuncSetAttribute(gemm_ts_kernel<OUT_I32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                    SMEM_TOTAL);
+    }, &n);
+    if (e != cudaSuccess) return e;
+    return n == LAUNCH_REGS ? cudaSuccess : cudaErrorInvalidConfiguration;
+}
 
 }  // namespace
 
@@ -782,23 +800,10 @@ cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cu
 
 cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, unsigned int *err,
                            cudaStream_t st) {
-    if (g_sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
-    }
-    const int ki = out_i32 ? 1 : 0;
+    const int sms = device_sms();
     auto kern = out_i32 ? gemm_ts_kernel<true> : gemm_ts_kernel<false>;
-    if (g_kernel_regs[ki] < 0) {
-        cudaFuncAttributes fa;
-        cudaError_t e = cudaFuncGetAttributes(&fa, kern);
-        if (e != cudaSuccess) return e;
-        g_kernel_regs[ki] = fa.numRegs;
-        e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_TOTAL);
-        if (e != cudaSuccess) return e;
-    }
-    // the register split above assumes the launch gets exactly this many
-    if (g_kernel_regs[ki] != LAUNCH_REGS) return cudaErrorInvalidConfiguration;
+    cudaError_t e = out_i32 ? prepare_ts_kernel<true>() : prepare_ts_kernel<false>();
+    if (e != cudaSuccess) return e;
 
     Params p{};
     CUtensorMap maps[4];
@@ -842,7 +847,7 @@ cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_
         if (p.br[i].M > 0 && (p.br[i].x_sumsq == nullptr || p.br[i].plan == nullptr)) p.single_ok = 0;
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
-    const int pairs = p.total_tiles < g_sms / 2 ? p.total_tiles : g_sms / 2;
+    const int pairs = p.total_tiles < sms / 2 ? p.total_tiles : sms / 2;
     kern<<<2 * pairs, THREADS, SMEM_TOTAL, st>>>(maps[0], maps[1], maps[2], maps[3], p);
     return cudaGetLastError();
 }

@@ -17,6 +17,7 @@
 #include <cuda_runtime.h>
 
 #include "common.cuh"
+#include "host_once.h"
 #include "launch.h"
 
 namespace w8a8 {
@@ -331,17 +332,7 @@ row_quant_long_kernel(const InT *__restrict__ in, const float *__restrict__ lam,
     }
 }
 
-int g_num_sms = 0;
-
-int num_sms() {
-    if (g_num_sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_num_sms, cudaDevAttrMultiProcessorCount, dev);
-        if (g_num_sms <= 0) g_num_sms = 148;
-    }
-    return g_num_sms;
-}
+int num_sms() { return device_sms(); }
 
 template <typename InT, bool IS_ACT, int CPT>
 cudaError_t launch_row_quant_cpt(const InT *in, const float *lam, int M, int K, int G,
@@ -349,13 +340,15 @@ cudaError_t launch_row_quant_cpt(const InT *in, const float *lam, int M, int K, 
     const int block = G < 256 ? 256 : G;
     const int teams = block / G;
     const int groups = (M + teams - 1) / teams;
-    static int per_sm_cache[2] = {0, 0};       // block = 256 or 512
-    int &per_sm = per_sm_cache[block == 256 ? 0 : 1];
-    if (per_sm == 0) {
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, row_quant_kernel<InT, IS_ACT, CPT>,
-                                                      block, 0);
-        if (per_sm < 1) per_sm = 1;
-    }
+    static PerDevice<int> setup[2];            // block = 256 or 512
+    int per_sm = 1;
+    cudaError_t e = setup[block == 256 ? 0 : 1].get([&](int &v) {
+        cudaError_t r = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, row_quant_kernel<InT, IS_ACT, CPT>,
+                                                                      block, 0);
+        if (v < 1) v = 1;
+        return r;
+    }, &per_sm);
+    if (e != cudaSuccess) return e;
     int grid = num_sms() * per_sm;
     if (grid > groups) grid = groups;
     if (grid < 1) grid = 1;
@@ -674,17 +667,19 @@ cudaError_t launch_act_quant_team(ActParams p, cudaStream_t st) {
     constexpr int kThreads = TW > 8 ? 32 * TW : 256;
     constexpr int kTeams = kThreads / (32 * TW);
     constexpr size_t smem = (size_t)(kThreads / 32) * S * U * 32 * 16;
-    static int per_sm = 0;
     auto kern = act_quant_team_kernel<U, TW, S, GELU, OUT16>;
-    if (per_sm == 0) {
+    static PerDevice<int> setup;
+    int per_sm = 1;
+    cudaError_t e = setup.get([&](int &v) {
         // always opted in: the static reduction array counts against the
         // 48 KB default too
-        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                             (int)smem);
-        if (e != cudaSuccess) return e;
-        cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, kThreads, smem);
-        if (per_sm < 1) per_sm = 1;
-    }
+        cudaError_t r = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem);
+        if (r != cudaSuccess) return r;
+        r = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&v, kern, kThreads, smem);
+        if (v < 1) v = 1;
+        return r;
+    }, &per_sm);
+    if (e != cudaSuccess) return e;
     const int M0 = p.br[0].M, M1 = p.br[1].M;
     int grid = num_sms() * per_sm;
     const int blocks_needed = (M0 + M1 + kTeams - 1) / kTeams;

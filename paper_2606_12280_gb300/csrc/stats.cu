@@ -24,22 +24,13 @@
 #include <cuda_runtime.h>
 
 #include "common.cuh"
+#include "host_once.h"
 #include "launch.h"
 
 namespace w8a8 {
 namespace {
 
-int g_sms = 0;
-
-int num_sms() {
-    if (g_sms == 0) {
-        int dev = 0;
-        cudaGetDevice(&dev);
-        cudaDeviceGetAttribute(&g_sms, cudaDevAttrMultiProcessorCount, dev);
-        if (g_sms <= 0) g_sms = 148;
-    }
-    return g_sms;
-}
+int num_sms() { return device_sms(); }
 
 // ----------------------------------------------------- packed fp32 helpers
 // Two fp32 lanes per instruction (sm_100 family).  Used only in the
@@ -430,25 +421,28 @@ tensor_quant_kernel(const uint16_t *__restrict__ X, const float *__restrict__ la
     }
 }
 
-// Row slabs so that a (gx x gy) grid fills the GPU once: gy = the resident
-// blocks of `kern` on all SMs divided by gx, at most one slab per row.
+// Resident blocks per SM of `kern` (no dynamic shared memory), looked up once
+// per device.
 template <typename Kern>
-int slabs_for(Kern kern, int threads, int rows, int gx) {
-    int per_sm = 0;
-    if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, kern, threads, 0) != cudaSuccess ||
-        per_sm < 1)
-        per_sm = 1;
+int blocks_per_sm(PerDevice<int> &cache, Kern kern, int threads) {
+    int v = 1;
+    if (cache.get([&](int &n) {
+            cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, threads, 0);
+            if (n < 1) n = 1;
+            return e;
+        }, &v) != cudaSuccess)
+        return 1;
+    return v;
+}
+
+// Row slabs so that a (gx x gy) grid fills the GPU once: gy = the resident
+// blocks on all SMs divided by gx, at most one slab per row.
+int slabs_for(int per_sm, int rows, int gx) {
     int gy = (num_sms() * per_sm) / gx;
     if (gy > rows) gy = rows;
     if (gy < 1) gy = 1;
     return gy;
 }
-
-// Cached slab counts per (kernel, gx, rows); the grid shape depends only on
-// the launch shape.
-struct SlabCache {
-    int gx = -1, rows = -1, gy = 0;
-};
 
 // One-shot statistics without caller accumulators: a file-scope scratch of
 // power sums (4 x max K doubles) then max-abs (max K floats), cleared at the
@@ -459,14 +453,10 @@ static __device__ __align__(256) unsigned char g_stats_scratch[kNoAllocMaxK * (4
 // Device address of the scratch on the current device, looked up once per
 // device (the lookup is not a stream operation: do it before any capture).
 void *stats_scratch_address() {
-    constexpr int kMaxDevices = 64;
-    static void *cache[kMaxDevices] = {};
-    int dev = 0;
-    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= kMaxDevices) return nullptr;
-    if (cache[dev]) return cache[dev];
+    static PerDevice<void *> addr;
     void *p = nullptr;
-    if (cudaGetSymbolAddress(&p, g_stats_scratch) != cudaSuccess) return nullptr;
-    cache[dev] = p;
+    if (addr.get([](void *&v) { return cudaGetSymbolAddress(&v, g_stats_scratch); }, &p) != cudaSuccess)
+        return nullptr;
     return p;
 }
 
@@ -475,13 +465,8 @@ void *stats_scratch_address() {
 cudaError_t launch_act_stats_update(const uint16_t *X, int T, int K, const float *shift,
                                     double *sums, float *absmax, cudaStream_t st) {
     const int gx = (K / 4 + 31) / 32;
-    static SlabCache cache;
-    if (cache.gx != gx || cache.rows != T) {
-        cache.gy = slabs_for(stats_update_kernel, 32 * kStatsWarps, T, gx);
-        cache.gx = gx;
-        cache.rows = T;
-    }
-    int gy = cache.gy;
+    static PerDevice<int> occ;
+    int gy = slabs_for(blocks_per_sm(occ, stats_update_kernel, 32 * kStatsWarps), T, gx);
     const int rows_per_slab = (T + gy - 1) / gy;
     gy = (T + rows_per_slab - 1) / rows_per_slab;
     stats_update_kernel<<<dim3(gx, gy), 32 * kStatsWarps, 0, st>>>(
@@ -502,14 +487,10 @@ cudaError_t launch_quant_act_per_tensor(const uint16_t *X, const float *lambda, 
     cudaError_t e = cudaMemsetAsync(amax, 0, sizeof(float), st);
     if (e != cudaSuccess) return e;
     const int gx = (K / 8 + 31) / 32;
-    static SlabCache c1, c2;
-    if (c1.gx != gx || c1.rows != M) {
-        c1.gy = slabs_for(tensor_absmax_kernel, 32 * kQWarps, M, gx);
-        c2.gy = slabs_for(tensor_quant_kernel, 32 * kQWarps, M, gx);
-        c1.gx = c2.gx = gx;
-        c1.rows = c2.rows = M;
-    }
-    const int rps1 = (M + c1.gy - 1) / c1.gy, rps2 = (M + c2.gy - 1) / c2.gy;
+    static PerDevice<int> occ1, occ2;
+    const int gy1 = slabs_for(blocks_per_sm(occ1, tensor_absmax_kernel, 32 * kQWarps), M, gx);
+    const int gy2 = slabs_for(blocks_per_sm(occ2, tensor_quant_kernel, 32 * kQWarps), M, gx);
+    const int rps1 = (M + gy1 - 1) / gy1, rps2 = (M + gy2 - 1) / gy2;
     tensor_absmax_kernel<<<dim3(gx, (M + rps1 - 1) / rps1), 32 * kQWarps, 0, st>>>(X, lambda, M, K,
                                                                                    rps1, amax);
     e = cudaGetLastError();
