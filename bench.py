@@ -228,8 +228,6 @@ def run_ours(args):
     if ws > 1:
         import torch.distributed as dist
         dist.init_process_group("nccl", device_id=dev)
-    if args.engine is not None:
-        w8a8.set_gemm_engine(args.engine)
     w8a8.lib()
 
     case = wl.workload_cases(args.workload)[0]
@@ -636,8 +634,7 @@ def run_ours(args):
     gemm_avg = sum(gemm_ms) / len(gemm_ms)
     quant_avg = sum(quant_ms) / len(quant_ms)
     gemm_tflops = ops_step / (gemm_avg * 1e-3) / 1e12
-    engine = w8a8.get_gemm_engine()
-    engine_name = "ts" if f16 else {2: "tc2", 1: "tc", 0: "mma"}[engine]
+    engine_name = "ts" if f16 else "tc2"
     peak_t = peaks["bf16_tflops"]
     quant_bytes = (2.0 + code_bytes) * M * K + 4.0 * M + 4.0 * K
     pt_bytes = 3.0 * M * K + 4.0 * M + 4.0 * K     # the per-tensor pass writes int8 codes
@@ -775,8 +772,6 @@ def main(argv=None):
     p.add_argument("--warmup", type=int, default=5)
     p.add_argument("--impl", choices=["ours", "reference"], default="ours")
     p.add_argument("--workload", default="qkv_m4608_k4096_n12288")
-    p.add_argument("--engine", type=int, default=None,
-                   help="int8 codes: 2 tcgen05 pairs (default), 1 tcgen05, 0 mma.sync")
     p.add_argument("--codes", choices=["f16", "int8"], default="f16",
                    help="container of the activation codes between a3 and the GEMM")
     p.add_argument("--no-cpu-baseline", action="store_true")

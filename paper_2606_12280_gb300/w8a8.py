@@ -32,8 +32,7 @@ SIGNATURES = {
     "w8a8_linear": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P],
     "w8a8_linear_dual": [_P, _I, _I, _P],
     "w8a8_debug_gemm_i32": [_P, _P, _I, _I, _I, _P, _P],
-    "w8a8_set_gemm_engine": [_I],
-    "w8a8_get_gemm_engine": [],
+    "w8a8_debug_linear_engine": [_I, _P, _I, _I, _I, _I, _P],
     "w8a8_device_status": [_P, ctypes.POINTER(ctypes.c_uint32)],
     "w8a8_debug_wait_timeout": [ctypes.c_uint32, _P],
     "w8a8_status_string": [_I],
@@ -140,7 +139,18 @@ def _ptr(t, dtype, name):
         raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
     if not t.is_contiguous():
         raise ValueError(f"{name} must be contiguous")
+    # the library launches on the current device and dereferences every
+    # pointer there
+    if t.device.index != torch.cuda.current_device():
+        raise ValueError(f"{name} is on {t.device}, the current device is cuda:{torch.cuda.current_device()}")
     return t.data_ptr()
+
+
+def _shape(t, shape, name):
+    """Refuse a tensor whose shape is not exactly `shape` (where the library
+    addresses it with strides that the shape fixes)."""
+    if t is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} has shape {tuple(t.shape)}, the call needs {tuple(shape)}")
 
 
 def _room(t, n, name):
@@ -210,12 +220,16 @@ def quant_act(X, smooth=None, Xq=None, x_scale=None, stream=None):
     return Xq, x_scale
 
 
+def _check_weights(Wq, N, K):
+    if tuple(Wq.shape) != (N, K):
+        raise ValueError(f"Wq has shape {tuple(Wq.shape)}, the activations need ({N}, {K})")
+
+
 def linear(Xq, x_scale, Wq, w_scale, bias=None, Y=None, stream=None):
     """Y = bf16((Xq Wq^T) * sx * sw + b): [M,N] bf16."""
     M, K = Xq.shape
     N = Wq.shape[0]
-    if Wq.shape[1] != K:
-        raise ValueError("Xq and Wq disagree on K")
+    _check_weights(Wq, N, K)
     if Y is None:
         Y = torch.empty(M, N, dtype=torch.bfloat16, device=Xq.device)
     _room(x_scale, M, "x_scale")
@@ -230,29 +244,34 @@ def linear(Xq, x_scale, Wq, w_scale, bias=None, Y=None, stream=None):
     return Y
 
 
-def linear_dual(branches, Ys=None, stream=None):
-    """One grouped launch over two branches.  branches: two tuples
-    (Xq, x_scale, Wq, w_scale, bias); returns [Y_cond, Y_uncond]."""
-    if len(branches) != 2:
-        raise ValueError("linear_dual takes exactly two branches")
+def _branch_array(branches, Ys, out_dtype=torch.bfloat16):
+    """Branch structs for two (or one) branches (Xq, x_scale, Wq, w_scale,
+    bias); returns (array, outputs, N, K)."""
     N, K = branches[0][2].shape
-    arr = (Branch * 2)()
+    arr = (Branch * len(branches))()
     out = []
     for i, (Xq, sx, Wq, sw, b) in enumerate(branches):
         if tuple(Wq.shape) != (N, K) or Xq.shape[1] != K:
             raise ValueError("branches must share N and K")
-        Y = Ys[i] if Ys is not None else torch.empty(Xq.shape[0], N, dtype=torch.bfloat16,
-                                                     device=Xq.device)
         M = Xq.shape[0]
+        Y = Ys[i] if Ys is not None else torch.empty(M, N, dtype=out_dtype, device=Xq.device)
         _room(sx, M, "x_scale")
         _room(sw, N, "w_scale")
         _room(b, N, "bias")
         _room(Y, M * N, "Y")
         arr[i] = Branch(_ptr(Xq, torch.int8, "Xq"), _ptr(sx, torch.float32, "x_scale"),
                         _ptr(Wq, torch.int8, "Wq"), _ptr(sw, torch.float32, "w_scale"),
-                        _ptr(b, torch.float32, "bias"), _ptr(Y, torch.bfloat16, "Y"),
-                        Xq.shape[0])
+                        _ptr(b, torch.float32, "bias"), _ptr(Y, out_dtype, "Y"), M)
         out.append(Y)
+    return arr, out, N, K
+
+
+def linear_dual(branches, Ys=None, stream=None):
+    """One grouped launch over two branches.  branches: two tuples
+    (Xq, x_scale, Wq, w_scale, bias); returns [Y_cond, Y_uncond]."""
+    if len(branches) != 2:
+        raise ValueError("linear_dual takes exactly two branches")
+    arr, out, N, K = _branch_array(branches, Ys)
     _check("w8a8_linear_dual", lib().w8a8_linear_dual(arr, N, K, _stream(stream)))
     return out
 
@@ -261,6 +280,7 @@ def debug_gemm_i32(Xq, Wq, acc=None, stream=None):
     """Exact int32 acc = Xq Wq^T (test export of the GEMM alone)."""
     M, K = Xq.shape
     N = Wq.shape[0]
+    _check_weights(Wq, N, K)
     if acc is None:
         acc = torch.empty(M, N, dtype=torch.int32, device=Xq.device)
     _room(acc, M * N, "acc")
@@ -270,13 +290,17 @@ def debug_gemm_i32(Xq, Wq, acc=None, stream=None):
     return acc
 
 
-def set_gemm_engine(engine: int) -> None:
-    """1 = tcgen05 tensor cores, 0 = legacy mma.sync s8, -1 = default."""
-    _check("w8a8_set_gemm_engine", lib().w8a8_set_gemm_engine(int(engine)))
-
-
-def get_gemm_engine() -> int:
-    return int(lib().w8a8_get_gemm_engine())
+def debug_linear_engine(engine: int, branches, Ys=None, out_i32=False, stream=None):
+    """Test anchor: the exact-integer product on a chosen int8-code engine (2
+    the product's tcgen05 CTA pairs, 1 tcgen05 single SMs, 0 mma.sync), per
+    call, on one or two branches (Xq, x_scale, Wq, w_scale, bias); returns the
+    outputs (bf16 Y, or int32 products when out_i32)."""
+    if len(branches) not in (1, 2):
+        raise ValueError("one or two branches")
+    arr, out, N, K = _branch_array(branches, Ys, torch.int32 if out_i32 else torch.bfloat16)
+    _check("w8a8_debug_linear_engine", lib().w8a8_debug_linear_engine(
+        int(engine), arr, len(branches), N, K, 1 if out_i32 else 0, _stream(stream)))
+    return out
 
 
 def device_status(stream=None) -> int:
@@ -425,6 +449,7 @@ def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, x_
     ``quant_act_f16codes(..., sumsq=)`` wrote for these codes."""
     M, K = Xq16.shape
     N = Wq.shape[0]
+    _check_weights(Wq, N, K)
     if Y is None:
         Y = torch.empty(M, N, dtype=torch.bfloat16, device=Xq16.device)
     _room(x_scale, M, "x_scale")
@@ -446,6 +471,7 @@ def debug_gemm_f16codes_i32(Xq16, Wq, plan=None, x_sumsq=None, acc=None, stream=
     """Exact int32 acc = Xq16 Wq^T (test export of the fp16-code GEMM)."""
     M, K = Xq16.shape
     N = Wq.shape[0]
+    _check_weights(Wq, N, K)
     if acc is None:
         acc = torch.empty(M, N, dtype=torch.int32, device=Xq16.device)
     if plan is not None:
@@ -540,8 +566,9 @@ def act_stats_update(X, sums, absmax, shift=None, stream=None):
     """Accumulate the per-channel power sums [4,K] fp64 and absmax [K] of X [T,K] bf16."""
     T, K = X.shape
     _room(shift, K, "shift")
-    _room(sums, 4 * K, "sums")
-    _room(absmax, K, "absmax")
+    # the library addresses the four planes at stride K
+    _shape(sums, (4, K), "sums")
+    _shape(absmax, (K,), "absmax")
     _check("w8a8_act_stats_update", lib().w8a8_act_stats_update(
         _ptr(X, torch.bfloat16, "X"), T, K, _ptr(shift, torch.float32, "shift"),
         _ptr(sums, torch.float64, "sums"), _ptr(absmax, torch.float32, "absmax"),
@@ -555,7 +582,8 @@ def act_stats_finalize(sums, absmax, count: int, shift=None, chan=None, tensor=N
         chan = torch.empty(4, K, dtype=torch.float32, device=absmax.device)
     if tensor is None:
         tensor = torch.empty(4, dtype=torch.float32, device=absmax.device)
-    _room(sums, 4 * K, "sums")
+    _shape(absmax, (K,), "absmax")
+    _shape(sums, (4, K), "sums")
     _room(shift, K, "shift")
     _room(chan, 4 * K, "chan")
     _room(tensor, 4, "tensor")
@@ -604,13 +632,24 @@ def layer_forward(X, protect: bool, N: int, K: int, smooth=None, Wq=None, w_scal
                   W_bf16=None, bias=None, Xq_work=None, x_scale_work=None, Y=None, stream=None):
     """Per-layer dispatch (protected -> bf16 linear, else a3 + a4 + a5)."""
     M = X.shape[0]
+    if tuple(X.shape) != (M, K):
+        raise ValueError(f"X has shape {tuple(X.shape)}, the layer needs ({M}, {K})")
     if Y is None:
         Y = torch.empty(M, N, dtype=torch.bfloat16, device=X.device)
-    if not protect:
+    _room(bias, N, "bias")
+    _room(Y, M * N, "Y")
+    if protect:
+        _room(W_bf16, N * K, "W_bf16")
+    else:
         if Xq_work is None:
             Xq_work = torch.empty(M, K, dtype=torch.int8, device=X.device)
         if x_scale_work is None:
             x_scale_work = torch.empty(M, dtype=torch.float32, device=X.device)
+        _room(smooth, K, "smooth")
+        _room(Wq, N * K, "Wq")
+        _room(w_scale, N, "w_scale")
+        _room(Xq_work, M * K, "Xq_work")
+        _room(x_scale_work, M, "x_scale_work")
     layer = Layer(1 if protect else 0, N, K, _ptr(smooth, torch.float32, "smooth"),
                   _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
                   _ptr(W_bf16, torch.bfloat16, "W_bf16"), _ptr(bias, torch.float32, "bias"))

@@ -125,18 +125,32 @@ def test_dual_validation(L):
     assert f(arr, 8, 16, None) == OK                      # both branches empty
 
 
+def test_debug_engine_validation(L):
+    """The earlier engines are reached only through the test entry point,
+    per call (no process-wide switch)."""
+    from paper_2606_12280_gb300.w8a8 import Branch
+    arr = (Branch * 2)()
+    for i in range(2):
+        arr[i] = Branch(A, A, A, A, None, A, 4)
+    f = L.w8a8_debug_linear_engine
+    assert f(3, arr, 1, 8, 16, 0, None) == INVALID        # no such engine
+    assert f(-1, arr, 1, 8, 16, 0, None) == INVALID
+    assert f(2, arr, 0, 8, 16, 0, None) == INVALID        # one or two branches
+    assert f(2, arr, 3, 8, 16, 0, None) == INVALID
+    assert f(2, None, 1, 8, 16, 0, None) == INVALID
+    assert f(1, arr, 2, 12, 16, 0, None) == SHAPE
+    arr[0].x_scale = None
+    assert f(0, arr, 1, 8, 16, 0, None) == INVALID        # scales needed for the bf16 output
+    arr[0].Y = U
+    assert f(0, arr, 1, 8, 16, 1, None) == MISALIGNED     # int32 output: scales unused
+    arr[0].M = 0
+    assert f(0, arr, 1, 8, 16, 1, None) == OK
+    assert not hasattr(L, "w8a8_set_gemm_engine")
+
+
 def test_wait_probe_validation(L):
     assert L.w8a8_debug_wait_timeout(0, None) == INVALID
     assert L.w8a8_debug_wait_timeout(2000001, None) == INVALID
-
-
-def test_engine_switch(L):
-    assert L.w8a8_set_gemm_engine(7) == INVALID
-    assert L.w8a8_set_gemm_engine(0) == OK
-    assert L.w8a8_get_gemm_engine() == 0
-    assert L.w8a8_set_gemm_engine(-1) == OK
-    assert L.w8a8_get_gemm_engine() == 2
-    assert L.w8a8_set_gemm_engine(3) == INVALID
 
 
 def test_binding_fails_loudly_without_library(monkeypatch, tmp_path):
@@ -290,6 +304,7 @@ def test_noalloc_stats_validation(L):
     assert f(A, 4, 32768 + 16, None, A, A, None) == SHAPE       # beyond the static scratch
     assert f(A, 4, 24, None, A, A, None) == SHAPE
     assert f(A, 0, 16, None, A, A, None) == INVALID            # no tokens
+    assert f(A, -3, 16, None, A, A, None) == INVALID           # negative count: T >= 1
     assert f(None, 4, 16, None, A, A, None) == INVALID
     assert f(A, 4, 16, None, U, A, None) == MISALIGNED
 

@@ -58,6 +58,10 @@ def cases(w8):
                                                                  "tensor": (4, f32)}),
         (w8.act_stats_noalloc, (X,), {"shift": (K, f32), "chan": (4 * K, f32), "tensor": (4, f32)}),
         (w8.linear_bf16, (X, e((N, K), bf16)), {"bias": (N, f32), "Y": (M * N, bf16)}),
+        (w8.layer_forward, (X, False, N, K), {"smooth": (K, f32), "Wq": (N * K, i8), "w_scale": (N, f32),
+                                              "bias": (N, f32), "Xq_work": (M * K, i8),
+                                              "x_scale_work": (M, f32), "Y": (M * N, bf16)}),
+        (w8.layer_forward, (X, True, N, K), {"W_bf16": (N * K, bf16), "bias": (N, f32), "Y": (M * N, bf16)}),
     ]
 
 
@@ -83,6 +87,36 @@ def test_inputs_sized_too(w8):
         w8.linear_gguf(e((M, K), bf16), e(N * 34 - 1, u8), 0, N)
     with pytest.raises(ValueError, match="sums"):
         w8.act_stats_update(e((M, K), bf16), e(4 * K - 1, f64), e(K, f32))
+
+
+def test_weights_match_the_activations(w8):
+    """A weight matrix narrower than the activations' K would be read past
+    its end: every GEMM entry refuses it."""
+    Xq, X16, short = e((M, K), i8), e((M, K), f16), e((N, K - 16), i8)
+    for call in (lambda: w8.linear(Xq, e(M, f32), short, e(N, f32)),
+                 lambda: w8.debug_gemm_i32(Xq, short),
+                 lambda: w8.linear_f16codes(X16, e(M, f32), short, e(N, f32)),
+                 lambda: w8.debug_gemm_f16codes_i32(X16, short)):
+        with pytest.raises(ValueError, match="Wq"):
+            call()
+
+
+def test_statistics_planes_exact_shape(w8):
+    """The library addresses the four power-sum planes at stride K: a wider
+    accumulator (enough elements, wrong stride) is refused, and so is an
+    absmax longer than the batch's K."""
+    X = e((M, K), bf16)
+    with pytest.raises(ValueError, match="sums"):
+        w8.act_stats_update(X, e((4, 2 * K), f64), e(K, f32))
+    with pytest.raises(ValueError, match="absmax"):
+        w8.act_stats_update(X, e((4, K), f64), e(2 * K, f32))
+    with pytest.raises(ValueError, match="sums"):
+        w8.act_stats_finalize(e((4, 2 * K), f64), e(K, f32), M)
+
+
+def test_layer_forward_checks_x(w8):
+    with pytest.raises(ValueError, match="X has shape"):
+        w8.layer_forward(e((M, K - 16), bf16), False, N, K)
 
 
 def test_dual_branches_sized(w8):

@@ -44,7 +44,8 @@ def codes(Xq16):
     return q.astype(np.int8)
 
 
-@pytest.mark.parametrize("M,K", [(1, 16), (300, 528), (257, 4096), (64, 16384)])
+@pytest.mark.parametrize("M,K", [(1, 16), (1000, 272), (300, 528), (77, 2064), (257, 4096), (40, 4112),
+                                 (64, 16384)])
 def test_quant_act_f16codes_exact(w8, oracle_mod, M, K):
     X = wl.random_bf16((M, K), seed=M + K, scale=2.0)
     X[0, :] = 0                                         # an all-zero token

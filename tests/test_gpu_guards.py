@@ -61,7 +61,7 @@ def check(*gs):
         assert g.intact()
 
 
-@pytest.mark.parametrize("M,K", [(131, 528), (37, 16384 + 16)])
+@pytest.mark.parametrize("M,K", [(131, 528), (1001, 4096), (37, 4112), (37, 16384 + 16)])
 def test_quant_act(w8, M, K):
     X = bf(wl.random_bf16((M, K), seed=M + K, scale=2.0))
     lam = t(wl.random_uniform_f32((K,), seed=K, lo=0.25, hi=4.0))
@@ -125,6 +125,7 @@ def test_linear_f16codes_and_i32(w8, with_plan):
     w8.debug_gemm_f16codes_i32(q16, Wq, plan=plan, x_sumsq=ss if with_plan else None, acc=acc.t)
     check(acc)
     assert torch.equal(acc.t, w8.debug_gemm_i32(q8, Wq))
+
 
 
 def test_linear_dual_both_containers(w8):

@@ -5,8 +5,9 @@ product bit-exact; bf16 outputs within 1 bf16 ulp (relative 2^-8), and in fact
 bit-identical because both sides follow the same pinned fp32 op order.  Sizes
 span several tiles with ragged tails; edge cases cover empty and single-row
 inputs, all-zero rows and columns, adversarial INT8 extremes and the largest K.
-All three GEMM engines (tcgen05 on SM pairs, tcgen05 on single SMs, and
-mma.sync) are checked.
+The product GEMM (tcgen05 on SM pairs) is checked through w8a8_linear and the
+earlier engines kept as test anchors (tcgen05 on single SMs, mma.sync)
+through the test-only entry point that takes the engine per call.
 """
 
 import numpy as np
@@ -17,7 +18,8 @@ from paper_2606_12280_gb300 import workloads as wl
 
 pytestmark = pytest.mark.gpu
 
-ENGINES = [2, 1, 0]
+ENGINES = ["tcgen05_pair", "tcgen05", "mma_sync"]
+DEBUG_ENGINE = {"tcgen05": 1, "mma_sync": 0}
 
 
 @pytest.fixture(scope="module")
@@ -27,14 +29,37 @@ def w8():
     from paper_2606_12280_gb300 import w8a8
     w8a8.lib()
     yield w8a8
-    w8a8.set_gemm_engine(-1)
 
 
-@pytest.fixture(params=ENGINES, ids=["tcgen05_pair", "tcgen05", "mma_sync"])
+class Engine:
+    """One GEMM engine behind the calls the tests make: the product engine
+    through w8a8_linear / w8a8_linear_dual / w8a8_debug_gemm_i32, the others
+    through the test-only entry point that takes the engine as an argument."""
+
+    def __init__(self, w8, name):
+        self.w8, self.name = w8, name
+
+    def linear(self, Xq, sx, Wq, sw, b=None, Y=None):
+        if self.name in DEBUG_ENGINE:
+            return self.w8.debug_linear_engine(DEBUG_ENGINE[self.name], [(Xq, sx, Wq, sw, b)],
+                                               Ys=None if Y is None else [Y])[0]
+        return self.w8.linear(Xq, sx, Wq, sw, b, Y=Y)
+
+    def debug_gemm_i32(self, Xq, Wq, acc=None):
+        if self.name in DEBUG_ENGINE:
+            return self.w8.debug_linear_engine(DEBUG_ENGINE[self.name], [(Xq, None, Wq, None, None)],
+                                               Ys=None if acc is None else [acc], out_i32=True)[0]
+        return self.w8.debug_gemm_i32(Xq, Wq, acc=acc)
+
+    def linear_dual(self, brs):
+        if self.name in DEBUG_ENGINE:
+            return self.w8.debug_linear_engine(DEBUG_ENGINE[self.name], brs)
+        return self.w8.linear_dual(brs)
+
+
+@pytest.fixture(params=ENGINES)
 def engine(request, w8):
-    w8.set_gemm_engine(request.param)
-    yield request.param
-    w8.set_gemm_engine(-1)
+    return Engine(w8, request.param)
 
 
 DEV = "cuda"
@@ -104,8 +129,11 @@ def test_quantize_weights(w8, oracle_mod, N, K, smooth):
     np.testing.assert_array_equal(sw.cpu().numpy(), sw_ref)
 
 
-@pytest.mark.parametrize("M,K", [(1, 16), (7, 48), (129, 528), (300, 4096), (33, 16384),
-                                 (5, 20016), (4608, 512)])
+# K spans every team width of the warp-team kernel (K <= 256, 512, 1024, 2048,
+# 4096, 8192, 16384 values per row, each with a ragged last chunk) and the
+# long-row kernel beyond
+@pytest.mark.parametrize("M,K", [(1, 16), (7, 48), (2, 256), (1000, 272), (129, 528), (77, 2064),
+                                 (300, 4096), (513, 4112), (40, 8208), (33, 16384), (5, 20016), (4608, 512)])
 @pytest.mark.parametrize("smooth", [True, False])
 def test_quant_act(w8, oracle_mod, M, K, smooth):
     c = wl.make_case(M, K, 16, seed=M + K, outlier_frac=0.01, outlier_mult=30.0)
@@ -145,7 +173,7 @@ GEMM_SHAPES = [(1, 8, 16), (7, 24, 48), (129, 136, 528), (300, 264, 1040),
 def test_gemm_i32_exact(w8, engine, oracle_mod, M, N, K):
     Xq = wl.random_int8((M, K), seed=M * 3 + K)
     Wq = wl.random_int8((N, K), seed=N * 5 + K)
-    acc = w8.debug_gemm_i32(t(Xq), t(Wq)).cpu().numpy()
+    acc = engine.debug_gemm_i32(t(Xq), t(Wq)).cpu().numpy()
     np.testing.assert_array_equal(acc, oracle_mod.gemm_i32(Xq, Wq))
 
 
@@ -170,7 +198,7 @@ def test_gemm_i32_adversarial_k16384(w8, engine, oracle_mod, pattern):
         g = np.random.default_rng(0)
         Xq = (g.integers(0, 2, (M, K)) * 254 - 127).astype(np.int8)
         Wq = (g.integers(0, 2, (N, K)) * 254 - 127).astype(np.int8)
-    acc = w8.debug_gemm_i32(t(Xq), t(Wq)).cpu().numpy()
+    acc = engine.debug_gemm_i32(t(Xq), t(Wq)).cpu().numpy()
     want = oracle_mod.gemm_i32(Xq, Wq)
     np.testing.assert_array_equal(acc, want)
 
@@ -181,7 +209,7 @@ def test_gemm_i32_max_k(w8, engine, oracle_mod):
     Xq[1] = -127
     Wq = np.full((8, K), 127, np.int8)
     Wq[2, ::2] = -127
-    acc = w8.debug_gemm_i32(t(Xq), t(Wq)).cpu().numpy()
+    acc = engine.debug_gemm_i32(t(Xq), t(Wq)).cpu().numpy()
     np.testing.assert_array_equal(acc, oracle_mod.gemm_i32(Xq, Wq))
 
 
@@ -193,7 +221,7 @@ def test_linear(w8, engine, oracle_mod, M, N, K, with_bias):
     sx = np.abs(wl.random_f32((M,), seed=M, scale=0.03)).astype(np.float32)
     sw = np.abs(wl.random_f32((N,), seed=N, scale=1e-4)).astype(np.float32)
     b = wl.random_f32((N,), seed=N + 1, scale=0.01) if with_bias else None
-    Y = w8.linear(t(Xq), t(sx), t(Wq), t(sw), t(b) if with_bias else None)
+    Y = engine.linear(t(Xq), t(sx), t(Wq), t(sw), t(b) if with_bias else None)
     want = oracle_mod.linear(Xq, sx, Wq, sw, b)
     assert_bf16_close(u16(Y), want)
     np.testing.assert_array_equal(u16(Y), want)   # same pinned op order
@@ -205,8 +233,8 @@ def test_linear_empty_and_dual_ragged(w8, engine, oracle_mod):
     sw = [np.abs(wl.random_f32((N,), seed=50 + i, scale=1e-4)).astype(np.float32) for i in range(2)]
     b = [wl.random_f32((N,), seed=60 + i, scale=0.01) for i in range(2)]
     # M = 0 is a no-op
-    Y0 = w8.linear(torch.empty(0, K, dtype=torch.int8, device=DEV),
-                   torch.empty(0, dtype=torch.float32, device=DEV), t(Wq[0]), t(sw[0]))
+    Y0 = engine.linear(torch.empty(0, K, dtype=torch.int8, device=DEV),
+                       torch.empty(0, dtype=torch.float32, device=DEV), t(Wq[0]), t(sw[0]))
     assert Y0.shape == (0, N)
     # branches of different M (one of them ragged, one empty)
     for Ms in ((129, 300), (0, 77)):
@@ -216,11 +244,11 @@ def test_linear_empty_and_dual_ragged(w8, engine, oracle_mod):
             sx = np.abs(wl.random_f32((M,), seed=80 + i + M, scale=0.03)).astype(np.float32)
             brs.append((t(Xq), t(sx), t(Wq[i]), t(sw[i]), t(b[i])))
             wants.append(oracle_mod.linear(Xq, sx, Wq[i], sw[i], b[i]) if M else None)
-        Ys = w8.linear_dual(brs)
+        Ys = engine.linear_dual(brs)
         for i, M in enumerate(Ms):
             if M:
                 np.testing.assert_array_equal(u16(Ys[i]), wants[i])
-                np.testing.assert_array_equal(u16(Ys[i]), u16(w8.linear(*brs[i])))
+                np.testing.assert_array_equal(u16(Ys[i]), u16(engine.linear(*brs[i])))
 
 
 def test_no_out_of_bounds_writes(w8, engine):
@@ -233,12 +261,12 @@ def test_no_out_of_bounds_writes(w8, engine):
     sw = torch.ones(N, device=DEV)
     buf = torch.full((guard + M * N + guard,), 0x7A7B, dtype=torch.int16, device=DEV)
     Y = buf[guard:guard + M * N].view(torch.bfloat16).view(M, N)
-    w8.linear(Xq, sx, Wq, sw, None, Y=Y)
+    engine.linear(Xq, sx, Wq, sw, None, Y=Y)
     torch.cuda.synchronize()
     assert torch.all(buf[:guard] == 0x7A7B) and torch.all(buf[guard + M * N:] == 0x7A7B)
     buf32 = torch.full((guard + M * N + guard,), 0x5A5A5A5A, dtype=torch.int32, device=DEV)
     acc = buf32[guard:guard + M * N].view(M, N)
-    w8.debug_gemm_i32(Xq, Wq, acc=acc)
+    engine.debug_gemm_i32(Xq, Wq, acc=acc)
     torch.cuda.synchronize()
     assert torch.all(buf32[:guard] == 0x5A5A5A5A) and torch.all(buf32[guard + M * N:] == 0x5A5A5A5A)
     assert w8.device_status() == 0

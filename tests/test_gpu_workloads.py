@@ -30,7 +30,7 @@ def w8():
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     from paper_2606_12280_gb300 import w8a8
-    w8a8.set_gemm_engine(-1)
+    w8a8.lib()
     return w8a8
 
 
