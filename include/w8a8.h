@@ -39,8 +39,9 @@
  *     W8A8_ERR_UNSUPPORTED_SHAPE, W8A8_ERR_MISALIGNED (a pointer not 16-byte
  *     aligned) leave the stream untouched.  W8A8_ERR_CUDA reports a launch
  *     failure.  The library keeps one device-side error word (see
- *     w8a8_device_status) and the fixed scratch of w8a8_act_stats_noalloc;
- *     it holds no other state (per-device kernel attributes are set once,
+ *     w8a8_device_status), the fixed scratch of w8a8_act_stats_noalloc and
+ *     the constant GELU table of w8a8_gelu_quant_act; it holds no other
+ *     state (per-device kernel attributes are set once,
  *     thread-safely), and calls on different streams or host threads do not
  *     affect one another.
  *   - Every pointer refers to memory of the CURRENT device (cudaSetDevice),
@@ -364,14 +365,15 @@ W8A8_API w8a8_status w8a8_quant_act_dual(const w8a8_act_branch *br, int K, void 
  * up-projection's bf16 output (the down-projections are the fragile layers
  * of Sec. 3, "Activation-fragility profiling and protection"; the paper does
  * not name the activation, the exact erf form is taken):
- *     g_mj = GELU(H_mj) = (H_mj / 2) * erfc(-H_mj / sqrt 2)   in fp32
+ *     g_mj = GELU(H_mj) = (H_mj / 2) * erfc(-H_mj / sqrt 2)
+ *            evaluated in binary64 and rounded once to fp32,
  *     then w8a8_quant_act's arithmetic on g (no rounding of g to bf16).
- * GELU is evaluated in fp32 with a fitted approximation, log2 erfc(|h|/sqrt 2)
- * as a degree-12 polynomial in min(|h|, 8)/4 - 1: g is within a relative
- * 2e-6 of GELU(H) for H >= -6 and 4e-6 for H >= -8 (below -8 both have
- * magnitude under |H| * 7e-16), so a code can differ from one computed with
- * the correctly rounded GELU only where x' * (127/a) lies within ~3e-4 of a
- * rounding tie (where it differs by one).
+ * g is exact as defined: H is bf16, so the pass reads g from a table that
+ * holds it for each of the 65536 bf16 bit patterns.  The library builds the
+ * table (256 KB of device memory, kept until the process exits) on each
+ * device the first time a GELU pass runs there, synchronously and outside
+ * the caller's stream: make that first call before capturing a stream into
+ * a CUDA graph (later calls are capturable).
  *   H [M,K] bf16, read.   smooth [K] fp32 or NULL.
  *   Xq [M,K] int8, x_scale [M] fp32, written.
  */
@@ -380,7 +382,8 @@ W8A8_API w8a8_status w8a8_gelu_quant_act(const uint16_t *H, const float *smooth,
 
 /*
  * Test export of the GELU that w8a8_gelu_quant_act uses: G[i] = g(H[i]) in
- * fp32 for n values (n >= 0).  H [n] bf16, read; G [n] fp32, written.
+ * fp32 for n values (n >= 0), read from the same table (built on first use
+ * as above).  H [n] bf16, read; G [n] fp32, written.
  */
 W8A8_API w8a8_status w8a8_debug_gelu(const uint16_t *H, int n, float *G, void *stream);
 

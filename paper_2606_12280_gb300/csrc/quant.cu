@@ -33,10 +33,11 @@ template <> struct Chunk<uint16_t> {        // 8 bf16 = 16 bytes
         v = __ldcs(reinterpret_cast<const uint4 *>(p));
     }
     __device__ __forceinline__ void zero() { v = make_uint4(0, 0, 0, 0); }
-    __device__ __forceinline__ float get(int e) const {
+    __device__ __forceinline__ uint32_t bits(int e) const {
         uint32_t w = (e < 2) ? v.x : (e < 4) ? v.y : (e < 6) ? v.z : v.w;
-        return bf16_bits_to_f32((e & 1) ? (w >> 16) : (w & 0xffffu));
+        return (e & 1) ? (w >> 16) : (w & 0xffffu);
     }
+    __device__ __forceinline__ float get(int e) const { return bf16_bits_to_f32(bits(e)); }
 };
 
 template <> struct Chunk<float> {           // 8 fp32 = 32 bytes
@@ -64,22 +65,6 @@ __device__ __forceinline__ float warp_max(float v) {
     return v;
 }
 
-// GELU(h) = h * Phi(h) = (h/2) erfc(-h/sqrt 2), the exact (erf) form, for
-// the FFN down-projection input.  With a = min(|h|, 8),
-//     log2 erfc(a/sqrt 2) ~= P(u),   u = a/4 - 1   (exact in fp32),
-// P of degree 12 fitted by least squares over a in [0, 8]
-// (fit_gelu_erfc.py beside this file), evaluated by Horner in fp32 with the
-// constant term lowered by 1, so that d = 2^P'(u) = erfc(a/sqrt 2)/2 =
-// Phi(-a); then GELU(h) = h d for h < 0 and h - h d for h >= 0 (one ex2, no
-// division).  Relative error of the result: below 2e-6 for h >= -6 and 4e-6
-// for h >= -8; below -8 the result has magnitude below |h| * 7e-16 like
-// GELU(h) itself.
-__device__ __forceinline__ float ex2_approx(float x) {
-    float r;
-    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
-    return r;
-}
-
 __device__ __forceinline__ uint64_t pk(float a, float b) {
     uint64_t r;
     asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(a), "f"(b));
@@ -104,73 +89,50 @@ __device__ __forceinline__ uint64_t add_pk(uint64_t a, uint64_t b) {
     return r;
 }
 
-__device__ __forceinline__ uint64_t mul_pk(uint64_t a, uint64_t b) {
-    uint64_t r;
-    asm("mul.rn.f32x2 %0, %1, %2;" : "=l"(r) : "l"(a), "l"(b));
-    return r;
-}
+}  // namespace
 
-__device__ __forceinline__ uint64_t splat(float c) { return pk(c, c); }
+// GELU(h) = h Phi(h) = (h/2) erfc(-h/sqrt 2), the exact (erf) form, for the
+// FFN down-projection input.  The fused pass only ever evaluates it at bf16
+// inputs, so it reads a table holding, for each of the 65536 bf16 bit
+// patterns, the value evaluated in binary64 and rounded once to fp32: exact
+// as defined, no approximation.  The table (256 KB) is built on each device
+// the first time a GELU pass runs there (build_gelu_table below) and then
+// only read.
+__device__ float g_gelu_table[65536];
 
-// h Phi(-|h|) from P = log2 erfc(|h|/sqrt 2) - 1 (= log2 Phi(-|h|)), then
-// GELU(h) = h - h Phi(-|h|) for h >= 0 and h Phi(-|h|) for h < 0.
-__device__ __forceinline__ float2 gelu_tail(float2 h, uint64_t p) {
-    const float2 lg = upk(p);
-    const float2 q = upk(mul_pk(pk(h.x, h.y), pk(ex2_approx(lg.x), ex2_approx(lg.y))));   // h Phi(-|h|)
-    return make_float2(h.x >= 0.0f ? h.x - q.x : q.x, h.y >= 0.0f ? h.y - q.y : q.y);
-}
+namespace {
 
-// GELU of two values with packed fp32 instructions (each packed operation
-// rounds like its scalar form), the degree-12 fit over |h| <= 8.
-__device__ __forceinline__ float2 gelu_erf2_long(float2 h) {
-    const uint64_t u = fma_pk(pk(fminf(fabsf(h.x), 8.0f), fminf(fabsf(h.y), 8.0f)), splat(0.25f),
-                              splat(-1.0f));
-    uint64_t p = splat(-0.00130923442f);
-    p = fma_pk(p, u, splat(0.00208183355f));
-    p = fma_pk(p, u, splat(0.00157369743f));
-    p = fma_pk(p, u, splat(-0.00497690868f));
-    p = fma_pk(p, u, splat(0.00688785873f));
-    p = fma_pk(p, u, splat(-0.0167602543f));
-    p = fma_pk(p, u, splat(0.039086014f));
-    p = fma_pk(p, u, splat(-0.0774176419f));
-    p = fma_pk(p, u, splat(0.146253109f));
-    p = fma_pk(p, u, splat(-0.274731398f));
-    p = fma_pk(p, u, splat(-11.0028801f));
-    p = fma_pk(p, u, splat(-24.3850517f));
-    p = fma_pk(p, u, splat(-14.9464674f));                  // C0 - 1: halves erfc
-    return gelu_tail(h, p);
-}
-
-// The degree-8 fit over |h| < 4 in v = |h|/2 - 1 (relative error of Phi
-// about 1e-6 in fp32, no worse than the long fit's there) at 8 instead of 12
-// multiply-adds.  Callers choose it for a whole warp's values at once, when
-// every one of them has |h| < 4 (most warps of Gaussian-like activations);
-// so a value's GELU may differ in the last bits with the company it keeps,
-// and a caller that evaluates a value twice uses gelu_erf (always the long
-// fit).
-__device__ __forceinline__ float2 gelu_erf2_short(float2 h) {
-    {
-        const uint64_t v = fma_pk(pk(fabsf(h.x), fabsf(h.y)), splat(0.5f), splat(-1.0f));
-        uint64_t p = splat(-0.000231636994f);
-        p = fma_pk(p, v, splat(-4.95363784e-05f));
-        p = fma_pk(p, v, splat(0.00274736318f));
-        p = fma_pk(p, v, splat(-0.0114125507f));
-        p = fma_pk(p, v, splat(0.0378777497f));
-        p = fma_pk(p, v, splat(-0.114114717f));
-        p = fma_pk(p, v, splat(-2.55564547f));
-        p = fma_pk(p, v, splat(-6.8476572f));
-        p = fma_pk(p, v, splat(-5.45798159f));               // S0 - 1: halves erfc
-        return gelu_tail(h, p);
+__global__ void gelu_table_kernel() {
+    const int i = blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < 65536) {
+        const double x = static_cast<double>(__uint_as_float(static_cast<uint32_t>(i) << 16));
+        g_gelu_table[i] = __double2float_rn(0.5 * x * erfc(-x / sqrt(2.0)));
     }
 }
 
-// One pair with the fit chosen by a vote of the active lanes (test export).
-__device__ __forceinline__ float2 gelu_erf2_vote(float2 h) {
-    if (__all_sync(__activemask(), fmaxf(fabsf(h.x), fabsf(h.y)) < 4.0f)) return gelu_erf2_short(h);
-    return gelu_erf2_long(h);
+// GELU of a bf16 bit pattern (the table holds every one).
+__device__ __forceinline__ float gelu_of_bits(uint32_t h16) { return __ldg(&g_gelu_table[h16 & 0xffffu]); }
+
+cudaError_t build_gelu_table();
+
+// The hot range of the table, |h| in [2^-10, 2^5) (bf16 patterns 0x3A80 ..
+// 0x41FF and their negatives: 15 KB), which a block copies into shared
+// memory; values outside it (rare) read the global table.
+constexpr uint32_t kGeluLo = 0x3A80u, kGeluN = 0x4200u - 0x3A80u;
+
+__device__ __forceinline__ float gelu_hot(const float *tab, uint32_t h16) {
+    h16 &= 0xffffu;
+    const uint32_t t = (h16 & 0x7fffu) - kGeluLo;          // wraps below the range
+    if (t < kGeluN) return tab[t + ((h16 & 0x8000u) ? kGeluN : 0u)];
+    return gelu_of_bits(h16);
 }
 
-__device__ __forceinline__ float gelu_erf(float h) { return gelu_erf2_long(make_float2(h, 0.0f)).x; }
+// Element e of a chunk as the pass reads it: the value, or GELU of it.
+template <bool GELU, typename C>
+__device__ __forceinline__ float input_value(const C &ch, int e) {
+    if constexpr (GELU) return gelu_of_bits(ch.bits(e));
+    else return ch.get(e);
+}
 
 // ------------------------------------------------------------- row quant
 //
@@ -300,7 +262,7 @@ row_quant_long_kernel(const InT *__restrict__ in, const float *__restrict__ lam,
             for (int e = 0; e < 8; ++e) {
                 float fe = 1.0f;
                 if (lam) { const float l = __ldg(lam + col0 + e); fe = IS_ACT ? __frcp_rn(l) : l; }
-                a = fmaxf(a, fabsf(__fmul_rn(GELU ? gelu_erf(ch.get(e)) : ch.get(e), fe)));
+                a = fmaxf(a, fabsf(__fmul_rn(input_value<GELU>(ch, e), fe)));
             }
         }
         a = warp_max(a);
@@ -321,7 +283,7 @@ row_quant_long_kernel(const InT *__restrict__ in, const float *__restrict__ lam,
                 for (int e = 0; e < 8; ++e) {
                     float fe = 1.0f;
                     if (lam) { const float l = __ldg(lam + col0 + e); fe = IS_ACT ? __frcp_rn(l) : l; }
-                    const float xs = __fmul_rn(GELU ? gelu_erf(ch.get(e)) : ch.get(e), fe);
+                    const float xs = __fmul_rn(input_value<GELU>(ch, e), fe);
                     const uint32_t b = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xs, inv))) & 0xffu;
                     if (e < 4) lo |= b << (8 * e);
                     else hi |= b << (8 * (e - 4));
@@ -459,6 +421,8 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
     const uint32_t ring = static_cast<uint32_t>(__cvta_generic_to_shared(ring_s)) +
                           static_cast<uint32_t>((warp * S * U * 32 + lane) * 16);
 
+    // GELU: the hot range of the table in shared memory (see gelu_hot)
+    __shared__ float gtab[GELU ? 2 * kGeluN : 1];
     const int gteam = blockIdx.x * kTeams + team;
     const bool second = gteam >= p.teams0;
     const ActBranch b = second ? p.br[1] : p.br[0];
@@ -480,6 +444,12 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
 #pragma unroll
     for (int k = 0; k < S - 1; ++k) issue(k);           // first rows in flight before the setup
 
+    if (GELU) {
+        for (int i = tid; i < static_cast<int>(2 * kGeluN); i += kThreads)
+            gtab[i] = __ldg(&g_gelu_table[i < static_cast<int>(kGeluN) ? kGeluLo + i
+                                                                       : 0x8000u + kGeluLo + (i - kGeluN)]);
+        __syncthreads();
+    }
     float2 r[U][4];                                         // 1/lambda of this lane's columns
 #pragma unroll
     for (int u = 0; u < U; ++u) {
@@ -516,27 +486,8 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
             const uint32_t wd[4] = {v.x, v.y, v.z, v.w};
 #pragma unroll
             for (int q = 0; q < 4; ++q)
-                xs[u][q] = make_float2(__uint_as_float(wd[q] << 16), __uint_as_float(wd[q] & 0xffff0000u));
-        }
-        if (GELU) {
-            // one fit for all of the warp's values of this row: the short
-            // one when every |h| < 4
-            float hm = 0.0f;
-#pragma unroll
-            for (int u = 0; u < U; ++u)
-#pragma unroll
-                for (int q = 0; q < 4; ++q) hm = fmaxf(hm, fmaxf(fabsf(xs[u][q].x), fabsf(xs[u][q].y)));
-            if (__all_sync(0xffffffffu, hm < 4.0f)) {
-#pragma unroll
-                for (int u = 0; u < U; ++u)
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) xs[u][q] = gelu_erf2_short(xs[u][q]);
-            } else {
-#pragma unroll
-                for (int u = 0; u < U; ++u)
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) xs[u][q] = gelu_erf2_long(xs[u][q]);
-            }
+                xs[u][q] = GELU ? make_float2(gelu_hot(gtab, wd[q]), gelu_hot(gtab, wd[q] >> 16))
+                                : make_float2(__uint_as_float(wd[q] << 16), __uint_as_float(wd[q] & 0xffff0000u));
         }
 #pragma unroll
         for (int u = 0; u < U; ++u) {
@@ -663,7 +614,7 @@ cudaError_t launch_act_quant_team(ActParams p, cudaStream_t st) {
     // (4608 rows on 608 teams for K = 4096), so a deeper ring only front-loads
     // the reads; 2 slices suit the 256-thread teams writing fp16 codes, 3
     // the int8 codes and the 16-warp teams of K > 8192
-    constexpr int S = GELU ? 4 : ((OUT16 && TW <= 8) ? 2 : 3);
+    constexpr int S = GELU ? 3 : ((OUT16 && TW <= 8) ? 2 : 3);
     constexpr int kThreads = TW > 8 ? 32 * TW : 256;
     constexpr int kTeams = kThreads / (32 * TW);
     constexpr size_t smem = (size_t)(kThreads / 32) * S * U * 32 * 16;
@@ -808,6 +759,8 @@ cudaError_t launch_quant_act(const uint16_t *X, const float *lambda, int M, int 
 cudaError_t launch_quant_act_f16codes(const uint16_t *X, const float *lambda, int M, int K,
                                      uint16_t *Xq16, float *x_scale, uint32_t *sumsq, bool gelu,
                                      cudaStream_t st) {
+    if (gelu)
+        if (cudaError_t e = build_gelu_table()) return e;
     ActParams p{};
     p.br[0] = ActBranch{X, lambda, reinterpret_cast<int8_t *>(Xq16), x_scale, M, sumsq};
     p.K = K;
@@ -843,12 +796,32 @@ cudaError_t launch_quant_act_dual(const QuantActBranch *br, int K, cudaStream_t 
 namespace {
 __global__ void gelu_values_kernel(const uint16_t *__restrict__ H, int n, float *__restrict__ G) {
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x)
-        G[i] = gelu_erf2_vote(make_float2(bf16_bits_to_f32(H[i]), 0.0f)).x;   // either fit, as the team kernel
+        G[i] = gelu_of_bits(H[i]);
+}
+
+// The GELU table of the current device, built once (synchronously, on a
+// stream of its own, so that every later launch on any stream finds it
+// complete; this first build is no stream operation of the caller's, so it
+// must not happen during a stream capture).
+cudaError_t build_gelu_table() {
+    static PerDevice<int> built;
+    int unused = 0;
+    return built.get([](int &) {
+        cudaStream_t s;
+        cudaError_t e = cudaStreamCreateWithFlags(&s, cudaStreamNonBlocking);
+        if (e != cudaSuccess) return e;
+        gelu_table_kernel<<<65536 / 256, 256, 0, s>>>();
+        e = cudaGetLastError();
+        cudaError_t e2 = cudaStreamSynchronize(s);
+        cudaStreamDestroy(s);
+        return e != cudaSuccess ? e : e2;
+    }, &unused);
 }
 }  // namespace
 
 cudaError_t launch_debug_gelu(const uint16_t *H, int n, float *G, cudaStream_t st) {
     if (n == 0) return cudaSuccess;
+    if (cudaError_t e = build_gelu_table()) return e;
     int grid = (n + 255) / 256;
     if (grid > num_sms() * 8) grid = num_sms() * 8;
     gelu_values_kernel<<<grid, 256, 0, st>>>(H, n, G);
@@ -857,6 +830,7 @@ cudaError_t launch_debug_gelu(const uint16_t *H, int n, float *G, cudaStream_t s
 
 cudaError_t launch_gelu_quant_act(const uint16_t *H, const float *lambda, int M, int K, int8_t *Xq,
                                   float *x_scale, cudaStream_t st) {
+    if (cudaError_t e = build_gelu_table()) return e;
     if (K <= 16384) {
         ActParams p{};
         p.br[0] = ActBranch{H, lambda, Xq, x_scale, M};
