@@ -424,9 +424,10 @@ W8A8_API w8a8_status w8a8_quant_act_per_tensor(const uint16_t *X, const float *s
  * [K] before the first call and keeps the total token count.  A shift near
  * each channel's mean (for example from a first batch) keeps the power sums
  * well conditioned.  Each thread sums at most 64 of its rows in fp32, adds at
- * most 64 such group sums in fp32, and only those into fp64: every returned
- * sum is within (2 * 64 + 4) * 2^-24 of
- * sum_t |X_tj - c_j|^p of its exact value.  T == 0 is a no-op.
+ * most 64 such group sums in fp32, a block adds its 8 warps' sums in fp32,
+ * and only those block sums are added into fp64: every returned sum is within
+ * (2 * 64 + 12) * 2^-24 of sum_t |X_tj - c_j|^p of its exact value.  T == 0
+ * is a no-op.
  *   X [T,K] bf16, read.   shift [K] fp32 or NULL, read.
  *   sums [4,K] fp64, absmax [K] fp32: read and written (accumulators).
  */

@@ -15,11 +15,12 @@
 //                          (the naive per-tensor arm of the activation-quant
 //                          ablation, Sec. 5, "What drives INT8 recovery")
 //
-// Layout of the streaming passes: a block is WR warps; lane l of every warp
-// owns the same few columns (fixed per thread, so per-column factors stay in
-// registers) and warp w takes rows w, w + WR, ... of the block's row slab, so
-// a warp reads one contiguous run of the row per instruction and consecutive
-// warps read consecutive rows.
+// Layout of the streaming passes: a block is 8 warps; lane l of every warp
+// owns the same 8 columns (fixed per thread, so per-column factors and sums
+// stay in registers) and warp w takes rows w, w + 8, ... of the block's row
+// slab, so a warp reads 512 contiguous bytes of a row per copy and
+// consecutive warps read consecutive rows.  Rows reach the threads through
+// per-thread cp.async rings in shared memory; the grids fill the GPU once.
 #include <cstdint>
 #include <cuda_runtime.h>
 
@@ -61,147 +62,233 @@ __device__ __forceinline__ float2 fma2(float2 a, float2 b, float2 c) {
     return r;
 }
 
+// ------------------------------------------------- streaming through rings
+//
+// The passes below stream rows through a per-thread ring of 16-byte slots in
+// shared memory filled with cp.async: a thread copies its own chunks and reads
+// back only those, so no barrier is needed, and the bytes in flight take no
+// registers.  One commit group per row: waiting until at most S - 1 groups
+// are pending makes the oldest row of an S-deep ring visible.
+__device__ __forceinline__ void ring_cp16(uint32_t dst, const void *src, bool valid) {
+    asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;" ::"r"(dst), "l"(src),
+                 "r"(valid ? 16 : 0) : "memory");
+}
+
+__device__ __forceinline__ void ring_commit() { asm volatile("cp.async.commit_group;" ::: "memory"); }
+
+template <int S>
+__device__ __forceinline__ void ring_wait() {
+    asm volatile("cp.async.wait_group %0;" ::"n"(S - 1) : "memory");
+}
+
+__device__ __forceinline__ void ring_drain() { asm volatile("cp.async.wait_group 0;" ::: "memory"); }
+
+__device__ __forceinline__ uint4 ring_lds(uint32_t a) {
+    uint4 v;
+    asm volatile("ld.shared.v4.u32 {%0, %1, %2, %3}, [%4];"
+                 : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(a));
+    return v;
+}
+
+// max(|a|, |b|) of each bf16 half (max.xorsign.abs keeps the larger
+// magnitude; the sign bit of the result is meaningless and is dropped by the
+// caller).  Exact.
+__device__ __forceinline__ uint32_t absmax_bf16x2(uint32_t m, uint32_t x) {
+    uint32_t r;
+    asm("max.xorsign.abs.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(m), "r"(x));
+    return r;
+}
+
+// Magnitudes of the two halves of a packed bf16 max-abs, as floats.
+__device__ __forceinline__ float absmax_lo(uint32_t m) { return __uint_as_float((m << 16) & 0x7fffffffu); }
+__device__ __forceinline__ float absmax_hi(uint32_t m) { return __uint_as_float(m & 0x7fff0000u); }
+
+// Programmatic dependent launch: a kernel launched with the
+// programmatic-serialization attribute may start while the previous kernel of
+// the stream still runs; grid_dependency_wait() returns once that kernel has
+// completed and its writes are visible (at once when launched without the
+// attribute).  allow_dependents() lets the next such kernel start.
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void allow_dependents() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 // ------------------------------------------------------------ statistics
 //
-// Lane l owns 4 consecutive channels of the block's 128 (one 8-byte load per
-// row) and the 8 warps of a block split the block's row slab.  Each thread
-// sums (x - c)^p in fp32 over groups of at most kGroup of its rows, adds the
-// group sums into fp32 level-2 sums (at most kGroup groups), and only those
-// into fp64 (at the end of the slab, or every kGroup groups); the block then
-// combines its warps in fp64 through shared memory and adds into the global
-// fp64 sums with atomics.  Rounding: every returned sum is within
-// (2 kGroup + 4) * 2^-24 of sum |x - c|^p of its exact value.
+// Lane l owns 8 consecutive channels of the block's 256 (one 16-byte chunk per
+// row) and the 8 warps of a block split the block's row slab (warp w takes
+// rows w, w + 8, ...).  Each thread streams its rows through a kStatsRing-deep
+// ring; the row loop is unrolled over the ring, so every slot address is a
+// constant, and only a warp's last (< 2 kStatsRing) rows test whether a row or
+// a refill exists.  Max-abs is kept as packed bf16 (one instruction per two
+// channels and row).
+//
+// Precision of the power sums: every sum is kept in fp32 on the SM.  A thread
+// sums (x - c)^p over groups of at most kGroup of its rows (level 1), adds the
+// group sums into level-2 sums (at most kGroup groups: the launch keeps a
+// thread's rows at or below kGroup^2), the block adds its 8 warps' sums, and
+// only the block's total is widened to fp64 and added into the caller's fp64
+// accumulators with atomics.  The error of every returned sum is at most
+// (63 + 63 + 7 + 4) * 2^-24 < (2 kGroup + 12) * 2^-24 of sum |x - c|^p (the
+// three fp32 summation levels, and the rounding of the terms (x - c)^p);
+// widening fp32 to fp64 is exact.  FP64 arithmetic runs at a small fraction
+// of the fp32 rate on this part, so none happens per element.
 constexpr int kStatsWarps = 8;
+constexpr int kStatsThreads = 32 * kStatsWarps;
 constexpr int kGroup = 64;
-constexpr int kUnroll = 16;
-static_assert(kGroup % kUnroll == 0, "whole unrolled batches per group");
+constexpr int kStatsRing = 6;                             // rows in flight per thread
+constexpr int kL2Pitch = 36;     // [q][lane] pitch: conflict-free both by lane and by channel
+constexpr int kMaxRowsPerThread = kGroup * kGroup;
+static_assert(kGroup >= 4 * kStatsRing, "a level-1 group absorbs the drain");
 
-struct Acc4 {                   // one moment for the thread's 4 channels
-    float2 a, b;
+struct StatsRed {
+    float lvl[kStatsWarps][32][kL2Pitch];  // per-thread sums [q = 8 p + e][lane]
+    float mx[kStatsWarps][32][8];           // per-thread maxima [lane][e]
+};
+constexpr int kStatsRingBytes = kStatsRing * kStatsThreads * 16;
+constexpr int kStatsSmem =
+    kStatsRingBytes > (int)sizeof(StatsRed) ? kStatsRingBytes : (int)sizeof(StatsRed);
+
+struct StatsAcc {
+    float2 g[4][4];         // level 1 [p][channel pair]
+    float2 l2[4][4];        // level 2
+    uint32_t mx[4];         // packed bf16 max-abs
+    float2 c[4];            // -shift
+    int in_group;
+
+    __device__ __forceinline__ void row(const uint4 v) {
+        const uint32_t wd[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+            mx[h] = absmax_bf16x2(mx[h], wd[h]);
+            const float2 x = make_float2(__uint_as_float(wd[h] << 16), __uint_as_float(wd[h] & 0xffff0000u));
+            const float2 d = add2(x, c[h]);
+            const float2 d2 = mul2(d, d);
+            g[0][h] = add2(g[0][h], d);
+            g[1][h] = add2(g[1][h], d2);
+            g[2][h] = fma2(d2, d, g[2][h]);
+            g[3][h] = fma2(d2, d2, g[3][h]);
+        }
+    }
+    __device__ __forceinline__ void fold() {
+#pragma unroll
+        for (int p = 0; p < 4; ++p)
+#pragma unroll
+            for (int h = 0; h < 4; ++h) {
+                l2[p][h] = add2(l2[p][h], g[p][h]);
+                g[p][h] = make_float2(0.f, 0.f);
+            }
+        in_group = 0;
+    }
 };
 
-__global__ void __launch_bounds__(32 * kStatsWarps, 2)
-stats_update_kernel(const uint2 *__restrict__ X4, int T, int K, const float *__restrict__ shift,
+__global__ void __launch_bounds__(kStatsThreads, 2)
+stats_update_kernel(const uint4 *__restrict__ X8, int T, int K, const float *__restrict__ shift,
                     int rows_per_slab, double *__restrict__ sums, float *__restrict__ absmax) {
-    __shared__ double red_s[kStatsWarps][16][32];     // per-thread fp64 sums [p][e]
-    __shared__ float lvl2[kStatsWarps][16][32];       // per-thread level-2 fp32 sums,
-                                                      // then the maxima [e] (48 KB total)
+    extern __shared__ __align__(16) unsigned char stats_smem[];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    const int quad = blockIdx.x * 32 + lane;            // 4-channel group index
-    const int kq = K / 4;
-    const bool active = quad < kq;
+    const int ko = K / 8;                                 // 8-channel groups per row
+    const int oct = blockIdx.x * 32 + lane;
+    const bool active = oct < ko;
     const int r0 = blockIdx.y * rows_per_slab;
     const int r1 = min(T, r0 + rows_per_slab);
-    constexpr int kStep = kStatsWarps * kUnroll;
+    // rows of this warp: r0 + w + 8 i, i < n
+    const int n = r1 - r0 > w ? (r1 - r0 - w + kStatsWarps - 1) / kStatsWarps : 0;
+    const size_t step = (size_t)kStatsWarps * ko;
+    const uint4 *nxt = X8 + (size_t)(r0 + w) * ko + (active ? oct : 0);   // next row to fetch
+    const uint32_t ring = static_cast<uint32_t>(__cvta_generic_to_shared(stats_smem)) + threadIdx.x * 16;
+    constexpr uint32_t kSlot = kStatsThreads * 16;
 
-    float2 c0 = make_float2(0.0f, 0.0f), c1 = c0;     // -shift
-    if (active && shift) {
-        const float4 sh = __ldg(reinterpret_cast<const float4 *>(shift) + quad);
-        c0 = make_float2(-sh.x, -sh.y);
-        c1 = make_float2(-sh.z, -sh.w);
-    }
-    const float2 z = make_float2(0.f, 0.f);
-    Acc4 g[4] = {{z, z}, {z, z}, {z, z}, {z, z}};      // level 1, p = 1..4
 #pragma unroll
-    for (int i = 0; i < 16; ++i) {
-        red_s[w][i][lane] = 0.0;
-        lvl2[w][i][lane] = 0.0f;
+    for (int u = 0; u < kStatsRing; ++u) {
+        if (u < n) ring_cp16(ring + u * kSlot, nxt, active);
+        nxt += step;
+        ring_commit();
     }
-    float mx[4] = {0.f, 0.f, 0.f, 0.f};
-    int rows_in_group = 0, groups = 0;
 
-    // level 1 -> level 2 (every kGroup rows), level 2 -> fp64 (every kGroup
-    // groups); both live in this thread's slots of shared memory
-    auto fold_group = [&]() {
+    StatsAcc acc;
+#pragma unroll
+    for (int h = 0; h < 4; ++h) {
+        acc.c[h] = make_float2(0.f, 0.f);
+        acc.mx[h] = 0u;
+#pragma unroll
+        for (int p = 0; p < 4; ++p) acc.g[p][h] = acc.l2[p][h] = make_float2(0.f, 0.f);
+    }
+    acc.in_group = 0;
+    if (active && shift) {
+        const float4 s0 = __ldg(reinterpret_cast<const float4 *>(shift) + 2 * oct);
+        const float4 s1 = __ldg(reinterpret_cast<const float4 *>(shift) + 2 * oct + 1);
+        acc.c[0] = make_float2(-s0.x, -s0.y);
+        acc.c[1] = make_float2(-s0.z, -s0.w);
+        acc.c[2] = make_float2(-s1.x, -s1.y);
+        acc.c[3] = make_float2(-s1.z, -s1.w);
+    }
+
+    // steady state: every row's slot is refilled with the row kStatsRing on
+    int i = 0;
+    for (; i + 2 * kStatsRing <= n; i += kStatsRing) {
+#pragma unroll
+        for (int u = 0; u < kStatsRing; ++u) {
+            ring_wait<kStatsRing>();
+            acc.row(ring_lds(ring + u * kSlot));
+            ring_cp16(ring + u * kSlot, nxt, active);
+            nxt += step;
+            ring_commit();
+        }
+        acc.in_group += kStatsRing;
+        if (acc.in_group > kGroup - 2 * kStatsRing) acc.fold();
+    }
+    // drain: the last n - i < 2 kStatsRing rows (in_group <= kGroup -
+    // 2 kStatsRing here, so they stay within one level-1 group)
+#pragma unroll
+    for (int u = 0; u < kStatsRing; ++u) {
+        if (i + u < n) {
+            ring_wait<kStatsRing>();
+            acc.row(ring_lds(ring + u * kSlot));
+            if (i + u + kStatsRing < n) ring_cp16(ring + u * kSlot, nxt, active);
+            nxt += step;
+            ring_commit();
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < kStatsRing; ++u) {
+        if (i + kStatsRing + u < n) {
+            ring_wait<kStatsRing>();
+            acc.row(ring_lds(ring + u * kSlot));
+            ring_commit();
+        }
+    }
+    ring_drain();
+    __syncthreads();                                      // the ring becomes the reduction area
+    StatsRed &sm = *reinterpret_cast<StatsRed *>(stats_smem);
+#pragma unroll
+    for (int p = 0; p < 4; ++p)
+#pragma unroll
+        for (int h = 0; h < 4; ++h) {
+            const float2 s = add2(acc.l2[p][h], acc.g[p][h]);
+            sm.lvl[w][8 * p + 2 * h][lane] = s.x;
+            sm.lvl[w][8 * p + 2 * h + 1][lane] = s.y;
+        }
+    reinterpret_cast<float4 *>(&sm.mx[w][lane][0])[0] =
+        make_float4(absmax_lo(acc.mx[0]), absmax_hi(acc.mx[0]), absmax_lo(acc.mx[1]), absmax_hi(acc.mx[1]));
+    reinterpret_cast<float4 *>(&sm.mx[w][lane][0])[1] =
+        make_float4(absmax_lo(acc.mx[2]), absmax_hi(acc.mx[2]), absmax_lo(acc.mx[3]), absmax_hi(acc.mx[3]));
+    __syncthreads();
+
+    // block totals: thread t combines channel t of the block (source lane t/8,
+    // entry e = t%8) over the 8 warps, for the 4 moments, and the maxima
+    const int t = threadIdx.x, sl = t >> 3, e = t & 7;
+    if (blockIdx.x * 256 + t < K && r0 < r1) {
+        float a = 0.f;
+#pragma unroll
+        for (int ww = 0; ww < kStatsWarps; ++ww) a = fmaxf(a, sm.mx[ww][sl][e]);
+        const size_t j = (size_t)blockIdx.x * 256 + t;
+        // non-negative floats order like their bit patterns
+        atomicMax(reinterpret_cast<unsigned int *>(absmax) + j, __float_as_uint(a));
 #pragma unroll
         for (int p = 0; p < 4; ++p) {
-            lvl2[w][4 * p + 0][lane] += g[p].a.x;
-            lvl2[w][4 * p + 1][lane] += g[p].a.y;
-            lvl2[w][4 * p + 2][lane] += g[p].b.x;
-            lvl2[w][4 * p + 3][lane] += g[p].b.y;
-            g[p].a = z;
-            g[p].b = z;
-        }
-        rows_in_group = 0;
-        ++groups;
-    };
-    auto fold_level2 = [&]() {
+            float s = 0.f;
 #pragma unroll
-        for (int i = 0; i < 16; ++i) {
-            red_s[w][i][lane] += lvl2[w][i][lane];
-            lvl2[w][i][lane] = 0.0f;
-        }
-        groups = 0;
-    };
-    auto load_batch = [&](int rb, uint2 (&v)[kUnroll]) {
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-            const int r = rb + u * kStatsWarps;
-            v[u] = (active && r < r1) ? __ldcs(X4 + (size_t)r * kq + quad) : make_uint2(0u, 0u);
-        }
-    };
-
-    // two batches of kUnroll rows in flight: the next one loads while this
-    // one is summed
-    uint2 v[kUnroll];
-    load_batch(r0 + w, v);
-    for (int rb = r0 + w; rb < r1; rb += kStep) {
-        uint2 vn[kUnroll];
-        load_batch(rb + kStep, vn);
-        // rows of this batch inside the slab
-        const int valid = min(kUnroll, (r1 - rb + kStatsWarps - 1) / kStatsWarps);
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) {
-            if (u < valid) {
-                const float2 xa = make_float2(__uint_as_float(v[u].x << 16), __uint_as_float(v[u].x & 0xffff0000u));
-                const float2 xb = make_float2(__uint_as_float(v[u].y << 16), __uint_as_float(v[u].y & 0xffff0000u));
-                mx[0] = fmaxf(mx[0], fabsf(xa.x));
-                mx[1] = fmaxf(mx[1], fabsf(xa.y));
-                mx[2] = fmaxf(mx[2], fabsf(xb.x));
-                mx[3] = fmaxf(mx[3], fabsf(xb.y));
-                const float2 da = add2(xa, c0), db = add2(xb, c1);
-                const float2 da2 = mul2(da, da), db2 = mul2(db, db);
-                g[0].a = add2(g[0].a, da);
-                g[0].b = add2(g[0].b, db);
-                g[1].a = add2(g[1].a, da2);
-                g[1].b = add2(g[1].b, db2);
-                g[2].a = fma2(da2, da, g[2].a);
-                g[2].b = fma2(db2, db, g[2].b);
-                g[3].a = fma2(da2, da2, g[3].a);
-                g[3].b = fma2(db2, db2, g[3].b);
-            }
-        }
-#pragma unroll
-        for (int u = 0; u < kUnroll; ++u) v[u] = vn[u];
-        rows_in_group += kUnroll;
-        if (rows_in_group >= kGroup) {
-            fold_group();
-            if (groups >= kGroup) fold_level2();
-        }
-    }
-    fold_group();
-    fold_level2();
-#pragma unroll
-    for (int e = 0; e < 4; ++e) lvl2[w][e][lane] = mx[e];   // own slots: no other thread reads them yet
-    __syncthreads();
-    // warp p (p < 4) reduces moment p, warp 4 the maxima: 4 channels per lane
-    if (active && r0 < r1 && w < 5) {
-        if (w < 4) {
-            double tot[4] = {0, 0, 0, 0};
-            for (int ww = 0; ww < kStatsWarps; ++ww)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) tot[e] += red_s[ww][4 * w + e][lane];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) atomicAdd(sums + (size_t)w * K + 4 * quad + e, tot[e]);
-        } else {
-            float a[4] = {0.f, 0.f, 0.f, 0.f};
-            for (int ww = 0; ww < kStatsWarps; ++ww)
-#pragma unroll
-                for (int e = 0; e < 4; ++e) a[e] = fmaxf(a[e], lvl2[ww][e][lane]);
-            // non-negative floats order like their bit patterns
-#pragma unroll
-            for (int e = 0; e < 4; ++e)
-                atomicMax(reinterpret_cast<unsigned int *>(absmax) + 4 * quad + e, __float_as_uint(a[e]));
+            for (int ww = 0; ww < kStatsWarps; ++ww) s += sm.lvl[ww][8 * p + e][sl];
+            atomicAdd(sums + (size_t)p * K + j, (double)s);
         }
     }
 }
@@ -299,9 +386,16 @@ stats_finalize_kernel(const double *__restrict__ sums, const float *__restrict__
 
 // ------------------------------------------------- per-tensor quantization
 //
-// Lane l owns 8 consecutive columns of the block's 256 (16-byte loads, 1/lambda
-// of its columns in registers).
+// Lane l owns 8 consecutive columns of the block's 256 (one 16-byte chunk per
+// row) and warp w takes rows w, w + 8, ... of the block's slab; rows stream
+// through a kPtRing-deep ring per thread.  The three launches (zero the
+// maximum, pass 1, pass 2) use programmatic dependent launch: pass 1 streams
+// X while the zeroing kernel finishes and waits only before its atomic; pass 2
+// starts its first copies and 1/lambda while pass 1 finishes and waits before
+// it reads the maximum.  X itself was complete before the first of them ran.
 constexpr int kQWarps = 8;
+constexpr int kPtRing = 8;
+constexpr int kPtSmem = kPtRing * 32 * kQWarps * 16;
 
 __device__ __forceinline__ float warp_max(float v) {
 #pragma unroll
@@ -314,34 +408,98 @@ __device__ __forceinline__ void load_recip(const float *lam, int col0, bool acti
     for (int e = 0; e < 8; ++e) r[e] = (lam != nullptr && active) ? __frcp_rn(__ldg(lam + col0 + e)) : 1.0f;
 }
 
+// Runs `one(slot address)` for each of a warp's n rows in order, streaming
+// them through the thread's ring (rows step `step` chunks apart, the first at
+// `nxt`; the ring's first kPtRing copies are already issued).
+template <typename F>
+__device__ __forceinline__ void pt_stream(int n, const uint4 *nxt, size_t step, uint32_t ring,
+                                          bool active, F &&one) {
+    constexpr uint32_t kSlot = 32 * kQWarps * 16;
+    nxt += kPtRing * step;
+    int i = 0;
+    for (; i + 2 * kPtRing <= n; i += kPtRing) {
+#pragma unroll
+        for (int u = 0; u < kPtRing; ++u) {
+            ring_wait<kPtRing>();
+            one(ring + u * kSlot);
+            ring_cp16(ring + u * kSlot, nxt, active);
+            nxt += step;
+            ring_commit();
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < kPtRing; ++u) {
+        if (i + u < n) {
+            ring_wait<kPtRing>();
+            one(ring + u * kSlot);
+            if (i + u + kPtRing < n) ring_cp16(ring + u * kSlot, nxt, active);
+            nxt += step;
+            ring_commit();
+        }
+    }
+#pragma unroll
+    for (int u = 0; u < kPtRing; ++u) {
+        if (i + kPtRing + u < n) {
+            ring_wait<kPtRing>();
+            one(ring + u * kSlot);
+            ring_commit();
+        }
+    }
+    ring_drain();
+}
+
+__device__ __forceinline__ void pt_prologue(int n, const uint4 *nxt, size_t step, uint32_t ring, bool active) {
+    constexpr uint32_t kSlot = 32 * kQWarps * 16;
+#pragma unroll
+    for (int u = 0; u < kPtRing; ++u) {
+        if (u < n) ring_cp16(ring + u * kSlot, nxt, active);
+        nxt += step;
+        ring_commit();
+    }
+}
+
+__global__ void zero_max_kernel(float *amax) {
+    allow_dependents();
+    *amax = 0.0f;
+}
+
+// Pass 1: max over the whole tensor of |x_mj / lambda_j| = |x_mj * r_j| with
+// r_j = rn(1 / lambda_j).  Rounding is monotone, so for each column
+// max_m fl(|x_mj| * r_j) = fl(r_j * max_m |x_mj|): a lane keeps the packed
+// bf16 max-abs of its 8 columns over its rows and multiplies by r_j once.
 __global__ void __launch_bounds__(32 * kQWarps)
 tensor_absmax_kernel(const uint16_t *__restrict__ X, const float *__restrict__ lam, int M, int K,
                      int rows_per_slab, float *__restrict__ amax) {
+    extern __shared__ __align__(16) unsigned char pt_smem[];
     __shared__ float red[kQWarps];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    const int col0 = (blockIdx.x * 32 + lane) * 8;
-    const bool active = col0 < K;
-    float r[8];
-    load_recip(lam, col0, active, r);
+    const int ko = K / 8;
+    const int oct = blockIdx.x * 32 + lane;
+    const bool active = oct < ko;
     const int r0 = blockIdx.y * rows_per_slab;
     const int r1 = min(M, r0 + rows_per_slab);
+    const int n = r1 - r0 > w ? (r1 - r0 - w + kQWarps - 1) / kQWarps : 0;
+    const size_t step = (size_t)kQWarps * ko;
+    const uint4 *first = reinterpret_cast<const uint4 *>(X) + (size_t)(r0 + w) * ko + (active ? oct : 0);
+    const uint32_t ring = static_cast<uint32_t>(__cvta_generic_to_shared(pt_smem)) + threadIdx.x * 16;
+    pt_prologue(n, first, step, ring, active);
+    allow_dependents();
+    uint32_t m[4] = {0u, 0u, 0u, 0u};
+    pt_stream(n, first, step, ring, active, [&](uint32_t slot) {
+        const uint4 v = ring_lds(slot);
+        m[0] = absmax_bf16x2(m[0], v.x);
+        m[1] = absmax_bf16x2(m[1], v.y);
+        m[2] = absmax_bf16x2(m[2], v.z);
+        m[3] = absmax_bf16x2(m[3], v.w);
+    });
     float a = 0.0f;
-    for (int rb = r0 + w; rb < r1; rb += kQWarps * 4) {
-        uint4 v[4];
+    if (active) {
+        float r[8];
+        load_recip(lam, oct * 8, true, r);
 #pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int row = rb + u * kQWarps;
-            v[u] = (active && row < r1) ? __ldcs(reinterpret_cast<const uint4 *>(X + (size_t)row * K + col0))
-                                        : make_uint4(0, 0, 0, 0);
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                a = fmaxf(a, fabsf(__fmul_rn(__uint_as_float(wd[e] << 16), r[2 * e])));
-                a = fmaxf(a, fabsf(__fmul_rn(__uint_as_float(wd[e] & 0xffff0000u), r[2 * e + 1])));
-            }
+        for (int h = 0; h < 4; ++h) {
+            a = fmaxf(a, __fmul_rn(absmax_lo(m[h]), r[2 * h]));
+            a = fmaxf(a, __fmul_rn(absmax_hi(m[h]), r[2 * h + 1]));
         }
     }
     a = warp_max(a);
@@ -349,7 +507,9 @@ tensor_absmax_kernel(const uint16_t *__restrict__ X, const float *__restrict__ l
     __syncthreads();
     if (threadIdx.x == 0) {
         float t = 0.0f;
-        for (int i = 0; i < kQWarps; ++i) t = fmaxf(t, red[i]);
+        for (int k = 0; k < kQWarps; ++k) t = fmaxf(t, red[k]);
+        grid_dependency_wait();                  // the zeroing kernel has completed
+        // non-negative floats order like their bit patterns
         atomicMax(reinterpret_cast<unsigned int *>(amax), __float_as_uint(t));
     }
 }
@@ -362,77 +522,103 @@ __device__ __forceinline__ uint32_t pack4_low_bytes(float a, float b, float c, f
     return __byte_perm(ab, cd, 0x5410);
 }
 
+// The 8 codes of one lane's chunk: q = rne(fl(x * r) * inv), clamped.
+template <bool FAST>
+__device__ __forceinline__ uint2 quant8(const uint4 v, const float (&r)[8], float inv) {
+    const uint32_t wd[4] = {v.x, v.y, v.z, v.w};
+    float xs[8];
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+        xs[2 * e] = __fmul_rn(__uint_as_float(wd[e] << 16), r[2 * e]);
+        xs[2 * e + 1] = __fmul_rn(__uint_as_float(wd[e] & 0xffff0000u), r[2 * e + 1]);
+    }
+    uint32_t word[2] = {0u, 0u};
+    if (FAST) {
+#pragma unroll
+        for (int h = 0; h < 2; ++h)
+            word[h] = pack4_low_bytes(__fadd_rn(__fmul_rn(xs[4 * h], inv), kRoundMagic),
+                                      __fadd_rn(__fmul_rn(xs[4 * h + 1], inv), kRoundMagic),
+                                      __fadd_rn(__fmul_rn(xs[4 * h + 2], inv), kRoundMagic),
+                                      __fadd_rn(__fmul_rn(xs[4 * h + 3], inv), kRoundMagic));
+    } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const uint32_t b = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xs[e], inv))) & 0xffu;
+            word[e >> 2] |= b << (8 * (e & 3));
+        }
+    }
+    return make_uint2(word[0], word[1]);
+}
+
+template <bool FAST>
+__device__ __forceinline__ void quant_rows(int n, const uint4 *first, size_t step, uint32_t ring,
+                                           bool active, const float (&r)[8], float inv, float scale,
+                                           bool zero, uint2 *dst, size_t dstep, float *xs_out,
+                                           bool write_scale) {
+    pt_stream(n, first, step, ring, active, [&](uint32_t slot) {
+        const uint4 v = ring_lds(slot);
+        if (write_scale) *xs_out = scale;
+        if (active) *dst = zero ? make_uint2(0u, 0u) : quant8<FAST>(v, r, inv);
+        dst += dstep;
+        xs_out += kQWarps;
+    });
+}
+
+// Pass 2: INT8 codes of x_mj / lambda_j with the one scale a / 127 (each lane
+// writes its 8 codes of a row as one 8-byte store; block column 0 writes the
+// row scales).
 __global__ void __launch_bounds__(32 * kQWarps)
 tensor_quant_kernel(const uint16_t *__restrict__ X, const float *__restrict__ lam, int M, int K,
                     int rows_per_slab, const float *__restrict__ amax, int8_t *__restrict__ Xq,
                     float *__restrict__ x_scale) {
+    extern __shared__ __align__(16) unsigned char pt_smem[];
     const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    const int col0 = (blockIdx.x * 32 + lane) * 8;
-    const bool active = col0 < K;
+    const int ko = K / 8;
+    const int oct = blockIdx.x * 32 + lane;
+    const bool active = oct < ko;
+    const int r0 = blockIdx.y * rows_per_slab;
+    const int r1 = min(M, r0 + rows_per_slab);
+    const int n = r1 - r0 > w ? (r1 - r0 - w + kQWarps - 1) / kQWarps : 0;
+    const size_t step = (size_t)kQWarps * ko;
+    const uint4 *first = reinterpret_cast<const uint4 *>(X) + (size_t)(r0 + w) * ko + (active ? oct : 0);
+    const uint32_t ring = static_cast<uint32_t>(__cvta_generic_to_shared(pt_smem)) + threadIdx.x * 16;
+    pt_prologue(n, first, step, ring, active);
     float r[8];
-    load_recip(lam, col0, active, r);
-    const float a = *amax;                       // written by the previous kernel
+    load_recip(lam, oct * 8, active, r);
+    grid_dependency_wait();                      // pass 1 has completed: the maximum is final
+    const float a = *amax;
     const bool zero = (a == 0.0f);
     const float inv = zero ? 0.0f : __fdiv_rn(127.0f, a);
     const float scale = zero ? 0.0f : __fdiv_rn(a, 127.0f);
     // a and 127/a finite: |x' * inv| <= 127 (1 + 2^-23), no clamp needed
     const bool fast = (a <= 3.402823466e38f) && (inv <= 3.402823466e38f);
-    const int r0 = blockIdx.y * rows_per_slab;
-    const int r1 = min(M, r0 + rows_per_slab);
-    for (int rb = r0 + w; rb < r1; rb += kQWarps * 4) {
-        uint4 v[4];
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int row = rb + u * kQWarps;
-            v[u] = (active && row < r1) ? __ldcs(reinterpret_cast<const uint4 *>(X + (size_t)row * K + col0))
-                                        : make_uint4(0, 0, 0, 0);
-        }
-#pragma unroll
-        for (int u = 0; u < 4; ++u) {
-            const int row = rb + u * kQWarps;
-            if (row >= r1) continue;
-            if (blockIdx.x == 0 && lane == 0) x_scale[row] = scale;
-            if (!active) continue;
-            const uint32_t wd[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-            float xs[8];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                xs[2 * e] = __fmul_rn(__uint_as_float(wd[e] << 16), r[2 * e]);
-                xs[2 * e + 1] = __fmul_rn(__uint_as_float(wd[e] & 0xffff0000u), r[2 * e + 1]);
-            }
-            uint32_t word[2] = {0u, 0u};
-            if (zero) {
-            } else if (fast) {
-#pragma unroll
-                for (int h = 0; h < 2; ++h)
-                    word[h] = pack4_low_bytes(__fadd_rn(__fmul_rn(xs[4 * h], inv), kRoundMagic),
-                                              __fadd_rn(__fmul_rn(xs[4 * h + 1], inv), kRoundMagic),
-                                              __fadd_rn(__fmul_rn(xs[4 * h + 2], inv), kRoundMagic),
-                                              __fadd_rn(__fmul_rn(xs[4 * h + 3], inv), kRoundMagic));
-            } else {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const uint32_t b = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xs[e], inv))) & 0xffu;
-                    word[e >> 2] |= b << (8 * (e & 3));
-                }
-            }
-            *reinterpret_cast<uint2 *>(Xq + (size_t)row * K + col0) = make_uint2(word[0], word[1]);
-        }
-    }
+    uint2 *dst = reinterpret_cast<uint2 *>(Xq + (size_t)(r0 + w) * K) + (active ? oct : 0);
+    const size_t dstep = (size_t)kQWarps * ko;   // 8-byte units between a warp's rows
+    float *xs_out = x_scale + r0 + w;
+    const bool write_scale = blockIdx.x == 0 && lane == 0;
+    if (fast)
+        quant_rows<true>(n, first, step, ring, active, r, inv, scale, zero, dst, dstep, xs_out, write_scale);
+    else
+        quant_rows<false>(n, first, step, ring, active, r, inv, scale, zero, dst, dstep, xs_out, write_scale);
 }
 
-// Resident blocks per SM of `kern` (no dynamic shared memory), looked up once
-// per device.
+// Zeroes n 4-byte words (the one-shot statistics' accumulators).
+__global__ void zero_words_kernel(uint32_t *p, size_t n) {
+    for (size_t i = (size_t)blockIdx.x * blockDim.x + threadIdx.x; i < n; i += (size_t)gridDim.x * blockDim.x)
+        p[i] = 0u;
+}
+
+// Sets the dynamic shared memory of `kern` and looks up its resident blocks
+// per SM with that much, once per device.
 template <typename Kern>
-int blocks_per_sm(PerDevice<int> &cache, Kern kern, int threads) {
-    int v = 1;
-    if (cache.get([&](int &n) {
-            cudaError_t e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, threads, 0);
-            if (n < 1) n = 1;
-            return e;
-        }, &v) != cudaSuccess)
-        return 1;
-    return v;
+cudaError_t kernel_setup(PerDevice<int> &cache, Kern kern, int threads, int smem, int *per_sm) {
+    return cache.get([&](int &n) {
+        cudaError_t e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+        if (e != cudaSuccess) return e;
+        e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&n, kern, threads, smem);
+        if (n < 1) n = 1;
+        return e;
+    }, per_sm);
 }
 
 // Row slabs so that a (gx x gy) grid fills the GPU once: gy = the resident
@@ -444,9 +630,27 @@ int slabs_for(int per_sm, int rows, int gx) {
     return gy;
 }
 
-// One-shot statistics without caller accumulators: a file-scope scratch of
-// power sums (4 x max K doubles) then max-abs (max K floats), cleared at the
-// start of every call.  Calls that overlap in time share it.
+// Launch with programmatic stream serialization (see grid_dependency_wait).
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(void (*kern)(KArgs...), dim3 grid, int threads, int smem, cudaStream_t st,
+                       Args... args) {
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = grid;
+    cfg.blockDim = dim3(threads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kern, static_cast<KArgs>(args)...);
+}
+
+// One-shot statistics without caller accumulators: a file-scope scratch that
+// holds, for a call with K channels, the power sums (4 x K doubles) followed
+// by the max-abs (K floats), cleared at the start of every call.  Calls that
+// overlap in time share it.
 constexpr int kNoAllocMaxK = W8A8_NOALLOC_STATS_MAX_K;
 static __device__ __align__(256) unsigned char g_stats_scratch[kNoAllocMaxK * (4 * sizeof(double) + sizeof(float))];
 
@@ -464,14 +668,27 @@ void *stats_scratch_address() {
 
 cudaError_t launch_act_stats_update(const uint16_t *X, int T, int K, const float *shift,
                                     double *sums, float *absmax, cudaStream_t st) {
-    const int gx = (K / 4 + 31) / 32;
     static PerDevice<int> occ;
-    int gy = slabs_for(blocks_per_sm(occ, stats_update_kernel, 32 * kStatsWarps), T, gx);
-    const int rows_per_slab = (T + gy - 1) / gy;
-    gy = (T + rows_per_slab - 1) / rows_per_slab;
-    stats_update_kernel<<<dim3(gx, gy), 32 * kStatsWarps, 0, st>>>(
-        reinterpret_cast<const uint2 *>(X), T, K, shift, rows_per_slab, sums, absmax);
-    return cudaGetLastError();
+    int per_sm = 1;
+    cudaError_t e = kernel_setup(occ, stats_update_kernel, kStatsThreads, kStatsSmem, &per_sm);
+    if (e != cudaSuccess) return e;
+    const int gx = (K / 8 + 31) / 32;
+    int gy = slabs_for(per_sm, T, gx);
+    // at least 8 rows per warp; at most kGroup^2 rows per thread
+    int rows_per_slab = (T + gy - 1) / gy;
+    if (rows_per_slab < 8 * kStatsWarps) rows_per_slab = 8 * kStatsWarps;
+    if (rows_per_slab > kStatsWarps * kMaxRowsPerThread) rows_per_slab = kStatsWarps * kMaxRowsPerThread;
+    // at most 65535 slabs per launch (a grid's y extent)
+    const long long rows_per_launch = 65535LL * rows_per_slab;
+    for (long long t0 = 0; t0 < T; t0 += rows_per_launch) {
+        const int rows = static_cast<int>(T - t0 < rows_per_launch ? T - t0 : rows_per_launch);
+        stats_update_kernel<<<dim3(gx, (rows + rows_per_slab - 1) / rows_per_slab), kStatsThreads,
+                              kStatsSmem, st>>>(reinterpret_cast<const uint4 *>(X + t0 * K), rows, K,
+                                                shift, rows_per_slab, sums, absmax);
+        e = cudaGetLastError();
+        if (e != cudaSuccess) return e;
+    }
+    return cudaSuccess;
 }
 
 cudaError_t launch_act_stats_finalize(const double *sums, const float *absmax, const float *shift,
@@ -484,35 +701,37 @@ cudaError_t launch_act_stats_finalize(const double *sums, const float *absmax, c
 
 cudaError_t launch_quant_act_per_tensor(const uint16_t *X, const float *lambda, int M, int K,
                                         int8_t *Xq, float *x_scale, float *amax, cudaStream_t st) {
-    cudaError_t e = cudaMemsetAsync(amax, 0, sizeof(float), st);
-    if (e != cudaSuccess) return e;
-    const int gx = (K / 8 + 31) / 32;
     static PerDevice<int> occ1, occ2;
-    const int gy1 = slabs_for(blocks_per_sm(occ1, tensor_absmax_kernel, 32 * kQWarps), M, gx);
-    const int gy2 = slabs_for(blocks_per_sm(occ2, tensor_quant_kernel, 32 * kQWarps), M, gx);
-    const int rps1 = (M + gy1 - 1) / gy1, rps2 = (M + gy2 - 1) / gy2;
-    tensor_absmax_kernel<<<dim3(gx, (M + rps1 - 1) / rps1), 32 * kQWarps, 0, st>>>(X, lambda, M, K,
-                                                                                   rps1, amax);
+    int per1 = 1, per2 = 1;
+    cudaError_t e = kernel_setup(occ1, tensor_absmax_kernel, 32 * kQWarps, kPtSmem, &per1);
+    if (e != cudaSuccess) return e;
+    e = kernel_setup(occ2, tensor_quant_kernel, 32 * kQWarps, kPtSmem, &per2);
+    if (e != cudaSuccess) return e;
+    zero_max_kernel<<<1, 1, 0, st>>>(amax);
     e = cudaGetLastError();
     if (e != cudaSuccess) return e;
-    tensor_quant_kernel<<<dim3(gx, (M + rps2 - 1) / rps2), 32 * kQWarps, 0, st>>>(
-        X, lambda, M, K, rps2, amax, Xq, x_scale);
-    return cudaGetLastError();
+    // pass 1 at two blocks per SM: pass 2's blocks start beside them
+    const int gx = (K / 8 + 31) / 32;
+    const int gy1 = slabs_for(per1 < 2 ? per1 : 2, M, gx);
+    const int gy2 = slabs_for(per2 < 2 ? per2 : 2, M, gx);
+    const int rps1 = (M + gy1 - 1) / gy1, rps2 = (M + gy2 - 1) / gy2;
+    e = launch_pdl(tensor_absmax_kernel, dim3(gx, (M + rps1 - 1) / rps1), 32 * kQWarps, kPtSmem, st,
+                   X, lambda, M, K, rps1, amax);
+    if (e != cudaSuccess) return e;
+    return launch_pdl(tensor_quant_kernel, dim3(gx, (M + rps2 - 1) / rps2), 32 * kQWarps, kPtSmem, st,
+                      X, lambda, M, K, rps2, static_cast<const float *>(amax), Xq, x_scale);
 }
-
-}  // namespace w8a8
-
-namespace w8a8 {
 
 cudaError_t launch_act_stats_noalloc(const uint16_t *X, int T, int K, const float *shift, float *chan,
                                      float *tensor, cudaStream_t st) {
     void *base = stats_scratch_address();
     if (!base) return cudaErrorInvalidSymbol;
     double *sums = static_cast<double *>(base);
-    float *absmax = reinterpret_cast<float *>(sums + 4 * static_cast<size_t>(kNoAllocMaxK));
-    cudaError_t e = cudaMemsetAsync(sums, 0, sizeof(double) * 4 * static_cast<size_t>(K), st);
-    if (e != cudaSuccess) return e;
-    e = cudaMemsetAsync(absmax, 0, sizeof(float) * static_cast<size_t>(K), st);
+    float *absmax = reinterpret_cast<float *>(sums + 4 * static_cast<size_t>(K));
+    const size_t words = 9 * static_cast<size_t>(K);      // 4K doubles and K floats
+    zero_words_kernel<<<(unsigned)((words + 1023) / 1024 < 256 ? (words + 1023) / 1024 : 256), 1024, 0, st>>>(
+        static_cast<uint32_t *>(base), words);
+    cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return e;
     e = launch_act_stats_update(X, T, K, shift, sums, absmax, st);
     if (e != cudaSuccess) return e;
