@@ -444,6 +444,9 @@ W8A8_API w8a8_status w8a8_act_stats_update(const uint16_t *X, int T, int K, cons
  *               about the grand mean).
  * A variance within the accumulation error of zero (at most 1e-5 of the
  * second power sum about the shift) is reported as 0, with kurtosis 0.
+ * chan must not overlap sums, absmax or shift (W8A8_ERR_INVALID_ARG): during
+ * the call its first floats hold per-32-channel partial sums, overwritten with
+ * their final values before the call completes (stream order).
  */
 W8A8_API w8a8_status w8a8_act_stats_finalize(const double *sums, const float *absmax,
                                              const float *shift, long long count, int K,

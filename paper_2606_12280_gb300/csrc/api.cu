@@ -19,6 +19,12 @@ __device__ unsigned int g_w8a8_device_error = 0;
 
 bool aligned16(const void *p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
 
+// Whether byte ranges [a, a + na) and [b, b + nb) overlap.
+bool overlaps(const void *a, size_t na, const void *b, size_t nb) {
+    const uintptr_t x = reinterpret_cast<uintptr_t>(a), y = reinterpret_cast<uintptr_t>(b);
+    return x < y + nb && y < x + na;
+}
+
 w8a8_status check_mk(int M, int K) {
     if (M < 0 || K <= 0 || (K % 16) != 0 || K > W8A8_MAX_K) return W8A8_ERR_UNSUPPORTED_SHAPE;
     return W8A8_OK;
@@ -348,6 +354,11 @@ w8a8_status w8a8_act_stats_finalize(const double *sums, const float *absmax, con
     if (!aligned16(sums) || !aligned16(absmax) || !aligned16(chan) || !aligned16(tensor) ||
         (shift && !aligned16(shift)))
         return W8A8_ERR_MISALIGNED;
+    const size_t k = static_cast<size_t>(K);
+    if (overlaps(chan, 4 * k * sizeof(float), sums, 4 * k * sizeof(double)) ||
+        overlaps(chan, 4 * k * sizeof(float), absmax, k * sizeof(float)) ||
+        (shift && overlaps(chan, 4 * k * sizeof(float), shift, k * sizeof(float))))
+        return W8A8_ERR_INVALID_ARG;
     return from_cuda(w8a8::launch_act_stats_finalize(sums, absmax, shift, count, K, chan, tensor,
                                                      as_stream(stream)));
 }

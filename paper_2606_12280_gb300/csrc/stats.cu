@@ -8,8 +8,9 @@
 //                          kurtosis of every linear's input, recorded over
 //                          the denoising trajectory, so the sums accumulate
 //                          over any number of calls)
-//   stats_finalize_kernel  per-channel and whole-tensor max-abs, mean,
-//                          population std and Pearson kurtosis from the sums
+//   stats_channels_kernel  per-channel max-abs, mean, population std and
+//   stats_tensor_kernel    Pearson kurtosis from the sums, then the same four
+//                          over the whole tensor
 //   tensor_absmax_kernel   max over the whole tensor of |x_mj / lambda_j|
 //   tensor_quant_kernel    INT8 codes of x_mj / lambda_j with that one scale
 //                          (the naive per-tensor arm of the activation-quant
@@ -321,60 +322,99 @@ __device__ __forceinline__ Central central(const double *sums, const float *shif
     return r;
 }
 
-constexpr int kFinThreads = 1024;
+// Finalize in two launches, with the work spread over the GPU (fp64 runs at a
+// small fraction of the fp32 rate here, so one block doing all K channels
+// takes far longer than the data movement):
+//   stats_channels_kernel  one warp per 32 channels: per-channel mean, std
+//                          and kurtosis into chan; and the warp's channels
+//                          pooled about their own mean mu_b (count 32 n):
+//                          M2_b = sum_j M2_j + n d_j^2,
+//                          M3_b = sum_j M3_j + 3 d_j M2_j + n d_j^3,
+//                          M4_b = sum_j M4_j + 4 d_j M3_j + 6 d_j^2 M2_j + n d_j^4
+//                          (d_j = mean_j - mu_b), with sum_j S2_j + n d_j^2 and
+//                          the max-abs.  These six fp64 numbers per warp are
+//                          kept in the first 12 floats per warp of chan's
+//                          max-abs plane, whose own values are written last.
+//   stats_tensor_kernel    one warp: pools the warps' summaries the same way
+//                          about the grand mean, writes tensor[4], then the
+//                          max-abs plane entries that held the summaries.
+constexpr int kFinWarpCh = 32;
+constexpr int kFinSummary = 6;                 // doubles per warp
 
-__device__ __forceinline__ double block_sum(double v, double *red) {
+__device__ __forceinline__ double warp_sum_f64(double v) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-    __syncthreads();
-    if (lane == 0) red[w] = v;
-    __syncthreads();
-    double t = 0.0;
-    for (int i = 0; i < kFinThreads / 32; ++i) t += red[i];
-    return t;
+    return v;
 }
 
-__global__ void __launch_bounds__(kFinThreads)
-stats_finalize_kernel(const double *__restrict__ sums, const float *__restrict__ absmax,
-                      const float *__restrict__ shift, double n, int K, float *__restrict__ chan,
-                      float *__restrict__ tensor) {
-    __shared__ double red[kFinThreads / 32];
-    double mean_sum = 0.0, amax = 0.0;
-    for (int j = threadIdx.x; j < K; j += kFinThreads) {
-        const Central c = central(sums, shift, K, j, n);
+__device__ __forceinline__ int fin_stash_floats(int K) {
+    return kFinSummary * 2 * ((K + kFinWarpCh - 1) / kFinWarpCh);
+}
+
+__global__ void __launch_bounds__(32)
+stats_channels_kernel(const double *__restrict__ sums, const float *__restrict__ absmax,
+                      const float *__restrict__ shift, double n, int K, float *__restrict__ chan) {
+    const int lane = threadIdx.x;
+    const int j = blockIdx.x * kFinWarpCh + lane;
+    const bool valid = j < K;
+    const int kb = min(kFinWarpCh, K - (int)blockIdx.x * kFinWarpCh);
+    Central c = {0.0, 0.0, 0.0, 0.0};
+    double s2 = 0.0;
+    float am = 0.0f;
+    if (valid) {
+        c = central(sums, shift, K, j, n);
+        s2 = sums[(size_t)K + j];
+        am = absmax[j];
         const double var = c.m2 / n;
-        chan[j] = absmax[j];
+        if (j >= fin_stash_floats(K)) chan[j] = am;
         chan[(size_t)K + j] = static_cast<float>(c.mean);
         chan[2 * (size_t)K + j] = static_cast<float>(sqrt(var));
         chan[3 * (size_t)K + j] = static_cast<float>(var > 0.0 ? (c.m4 / n) / (var * var) : 0.0);
-        mean_sum += c.mean;
-        amax = fmax(amax, (double)absmax[j]);
     }
-    // whole tensor: pool the channels about the grand mean mu (all channels
-    // have n rows), with delta_j = mean_j - mu:
-    //   M2 = sum_j M2_j + n delta_j^2,
-    //   M4 = sum_j M4_j + 4 delta_j M3_j + 6 delta_j^2 M2_j + n delta_j^4
-    const double mu = block_sum(mean_sum, red) / K;
-    double t2 = 0.0, t4 = 0.0, ss = 0.0;
-    for (int j = threadIdx.x; j < K; j += kFinThreads) {
-        const Central c = central(sums, shift, K, j, n);
-        const double dl = c.mean - mu;
-        t2 += c.m2 + n * dl * dl;
-        t4 += c.m4 + 4.0 * dl * c.m3 + 6.0 * dl * dl * c.m2 + n * dl * dl * dl * dl;
-        // size of the pooled second moment's terms about mu, for the
-        // constant-tensor test (same criterion as per channel)
-        ss += sums[(size_t)K + j] + n * dl * dl;
-    }
-    const double T2 = block_sum(t2, red), T4 = block_sum(t4, red), SS = block_sum(ss, red);
+    const double mu_b = warp_sum_f64(valid ? c.mean : 0.0) / kb;
+    const double d = valid ? c.mean - mu_b : 0.0;
+    const double M2 = warp_sum_f64(valid ? c.m2 + n * d * d : 0.0);
+    const double M3 = warp_sum_f64(valid ? c.m3 + 3.0 * d * c.m2 + n * d * d * d : 0.0);
+    const double M4 = warp_sum_f64(valid ? c.m4 + 4.0 * d * c.m3 + 6.0 * d * d * c.m2 + n * d * d * d * d : 0.0);
+    const double SS = warp_sum_f64(valid ? s2 + n * d * d : 0.0);
 #pragma unroll
-    for (int o = 16; o > 0; o >>= 1) amax = fmax(amax, __shfl_xor_sync(0xffffffffu, amax, o));
-    __syncthreads();
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = amax;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-        double am = 0.0;
-        for (int i = 0; i < kFinThreads / 32; ++i) am = fmax(am, red[i]);
+    for (int o = 16; o > 0; o >>= 1) am = fmaxf(am, __shfl_xor_sync(0xffffffffu, am, o));
+    if (lane == 0) {
+        double *st = reinterpret_cast<double *>(chan) + (size_t)kFinSummary * blockIdx.x;
+        st[0] = mu_b;
+        st[1] = M2;
+        st[2] = M3;
+        st[3] = M4;
+        st[4] = SS;
+        st[5] = am;
+    }
+}
+
+__global__ void __launch_bounds__(32)
+stats_tensor_kernel(const float *__restrict__ absmax, double n, int K, float *__restrict__ chan,
+                    float *__restrict__ tensor) {
+    const int lane = threadIdx.x;
+    const int G = (K + kFinWarpCh - 1) / kFinWarpCh;
+    const double *st = reinterpret_cast<const double *>(chan);
+    // grand mean: the warps' means weighted by their channel counts
+    double ms = 0.0;
+    for (int b = lane; b < G; b += 32) ms += st[kFinSummary * b] * min(kFinWarpCh, K - b * kFinWarpCh);
+    const double mu = warp_sum_f64(ms) / K;
+    double t2 = 0.0, t4 = 0.0, ss = 0.0, am = 0.0;
+    for (int b = lane; b < G; b += 32) {
+        const double *s = st + kFinSummary * b;
+        const double nb = n * min(kFinWarpCh, K - b * kFinWarpCh);
+        const double d = s[0] - mu;
+        t2 += s[1] + nb * d * d;
+        t4 += s[3] + 4.0 * d * s[2] + 6.0 * d * d * s[1] + nb * d * d * d * d;
+        ss += s[4] + nb * d * d;
+        am = fmax(am, s[5]);
+    }
+    const double T2 = warp_sum_f64(t2), T4 = warp_sum_f64(t4), SS = warp_sum_f64(ss);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) am = fmax(am, __shfl_xor_sync(0xffffffffu, am, o));
+    __syncwarp();                                         // every summary has been read
+    if (lane == 0) {
         const double nt = n * K;
         const double var = (T2 > 1e-5 * SS) ? T2 / nt : 0.0;
         tensor[0] = static_cast<float>(am);
@@ -382,6 +422,10 @@ stats_finalize_kernel(const double *__restrict__ sums, const float *__restrict__
         tensor[2] = static_cast<float>(sqrt(var));
         tensor[3] = static_cast<float>(var > 0.0 ? (T4 / nt) / (var * var) : 0.0);
     }
+    // the max-abs plane entries that held the summaries (R is a multiple of 4)
+    const int R4 = min(K, fin_stash_floats(K)) / 4;
+    for (int q = lane; q < R4; q += 32)
+        reinterpret_cast<float4 *>(chan)[q] = reinterpret_cast<const float4 *>(absmax)[q];
 }
 
 // ------------------------------------------------- per-tensor quantization
@@ -694,8 +738,11 @@ cudaError_t launch_act_stats_update(const uint16_t *X, int T, int K, const float
 cudaError_t launch_act_stats_finalize(const double *sums, const float *absmax, const float *shift,
                                       long long count, int K, float *chan, float *tensor,
                                       cudaStream_t st) {
-    stats_finalize_kernel<<<1, kFinThreads, 0, st>>>(sums, absmax, shift, (double)count, K, chan,
-                                                     tensor);
+    stats_channels_kernel<<<(K + kFinWarpCh - 1) / kFinWarpCh, 32, 0, st>>>(sums, absmax, shift,
+                                                                           (double)count, K, chan);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    stats_tensor_kernel<<<1, 32, 0, st>>>(absmax, (double)count, K, chan, tensor);
     return cudaGetLastError();
 }
 

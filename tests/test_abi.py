@@ -177,6 +177,15 @@ def test_per_tensor_and_stats_validation(L):
     assert fin(A, A, None, 0, 16, A, A, None) == INVALID          # count
     assert fin(A, A, None, 5, 16, A, None, None) == INVALID
     assert fin(A, A, None, 5, 8, A, A, None) == SHAPE
+    # chan may not overlap the inputs (it carries partial sums during the call)
+    base = 1 << 20
+    chan = ctypes.c_void_p(base)
+    assert fin(ctypes.c_void_p(base + 4 * 16 * 4 - 16), ctypes.c_void_p(base + 4096), None, 5, 16,
+               chan, A, None) == INVALID                          # sums
+    assert fin(ctypes.c_void_p(base + 4096), ctypes.c_void_p(base + 16), None, 5, 16,
+               chan, A, None) == INVALID                          # absmax
+    assert fin(ctypes.c_void_p(base + 4096), ctypes.c_void_p(base + 8192), ctypes.c_void_p(base + 128),
+               5, 16, chan, A, None) == INVALID                   # shift
 
 
 def test_linear_bf16_and_layer_validation(L):
