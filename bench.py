@@ -216,6 +216,19 @@ GEMM_TRAFFIC_BYTES = {("ts", "qkv_m4608_k4096_n12288"): 176.97e6}
 
 # ------------------------------------------------ the other configurations
 
+_WS = {}
+
+
+def _gemm_ws(dev):
+    """The fp16-code GEMM's split-K workspace (one per device: every GEMM of
+    this benchmark runs on one stream at a time)."""
+    key = str(torch.device(dev))
+    if key not in _WS:
+        from paper_2606_12280_gb300 import w8a8
+        _WS[key] = w8a8.gemm_workspace(dev)
+    return _WS[key]
+
+
 def _bf_dev(a, dev):
     import torch
     return torch.from_numpy(np.ascontiguousarray(a).view(np.int16)).view(torch.bfloat16).to(dev)
@@ -243,7 +256,7 @@ def config_single(w8a8, wl, dev):
     Y8 = w8a8.linear(Xq, sx, Wq, sw, b)
     ss = torch.empty(M, dtype=torch.int32, device=dev)
     q16, sx16 = w8a8.quant_act_f16codes(_bf_dev(case.X[0], dev), lam, sumsq=ss)
-    Y16 = w8a8.linear_f16codes(q16, sx16, Wq, sw, b, plan=w8a8.chunk_plan(Wq), x_sumsq=ss)
+    Y16 = w8a8.linear_f16codes(q16, sx16, Wq, sw, b, plan=w8a8.chunk_plan(Wq), x_sumsq=ss, workspace=_gemm_ws(dev))
     torch.cuda.synchronize()
     ulp = lambda y: int(np.abs(_u16(y).astype(np.int32) - ref["Y"].astype(np.int32)).max())
     checks = {
@@ -296,7 +309,7 @@ def config_ffn_pair(w8a8, wl, dev, isolated, codes, with_oracle):
 
         def gemm(i, st):
             if f16:
-                w8a8.linear_f16codes(q, sx, Wq, sw, b, Y=Y, plan=plan, x_sumsq=ss, stream=st)
+                w8a8.linear_f16codes(q, sx, Wq, sw, b, Y=Y, plan=plan, x_sumsq=ss, stream=st, workspace=_gemm_ws(dev))
             else:
                 w8a8.linear(q, sx, Wq, sw, b, Y=Y, stream=st)
 
@@ -406,7 +419,7 @@ def run_ours(args):
     def gemm(j, st):
         if f16:
             w8a8.linear_f16codes(Xqs[j], sxs[j], Wqs[j], sw, bias, Y=Ys[j], plan=plan, x_sumsq=sss[j],
-                                 stream=st)
+                                 stream=st, workspace=_gemm_ws(dev))
         else:
             w8a8.linear(Xqs[j], sxs[j], Wqs[j], sw, bias, Y=Ys[j], stream=st)
 
@@ -652,7 +665,7 @@ def run_ours(args):
         other_gemm = isolated(lambda i, st: w8a8.linear_f16codes(Xq_o[i % 2], sxs[i % n_sets],
                                                                  Wqs[i % n_sets], sw, bias, Y=Ys[i % n_sets],
                                                                  plan=plan, x_sumsq=sss[i % n_sets],
-                                                                 stream=st), 10)
+                                                                 stream=st, workspace=_gemm_ws(dev)), 10)
     del Xq_o
 
     # the pieces around the layer, each alone in a CUDA graph on the same
@@ -723,7 +736,7 @@ def run_ours(args):
     def dual_gemm(i, st):
         w8a8.linear_dual_f16codes([(dq[i % 2][b][0], dq[i % 2][b][1], dual_in[b][2], dual_in[b][3],
                                     dual_in[b][4], dual_in[b][5], dq[i % 2][b][2]) for b in range(2)],
-                                  Ys=dY[i % 2], stream=st)
+                                  Ys=dY[i % 2], stream=st, workspace=_gemm_ws(dev))
 
     dual_g_iso = isolated(dual_gemm, 10)
     # the dual steps pipelined like the headline step: step i+1's a3 on a
@@ -798,7 +811,7 @@ def run_ours(args):
                 w8a8.quant_act_dual_f16codes([(bi[0], bi[1]) for bi in br_in], out=[bi[6] for bi in br_in],
                                              stream=st)
                 w8a8.linear_dual_f16codes([(bi[6][0], bi[6][1], bi[2], bi[3], bi[4], bi[5], bi[6][2])
-                                           for bi in br_in], Ys=[bi[7] for bi in br_in], stream=st)
+                                           for bi in br_in], Ys=[bi[7] for bi in br_in], stream=st, workspace=_gemm_ws(dev))
 
             fns.append(lin)
             ops_b += 2 * 2.0 * Mb * Kb * Nb
@@ -872,7 +885,8 @@ def run_ours(args):
                                  "(roofline, act_quant.ms_in_step) from a second pass of K "
                                  "stream-launched steps with events around each kernel",
                        "codes": f"{args.codes} container of the int8 activation codes",
-                       "gemm_engine": {"ts": "tcgen05 cta pair, weights in TMEM, drain plan + token sums",
+                       "gemm_engine": {"ts": "tcgen05 cta pair, weights in TMEM, drain plan + token sums, "
+                                             "last round of tiles split over K (workspace)",
                                        "tc2": "tcgen05 cta pair", "tc": "tcgen05",
                                        "mma": "mma.sync"}[engine_name]},
             "roofline": {"bound": "tensor", "achieved": gemm_tflops, "peak": peak_t,

@@ -225,21 +225,35 @@ W8A8_API w8a8_status w8a8_quant_act_f16codes(const uint16_t *X, const float *smo
  *     its largest weight-row sum of squares is at most 2^48 has every partial
  *     sum within 2^24 (Cauchy-Schwarz) and is accumulated without a drain.
  *     Sums of other codes void the exactness guarantee.
+ *   workspace: NULL, or w8a8_gemm_workspace_size() bytes of device memory
+ *     (16-byte aligned) that the caller zeroed once before its first use.
+ *     The output tiles (256 x 256) fill the GPU's CTA pairs in rounds; with a
+ *     workspace, as many tiles as a last, partial round would hold (all
+ *     tiles, when there are fewer tiles than pairs) are split over K between
+ *     pairs in the first round, their int32 partial sums meet in the
+ *     workspace, and the part that finishes last adds them (integer sums:
+ *     the result is the same bits as without a workspace).  The kernel leaves the workspace's
+ *     counters zero; after a call that returned an error, zero it again.
+ *     Calls that overlap in time need workspaces of their own.
  */
 W8A8_API w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale,
                                           const int8_t *Wq, const float *w_scale,
                                           const float *bias, int M, int N, int K,
                                           const uint32_t *chunk_plan, const uint32_t *x_sumsq,
-                                          uint16_t *Y, void *stream);
+                                          uint16_t *Y, void *workspace, void *stream);
+
+/* Bytes of the workspace of w8a8_linear_f16codes on the current device (one
+ * int32 256 x 256 tile per CTA pair, and counters). */
+W8A8_API long long w8a8_gemm_workspace_size(void);
 
 /*
  * Test export of the product above alone: acc = Xq16 Wq^T as int32 [M,N],
- * written.  Same shape rules, plan and token sums.
+ * written.  Same shape rules, plan, token sums and workspace.
  */
 W8A8_API w8a8_status w8a8_debug_gemm_f16codes_i32(const uint16_t *Xq16, const int8_t *Wq, int M,
                                                   int N, int K, const uint32_t *chunk_plan,
                                                   const uint32_t *x_sumsq, int32_t *acc,
-                                                  void *stream);
+                                                  void *workspace, void *stream);
 
 /* One branch of the dual-branch layer with fp16 codes (a6 on this path). */
 typedef struct {
@@ -275,9 +289,11 @@ W8A8_API w8a8_status w8a8_quant_act_dual_f16codes(const w8a8_act_branch16 *br, i
  * a4 + a5 of both branches in one grouped launch (a6) with fp16 codes: the
  * tile space covers both branches, each tile with its own branch's operands,
  * plan and token sums; results as two w8a8_linear_f16codes calls, bitwise.
- * The branches share N and K.
+ * The branches share N and K.  workspace as w8a8_linear_f16codes (the last
+ * round's tiles of both branches are split).
  */
-W8A8_API w8a8_status w8a8_linear_dual_f16codes(const w8a8_branch16 *br, int N, int K, void *stream);
+W8A8_API w8a8_status w8a8_linear_dual_f16codes(const w8a8_branch16 *br, int N, int K,
+                                               void *workspace, void *stream);
 
 /*
  * Drain plan of an int8 weight matrix for w8a8_linear_f16codes (no

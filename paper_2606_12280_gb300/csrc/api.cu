@@ -228,8 +228,10 @@ w8a8_status w8a8_quant_act_dual_f16codes(const w8a8_act_branch16 *br, int K, voi
     return from_cuda(w8a8::launch_quant_act_dual_f16codes(b, K, as_stream(stream)));
 }
 
-w8a8_status w8a8_linear_dual_f16codes(const w8a8_branch16 *br, int N, int K, void *stream) {
+w8a8_status w8a8_linear_dual_f16codes(const w8a8_branch16 *br, int N, int K, void *workspace,
+                                      void *stream) {
     if (!br) return W8A8_ERR_INVALID_ARG;
+    if (workspace && !aligned16(workspace)) return W8A8_ERR_MISALIGNED;
     if (w8a8_status e = check_nk(N, K)) return e;
     w8a8::GemmBranch b[2];
     for (int i = 0; i < 2; ++i) {
@@ -244,7 +246,7 @@ w8a8_status w8a8_linear_dual_f16codes(const w8a8_branch16 *br, int N, int K, voi
     if (b[0].M == 0 && b[1].M == 0) return W8A8_OK;
     unsigned int *err = device_error_word();
     if (!err) return W8A8_ERR_CUDA;
-    return from_cuda(w8a8::launch_gemm_ts(b, 2, N, K, false, err, as_stream(stream)));
+    return from_cuda(w8a8::launch_gemm_ts(b, 2, N, K, false, workspace, err, as_stream(stream)));
 }
 
 w8a8_status w8a8_gelu_quant_act(const uint16_t *H, const float *smooth, int M, int K, int8_t *Xq,
@@ -282,8 +284,9 @@ w8a8_status w8a8_quant_act_f16codes(const uint16_t *X, const float *smooth, int 
 w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale, const int8_t *Wq,
                                  const float *w_scale, const float *bias, int M, int N, int K,
                                  const uint32_t *chunk_plan, const uint32_t *x_sumsq, uint16_t *Y,
-                                 void *stream) {
+                                 void *workspace, void *stream) {
     if (w8a8_status e = check_nk(N, K)) return e;
+    if (workspace && !aligned16(workspace)) return W8A8_ERR_MISALIGNED;
     if (w8a8_status e = check_mk(M, K)) return e;
     w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), x_scale, Wq, w_scale, bias, Y, M, x_sumsq,
                        chunk_plan};
@@ -292,13 +295,14 @@ w8a8_status w8a8_linear_f16codes(const uint16_t *Xq16, const float *x_scale, con
     if (M == 0) return W8A8_OK;
     unsigned int *err = device_error_word();
     if (!err) return W8A8_ERR_CUDA;
-    return from_cuda(w8a8::launch_gemm_ts(&b, 1, N, K, false, err, as_stream(stream)));
+    return from_cuda(w8a8::launch_gemm_ts(&b, 1, N, K, false, workspace, err, as_stream(stream)));
 }
 
 w8a8_status w8a8_debug_gemm_f16codes_i32(const uint16_t *Xq16, const int8_t *Wq, int M, int N, int K,
                                          const uint32_t *chunk_plan, const uint32_t *x_sumsq, int32_t *acc,
-                                         void *stream) {
+                                         void *workspace, void *stream) {
     if (w8a8_status e = check_nk(N, K)) return e;
+    if (workspace && !aligned16(workspace)) return W8A8_ERR_MISALIGNED;
     if (w8a8_status e = check_mk(M, K)) return e;
     w8a8::GemmBranch b{reinterpret_cast<const int8_t *>(Xq16), nullptr, Wq, nullptr, nullptr, acc, M, x_sumsq,
                        chunk_plan};
@@ -307,8 +311,10 @@ w8a8_status w8a8_debug_gemm_f16codes_i32(const uint16_t *Xq16, const int8_t *Wq,
     if (M == 0) return W8A8_OK;
     unsigned int *err = device_error_word();
     if (!err) return W8A8_ERR_CUDA;
-    return from_cuda(w8a8::launch_gemm_ts(&b, 1, N, K, true, err, as_stream(stream)));
+    return from_cuda(w8a8::launch_gemm_ts(&b, 1, N, K, true, workspace, err, as_stream(stream)));
 }
+
+long long w8a8_gemm_workspace_size(void) { return w8a8::gemm_ts_workspace_bytes(); }
 
 long long w8a8_chunk_plan_size(int N, int K) {
     if (N <= 0 || K <= 0) return 1;

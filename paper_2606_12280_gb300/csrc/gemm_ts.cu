@@ -105,8 +105,9 @@ constexpr uint32_t BAR_TFLAG = BAR_DRAIN + 8;              // a tile's single-ru
 constexpr uint32_t OFF_TFLAG = BAR_TFLAG + 16;             // the flags (two tiles in flight)
 constexpr uint32_t OFF_TMEM = OFF_TFLAG + 8;
 constexpr uint32_t OFF_ABORT = OFF_TMEM + 4;
+constexpr uint32_t OFF_SPLIT = OFF_ABORT + 4;                // a split part's arrival order
 constexpr uint32_t SMEM_BARRIERS = 512;
-static_assert(OFF_ABORT + 4 - OFF_BAR <= SMEM_BARRIERS, "barrier area");
+static_assert(OFF_SPLIT + 4 - OFF_BAR <= SMEM_BARRIERS, "barrier area");
 // per epilogue warp: the activation scales of its 128 tokens
 constexpr uint32_t OFF_EPI = OFF_BAR + SMEM_BARRIERS;
 constexpr uint32_t EPI_BYTES = (PAIR_T / 2) * 4;
@@ -140,6 +141,13 @@ struct Params {
     int single_ok;
     unsigned int *err;
     uint64_t wait_limit_ns;
+    // work units: first the split_tiles last tiles as `split` parts each
+    // over consecutive K chunks (split = 1: none), then tiles 0 ..
+    // full_tiles - 1 whole; a part's int32 sums go to ws, and the last part
+    // of a tile to arrive (ws_cnt) adds them up and runs the epilogue
+    int full_tiles, split, split_tiles, total_units;
+    int32_t *ws;               // [split_tiles][split][PAIR_T tokens][PAIR_F features]
+    unsigned int *ws_cnt;      // [split_tiles][2 CTAs], zero between calls
 };
 
 struct Tile {
@@ -153,6 +161,34 @@ __device__ __forceinline__ Tile tile_coords(const Params &p, int t) {
     const int tt = p.br[r.branch].t_tiles;
     r.t0 = (local % tt) * PAIR_T;
     r.f0 = (local / tt) * PAIR_F;
+    return r;
+}
+
+struct Unit {
+    int tile;          // output tile
+    int ci0, ci1;      // K chunks [ci0, ci1)
+    int part, slot;    // split part, split tile index (-1: a whole tile)
+};
+
+// The split parts come first, in the pairs' first round: the exchange of
+// partial sums then overlaps the whole tiles that follow instead of
+// lengthening the end of the kernel.
+__device__ __forceinline__ Unit unit_coords(const Params &p, int u, int NC) {
+    Unit r;
+    const int nsplit = p.split_tiles * p.split;
+    if (u >= nsplit) {
+        r.tile = u - nsplit;
+        r.ci0 = 0;
+        r.ci1 = NC;
+        r.part = 0;
+        r.slot = -1;
+    } else {
+        r.slot = u / p.split;
+        r.part = u - r.slot * p.split;
+        r.tile = p.full_tiles + r.slot;
+        r.ci0 = r.part * NC / p.split;
+        r.ci1 = (r.part + 1) * NC / p.split;
+    }
     return r;
 }
 
@@ -246,18 +282,20 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
             mbar_arrive(sb + BAR_TFLAG + 8 * (n & 1));
         }
     };
-    bool single = use_single && pair < p.total_tiles && tile_single_run(p, pair, lane);
-    if (pair < p.total_tiles) publish(0, single);
-    int n = 0;                         // tiles so far
-    for (int t = pair; ok && t < p.total_tiles; t += npairs, ++n) {
+    bool single = use_single && pair < p.total_units && tile_single_run(p, unit_coords(p, pair, NC).tile, lane);
+    if (pair < p.total_units) publish(0, single);
+    int n = 0;                         // units so far
+    for (int u = pair; ok && u < p.total_units; u += npairs, ++n) {
+        const Unit un = unit_coords(p, u, NC);
+        const int t = un.tile;
         const Tile tc = tile_coords(p, t);
         const int fb = tc.f0 / PAIR_F;
         const uint32_t *plan = p.br[tc.branch].plan;
         int32_t run[RUN];
 #pragma unroll
         for (int i = 0; i < RUN; ++i) run[i] = 0;
-        for (int ci = 0; ci < NC; ++ci) {
-            if (ci != NC - 1 && (single || !plan_drains(p, plan, fb, ci, NC))) continue;
+        for (int ci = un.ci0; ci < un.ci1; ++ci) {
+            if (ci != un.ci1 - 1 && (single || !plan_drains(p, plan, fb, ci, NC))) continue;
             if (!mbar_wait_cluster(sb + BAR_ACCFULL, c & 1, wc, ERR_EPILOGUE)) {
                 ok = false;
                 break;
@@ -305,12 +343,54 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
             ++c;
         }
         if (!ok) break;
-        // the next tile's decision, before this tile's stores
-        const bool raw = single;
+        // the next unit's decision, before this unit's stores
+        bool raw = single;
         if (use_single) {
-            const int tn = t + npairs;
-            single = tn < p.total_tiles && tile_single_run(p, tn, lane);
-            if (tn < p.total_tiles) publish(n + 1, single);
+            const int un_next = u + npairs;
+            single = un_next < p.total_units && tile_single_run(p, unit_coords(p, un_next, NC).tile, lane);
+            if (un_next < p.total_units) publish(n + 1, single);
+        }
+        if (un.slot >= 0) {
+            // a part of a split tile: this warp's 32 features x 128 tokens of
+            // int32 sums go to the workspace, and the warp of the part that
+            // arrives last adds the other parts' and stores the tile (integer
+            // sums: exact in any order).  Each warp counts its own arrivals,
+            // so no warp waits for another.
+            if (raw) {
+#pragma unroll
+                for (int i = 0; i < RUN; ++i) run[i] = exact_int(static_cast<uint32_t>(run[i]));
+                raw = false;
+            }
+            const size_t at = (size_t)h * (PAIR_T / 2) * PAIR_F + rank * CTA_F + q * 32 + lane;
+            const size_t part_elems = (size_t)PAIR_T * PAIR_F;
+            int32_t *mine = p.ws + (size_t)(un.slot * p.split + un.part) * part_elems + at;
+#pragma unroll
+            for (int i = 0; i < RUN; ++i) __stcg(mine + (size_t)i * PAIR_F, run[i]);
+            __threadfence();
+            __syncwarp();
+            unsigned int *cnt = p.ws_cnt + (size_t)un.slot * 16 + rank * 8 + (warp - 8);
+            unsigned int order = 0;
+            if (lane == 0) order = atomicAdd(cnt, 1u);
+            order = __shfl_sync(0xffffffffu, order, 0);
+            if (order != static_cast<unsigned int>(p.split - 1)) {
+                __syncwarp();
+                continue;
+            }
+            __threadfence();
+            for (int pp = 0; pp < p.split; ++pp) {
+                if (pp == un.part) continue;
+                const int32_t *other = p.ws + (size_t)(un.slot * p.split + pp) * part_elems + at;
+                // 32 loads in flight per batch
+#pragma unroll
+                for (int jb = 0; jb < RUN; jb += 32) {
+                    int32_t tmp[32];
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) tmp[i] = __ldcg(other + (size_t)(jb + i) * PAIR_F);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) run[jb + i] += tmp[i];
+                }
+            }
+            if (lane == 0) *cnt = 0u;          // every part has arrived: ready for the next call
         }
         // one representation for the stores: int32 for the int32 export,
         // fp32 (the exact value, |acc| <= 2^24 or rounded as (float)acc)
@@ -466,11 +546,13 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
             if (lane == 0) {
                 uint32_t j = 0;
                 bool ok = true;
-                for (int t = pair; ok && t < p.total_tiles; t += npairs) {
-                    const Tile tl = tile_coords(p, t);
+                for (int u = pair; ok && u < p.total_units; u += npairs) {
+                    const Unit un = unit_coords(p, u, NC);
+                    const Tile tl = tile_coords(p, un.tile);
                     const CUtensorMap *mW = tl.branch ? &tmW1 : &tmW0;
                     const int frow = tl.f0 + static_cast<int>(rank) * CTA_F;
-                    for (int ks = 0; ks < NS; ++ks, ++j) {
+                    const int ks_end = min(NS, un.ci1 * KC_STAGES);
+                    for (int ks = un.ci0 * KC_STAGES; ks < ks_end; ++ks, ++j) {
                         const uint32_t s = j % S8;
                         if (!mbar_wait(sb + BAR_EMPTY8 + 8 * s, ((j / S8) & 1) ^ 1, wc, ERR_PRODUCER)) {
                             ok = false;
@@ -495,11 +577,13 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
             if (lane == 0) {
                 uint32_t j = 0;
                 bool ok = true;
-                for (int t = pair; ok && t < p.total_tiles; t += npairs) {
-                    const Tile tl = tile_coords(p, t);
+                for (int u = pair; ok && u < p.total_units; u += npairs) {
+                    const Unit un = unit_coords(p, u, NC);
+                    const Tile tl = tile_coords(p, un.tile);
                     const CUtensorMap *mX = tl.branch ? &tmX1 : &tmX0;
                     const int trow = tl.t0 + static_cast<int>(rank) * CTA_T;
-                    for (int ks = 0; ks < NS; ++ks, ++j) {
+                    const int ks_end = min(NS, un.ci1 * KC_STAGES);
+                    for (int ks = un.ci0 * KC_STAGES; ks < ks_end; ++ks, ++j) {
                         const uint32_t s = j % SX;
                         if (!mbar_wait_cluster(sb + BAR_SEMPTY + 8 * s, ((j / SX) & 1) ^ 1, wc, ERR_PRODUCER)) {
                             ok = false;
@@ -525,14 +609,15 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
                 uint32_t j = 0, c = 0;         // stages, drains so far
                 bool ok = true;
                 const bool use_single = p.single_ok != 0;
-                int n = 0;                     // tiles so far
-                for (int t = pair; ok && t < p.total_tiles; t += npairs, ++n) {
-                    const Tile tc = tile_coords(p, t);
+                int n = 0;                     // units so far
+                for (int u = pair; ok && u < p.total_units; u += npairs, ++n) {
+                    const Unit un = unit_coords(p, u, NC);
+                    const Tile tc = tile_coords(p, un.tile);
                     const int fb = tc.f0 / PAIR_F;
                     const uint32_t *plan = p.br[tc.branch].plan;
                     bool single = false;       // the tile is one run (published by the epilogue)
                     bool fresh = true;         // the next MMA starts a new accumulation
-                    for (int ci = 0; ok && ci < NC; ++ci) {
+                    for (int ci = un.ci0; ok && ci < un.ci1; ++ci) {
                         if (fresh) {
                             // the epilogue has drained the previous accumulation
                             if (!mbar_wait_cluster(sb + BAR_ACCEMPTY, (c & 1) ^ 1, wc, ERR_MMA)) {
@@ -570,14 +655,14 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
                             }
                             mma_commit_pair_multicast(sb + BAR_SEMPTY + 8 * sa, 0x3);
                         }
-                        if (use_single && ci == 0 && ok) {
+                        if (use_single && ci == un.ci0 && ok) {
                             if (!mbar_wait(sb + BAR_TFLAG + 8 * (n & 1), (n >> 1) & 1, wc, ERR_MMA)) {
                                 ok = false;
                                 break;
                             }
                             single = ld_shared_s32(sb + OFF_TFLAG + 4 * (n & 1)) != 0;
                         }
-                        fresh = ci == NC - 1 || (!single && plan_drains(p, plan, fb, ci, NC));
+                        fresh = ci == un.ci1 - 1 || (!single && plan_drains(p, plan, fb, ci, NC));
                         if (ok && fresh) {
                             mma_commit_pair_multicast(sb + BAR_ACCFULL, 0x3);
                             ++c;
@@ -599,8 +684,10 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
             const uint32_t a_lane = tmem + (static_cast<uint32_t>((warp & 3) * 32) << 16) + A_COL0;
             uint32_t j = 0;
             bool ok = true;
-            for (int t = pair; ok && t < p.total_tiles; t += npairs) {
-                for (int ks = 0; ks < NS; ++ks, ++j) {
+            for (int u = pair; ok && u < p.total_units; u += npairs) {
+                const Unit un = unit_coords(p, u, NC);
+                const int ks_end = min(NS, un.ci1 * KC_STAGES);
+                for (int ks = un.ci0 * KC_STAGES; ks < ks_end; ++ks, ++j) {
                     const uint32_t s8 = j % S8, sa = j % SA;
                     // every lane waits; __all_sync keeps the warp's control flow
                     // uniform if a wait gives up
@@ -798,8 +885,20 @@ cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cu
     return cudaGetLastError();
 }
 
-cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, unsigned int *err,
-                           cudaStream_t st) {
+// Split-K workspace: the arrival counters (16 per split tile: one per
+// epilogue warp of each CTA), then one int32 partial tile per split part.  A
+// launch splits at most as many parts as there are CTA pairs.
+namespace {
+constexpr size_t kWsCounterBytes(int pairs) { return ((size_t)pairs * 16 * 4 + 255) / 256 * 256; }
+}  // namespace
+
+long long gemm_ts_workspace_bytes() {
+    const int P = device_sms() / 2;
+    return static_cast<long long>(kWsCounterBytes(P) + (size_t)P * PAIR_T * PAIR_F * 4);
+}
+
+cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, void *workspace,
+                           unsigned int *err, cudaStream_t st) {
     const int sms = device_sms();
     auto kern = out_i32 ? gemm_ts_kernel<true> : gemm_ts_kernel<false>;
     cudaError_t e = out_i32 ? prepare_ts_kernel<true>() : prepare_ts_kernel<false>();
@@ -847,7 +946,30 @@ cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_
         if (p.br[i].M > 0 && (p.br[i].x_sumsq == nullptr || p.br[i].plan == nullptr)) p.single_ok = 0;
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
-    const int pairs = p.total_tiles < sms / 2 ? p.total_tiles : sms / 2;
+    // The tiles fill the CTA pairs in rounds; a last, partial round would
+    // leave pairs idle, so with a workspace R = T mod pairs tiles are split
+    // into s parts of consecutive K chunks (s R <= pairs, s <= chunks), one
+    // part per pair, run in the first round.  With fewer tiles than pairs,
+    // every tile is split.
+    const int P = sms / 2;
+    const int T = p.total_tiles;
+    const int NC = (K + KC - 1) / KC;
+    p.full_tiles = T;
+    p.split = 1;
+    p.split_tiles = 0;
+    if (workspace != nullptr && NC >= 2) {
+        const int rem = T % P;
+        const int s = rem > 0 ? min(P / rem, NC) : 1;
+        if (s >= 2) {
+            p.full_tiles = T - rem;
+            p.split = s;
+            p.split_tiles = rem;
+            p.ws_cnt = static_cast<unsigned int *>(workspace);
+            p.ws = reinterpret_cast<int32_t *>(static_cast<char *>(workspace) + kWsCounterBytes(P));
+        }
+    }
+    p.total_units = p.full_tiles + p.split_tiles * p.split;
+    const int pairs = p.total_units < P ? p.total_units : P;
     kern<<<2 * pairs, THREADS, SMEM_TOTAL, st>>>(maps[0], maps[1], maps[2], maps[3], p);
     return cudaGetLastError();
 }

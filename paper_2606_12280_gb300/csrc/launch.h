@@ -75,8 +75,12 @@ cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K,
 // activation codes as fp16 values (2 bytes each), Wq the int8 weights.  A
 // branch's plan (from launch_chunk_plan on its Wq) and x_sumsq (from a3) let
 // the accumulation skip drains where they bound the partial sums.
-cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, unsigned int *err,
-                           cudaStream_t st);
+// workspace: NULL, or gemm_ts_workspace_bytes() bytes whose counters are
+// zero (the kernel leaves them zero): the last, partial round of tiles is
+// then split over K between the idle CTA pairs.
+cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, void *workspace,
+                           unsigned int *err, cudaStream_t st);
+long long gemm_ts_workspace_bytes();
 int chunk_plan_words(int K);    // per block of 256 weight rows
 cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cudaStream_t st);
 

@@ -48,11 +48,12 @@ SIGNATURES = {
     "w8a8_linear_gguf": [_P, _P, _I, _P, _I, _I, _I, _P, _P],
     "w8a8_debug_gguf_dequant": [_P, _I, _I, _I, _P, _P],
     "w8a8_quant_act_f16codes": [_P, _P, _I, _I, _P, _P, _P, _I, _P],
-    "w8a8_linear_f16codes": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P],
-    "w8a8_debug_gemm_f16codes_i32": [_P, _P, _I, _I, _I, _P, _P, _P, _P],
+    "w8a8_linear_f16codes": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P, _P],
+    "w8a8_gemm_workspace_size": [],
+    "w8a8_debug_gemm_f16codes_i32": [_P, _P, _I, _I, _I, _P, _P, _P, _P, _P],
     "w8a8_chunk_plan_size": [_I, _I],
     "w8a8_quant_act_dual_f16codes": [_P, _I, _P],
-    "w8a8_linear_dual_f16codes": [_P, _I, _I, _P],
+    "w8a8_linear_dual_f16codes": [_P, _I, _I, _P, _P],
     "w8a8_chunk_plan": [_P, _I, _I, _P, _P],
     "w8a8_act_stats_noalloc": [_P, _I, _I, _P, _P, _P, _P],
 }
@@ -116,6 +117,7 @@ def lib() -> ctypes.CDLL:
                 fn.restype = ctypes.c_int
             L.w8a8_status_string.restype = ctypes.c_char_p
             L.w8a8_chunk_plan_size.restype = ctypes.c_longlong
+            L.w8a8_gemm_workspace_size.restype = ctypes.c_longlong
             _lib = L
     return _lib
 
@@ -376,10 +378,11 @@ def quant_act_dual_f16codes(branches, out=None, stream=None):
     return res
 
 
-def linear_dual_f16codes(branches, Ys=None, stream=None):
+def linear_dual_f16codes(branches, Ys=None, workspace=None, stream=None):
     """One grouped launch over two branches with fp16 codes.  branches: two
     tuples (Xq16, x_scale, Wq, w_scale, bias, plan, x_sumsq) (plan and x_sumsq
-    may be None); returns [Y_cond, Y_uncond]."""
+    may be None); returns [Y_cond, Y_uncond].  workspace: None or
+    ``gemm_workspace()`` (see ``linear_f16codes``)."""
     if len(branches) != 2:
         raise ValueError("linear_dual_f16codes takes exactly two branches")
     N, K = branches[0][2].shape
@@ -403,7 +406,8 @@ def linear_dual_f16codes(branches, Ys=None, stream=None):
                           _ptr(b, torch.float32, "bias"), _ptr(Y, torch.bfloat16, "Y"), Xq16.shape[0],
                           _ptr(plan, torch.int32, "plan"), _ptr(ss, torch.int32, "x_sumsq"))
         out.append(Y)
-    _check("w8a8_linear_dual_f16codes", lib().w8a8_linear_dual_f16codes(arr, N, K, _stream(stream)))
+    _check("w8a8_linear_dual_f16codes", lib().w8a8_linear_dual_f16codes(arr, N, K, _workspace(workspace),
+                                                                         _stream(stream)))
     return out
 
 
@@ -443,10 +447,13 @@ def quant_act_f16codes(X, smooth=None, Xq16=None, x_scale=None, gelu=False, sums
     return Xq16, x_scale
 
 
-def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, x_sumsq=None, stream=None):
+def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, x_sumsq=None, workspace=None,
+                    stream=None):
     """a4 + a5 with fp16-coded activations: Y = bf16((Xq Wq^T) * sx * sw + b).
     plan: None or ``chunk_plan(Wq)``; x_sumsq: None or the token sums that
-    ``quant_act_f16codes(..., sumsq=)`` wrote for these codes."""
+    ``quant_act_f16codes(..., sumsq=)`` wrote for these codes; workspace: None
+    or ``gemm_workspace()`` (the last round of tiles is then split over K
+    between idle SM pairs; same bits)."""
     M, K = Xq16.shape
     N = Wq.shape[0]
     _check_weights(Wq, N, K)
@@ -463,11 +470,12 @@ def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, x_
         _ptr(Xq16, torch.float16, "Xq16"), _ptr(x_scale, torch.float32, "x_scale"),
         _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
         _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(plan, torch.int32, "plan"),
-        _ptr(x_sumsq, torch.int32, "x_sumsq"), _ptr(Y, torch.bfloat16, "Y"), _stream(stream)))
+        _ptr(x_sumsq, torch.int32, "x_sumsq"), _ptr(Y, torch.bfloat16, "Y"), _workspace(workspace),
+        _stream(stream)))
     return Y
 
 
-def debug_gemm_f16codes_i32(Xq16, Wq, plan=None, x_sumsq=None, acc=None, stream=None):
+def debug_gemm_f16codes_i32(Xq16, Wq, plan=None, x_sumsq=None, acc=None, workspace=None, stream=None):
     """Exact int32 acc = Xq16 Wq^T (test export of the fp16-code GEMM)."""
     M, K = Xq16.shape
     N = Wq.shape[0]
@@ -481,8 +489,29 @@ def debug_gemm_f16codes_i32(Xq16, Wq, plan=None, x_sumsq=None, acc=None, stream=
     _check("w8a8_debug_gemm_f16codes_i32", lib().w8a8_debug_gemm_f16codes_i32(
         _ptr(Xq16, torch.float16, "Xq16"), _ptr(Wq, torch.int8, "Wq"), M, N, K,
         _ptr(plan, torch.int32, "plan"), _ptr(x_sumsq, torch.int32, "x_sumsq"),
-        _ptr(acc, torch.int32, "acc"), _stream(stream)))
+        _ptr(acc, torch.int32, "acc"), _workspace(workspace), _stream(stream)))
     return acc
+
+
+def gemm_workspace_size() -> int:
+    """Bytes of the fp16-code GEMM's workspace on the current device."""
+    return int(lib().w8a8_gemm_workspace_size())
+
+
+def gemm_workspace(device=None):
+    """A zeroed workspace for ``linear_f16codes`` / ``linear_dual_f16codes``
+    on `device` (a uint8 tensor; calls that overlap in time need their own)."""
+    device = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    with torch.cuda.device(device):
+        return torch.zeros(gemm_workspace_size(), dtype=torch.uint8, device=device)
+
+
+def _workspace(ws):
+    if ws is None:
+        return None
+    if ws.dtype != torch.uint8 or ws.numel() < gemm_workspace_size():
+        raise ValueError("workspace: a uint8 tensor of gemm_workspace_size() bytes (gemm_workspace())")
+    return _ptr(ws, torch.uint8, "workspace")
 
 
 def chunk_plan_size(N: int, K: int) -> int:

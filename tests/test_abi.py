@@ -277,18 +277,20 @@ def test_f16codes_validation(L):
     assert f(A, None, 4, 16, A, A, U, 0, None) == MISALIGNED          # sumsq
     assert f(None, None, 0, 16, None, None, None, 0, None) == OK
     g = L.w8a8_linear_f16codes
-    assert g(A, A, A, A, None, 4, 12, 16, None, None, A, None) == SHAPE
-    assert g(None, A, A, A, None, 4, 8, 16, None, None, A, None) == INVALID
-    assert g(A, A, U, A, None, 4, 8, 16, None, None, A, None) == MISALIGNED
-    assert g(A, A, A, A, None, 4, 8, 16, U, None, A, None) == MISALIGNED      # plan
-    assert g(A, A, A, A, None, 4, 8, 16, A, U, A, None) == MISALIGNED         # token sums
-    assert g(A, A, A, A, None, 0, 8, 16, None, None, A, None) == OK
+    assert g(A, A, A, A, None, 4, 12, 16, None, None, A, None, None) == SHAPE
+    assert g(None, A, A, A, None, 4, 8, 16, None, None, A, None, None) == INVALID
+    assert g(A, A, U, A, None, 4, 8, 16, None, None, A, None, None) == MISALIGNED
+    assert g(A, A, A, A, None, 4, 8, 16, U, None, A, None, None) == MISALIGNED      # plan
+    assert g(A, A, A, A, None, 4, 8, 16, A, U, A, None, None) == MISALIGNED         # token sums
+    assert g(A, A, A, A, None, 0, 8, 16, None, None, A, None, None) == OK
+    assert g(A, A, A, A, None, 4, 8, 16, None, None, A, U, None) == MISALIGNED   # workspace
     d = L.w8a8_debug_gemm_f16codes_i32
-    assert d(A, A, 4, 12, 16, None, None, A, None) == SHAPE
-    assert d(None, A, 4, 8, 16, None, None, A, None) == INVALID
-    assert d(A, U, 4, 8, 16, None, None, A, None) == MISALIGNED
-    assert d(A, A, 4, 8, 16, None, U, A, None) == MISALIGNED
-    assert d(A, A, 0, 8, 16, None, None, A, None) == OK
+    assert d(A, A, 4, 12, 16, None, None, A, None, None) == SHAPE
+    assert d(None, A, 4, 8, 16, None, None, A, None, None) == INVALID
+    assert d(A, U, 4, 8, 16, None, None, A, None, None) == MISALIGNED
+    assert d(A, A, 4, 8, 16, None, U, A, None, None) == MISALIGNED
+    assert d(A, A, 0, 8, 16, None, None, A, None, None) == OK
+    assert d(A, A, 4, 8, 16, None, None, A, U, None) == MISALIGNED             # workspace
 
 
 def test_chunk_plan_validation(L):
@@ -339,13 +341,14 @@ def test_dual_f16codes_validation(L):
     for i in range(2):
         ga[i] = Branch16(A, A, A, A, None, A, 4, None, None)
     g = L.w8a8_linear_dual_f16codes
-    assert g(None, 8, 16, None) == INVALID
-    assert g(ga, 12, 16, None) == SHAPE
+    assert g(None, 8, 16, None, None) == INVALID
+    assert g(ga, 12, 16, None, None) == SHAPE
+    assert g(ga, 8, 16, U, None) == MISALIGNED                # workspace
     ga[1].chunk_plan = U
-    assert g(ga, 8, 16, None) == MISALIGNED
+    assert g(ga, 8, 16, None, None) == MISALIGNED
     ga[1].chunk_plan = None
     ga[1].Wq = None
-    assert g(ga, 8, 16, None) == INVALID
+    assert g(ga, 8, 16, None, None) == INVALID
     ga[0] = Branch16(None, None, None, None, None, None, 0, None, None)
     ga[1] = Branch16(None, None, None, None, None, None, 0, None, None)
-    assert g(ga, 8, 16, None) == OK                      # both branches empty
+    assert g(ga, 8, 16, None, None) == OK                      # both branches empty
