@@ -211,7 +211,7 @@ METRIC = "W8A8 linear INT8 TOPS (act-quant + INT8 GEMM + fused dequant epilogue)
 # int8-code engine, gemm_ts_*.md for the fp16-code one); valid only for the
 # kernel version profiled there (removed whenever that kernel changes, until
 # the capture is repeated).
-GEMM_TRAFFIC_BYTES = {("ts", "qkv_m4608_k4096_n12288"): 176.97e6}
+GEMM_TRAFFIC_BYTES = {("ts", "qkv_m4608_k4096_n12288"): 196.05e6}
 
 
 # ------------------------------------------------ the other configurations
@@ -222,9 +222,10 @@ _WS = {}
 def _gemm_ws(dev):
     """The fp16-code GEMM's split-K workspace (one per device: every GEMM of
     this benchmark runs on one stream at a time)."""
+    import torch
+    from paper_2606_12280_gb300 import w8a8
     key = str(torch.device(dev))
     if key not in _WS:
-        from paper_2606_12280_gb300 import w8a8
         _WS[key] = w8a8.gemm_workspace(dev)
     return _WS[key]
 
@@ -416,10 +417,13 @@ def run_ours(args):
         else:
             w8a8.quant_act(Xs[j], lam, Xq=Xqs[j], x_scale=sxs[j], stream=st)
 
-    def gemm(j, st):
+    # split: the last partial round of tiles split over K between CTA pairs
+    # (a workspace); the pipelined graph runs without it, because there the
+    # next step's a3 fills the SMs that round leaves idle
+    def gemm(j, st, split=True):
         if f16:
             w8a8.linear_f16codes(Xqs[j], sxs[j], Wqs[j], sw, bias, Y=Ys[j], plan=plan, x_sumsq=sss[j],
-                                 stream=st, workspace=_gemm_ws(dev))
+                                 stream=st, workspace=_gemm_ws(dev) if split else None)
         else:
             w8a8.linear(Xqs[j], sxs[j], Wqs[j], sw, bias, Y=Ys[j], stream=st)
 
@@ -472,7 +476,7 @@ def run_ours(args):
                     q_done = torch.cuda.Event()
                     q_done.record(side)
                 cs.wait_event(q_done)
-                gemm(j, cs)
+                gemm(j, cs, split=False)
                 g_done = torch.cuda.Event()
                 g_done.record(cs)
                 gemm_done.append(g_done)
@@ -885,6 +889,10 @@ def run_ours(args):
                                  "(roofline, act_quant.ms_in_step) from a second pass of K "
                                  "stream-launched steps with events around each kernel",
                        "codes": f"{args.codes} container of the int8 activation codes",
+                       "split_k": ("serial steps, the per-kernel pass (roofline) and the GEMM's sustained "
+                                   "loop split the partial round of tiles over K (workspace); the pipelined "
+                                   "graph does not, its next a3 fills the SMs that round leaves idle")
+                                  if f16 else None,
                        "gemm_engine": {"ts": "tcgen05 cta pair, weights in TMEM, drain plan + token sums, "
                                              "last round of tiles split over K (workspace)",
                                        "tc2": "tcgen05 cta pair", "tc": "tcgen05",
