@@ -228,11 +228,12 @@ W8A8_API w8a8_status w8a8_quant_act_f16codes(const uint16_t *X, const float *smo
  *   workspace: NULL, or w8a8_gemm_workspace_size() bytes of device memory
  *     (16-byte aligned) that the caller zeroed once before its first use.
  *     The output tiles (256 x 256) fill the GPU's CTA pairs in rounds; with a
- *     workspace, as many tiles as a last, partial round would hold (all
- *     tiles, when there are fewer tiles than pairs) are split over K between
- *     pairs in the first round, their int32 partial sums meet in the
- *     workspace, and the part that finishes last adds them (integer sums:
- *     the result is the same bits as without a workspace).  The kernel leaves the workspace's
+ *     workspace and at most 12 full rounds, as many tiles as a last,
+ *     partial round would hold (all tiles, when there are fewer tiles than
+ *     pairs) are split over K between pairs in the first round, their int32
+ *     partial sums meet in the workspace, and the part that finishes last
+ *     adds them (integer sums: the result is the same bits as without a
+ *     workspace).  The kernel leaves the workspace's
  *     counters zero; after a call that returned an error, zero it again.
  *     Calls that overlap in time need workspaces of their own.
  */
