@@ -22,6 +22,7 @@
 #include "host_once.h"
 #include "launch.h"
 #include "tc_ptx.cuh"
+#include "tile_order.cuh"
 
 namespace w8a8 {
 namespace {
@@ -77,9 +78,18 @@ struct Params {
     uint16_t *Y;
     int M, N, K;
     int m_tiles, total_tiles, k_blocks;
+    int n_tiles, group;        // feature tiles; tile order (tile_order.cuh)
     unsigned int *err;
     uint64_t wait_limit_ns;
 };
+
+// Row offsets of tile t's tokens (m0) and features (n0).
+__device__ __forceinline__ void tile_mn(const Params &p, int t, int &m0, int &n0) {
+    int mi, ni;
+    grouped_tile(t, p.m_tiles, p.n_tiles, p.group, mi, ni);
+    m0 = mi * PAIR_M;
+    n0 = ni * PAIR_N;
+}
 
 __device__ __forceinline__ uint32_t bf16_rne_bits(float f) {
     uint32_t u = __float_as_uint(f);
@@ -97,8 +107,8 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
         const uint32_t buf = c & 1;
         if (!mbar_wait_cluster(sb + BAR_ACCFULL + 8 * buf, (c >> 1) & 1, wc, ERR_EPILOGUE)) break;
         tc_fence_after();
-        const int m0 = (t % p.m_tiles) * PAIR_M;
-        const int n0 = (t / p.m_tiles) * PAIR_N;
+        int m0, n0;
+        tile_mn(p, t, m0, n0);
         const int m = m0 + static_cast<int>(rank) * CTA_M + q * 32 + lane;
         const uint32_t base = tmem + (static_cast<uint32_t>(q * 32) << 16) + buf * PAIR_N;
         uint16_t *out = p.Y + (size_t)m * p.N + n0;
@@ -197,8 +207,10 @@ gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
             uint32_t j = 0;
             bool ok = true;
             for (int t = pair; ok && t < p.total_tiles; t += npairs) {
-                const int arow = (t % p.m_tiles) * PAIR_M + static_cast<int>(rank) * CTA_M;
-                const int brow = (t / p.m_tiles) * PAIR_N + static_cast<int>(rank) * CTA_N;
+                int m0, n0;
+                tile_mn(p, t, m0, n0);
+                const int arow = m0 + static_cast<int>(rank) * CTA_M;
+                const int brow = n0 + static_cast<int>(rank) * CTA_N;
                 for (int ks = 0; ks < NS; ++ks, ++j) {
                     const uint32_t st = j % S;
                     if (!mbar_wait_cluster(sb + BAR_EMPTY + 8 * st, ((j / S) & 1) ^ 1, wc, ERR_PRODUCER)) {
@@ -324,8 +336,11 @@ cudaError_t launch_gemm_bf16(const uint16_t *X, const uint16_t *W, const float *
     p.N = N;
     p.K = K;
     p.m_tiles = (M + PAIR_M - 1) / PAIR_M;
-    p.total_tiles = p.m_tiles * ((N + PAIR_N - 1) / PAIR_N);
+    p.n_tiles = (N + PAIR_N - 1) / PAIR_N;
+    p.total_tiles = p.m_tiles * p.n_tiles;
     p.k_blocks = (K + BK - 1) / BK;
+    // tile order (tile_order.cuh): bf16 activations and weights
+    p.group = tile_group(2LL * K * M, 2LL * PAIR_N * K, p.n_tiles);
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
     const int pairs = p.total_tiles < sms / 2 ? p.total_tiles : sms / 2;

@@ -30,6 +30,7 @@
 #include "host_once.h"
 #include "launch.h"
 #include "tc_ptx.cuh"
+#include "tile_order.cuh"
 
 namespace w8a8 {
 namespace {
@@ -104,6 +105,7 @@ struct Params {
     uint16_t *Y;
     int M, N, K;
     int t_tiles, total_tiles, spans;           // spans = K / 256 per tile
+    int f_tiles, group;                        // feature tiles; tile order (tile_order.cuh)
     unsigned int *err;
     uint64_t wait_limit_ns;
 };
@@ -291,8 +293,10 @@ __device__ __forceinline__ void arrive_leader(uint32_t bar, uint32_t rank) {
 }
 
 __device__ __forceinline__ void tile_coords(const Params &p, int t, int &t0, int &f0) {
-    t0 = (t % p.t_tiles) * PAIR_T;
-    f0 = (t / p.t_tiles) * PAIR_F;
+    int ti, fi;
+    grouped_tile(t, p.t_tiles, p.f_tiles, p.group, ti, fi);
+    t0 = ti * PAIR_T;
+    f0 = fi * PAIR_F;
 }
 
 template <int FMT>
@@ -654,7 +658,10 @@ cudaError_t launch_fmt(const uint16_t *X, const uint8_t *Wraw, const float *bias
     p.N = N;
     p.K = K;
     p.t_tiles = (M + PAIR_T - 1) / PAIR_T;
-    p.total_tiles = p.t_tiles * ((N + PAIR_F - 1) / PAIR_F);
+    p.f_tiles = (N + PAIR_F - 1) / PAIR_F;
+    p.total_tiles = p.t_tiles * p.f_tiles;
+    // tile order (tile_order.cuh): bf16 activations, raw blocks of row_bytes per row
+    p.group = tile_group(2LL * K * M, static_cast<long long>(PAIR_F) * row_bytes, p.f_tiles);
     p.spans = static_cast<int>(spans);
     p.err = err;
     p.wait_limit_ns = 2000000000ull;

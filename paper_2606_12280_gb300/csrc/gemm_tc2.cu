@@ -33,6 +33,7 @@
 #include "host_once.h"
 #include "launch.h"
 #include "tc_ptx.cuh"
+#include "tile_order.cuh"
 
 namespace w8a8 {
 namespace {
@@ -147,6 +148,7 @@ struct Params {
     int N, K;
     int total_tiles;
     int k_blocks;
+    int n_tiles, group;        // feature tiles; tile order (tile_order.cuh)
     unsigned int *err;
     uint64_t wait_limit_ns;
 };
@@ -159,9 +161,10 @@ __device__ __forceinline__ Tile tile_coords(const Params &p, int t) {
     Tile r;
     r.branch = t >= p.br[0].tiles ? 1 : 0;
     const int local = t - (r.branch ? p.br[0].tiles : 0);
-    const int mt = p.br[r.branch].m_tiles;
-    r.m0 = (local % mt) * PAIR_M;
-    r.n0 = (local / mt) * PAIR_N;
+    int mi, ni;
+    grouped_tile(local, p.br[r.branch].m_tiles, p.n_tiles, p.group, mi, ni);
+    r.m0 = mi * PAIR_M;
+    r.n0 = ni * PAIR_N;
     return r;
 }
 
@@ -678,6 +681,10 @@ cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K, bool out
     p.K = K;
     p.total_tiles = p.br[0].tiles + p.br[1].tiles;
     p.k_blocks = (K + BK - 1) / BK;
+    // tile order (tile_order.cuh): activation codes of 1 or 2 bytes, int8 weights
+    p.n_tiles = (N + PAIR_N - 1) / PAIR_N;
+    p.group = tile_group((a16 ? 2LL : 1LL) * K * (p.br[0].M > p.br[1].M ? p.br[0].M : p.br[1].M),
+                         static_cast<long long>(PAIR_N) * K, p.n_tiles);
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
     const int pairs = p.total_tiles < sms / 2 ? p.total_tiles : sms / 2;

@@ -45,6 +45,7 @@
 #include "host_once.h"
 #include "launch.h"
 #include "tc_ptx.cuh"
+#include "tile_order.cuh"
 
 namespace w8a8 {
 namespace {
@@ -158,24 +159,15 @@ struct Tile {
     int branch, t0, f0;
 };
 
-// Tile t of the launch's tile space.  Groups of group_f feature blocks in
-// turn; within a group, tile i covers token tile i / Gg and feature block i %
-// Gg of the group (Gg its number of blocks), so the tiles that run at the
-// same time share a few token tiles and the group's weights, which stay in
-// L2 while all token tiles stream past once per group.  With group_f = 1
-// this is the plain order: token tiles fastest.
+// Tile t of the launch's tile space, in the order of tile_order.cuh.
 __device__ __forceinline__ Tile tile_coords(const Params &p, int t) {
     Tile r;
     r.branch = t >= p.br[0].tiles ? 1 : 0;
     const int local = t - (r.branch ? p.br[0].tiles : 0);
-    const int tt = p.br[r.branch].t_tiles;
-    const int G = p.group_f;
-    const int g = local / (G * tt);
-    const int i = local - g * G * tt;
-    const int Gg = min(G, p.f_tiles - g * G);
-    const int ti = i / Gg;
+    int ti, fi;
+    grouped_tile(local, p.br[r.branch].t_tiles, p.f_tiles, p.group_f, ti, fi);
     r.t0 = ti * PAIR_T;
-    r.f0 = (g * G + (i - ti * Gg)) * PAIR_F;
+    r.f0 = fi * PAIR_F;
     return r;
 }
 
@@ -906,7 +898,6 @@ cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cu
 namespace {
 constexpr size_t kWsCounterBytes(int pairs) { return ((size_t)pairs * 16 * 4 + 255) / 256 * 256; }
 constexpr int kSplitMaxRounds = 12;
-constexpr long long kL2ResidentBytes = 48ll << 20;    // what the order plans to keep in L2
 }  // namespace
 
 long long gemm_ts_workspace_bytes() {
@@ -956,23 +947,10 @@ cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_
     p.N = N;
     p.K = K;
     p.total_tiles = p.br[0].tiles + p.br[1].tiles;
-    // While a branch's activation codes fit in L2 with room to spare, token
-    // tiles go fastest (the codes stay resident, every weight block is read
-    // once); beyond that, groups of feature blocks whose weights fit in L2
-    // (~40 MB) keep the weights resident while the codes stream past once per
-    // group, instead of once per round of tiles.
+    // tile order (tile_order.cuh): the codes are 2 bytes, the weights 1
     p.f_tiles = f_tiles;
-    p.group_f = 1;
-    {
-        const long long codes_bytes = 2LL * K * (p.br[0].M > p.br[1].M ? p.br[0].M : p.br[1].M);
-        if (codes_bytes > kL2ResidentBytes) {
-            const long long block_bytes = static_cast<long long>(PAIR_F) * K;
-            long long g = kL2ResidentBytes * 5 / 6 / block_bytes;
-            if (g < 1) g = 1;
-            if (g > f_tiles) g = f_tiles;
-            p.group_f = static_cast<int>(g);
-        }
-    }
+    p.group_f = tile_group(2LL * K * (p.br[0].M > p.br[1].M ? p.br[0].M : p.br[1].M),
+                           static_cast<long long>(PAIR_F) * K, f_tiles);
     p.k_blocks = (K + BK - 1) / BK;
     p.plan_words = chunk_plan_words(K);
     p.single_ok = 1;

@@ -88,3 +88,46 @@ def test_grouped_order_dual(w8):
     acc = w8.debug_gemm_f16codes_i32(brs[1][0], brs[1][2], plan=brs[1][5])
     assert torch.equal(singles[1].view(torch.int16),
                        epilogue(acc, brs[1][1], brs[1][3], brs[1][4]).view(torch.int16))
+
+
+# ------------------------------------------- the other engines, same order
+
+def test_grouped_order_int8_engine(w8):
+    # int8 codes of 12800 x 4096 (52 MB): above the threshold for 1-byte codes
+    M, N, K = 12800, 1040, 4096
+    q, w, sx, sw, b = operands(M, N, K, 21)
+    acc = w8.debug_gemm_i32(q.to(torch.int8), w.to(torch.int8))
+    assert torch.equal(acc.to(torch.int64), exact_product(q, w))
+    Y = w8.linear(q.to(torch.int8), sx, w.to(torch.int8), sw, b)
+    assert torch.equal(Y.view(torch.int16), epilogue(acc, sx, sw, b).view(torch.int16))
+
+
+def test_grouped_order_bf16_layer(w8):
+    # bf16 activations of 6400 x 4096 (52 MB): within half a bf16 ulp plus the
+    # fp32 accumulation bound (K/16 + 16) 2^-22 sum |x w| of the exact product
+    M, N, K = 6400, 2304, 4096
+    g = torch.Generator(device=DEV).manual_seed(5)
+    X = torch.randn(M, K, generator=g, device=DEV).to(torch.bfloat16)
+    W = (torch.randn(N, K, generator=g, device=DEV) * 0.05).to(torch.bfloat16)
+    b = torch.randn(N, generator=g, device=DEV) * 0.1
+    Y = w8.linear_bf16(X, W, b).double()
+    Xd, Wd = X.double(), W.double()
+    ref = Xd @ Wd.T + b.double()[None, :]
+    absum = Xd.abs() @ Wd.abs().T
+    ulp = torch.pow(2.0, torch.floor(torch.log2(ref.abs().clamp_min(1e-30))) - 7)
+    bound = 0.5 * ulp + (K / 16 + 16) * 2.0 ** -22 * absum + 1e-30
+    assert bool(((Y - ref).abs() <= bound).all())
+
+
+@pytest.mark.parametrize("fmt", [0, 1])
+def test_grouped_order_gguf_equals_bf16_layer(w8, fmt):
+    # the GGUF layer equals the bf16 layer on its decoded weights bitwise,
+    # whatever order either visits its tiles in
+    from paper_2606_12280_gb300 import workloads as wl
+    M, N, K = 6400, 1024, 4096
+    raw = torch.from_numpy(wl.random_gguf(fmt, N, K, seed=fmt + 3)).to(DEV)
+    g = torch.Generator(device=DEV).manual_seed(9)
+    X = torch.randn(M, K, generator=g, device=DEV).to(torch.bfloat16)
+    b = torch.randn(N, generator=g, device=DEV) * 0.1
+    Wd = w8.debug_gguf_dequant(raw, fmt, N, K)
+    assert torch.equal(w8.linear_gguf(X, raw, fmt, N, b), w8.linear_bf16(X, Wd, b))
