@@ -159,15 +159,25 @@ struct Tile {
     int branch, t0, f0;
 };
 
-// Tile t of the launch's tile space, in the order of tile_order.cuh.
+// Tile t of the launch's tile space: token tiles fastest, or (GROUPED) in
+// groups of feature blocks as tile_order.cuh describes.  The plain order is
+// its own instantiation: the benchmarked shapes use it, and a kernel whose
+// tile loop carried the grouped arithmetic measured ~1 % slower on them.
+template <bool GROUPED>
 __device__ __forceinline__ Tile tile_coords(const Params &p, int t) {
     Tile r;
     r.branch = t >= p.br[0].tiles ? 1 : 0;
     const int local = t - (r.branch ? p.br[0].tiles : 0);
-    int ti, fi;
-    grouped_tile(local, p.br[r.branch].t_tiles, p.f_tiles, p.group_f, ti, fi);
-    r.t0 = ti * PAIR_T;
-    r.f0 = fi * PAIR_F;
+    const int tt = p.br[r.branch].t_tiles;
+    if (GROUPED) {
+        int ti, fi;
+        grouped_tile(local, tt, p.f_tiles, p.group_f, ti, fi);
+        r.t0 = ti * PAIR_T;
+        r.f0 = fi * PAIR_F;
+    } else {
+        r.t0 = (local % tt) * PAIR_T;
+        r.f0 = (local / tt) * PAIR_F;
+    }
     return r;
 }
 
@@ -213,8 +223,9 @@ __device__ __forceinline__ bool plan_drains(const Params &p, const uint32_t *pla
 // so max_t ||a_t||^2 * max_f ||w_f||^2 <= 2^48 over the tile's 256 tokens and
 // 256 weight rows keeps every one within 2^24, exact in fp32.  Warp-wide: all
 // lanes take part.
+template <bool GROUPED>
 __device__ __forceinline__ bool tile_single_run(const Params &p, int t, int lane) {
-    const Tile tl = tile_coords(p, t);
+    const Tile tl = tile_coords<GROUPED>(p, t);
     const BranchArgs &br = p.br[tl.branch];
     uint32_t m = 0;
 #pragma unroll
@@ -270,7 +281,7 @@ __device__ __forceinline__ void arrive_leader(uint32_t bar, uint32_t rank) {
     else mbar_arrive_cluster_relaxed(mapa_shared(bar, 0));
 }
 
-template <bool OUT_I32>
+template <bool OUT_I32, bool GROUPED>
 __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint32_t tmem,
                                               const WaitCtx &wc, int warp, int lane, int NC,
                                               uint32_t rank, int pair, int npairs) {
@@ -289,13 +300,13 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
             mbar_arrive(sb + BAR_TFLAG + 8 * (n & 1));
         }
     };
-    bool single = use_single && pair < p.total_units && tile_single_run(p, unit_coords(p, pair, NC).tile, lane);
+    bool single = use_single && pair < p.total_units && tile_single_run<GROUPED>(p, unit_coords(p, pair, NC).tile, lane);
     if (pair < p.total_units) publish(0, single);
     int n = 0;                         // units so far
     for (int u = pair; ok && u < p.total_units; u += npairs, ++n) {
         const Unit un = unit_coords(p, u, NC);
         const int t = un.tile;
-        const Tile tc = tile_coords(p, t);
+        const Tile tc = tile_coords<GROUPED>(p, t);
         const int fb = tc.f0 / PAIR_F;
         const uint32_t *plan = p.br[tc.branch].plan;
         int32_t run[RUN];
@@ -354,7 +365,7 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
         bool raw = single;
         if (use_single) {
             const int un_next = u + npairs;
-            single = un_next < p.total_units && tile_single_run(p, unit_coords(p, un_next, NC).tile, lane);
+            single = un_next < p.total_units && tile_single_run<GROUPED>(p, unit_coords(p, un_next, NC).tile, lane);
             if (un_next < p.total_units) publish(n + 1, single);
         }
         if (un.slot >= 0) {
@@ -410,7 +421,7 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
                 run[i] = static_cast<int32_t>(__float_as_uint(__int2float_rn(run[i])));
             }
         }
-        const Tile tl = tile_coords(p, t);
+        const Tile tl = tile_coords<GROUPED>(p, t);
         const BranchArgs &br = p.br[tl.branch];
         const int f = tl.f0 + static_cast<int>(rank) * CTA_F + q * 32 + lane;   // output feature
         const int tok0 = tl.t0 + h * (PAIR_T / 2);
@@ -489,7 +500,7 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
     }
 }
 
-template <bool OUT_I32>
+template <bool OUT_I32, bool GROUPED>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(THREADS, 1)
 gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__ CUtensorMap tmW0,
                const __grid_constant__ CUtensorMap tmX1, const __grid_constant__ CUtensorMap tmW1,
@@ -544,7 +555,7 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
 
     if (warp >= 8) {
         asm volatile("setmaxnreg.inc.sync.aligned.u32 %0;" ::"n"(REGS_HIGH));
-        if (run_ok) epilogue_role<OUT_I32>(p, sb, tmem, wc, warp, lane, NC, rank, pair, npairs);
+        if (run_ok) epilogue_role<OUT_I32, GROUPED>(p, sb, tmem, wc, warp, lane, NC, rank, pair, npairs);
     } else {
         asm volatile("setmaxnreg.dec.sync.aligned.u32 %0;" ::"n"(REGS_LOW));
         if (!run_ok) {
@@ -555,7 +566,7 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
                 bool ok = true;
                 for (int u = pair; ok && u < p.total_units; u += npairs) {
                     const Unit un = unit_coords(p, u, NC);
-                    const Tile tl = tile_coords(p, un.tile);
+                    const Tile tl = tile_coords<GROUPED>(p, un.tile);
                     const CUtensorMap *mW = tl.branch ? &tmW1 : &tmW0;
                     const int frow = tl.f0 + static_cast<int>(rank) * CTA_F;
                     const int ks_end = min(NS, un.ci1 * KC_STAGES);
@@ -586,7 +597,7 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
                 bool ok = true;
                 for (int u = pair; ok && u < p.total_units; u += npairs) {
                     const Unit un = unit_coords(p, u, NC);
-                    const Tile tl = tile_coords(p, un.tile);
+                    const Tile tl = tile_coords<GROUPED>(p, un.tile);
                     const CUtensorMap *mX = tl.branch ? &tmX1 : &tmX0;
                     const int trow = tl.t0 + static_cast<int>(rank) * CTA_T;
                     const int ks_end = min(NS, un.ci1 * KC_STAGES);
@@ -619,7 +630,7 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
                 int n = 0;                     // units so far
                 for (int u = pair; ok && u < p.total_units; u += npairs, ++n) {
                     const Unit un = unit_coords(p, u, NC);
-                    const Tile tc = tile_coords(p, un.tile);
+                    const Tile tc = tile_coords<GROUPED>(p, un.tile);
                     const int fb = tc.f0 / PAIR_F;
                     const uint32_t *plan = p.br[tc.branch].plan;
                     bool single = false;       // the tile is one run (published by the epilogue)
@@ -861,17 +872,17 @@ bool make_map(CUtensorMap *m, CUtensorMapDataType dt, const void *base, uint64_t
 // Per variant and device: the dynamic shared memory limit set and the
 // registers ptxas gave the kernel (the register split assumes exactly
 // LAUNCH_REGS at launch).
-template <bool OUT_I32>
+template <bool OUT_I32, bool GROUPED>
 cudaError_t prepare_ts_kernel() {
     static PerDevice<int> regs;
     int n = 0;
     cudaError_t e = regs.get([](int &v) {
         cudaFuncAttributes fa;
-        cudaError_t r = cudaFuncGetAttributes(&fa, gemm_ts_kernel<OUT_I32>);
+        cudaError_t r = cudaFuncGetAttributes(&fa, gemm_ts_kernel<OUT_I32, GROUPED>);
         if (r != cudaSuccess) return r;
         v = fa.numRegs;
-        return cudaFuncSetAttribute(gemm_ts_kernel<OUT_I32>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                    SMEM_TOTAL);
+        return cudaFuncSetAttribute(gemm_ts_kernel<OUT_I32, GROUPED>,
+                                    cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_TOTAL);
     }, &n);
     if (e != cudaSuccess) return e;
     return n == LAUNCH_REGS ? cudaSuccess : cudaErrorInvalidConfiguration;
@@ -908,10 +919,6 @@ long long gemm_ts_workspace_bytes() {
 cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, void *workspace,
                            unsigned int *err, cudaStream_t st) {
     const int sms = device_sms();
-    auto kern = out_i32 ? gemm_ts_kernel<true> : gemm_ts_kernel<false>;
-    cudaError_t e = out_i32 ? prepare_ts_kernel<true>() : prepare_ts_kernel<false>();
-    if (e != cudaSuccess) return e;
-
     Params p{};
     CUtensorMap maps[4];
     int first = -1;
@@ -985,6 +992,12 @@ cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_
     }
     p.total_units = p.full_tiles + p.split_tiles * p.split;
     const int pairs = p.total_units < P ? p.total_units : P;
+    const bool grouped = p.group_f > 1;
+    auto kern = out_i32 ? (grouped ? gemm_ts_kernel<true, true> : gemm_ts_kernel<true, false>)
+                        : (grouped ? gemm_ts_kernel<false, true> : gemm_ts_kernel<false, false>);
+    cudaError_t e = out_i32 ? (grouped ? prepare_ts_kernel<true, true>() : prepare_ts_kernel<true, false>())
+                            : (grouped ? prepare_ts_kernel<false, true>() : prepare_ts_kernel<false, false>());
+    if (e != cudaSuccess) return e;
     kern<<<2 * pairs, THREADS, SMEM_TOTAL, st>>>(maps[0], maps[1], maps[2], maps[3], p);
     return cudaGetLastError();
 }

@@ -15,6 +15,11 @@ namespace w8a8 {
 // Token tile ti and feature block fi of tile `local` (G = 1: the plain order,
 // token tile fastest).  A bijection of [0, tt * nf).
 __device__ __forceinline__ void grouped_tile(int local, int tt, int nf, int G, int &ti, int &fi) {
+    if (G == 1) {                      // the plain order, with one division
+        fi = local / tt;
+        ti = local - fi * tt;
+        return;
+    }
     const int g = local / (G * tt);
     const int i = local - g * G * tt;
     const int Gg = min(G, nf - g * G);
