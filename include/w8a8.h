@@ -139,11 +139,30 @@ W8A8_API w8a8_status w8a8_quant_act(const uint16_t *X, const float *smooth, int 
  * The product runs exactly on the fp16 tensor datapath (every int8 is an
  * fp16 value, products are exact in fp32; partial sums of at most 1024
  * products stay below 2^24 and are drained into int32).
+ *   chunk_plan: NULL, or the plan that w8a8_chunk_plan wrote for this Wq
+ *     (same N, K); used with a workspace (see w8a8_linear_f16codes).  A
+ *     plan of other weights voids the exactness guarantee.
+ *   workspace: NULL, or w8a8_linear_workspace_size(M, K) bytes of device
+ *     memory (16-byte aligned) that the caller zeroed once before its first
+ *     use.  Without one, both operands are converted to fp16 in shared
+ *     memory inside the GEMM.  With one, a streaming pass first writes the
+ *     codes as fp16 values and each token's sum of squared codes into it
+ *     (3MK + 4M bytes moved, the fp16 codes left in L2), and the GEMM of
+ *     w8a8_linear_f16codes runs on them (the weights converted into tensor
+ *     memory, the split-K area of the same workspace).  Same bits either
+ *     way.  Calls that overlap in time need workspaces of their own.
  */
 W8A8_API w8a8_status w8a8_linear(const int8_t *Xq, const float *x_scale,
                         const int8_t *Wq, const float *w_scale,
                         const float *bias, int M, int N, int K, uint16_t *Y,
-                        void *stream);
+                        const uint32_t *chunk_plan, void *workspace, void *stream);
+
+/* Bytes of the workspace of w8a8_linear (tokens = M) and w8a8_linear_dual
+ * (tokens = M0 + M1) for K on the current device: 2 * tokens * K for the
+ * fp16 codes, 4 * tokens for the token sums, w8a8_gemm_workspace_size() for
+ * the split-K area, and 1024 bytes of alignment.  0 for tokens < 0 or
+ * K <= 0. */
+W8A8_API long long w8a8_linear_workspace_size(long long tokens, int K);
 
 /* One branch of the dual-branch (classifier-free guidance) layer. */
 typedef struct {
@@ -154,6 +173,7 @@ typedef struct {
     const float *bias;     /* [N] fp32 or NULL */
     uint16_t *Y;           /* [M,N] bf16, written */
     int M;                 /* tokens of this branch, >= 0 */
+    const uint32_t *chunk_plan;  /* this branch's weights' plan or NULL */
 } w8a8_branch;
 
 /*
@@ -164,16 +184,20 @@ typedef struct {
  * own M, activations, weights, scales, bias and output.  Results are
  * bitwise identical to two w8a8_linear calls.
  *   br  host pointer to an array of 2 w8a8_branch (read during the call only).
+ *   workspace: NULL, or w8a8_linear_workspace_size(M0 + M1, K) bytes, as
+ *     for w8a8_linear (one streaming pass for both branches' codes).
  */
 W8A8_API w8a8_status w8a8_linear_dual(const w8a8_branch *br, int N, int K,
-                             void *stream);
+                             void *workspace, void *stream);
 
 /*
  * Test export of a4 alone: acc = Xq Wq^T as int32 [M,N], written, so that the
- * exact integer product can be compared bit for bit.  Same shape rules.
+ * exact integer product can be compared bit for bit.  Same shape rules,
+ * chunk_plan and workspace as w8a8_linear.
  */
 W8A8_API w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int M,
-                                int N, int K, int32_t *acc, void *stream);
+                                int N, int K, int32_t *acc, const uint32_t *chunk_plan,
+                                void *workspace, void *stream);
 
 /*
  * Test anchors (no counterpart in the paper): the same exact-integer product

@@ -79,6 +79,19 @@ w8a8_status run_gemm(const w8a8::GemmBranch *br, int nb, int N, int K, bool out_
     return from_cuda(w8a8::launch_gemm_tc2(br, nb, N, K, out_i32, false, err, st));
 }
 
+// The same with a workspace: the codes expanded to fp16 values (with token
+// sums) by a streaming pass, then the GEMM with the weights in tensor memory.
+w8a8_status run_gemm_ws(const w8a8::GemmBranch *br, int nb, int N, int K, bool out_i32, void *workspace,
+                        cudaStream_t st) {
+    if (!workspace) return run_gemm(br, nb, N, K, out_i32, st);
+    if (!aligned16(workspace)) return W8A8_ERR_MISALIGNED;
+    for (int i = 0; i < nb; ++i)
+        if (br[i].M > 0 && br[i].plan && !aligned16(br[i].plan)) return W8A8_ERR_MISALIGNED;
+    unsigned int *err = device_error_word();
+    if (!err) return W8A8_ERR_CUDA;
+    return from_cuda(w8a8::launch_linear_codes8(br, nb, N, K, out_i32, workspace, err, st));
+}
+
 // The same product on the earlier engines, kept as test anchors and never on
 // a product call: 1 = tcgen05 on single SMs, 0 = mma.sync s8; 2 is the
 // product engine.
@@ -148,37 +161,44 @@ w8a8_status w8a8_quant_act(const uint16_t *X, const float *smooth, int M, int K,
 
 w8a8_status w8a8_linear(const int8_t *Xq, const float *x_scale, const int8_t *Wq,
                         const float *w_scale, const float *bias, int M, int N, int K,
-                        uint16_t *Y, void *stream) {
+                        uint16_t *Y, const uint32_t *chunk_plan, void *workspace, void *stream) {
     if (w8a8_status e = check_nk(N, K)) return e;
     if (w8a8_status e = check_mk(M, K)) return e;
-    w8a8::GemmBranch b{Xq, x_scale, Wq, w_scale, bias, Y, M};
+    w8a8::GemmBranch b{Xq, x_scale, Wq, w_scale, bias, Y, M, nullptr, chunk_plan};
     if (w8a8_status e = check_branch(b, true, N, K)) return e;
+    if (workspace && !aligned16(workspace)) return W8A8_ERR_MISALIGNED;
     if (M == 0) return W8A8_OK;
-    return run_gemm(&b, 1, N, K, false, as_stream(stream));
+    return run_gemm_ws(&b, 1, N, K, false, workspace, as_stream(stream));
 }
 
-w8a8_status w8a8_linear_dual(const w8a8_branch *br, int N, int K, void *stream) {
+long long w8a8_linear_workspace_size(long long tokens, int K) {
+    return w8a8::linear_codes8_workspace_bytes(tokens, K);
+}
+
+w8a8_status w8a8_linear_dual(const w8a8_branch *br, int N, int K, void *workspace, void *stream) {
     if (!br) return W8A8_ERR_INVALID_ARG;
     if (w8a8_status e = check_nk(N, K)) return e;
+    if (workspace && !aligned16(workspace)) return W8A8_ERR_MISALIGNED;
     w8a8::GemmBranch b[2];
     for (int i = 0; i < 2; ++i) {
         b[i] = w8a8::GemmBranch{br[i].Xq, br[i].x_scale, br[i].Wq, br[i].w_scale,
-                                br[i].bias, br[i].Y, br[i].M};
+                                br[i].bias, br[i].Y, br[i].M, nullptr, br[i].chunk_plan};
         if (w8a8_status e = check_mk(br[i].M, K)) return e;
         if (w8a8_status e = check_branch(b[i], true, N, K)) return e;
     }
     if (b[0].M == 0 && b[1].M == 0) return W8A8_OK;
-    return run_gemm(b, 2, N, K, false, as_stream(stream));
+    return run_gemm_ws(b, 2, N, K, false, workspace, as_stream(stream));
 }
 
 w8a8_status w8a8_debug_gemm_i32(const int8_t *Xq, const int8_t *Wq, int M, int N, int K,
-                                int32_t *acc, void *stream) {
+                                int32_t *acc, const uint32_t *chunk_plan, void *workspace, void *stream) {
     if (w8a8_status e = check_nk(N, K)) return e;
     if (w8a8_status e = check_mk(M, K)) return e;
-    w8a8::GemmBranch b{Xq, nullptr, Wq, nullptr, nullptr, acc, M};
+    w8a8::GemmBranch b{Xq, nullptr, Wq, nullptr, nullptr, acc, M, nullptr, chunk_plan};
     if (w8a8_status e = check_branch(b, false, N, K)) return e;
+    if (workspace && !aligned16(workspace)) return W8A8_ERR_MISALIGNED;
     if (M == 0) return W8A8_OK;
-    return run_gemm(&b, 1, N, K, true, as_stream(stream));
+    return run_gemm_ws(&b, 1, N, K, true, workspace, as_stream(stream));
 }
 
 w8a8_status w8a8_debug_linear_engine(int engine, const w8a8_branch *br, int nb, int N, int K, int out_i32,
@@ -187,7 +207,8 @@ w8a8_status w8a8_debug_linear_engine(int engine, const w8a8_branch *br, int nb, 
     if (w8a8_status e = check_nk(N, K)) return e;
     w8a8::GemmBranch b[2];
     for (int i = 0; i < nb; ++i) {
-        b[i] = w8a8::GemmBranch{br[i].Xq, br[i].x_scale, br[i].Wq, br[i].w_scale, br[i].bias, br[i].Y, br[i].M};
+        b[i] = w8a8::GemmBranch{br[i].Xq, br[i].x_scale, br[i].Wq, br[i].w_scale, br[i].bias, br[i].Y, br[i].M,
+                                nullptr, nullptr};
         if (w8a8_status e = check_mk(br[i].M, K)) return e;
         if (w8a8_status e = check_branch(b[i], out_i32 == 0, N, K)) return e;
     }

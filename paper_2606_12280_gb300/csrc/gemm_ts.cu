@@ -835,6 +835,63 @@ chunk_plan_kernel(const int8_t *__restrict__ Wq, int N, int K, int NC, int words
     }
 }
 
+// ------------------------------------------ int8 codes into this engine
+//
+// The int8 codes that a3 writes (w8a8_quant_act) reach this engine through
+// one streaming pass: each warp takes one token row, reads its codes 8 per
+// lane (256 bytes per warp instruction), writes them as fp16 values (the
+// weights' conversion; 512 bytes per store instruction) and sums their
+// squares exactly with dp4a: |code| <= 128 and K < 2^18 keep every sum
+// below 2^32, and the int32 adds wrap like the uint32 ones.  The fp16 codes
+// (2MK bytes) are written back into L2, where the GEMM that follows finds
+// them.  One launch covers both branches of a dual call: rows [0, M0) are
+// branch 0's, the rest branch 1's.
+struct ExpandBranch {
+    const int8_t *Xq;
+    uint16_t *Xq16;
+    uint32_t *sumsq;
+    int M;
+};
+
+constexpr int kExpandThreads = 256;
+constexpr int kExpandBatch = 16;                      // 8-code loads in flight per lane
+
+__global__ void __launch_bounds__(kExpandThreads)
+expand_codes_kernel(const __grid_constant__ ExpandBranch b0, const __grid_constant__ ExpandBranch b1, int K) {
+    const int lane = threadIdx.x & 31;
+    int row = (blockIdx.x * kExpandThreads + threadIdx.x) >> 5;
+    const bool second = row >= b0.M;
+    const ExpandBranch &b = second ? b1 : b0;
+    if (second) row -= b0.M;
+    if (row >= b.M) return;                           // whole warps leave together
+    const int n8 = K / 8;                             // 8-code groups per row
+    const uint2 *src = reinterpret_cast<const uint2 *>(b.Xq + (size_t)row * K);
+    uint4 *dst = reinterpret_cast<uint4 *>(b.Xq16 + (size_t)row * K);
+    int ss = 0;
+    for (int g0 = 0; g0 < n8; g0 += 32 * kExpandBatch) {
+        uint2 v[kExpandBatch];
+#pragma unroll
+        for (int i = 0; i < kExpandBatch; ++i) {
+            const int g = g0 + i * 32 + lane;
+            v[i] = g < n8 ? __ldcs(src + g) : make_uint2(0u, 0u);
+        }
+#pragma unroll
+        for (int i = 0; i < kExpandBatch; ++i) {
+            const int g = g0 + i * 32 + lane;
+            if (g < n8) {
+                uint4 o;
+                i8x4_to_f16x4(v[i].x, o.x, o.y);
+                i8x4_to_f16x4(v[i].y, o.z, o.w);
+                dst[g] = o;
+                ss = __dp4a(static_cast<int>(v[i].x), static_cast<int>(v[i].x), ss);
+                ss = __dp4a(static_cast<int>(v[i].y), static_cast<int>(v[i].y), ss);
+            }
+        }
+    }
+    const uint32_t t = __reduce_add_sync(0xffffffffu, static_cast<uint32_t>(ss));
+    if (lane == 0) b.sumsq[row] = t;
+}
+
 // ------------------------------------------------------------------ host
 
 typedef CUresult (*EncodeTiledFn)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *,
@@ -1000,6 +1057,51 @@ cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_
     if (e != cudaSuccess) return e;
     kern<<<2 * pairs, THREADS, SMEM_TOTAL, st>>>(maps[0], maps[1], maps[2], maps[3], p);
     return cudaGetLastError();
+}
+
+// The int8-code linear on this engine.  Workspace layout: the split-K area
+// (gemm_ts_workspace_bytes(), first, so that its counters stay where the
+// caller zeroed them), then each branch's fp16 codes and each branch's
+// token sums, every piece starting on a 256-byte boundary.
+namespace {
+constexpr size_t round256(size_t n) { return (n + 255) / 256 * 256; }
+}  // namespace
+
+long long linear_codes8_workspace_bytes(long long tokens, int K) {
+    if (tokens < 0 || K <= 0) return 0;
+    return gemm_ts_workspace_bytes() + 2 * tokens * K + 4 * tokens + 4 * 256;
+}
+
+cudaError_t launch_linear_codes8(const GemmBranch *br, int nb, int N, int K, bool out_i32, void *workspace,
+                                 unsigned int *err, cudaStream_t st) {
+    char *w = static_cast<char *>(workspace);
+    size_t off = static_cast<size_t>(gemm_ts_workspace_bytes());
+    ExpandBranch eb[2] = {{nullptr, nullptr, nullptr, 0}, {nullptr, nullptr, nullptr, 0}};
+    GemmBranch gb[2];
+    for (int i = 0; i < nb; ++i) {
+        gb[i] = br[i];
+        if (br[i].M <= 0) continue;
+        eb[i].Xq = br[i].Xq;
+        eb[i].M = br[i].M;
+        eb[i].Xq16 = reinterpret_cast<uint16_t *>(w + off);
+        off += round256(2 * static_cast<size_t>(br[i].M) * K);
+    }
+    for (int i = 0; i < nb; ++i) {
+        if (br[i].M <= 0) continue;
+        eb[i].sumsq = reinterpret_cast<uint32_t *>(w + off);
+        off += round256(4 * static_cast<size_t>(br[i].M));
+        gb[i].Xq = reinterpret_cast<const int8_t *>(eb[i].Xq16);
+        gb[i].x_sumsq = eb[i].sumsq;
+    }
+    const long long rows = static_cast<long long>(eb[0].M) + eb[1].M;
+    if (rows == 0) return cudaSuccess;
+    const int rows_per_block = kExpandThreads / 32;
+    const long long blocks = (rows + rows_per_block - 1) / rows_per_block;
+    if (blocks > 0x7fffffffLL) return cudaErrorInvalidValue;
+    expand_codes_kernel<<<static_cast<unsigned int>(blocks), kExpandThreads, 0, st>>>(eb[0], eb[1], K);
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    return launch_gemm_ts(gb, nb, N, K, out_i32, workspace, err, st);
 }
 
 }  // namespace w8a8

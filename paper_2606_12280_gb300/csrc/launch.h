@@ -81,6 +81,13 @@ cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K,
 cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_i32, void *workspace,
                            unsigned int *err, cudaStream_t st);
 long long gemm_ts_workspace_bytes();
+// The same engine on int8 codes: one streaming pass writes each branch's
+// codes as fp16 values and its token sums of squares into the workspace
+// (linear_codes8_workspace_bytes(M0 + M1, K) bytes, the split-K counters
+// zeroed once), then the GEMM above runs on them with the branch's plan.
+long long linear_codes8_workspace_bytes(long long tokens, int K);
+cudaError_t launch_linear_codes8(const GemmBranch *br, int nb, int N, int K, bool out_i32, void *workspace,
+                                 unsigned int *err, cudaStream_t st);
 int chunk_plan_words(int K);    // per block of 256 weight rows
 cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cudaStream_t st);
 

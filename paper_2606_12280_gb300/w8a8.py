@@ -29,9 +29,10 @@ SIGNATURES = {
     "w8a8_smooth_scales": [_P, _P, _I, _I, _F, _P, _P],
     "w8a8_quantize_weights": [_P, _P, _I, _I, _P, _P, _P],
     "w8a8_quant_act": [_P, _P, _I, _I, _P, _P, _P],
-    "w8a8_linear": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P],
-    "w8a8_linear_dual": [_P, _I, _I, _P],
-    "w8a8_debug_gemm_i32": [_P, _P, _I, _I, _I, _P, _P],
+    "w8a8_linear": [_P, _P, _P, _P, _P, _I, _I, _I, _P, _P, _P, _P],
+    "w8a8_linear_workspace_size": [ctypes.c_longlong, _I],
+    "w8a8_linear_dual": [_P, _I, _I, _P, _P],
+    "w8a8_debug_gemm_i32": [_P, _P, _I, _I, _I, _P, _P, _P, _P],
     "w8a8_debug_linear_engine": [_I, _P, _I, _I, _I, _I, _P],
     "w8a8_device_status": [_P, ctypes.POINTER(ctypes.c_uint32)],
     "w8a8_debug_wait_timeout": [ctypes.c_uint32, _P],
@@ -72,7 +73,7 @@ class W8A8Error(RuntimeError):
 class Branch(ctypes.Structure):
     """Mirror of ``w8a8_branch``."""
     _fields_ = [("Xq", _P), ("x_scale", _P), ("Wq", _P), ("w_scale", _P),
-                ("bias", _P), ("Y", _P), ("M", _I)]
+                ("bias", _P), ("Y", _P), ("M", _I), ("chunk_plan", _P)]
 
 
 class ActBranch(ctypes.Structure):
@@ -118,6 +119,7 @@ def lib() -> ctypes.CDLL:
             L.w8a8_status_string.restype = ctypes.c_char_p
             L.w8a8_chunk_plan_size.restype = ctypes.c_longlong
             L.w8a8_gemm_workspace_size.restype = ctypes.c_longlong
+            L.w8a8_linear_workspace_size.restype = ctypes.c_longlong
             _lib = L
     return _lib
 
@@ -227,8 +229,11 @@ def _check_weights(Wq, N, K):
         raise ValueError(f"Wq has shape {tuple(Wq.shape)}, the activations need ({N}, {K})")
 
 
-def linear(Xq, x_scale, Wq, w_scale, bias=None, Y=None, stream=None):
-    """Y = bf16((Xq Wq^T) * sx * sw + b): [M,N] bf16."""
+def linear(Xq, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, workspace=None, stream=None):
+    """Y = bf16((Xq Wq^T) * sx * sw + b): [M,N] bf16.  workspace: None, or
+    ``linear_workspace(M, K)`` (the codes are then expanded to fp16 values
+    and run on the GEMM of ``linear_f16codes``, with ``plan`` =
+    ``chunk_plan(Wq)`` or None; same bits)."""
     M, K = Xq.shape
     N = Wq.shape[0]
     _check_weights(Wq, N, K)
@@ -238,21 +243,49 @@ def linear(Xq, x_scale, Wq, w_scale, bias=None, Y=None, stream=None):
     _room(w_scale, N, "w_scale")
     _room(bias, N, "bias")
     _room(Y, M * N, "Y")
+    if plan is not None:
+        _room(plan, chunk_plan_size(N, K), "plan")
     _check("w8a8_linear", lib().w8a8_linear(
         _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"),
         _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
         _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(Y, torch.bfloat16, "Y"),
-        _stream(stream)))
+        _ptr(plan, torch.int32, "plan"), _linear_ws(workspace, M, K), _stream(stream)))
     return Y
+
+
+def linear_workspace_size(tokens: int, K: int) -> int:
+    """Bytes of the workspace of ``linear`` (tokens = M) or ``linear_dual``
+    (tokens = M0 + M1) on the current device."""
+    return int(lib().w8a8_linear_workspace_size(int(tokens), int(K)))
+
+
+def linear_workspace(tokens: int, K: int, device=None):
+    """A zeroed workspace for ``linear`` / ``linear_dual`` with up to `tokens`
+    tokens of K channels (a uint8 tensor; calls that overlap in time need
+    their own)."""
+    device = torch.device("cuda", torch.cuda.current_device()) if device is None else torch.device(device)
+    with torch.cuda.device(device):
+        return torch.zeros(linear_workspace_size(tokens, K), dtype=torch.uint8, device=device)
+
+
+def _linear_ws(ws, tokens, K):
+    if ws is None:
+        return None
+    if ws.dtype != torch.uint8 or ws.numel() < linear_workspace_size(tokens, K):
+        raise ValueError("workspace: a uint8 tensor of linear_workspace_size(tokens, K) bytes "
+                         "(linear_workspace())")
+    return _ptr(ws, torch.uint8, "workspace")
 
 
 def _branch_array(branches, Ys, out_dtype=torch.bfloat16):
     """Branch structs for two (or one) branches (Xq, x_scale, Wq, w_scale,
-    bias); returns (array, outputs, N, K)."""
+    bias[, plan]); returns (array, outputs, N, K)."""
     N, K = branches[0][2].shape
     arr = (Branch * len(branches))()
     out = []
-    for i, (Xq, sx, Wq, sw, b) in enumerate(branches):
+    for i, br in enumerate(branches):
+        Xq, sx, Wq, sw, b = br[:5]
+        plan = br[5] if len(br) > 5 else None
         if tuple(Wq.shape) != (N, K) or Xq.shape[1] != K:
             raise ValueError("branches must share N and K")
         M = Xq.shape[0]
@@ -261,34 +294,44 @@ def _branch_array(branches, Ys, out_dtype=torch.bfloat16):
         _room(sw, N, "w_scale")
         _room(b, N, "bias")
         _room(Y, M * N, "Y")
+        if plan is not None:
+            _room(plan, chunk_plan_size(N, K), "plan")
         arr[i] = Branch(_ptr(Xq, torch.int8, "Xq"), _ptr(sx, torch.float32, "x_scale"),
                         _ptr(Wq, torch.int8, "Wq"), _ptr(sw, torch.float32, "w_scale"),
-                        _ptr(b, torch.float32, "bias"), _ptr(Y, out_dtype, "Y"), M)
+                        _ptr(b, torch.float32, "bias"), _ptr(Y, out_dtype, "Y"), M,
+                        _ptr(plan, torch.int32, "plan"))
         out.append(Y)
     return arr, out, N, K
 
 
-def linear_dual(branches, Ys=None, stream=None):
+def linear_dual(branches, Ys=None, workspace=None, stream=None):
     """One grouped launch over two branches.  branches: two tuples
-    (Xq, x_scale, Wq, w_scale, bias); returns [Y_cond, Y_uncond]."""
+    (Xq, x_scale, Wq, w_scale, bias[, plan]); workspace: None or
+    ``linear_workspace(M0 + M1, K)``; returns [Y_cond, Y_uncond]."""
     if len(branches) != 2:
         raise ValueError("linear_dual takes exactly two branches")
     arr, out, N, K = _branch_array(branches, Ys)
-    _check("w8a8_linear_dual", lib().w8a8_linear_dual(arr, N, K, _stream(stream)))
+    tokens = sum(int(br[0].shape[0]) for br in branches)
+    _check("w8a8_linear_dual", lib().w8a8_linear_dual(arr, N, K, _linear_ws(workspace, tokens, K),
+                                                       _stream(stream)))
     return out
 
 
-def debug_gemm_i32(Xq, Wq, acc=None, stream=None):
-    """Exact int32 acc = Xq Wq^T (test export of the GEMM alone)."""
+def debug_gemm_i32(Xq, Wq, acc=None, plan=None, workspace=None, stream=None):
+    """Exact int32 acc = Xq Wq^T (test export of the GEMM alone; plan and
+    workspace as for ``linear``)."""
     M, K = Xq.shape
     N = Wq.shape[0]
     _check_weights(Wq, N, K)
     if acc is None:
         acc = torch.empty(M, N, dtype=torch.int32, device=Xq.device)
     _room(acc, M * N, "acc")
+    if plan is not None:
+        _room(plan, chunk_plan_size(N, K), "plan")
     _check("w8a8_debug_gemm_i32", lib().w8a8_debug_gemm_i32(
         _ptr(Xq, torch.int8, "Xq"), _ptr(Wq, torch.int8, "Wq"), M, N, K,
-        _ptr(acc, torch.int32, "acc"), _stream(stream)))
+        _ptr(acc, torch.int32, "acc"), _ptr(plan, torch.int32, "plan"), _linear_ws(workspace, M, K),
+        _stream(stream)))
     return acc
 
 

@@ -94,35 +94,51 @@ def test_weight_and_smooth_validation(L):
 
 def test_linear_validation(L):
     f = L.w8a8_linear
-    assert f(A, A, A, A, None, 4, 12, 16, A, None) == SHAPE     # N % 8
-    assert f(A, A, A, A, None, 4, 8, 24, A, None) == SHAPE      # K % 16
-    assert f(A, A, A, A, None, -2, 8, 16, A, None) == SHAPE
-    assert f(None, A, A, A, None, 4, 8, 16, A, None) == INVALID
-    assert f(A, None, A, A, None, 4, 8, 16, A, None) == INVALID
-    assert f(A, A, A, A, None, 4, 8, 16, None, None) == INVALID
-    assert f(A, A, U, A, None, 4, 8, 16, A, None) == MISALIGNED
-    assert f(A, A, A, A, U, 4, 8, 16, A, None) == MISALIGNED    # bias
-    assert f(A, A, A, A, None, 0, 8, 16, A, None) == OK          # empty batch
+    assert f(A, A, A, A, None, 4, 12, 16, A, None, None, None) == SHAPE     # N % 8
+    assert f(A, A, A, A, None, 4, 8, 24, A, None, None, None) == SHAPE      # K % 16
+    assert f(A, A, A, A, None, -2, 8, 16, A, None, None, None) == SHAPE
+    assert f(None, A, A, A, None, 4, 8, 16, A, None, None, None) == INVALID
+    assert f(A, None, A, A, None, 4, 8, 16, A, None, None, None) == INVALID
+    assert f(A, A, A, A, None, 4, 8, 16, None, None, None, None) == INVALID
+    assert f(A, A, U, A, None, 4, 8, 16, A, None, None, None) == MISALIGNED
+    assert f(A, A, A, A, U, 4, 8, 16, A, None, None, None) == MISALIGNED    # bias
+    assert f(A, A, A, A, None, 4, 8, 16, A, None, U, None) == MISALIGNED    # workspace
+    assert f(A, A, A, A, None, 4, 8, 16, A, U, A, None) == MISALIGNED       # plan, with a workspace
+    assert f(A, A, A, A, None, 0, 8, 16, A, None, None, None) == OK          # empty batch
+    assert f(A, A, A, A, None, 0, 8, 16, A, None, A, None) == OK
     g = L.w8a8_debug_gemm_i32
-    assert g(A, A, 4, 8, 15, A, None) == SHAPE
-    assert g(A, None, 4, 8, 16, A, None) == INVALID
+    assert g(A, A, 4, 8, 15, A, None, None, None) == SHAPE
+    assert g(A, None, 4, 8, 16, A, None, None, None) == INVALID
+    assert g(A, A, 4, 8, 16, A, None, U, None) == MISALIGNED
+
+
+def test_linear_workspace_size(L):
+    base = L.w8a8_gemm_workspace_size()
+    assert L.w8a8_linear_workspace_size(4608, 4096) == base + 2 * 4608 * 4096 + 4 * 4608 + 1024
+    assert L.w8a8_linear_workspace_size(0, 4096) == base + 1024
+    assert L.w8a8_linear_workspace_size(-1, 4096) == 0
+    assert L.w8a8_linear_workspace_size(16, 0) == 0
 
 
 def test_dual_validation(L):
     from paper_2606_12280_gb300.w8a8 import Branch
     arr = (Branch * 2)()
     for i in range(2):
-        arr[i] = Branch(A, A, A, A, None, A, 4)
+        arr[i] = Branch(A, A, A, A, None, A, 4, None)
     f = L.w8a8_linear_dual
-    assert f(None, 8, 16, None) == INVALID
-    assert f(arr, 12, 16, None) == SHAPE
+    assert f(None, 8, 16, None, None) == INVALID
+    assert f(arr, 12, 16, None, None) == SHAPE
+    assert f(arr, 8, 16, U, None) == MISALIGNED           # workspace
+    arr[1].chunk_plan = U
+    assert f(arr, 8, 16, A, None) == MISALIGNED           # plan, with a workspace
+    arr[1].chunk_plan = None
     arr[1].Wq = U
-    assert f(arr, 8, 16, None) == MISALIGNED
+    assert f(arr, 8, 16, None, None) == MISALIGNED
     arr[1].Wq = None
-    assert f(arr, 8, 16, None) == INVALID
+    assert f(arr, 8, 16, None, None) == INVALID
     arr[0].M = 0
-    arr[1] = Branch(None, None, None, None, None, None, 0)
-    assert f(arr, 8, 16, None) == OK                      # both branches empty
+    arr[1] = Branch(None, None, None, None, None, None, 0, None)
+    assert f(arr, 8, 16, None, None) == OK                # both branches empty
 
 
 def test_debug_engine_validation(L):
@@ -131,7 +147,7 @@ def test_debug_engine_validation(L):
     from paper_2606_12280_gb300.w8a8 import Branch
     arr = (Branch * 2)()
     for i in range(2):
-        arr[i] = Branch(A, A, A, A, None, A, 4)
+        arr[i] = Branch(A, A, A, A, None, A, 4, None)
     f = L.w8a8_debug_linear_engine
     assert f(3, arr, 1, 8, 16, 0, None) == INVALID        # no such engine
     assert f(-1, arr, 1, 8, 16, 0, None) == INVALID

@@ -31,10 +31,10 @@ int main(void) {
     int8_t *Xq = (int8_t *)a, *Wq = (int8_t *)(a + 0x1000);
     float *s = (float *)(a + 0x2000);
     uint16_t *Y = (uint16_t *)(a + 0x3000);
-    printf("%d\n", (int)w8a8_linear(Xq, s, Wq, s, 0, 16, 8, 15, Y, 0));          /* K % 16 != 0 */
-    printf("%d\n", (int)w8a8_linear(Xq, s, Wq, s, 0, 16, 8, 16, (uint16_t *)(a + 2), 0)); /* misaligned */
+    printf("%d\n", (int)w8a8_linear(Xq, s, Wq, s, 0, 16, 8, 15, Y, 0, 0, 0));    /* K % 16 != 0 */
+    printf("%d\n", (int)w8a8_linear(Xq, s, Wq, s, 0, 16, 8, 16, (uint16_t *)(a + 2), 0, 0, 0)); /* misaligned */
     printf("%d\n", (int)w8a8_quant_act(0, 0, 4, 16, Xq, s, 0));                   /* null X */
-    printf("%d\n", (int)w8a8_linear(Xq, s, Wq, s, 0, 0, 8, 16, Y, 0));           /* M == 0: no-op */
+    printf("%d\n", (int)w8a8_linear(Xq, s, Wq, s, 0, 0, 8, 16, Y, 0, 0, 0));     /* M == 0: no-op */
     return 0;
 }
 """
