@@ -539,19 +539,26 @@ typedef struct {
     const float *w_scale;      /* W8A8: [N] fp32 */
     const uint16_t *W_bf16;    /* protected: [N,K] bf16 */
     const float *bias;         /* [N] fp32 or NULL, both paths */
+    const uint32_t *chunk_plan;  /* W8A8: w8a8_chunk_plan of Wq, or NULL */
 } w8a8_layer;
 
 /*
  * Per-layer dispatch: a protected layer runs w8a8_linear_bf16 on X; any other
- * layer runs w8a8_quant_act (into the caller's workspace) and w8a8_linear.
+ * layer quantizes X (a3) and runs the quantized linear (a4 + a5).
  *   layer  host pointer, read during the call only.
  *   X [M,K] bf16, read.   Y [M,N] bf16, written.
- *   Xq_work [M,K] int8 and x_scale_work [M] fp32: workspace of the W8A8 path
- *   (ignored, may be NULL, for a protected layer).
+ *   x_scale_work [M] fp32: the token scales (W8A8 path; ignored, may be
+ *   NULL, for a protected layer).
+ *   workspace: NULL, or w8a8_linear_workspace_size(M, K) bytes as for
+ *     w8a8_linear.  With one and K <= 16384, a3 writes the codes as fp16
+ *     values with their token sums into it (w8a8_quant_act_f16codes) and the
+ *     fp16-code GEMM runs on them; Xq_work is then unused and may be NULL.
+ *     Otherwise w8a8_quant_act writes Xq_work [M,K] int8 and w8a8_linear runs
+ *     with the workspace (or without one).  Same bits on every path.
  */
 W8A8_API w8a8_status w8a8_layer_forward(const w8a8_layer *layer, const uint16_t *X, int M,
                                         int8_t *Xq_work, float *x_scale_work, uint16_t *Y,
-                                        void *stream);
+                                        void *workspace, void *stream);
 
 /*
  * Choice of the protected set (Sec. 3: the N most fragile of the model's

@@ -441,7 +441,7 @@ w8a8_status w8a8_debug_gguf_dequant(const uint8_t *Wraw, int fmt, int N, int K, 
 }
 
 w8a8_status w8a8_layer_forward(const w8a8_layer *layer, const uint16_t *X, int M, int8_t *Xq_work,
-                               float *x_scale_work, uint16_t *Y, void *stream) {
+                               float *x_scale_work, uint16_t *Y, void *workspace, void *stream) {
     if (!layer) return W8A8_ERR_INVALID_ARG;
     const int N = layer->N, K = layer->K;
     if (w8a8_status e = check_nk(N, K)) return e;
@@ -451,14 +451,33 @@ w8a8_status w8a8_layer_forward(const w8a8_layer *layer, const uint16_t *X, int M
         return w8a8_linear_bf16(X, layer->W_bf16, layer->bias, M, N, K, Y, stream);
     }
     if (!layer->Wq || !layer->w_scale) return W8A8_ERR_INVALID_ARG;
+    if (workspace && !aligned16(workspace)) return W8A8_ERR_MISALIGNED;
     if (M == 0) return W8A8_OK;
-    if (!Xq_work || !x_scale_work) return W8A8_ERR_INVALID_ARG;
+    const bool direct16 = workspace != nullptr && K <= 16384;   // a3 writes fp16 codes into the workspace
+    if (!x_scale_work || (!direct16 && !Xq_work)) return W8A8_ERR_INVALID_ARG;
+    if (layer->chunk_plan && !aligned16(layer->chunk_plan)) return W8A8_ERR_MISALIGNED;
     // validate the GEMM's arguments before anything is enqueued
-    w8a8::GemmBranch b{Xq_work, x_scale_work, layer->Wq, layer->w_scale, layer->bias, Y, M};
+    w8a8::GemmBranch b{direct16 ? reinterpret_cast<const int8_t *>(workspace) : Xq_work, x_scale_work,
+                       layer->Wq, layer->w_scale, layer->bias, Y, M, nullptr, layer->chunk_plan};
     if (w8a8_status e = check_branch(b, true, N, K)) return e;
+    if (!X) return W8A8_ERR_INVALID_ARG;
+    if (!aligned16(X) || (layer->smooth && !aligned16(layer->smooth))) return W8A8_ERR_MISALIGNED;
+    cudaStream_t st = as_stream(stream);
+    if (direct16) {
+        unsigned int *err = device_error_word();
+        if (!err) return W8A8_ERR_CUDA;
+        uint16_t *q16 = nullptr;
+        uint32_t *ss = nullptr;
+        w8a8::linear_workspace_views(workspace, M, K, &q16, &ss);
+        cudaError_t e = w8a8::launch_quant_act_f16codes(X, layer->smooth, M, K, q16, x_scale_work, ss, false, st);
+        if (e != cudaSuccess) return W8A8_ERR_CUDA;
+        b.Xq = reinterpret_cast<const int8_t *>(q16);
+        b.x_sumsq = ss;
+        return from_cuda(w8a8::launch_gemm_ts(&b, 1, N, K, false, workspace, err, st));
+    }
     if (w8a8_status e = w8a8_quant_act(X, layer->smooth, M, K, Xq_work, x_scale_work, stream))
         return e;
-    return run_gemm(&b, 1, N, K, false, as_stream(stream));
+    return run_gemm_ws(&b, 1, N, K, false, workspace, st);
 }
 
 w8a8_status w8a8_select_protected(const float *score, int L, int n_protect, int *protect_flags) {

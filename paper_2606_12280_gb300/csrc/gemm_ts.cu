@@ -1072,6 +1072,13 @@ long long linear_codes8_workspace_bytes(long long tokens, int K) {
     return gemm_ts_workspace_bytes() + 2 * tokens * K + 4 * tokens + 4 * 256;
 }
 
+void linear_workspace_views(void *workspace, int M, int K, uint16_t **codes16, uint32_t **sumsq) {
+    char *w = static_cast<char *>(workspace);
+    const size_t off = static_cast<size_t>(gemm_ts_workspace_bytes());
+    *codes16 = reinterpret_cast<uint16_t *>(w + off);
+    *sumsq = reinterpret_cast<uint32_t *>(w + off + round256(2 * static_cast<size_t>(M) * K));
+}
+
 cudaError_t launch_linear_codes8(const GemmBranch *br, int nb, int N, int K, bool out_i32, void *workspace,
                                  unsigned int *err, cudaStream_t st) {
     char *w = static_cast<char *>(workspace);

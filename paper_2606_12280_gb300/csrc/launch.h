@@ -88,6 +88,9 @@ long long gemm_ts_workspace_bytes();
 long long linear_codes8_workspace_bytes(long long tokens, int K);
 cudaError_t launch_linear_codes8(const GemmBranch *br, int nb, int N, int K, bool out_i32, void *workspace,
                                  unsigned int *err, cudaStream_t st);
+// The single-branch layout of that workspace: where the fp16 codes and the
+// token sums of M tokens go (a3 may write them there directly).
+void linear_workspace_views(void *workspace, int M, int K, uint16_t **codes16, uint32_t **sumsq);
 int chunk_plan_words(int K);    // per block of 256 weight rows
 cudaError_t launch_chunk_plan(const int8_t *Wq, int N, int K, uint32_t *plan, cudaStream_t st);
 

@@ -41,7 +41,7 @@ SIGNATURES = {
     "w8a8_act_stats_update": [_P, _I, _I, _P, _P, _P, _P],
     "w8a8_act_stats_finalize": [_P, _P, _P, ctypes.c_longlong, _I, _P, _P, _P],
     "w8a8_linear_bf16": [_P, _P, _P, _I, _I, _I, _P, _P],
-    "w8a8_layer_forward": [_P, _P, _I, _P, _P, _P, _P],
+    "w8a8_layer_forward": [_P, _P, _I, _P, _P, _P, _P, _P],
     "w8a8_select_protected": [_P, _I, _I, _P],
     "w8a8_quant_act_dual": [_P, _I, _P],
     "w8a8_gelu_quant_act": [_P, _P, _I, _I, _P, _P, _P],
@@ -95,7 +95,7 @@ class Branch16(ctypes.Structure):
 class Layer(ctypes.Structure):
     """Mirror of ``w8a8_layer``."""
     _fields_ = [("protect", _I), ("N", _I), ("K", _I), ("smooth", _P), ("Wq", _P),
-                ("w_scale", _P), ("W_bf16", _P), ("bias", _P)]
+                ("w_scale", _P), ("W_bf16", _P), ("bias", _P), ("chunk_plan", _P)]
 
 
 _lock = threading.Lock()
@@ -701,8 +701,12 @@ def linear_bf16(X, W, bias=None, Y=None, stream=None):
 
 
 def layer_forward(X, protect: bool, N: int, K: int, smooth=None, Wq=None, w_scale=None,
-                  W_bf16=None, bias=None, Xq_work=None, x_scale_work=None, Y=None, stream=None):
-    """Per-layer dispatch (protected -> bf16 linear, else a3 + a4 + a5)."""
+                  W_bf16=None, bias=None, Xq_work=None, x_scale_work=None, Y=None, plan=None,
+                  workspace=None, stream=None):
+    """Per-layer dispatch (protected -> bf16 linear, else a3 + a4 + a5).
+    workspace: None or ``linear_workspace(M, K)``; with it (K <= 16384) a3
+    writes fp16 codes into it and Xq_work is not needed; plan: None or
+    ``chunk_plan(Wq)``."""
     M = X.shape[0]
     if tuple(X.shape) != (M, K):
         raise ValueError(f"X has shape {tuple(X.shape)}, the layer needs ({M}, {K})")
@@ -713,7 +717,7 @@ def layer_forward(X, protect: bool, N: int, K: int, smooth=None, Wq=None, w_scal
     if protect:
         _room(W_bf16, N * K, "W_bf16")
     else:
-        if Xq_work is None:
+        if Xq_work is None and (workspace is None or K > 16384):
             Xq_work = torch.empty(M, K, dtype=torch.int8, device=X.device)
         if x_scale_work is None:
             x_scale_work = torch.empty(M, dtype=torch.float32, device=X.device)
@@ -722,13 +726,17 @@ def layer_forward(X, protect: bool, N: int, K: int, smooth=None, Wq=None, w_scal
         _room(w_scale, N, "w_scale")
         _room(Xq_work, M * K, "Xq_work")
         _room(x_scale_work, M, "x_scale_work")
+        if plan is not None:
+            _room(plan, chunk_plan_size(N, K), "plan")
+    ws = None if protect else _linear_ws(workspace, M, K)
     layer = Layer(1 if protect else 0, N, K, _ptr(smooth, torch.float32, "smooth"),
                   _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
-                  _ptr(W_bf16, torch.bfloat16, "W_bf16"), _ptr(bias, torch.float32, "bias"))
+                  _ptr(W_bf16, torch.bfloat16, "W_bf16"), _ptr(bias, torch.float32, "bias"),
+                  None if protect else _ptr(plan, torch.int32, "plan"))
     _check("w8a8_layer_forward", lib().w8a8_layer_forward(
         ctypes.byref(layer), _ptr(X, torch.bfloat16, "X"), M,
         _ptr(Xq_work, torch.int8, "Xq_work"), _ptr(x_scale_work, torch.float32, "x_scale_work"),
-        _ptr(Y, torch.bfloat16, "Y"), _stream(stream)))
+        _ptr(Y, torch.bfloat16, "Y"), ws, _stream(stream)))
     return Y
 
 

@@ -212,15 +212,21 @@ def test_linear_bf16_and_layer_validation(L):
     assert f(A, A, U, 4, 8, 16, A, None) == MISALIGNED
     assert f(None, None, None, 0, 8, 16, None, None) == OK       # empty batch
     g = L.w8a8_layer_forward
-    assert g(None, A, 4, A, A, A, None) == INVALID
-    prot = Layer(1, 8, 16, None, None, None, None, None)
-    assert g(ctypes.byref(prot), A, 4, None, None, A, None) == INVALID   # no bf16 weights
-    q = Layer(0, 8, 16, None, A, A, None, None)
-    assert g(ctypes.byref(q), A, 4, None, A, A, None) == INVALID        # no workspace
-    assert g(ctypes.byref(q), A, 4, U, A, A, None) == MISALIGNED
-    assert g(ctypes.byref(q), A, 0, None, None, A, None) == OK
-    bad = Layer(0, 12, 16, None, A, A, None, None)
-    assert g(ctypes.byref(bad), A, 4, A, A, A, None) == SHAPE
+    assert g(None, A, 4, A, A, A, None, None) == INVALID
+    prot = Layer(1, 8, 16, None, None, None, None, None, None)
+    assert g(ctypes.byref(prot), A, 4, None, None, A, None, None) == INVALID   # no bf16 weights
+    q = Layer(0, 8, 16, None, A, A, None, None, None)
+    assert g(ctypes.byref(q), A, 4, None, A, A, None, None) == INVALID        # no codes buffer
+    assert g(ctypes.byref(q), A, 4, A, None, A, A, None) == INVALID           # no scales
+    assert g(ctypes.byref(q), A, 4, U, A, A, None, None) == MISALIGNED
+    assert g(ctypes.byref(q), A, 4, None, A, A, U, None) == MISALIGNED        # workspace
+    assert g(ctypes.byref(q), U, 4, None, A, A, A, None) == MISALIGNED        # X, fp16-code path
+    assert g(ctypes.byref(q), None, 4, None, A, A, A, None) == INVALID
+    qp = Layer(0, 8, 16, None, A, A, None, None, U)
+    assert g(ctypes.byref(qp), A, 4, None, A, A, A, None) == MISALIGNED       # plan
+    assert g(ctypes.byref(q), A, 0, None, None, A, None, None) == OK
+    bad = Layer(0, 12, 16, None, A, A, None, None, None)
+    assert g(ctypes.byref(bad), A, 4, A, A, A, None, None) == SHAPE
 
 
 def test_select_protected():

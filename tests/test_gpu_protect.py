@@ -225,6 +225,11 @@ def test_layer_forward_dispatch(w8, oracle_mod):
     assert torch.equal(Yq, w8.linear(Xq, sx, Wq, sw, bias))
     Yp = w8.layer_forward(X, True, N, K, W_bf16=Wb, bias=bias)
     assert torch.equal(Yp, w8.linear_bf16(X, Wb, bias))
+    # with a workspace: fp16 codes written into it, the weights-in-TMEM GEMM
+    ws = w8.linear_workspace(M, K)
+    for plan in (None, w8.chunk_plan(Wq)):
+        Yw = w8.layer_forward(X, False, N, K, smooth=lam, Wq=Wq, w_scale=sw, bias=bias, plan=plan, workspace=ws)
+        assert torch.equal(Yw, Yq)
     # and against the oracle: the W8A8 path bit-exact
     lam_h = oracle_mod.smooth_scales(oracle_mod.channel_absmax(case.X_cal), case.W[0], case.alpha)
     Wq_h, sw_h = oracle_mod.quantize_weights(case.W[0], lam_h)
@@ -232,3 +237,19 @@ def test_layer_forward_dispatch(w8, oracle_mod):
                                                 "w_scale": sw_h, "W_bf16": None,
                                                 "bias": case.bias[0]})
     np.testing.assert_array_equal(u16(Yq), want)
+
+
+def test_layer_forward_workspace_long_k(w8):
+    # K > 16384: int8 codes, then the expansion pass in the workspace
+    M, N, K = 300, 264, 16400
+    g = torch.Generator(device=DEV).manual_seed(8)
+    X = torch.randn(M, K, generator=g, device=DEV).to(torch.bfloat16)
+    W = torch.randn(N, K, generator=g, device=DEV) * 0.02
+    lam = torch.rand(K, generator=g, device=DEV) + 0.5
+    Wq, sw = w8.quantize_weights(W, lam)
+    bias = torch.randn(N, generator=g, device=DEV) * 0.01
+    Y0 = w8.layer_forward(X, False, N, K, smooth=lam, Wq=Wq, w_scale=sw, bias=bias)
+    Y1 = w8.layer_forward(X, False, N, K, smooth=lam, Wq=Wq, w_scale=sw, bias=bias, plan=w8.chunk_plan(Wq),
+                          workspace=w8.linear_workspace(M, K))
+    assert torch.equal(Y0, Y1)
+    assert w8.device_status() == 0
