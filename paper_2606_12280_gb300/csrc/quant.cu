@@ -409,6 +409,9 @@ __device__ __forceinline__ uint32_t pack_f16(float a, float b) {
 template <int U, int TW, int S, bool GELU, bool OUT16>
 __global__ void __launch_bounds__(TW > 8 ? 32 * TW : 256)
 act_quant_team_kernel(const __grid_constant__ ActParams p) {
+    // a dependent GEMM launched programmatically may set itself up on SMs as
+    // they free up; it reads nothing of this pass before the pass completes
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     constexpr int kThreads = TW > 8 ? 32 * TW : 256;
     constexpr int kTeams = kThreads / (32 * TW);
     extern __shared__ __align__(16) uint4 ring_s[];
