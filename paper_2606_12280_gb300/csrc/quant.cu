@@ -404,6 +404,68 @@ __device__ __forceinline__ uint32_t pack_f16(float a, float b) {
     return r;
 }
 
+// The codes of one chunk of 8 smoothed values x' (x[q] = columns 2q, 2q+1)
+// with inv = 127/a: int8 bytes packed in .x/.y, or (OUT16) fp16 values in
+// .x .. .w.  OUT16 with want_ss adds the squared codes: exactly, as fp32
+// pairs in ssq on the fast path (integers below 2^24: a lane's U <= 4 chunks
+// give at most 4U codes of at most 127^2 per component) or as integers in ss.
+template <bool OUT16>
+__device__ __forceinline__ uint4 quant_chunk(const float2 (&x)[4], float inv, bool zero_row, bool fast,
+                                             bool want_ss, uint32_t &ss, uint64_t &ssq) {
+    uint4 o = make_uint4(0u, 0u, 0u, 0u);
+    if (zero_row) return o;
+    if (OUT16) {
+        uint32_t hw[4];
+        if (fast) {
+            // rne(x' * inv) as an fp32 integer: the product rounded once
+            // (scalar multiplies, never fused), the magic sum (in [2^23,
+            // 2^24], where one packed add rounds both values to integers as
+            // the scalar add would), minus the magic (exact)
+            const uint64_t magic = pk(kRoundMagic, kRoundMagic);
+            const uint64_t nmagic = pk(-kRoundMagic, -kRoundMagic);
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const uint64_t c = add_pk(add_pk(pk(__fmul_rn(x[q].x, inv), __fmul_rn(x[q].y, inv)), magic), nmagic);
+                const float2 cf = upk(c);
+                hw[q] = pack_f16(cf.x, cf.y);
+                if (want_ss) ssq = fma_pk(c, c, ssq);
+            }
+        } else {
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+                const int q0 = quantize_rne_clamp(__fmul_rn(x[q].x, inv));
+                const int q1 = quantize_rne_clamp(__fmul_rn(x[q].y, inv));
+                hw[q] = pack_f16(static_cast<float>(q0), static_cast<float>(q1));
+                ss += static_cast<uint32_t>(q0 * q0 + q1 * q1);
+            }
+        }
+        return make_uint4(hw[0], hw[1], hw[2], hw[3]);
+    }
+    uint32_t word[2] = {0u, 0u};
+    if (fast) {
+        // the products rounded once (scalar multiplies), their magic sums two
+        // at a time (one packed add, each value rounded to an integer as the
+        // scalar add would)
+        const uint64_t magic = pk(kRoundMagic, kRoundMagic);
+#pragma unroll
+        for (int h = 0; h < 2; ++h) {
+            const float2 s0 = upk(add_pk(pk(__fmul_rn(x[2 * h].x, inv), __fmul_rn(x[2 * h].y, inv)), magic));
+            const float2 s1 = upk(add_pk(pk(__fmul_rn(x[2 * h + 1].x, inv), __fmul_rn(x[2 * h + 1].y, inv)), magic));
+            word[h] = pack4_low_bytes(s0.x, s0.y, s1.x, s1.y);
+        }
+    } else {
+#pragma unroll
+        for (int e = 0; e < 8; ++e) {
+            const float xv = (e & 1) ? x[e >> 1].y : x[e >> 1].x;
+            const uint32_t q8 = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xv, inv))) & 0xffu;
+            word[e >> 2] |= q8 << (8 * (e & 3));
+        }
+    }
+    o.x = word[0];
+    o.y = word[1];
+    return o;
+}
+
 // OUT16: the codes are written as fp16 values (uint16 bit patterns, 2 bytes
 // each) instead of int8, for the GEMM that takes A without converting it.
 template <int U, int TW, int S, bool GELU, bool OUT16>
@@ -521,69 +583,14 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
         uint2 *qr = reinterpret_cast<uint2 *>(b.Xq + (size_t)row * K);
         uint4 *qr16 = reinterpret_cast<uint4 *>(b.Xq + 2 * (size_t)row * K);
         uint32_t ss = 0;
-        // fp16-code fast path: the lane's squared codes summed as fp32 pairs
-        // (integers below 2^24: at most 4U codes of 127^2 per component, so
-        // every sum is exact)
         uint64_t ssq = 0;
 #pragma unroll
         for (int u = 0; u < U; ++u) {
             const int c = (u * TW + tw) * 32 + lane;
             if (c >= cpr) continue;
-            if (OUT16) {
-                uint32_t hw[4] = {0u, 0u, 0u, 0u};
-                if (zero_row) {
-                } else if (fast) {
-                    // rne(x' * inv) as an fp32 integer: the product rounded
-                    // once (scalar multiplies, never fused), the magic sum
-                    // (in [2^23, 2^24], where one packed add rounds both
-                    // values to integers as the scalar add would), minus the
-                    // magic (exact)
-                    const uint64_t magic = pk(kRoundMagic, kRoundMagic);
-                    const uint64_t nmagic = pk(-kRoundMagic, -kRoundMagic);
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const uint64_t c = add_pk(add_pk(pk(__fmul_rn(xs[u][q].x, inv),
-                                                            __fmul_rn(xs[u][q].y, inv)), magic), nmagic);
-                        const float2 cf = upk(c);
-                        hw[q] = pack_f16(cf.x, cf.y);
-                        if (want_ss) ssq = fma_pk(c, c, ssq);
-                    }
-                } else {
-#pragma unroll
-                    for (int q = 0; q < 4; ++q) {
-                        const int q0 = quantize_rne_clamp(__fmul_rn(xs[u][q].x, inv));
-                        const int q1 = quantize_rne_clamp(__fmul_rn(xs[u][q].y, inv));
-                        hw[q] = pack_f16(static_cast<float>(q0), static_cast<float>(q1));
-                        ss += static_cast<uint32_t>(q0 * q0 + q1 * q1);
-                    }
-                }
-                qr16[c] = make_uint4(hw[0], hw[1], hw[2], hw[3]);
-                continue;
-            }
-            uint32_t word[2] = {0u, 0u};
-            if (zero_row) {
-            } else if (fast) {
-                // the products rounded once (scalar multiplies), their magic
-                // sums two at a time (one packed add, each value rounded to
-                // an integer as the scalar add would)
-                const uint64_t magic = pk(kRoundMagic, kRoundMagic);
-#pragma unroll
-                for (int h = 0; h < 2; ++h) {
-                    const float2 s0 = upk(add_pk(pk(__fmul_rn(xs[u][2 * h].x, inv),
-                                                    __fmul_rn(xs[u][2 * h].y, inv)), magic));
-                    const float2 s1 = upk(add_pk(pk(__fmul_rn(xs[u][2 * h + 1].x, inv),
-                                                    __fmul_rn(xs[u][2 * h + 1].y, inv)), magic));
-                    word[h] = pack4_low_bytes(s0.x, s0.y, s1.x, s1.y);
-                }
-            } else {
-#pragma unroll
-                for (int e = 0; e < 8; ++e) {
-                    const float xv = (e & 1) ? xs[u][e >> 1].y : xs[u][e >> 1].x;
-                    const uint32_t q8 = static_cast<uint32_t>(quantize_rne_clamp(__fmul_rn(xv, inv))) & 0xffu;
-                    word[e >> 2] |= q8 << (8 * (e & 3));
-                }
-            }
-            qr[c] = make_uint2(word[0], word[1]);
+            const uint4 o = quant_chunk<OUT16>(xs[u], inv, zero_row, fast, want_ss, ss, ssq);
+            if (OUT16) qr16[c] = o;
+            else qr[c] = make_uint2(o.x, o.y);
         }
         if (want_ss) {
             const float2 sf = upk(ssq);
