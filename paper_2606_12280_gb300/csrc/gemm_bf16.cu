@@ -197,6 +197,7 @@ gemm_bf16_kernel(const __grid_constant__ CUtensorMap tmA, const __grid_constant_
     const uint32_t peer_tmem = ld_shared_cluster_u32(mapa_shared(sb + OFF_TMEM, rank ^ 1u));
     const bool run_ok = (tmem == peer_tmem);
     if (!run_ok && threadIdx.x == 0) atomicOr(p.err, ERR_TMEM_PAIR);
+    wait_prior_grid();
     const WaitCtx wc{sb + OFF_ABORT, p.err, p.wait_limit_ns};
     const int NS = (p.k_blocks + SUB - 1) / SUB;           // stages per tile
 
@@ -344,8 +345,7 @@ cudaError_t launch_gemm_bf16(const uint16_t *X, const uint16_t *W, const float *
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
     const int pairs = p.total_tiles < sms / 2 ? p.total_tiles : sms / 2;
-    gemm_bf16_kernel<<<2 * pairs, THREADS, SMEM_TOTAL, st>>>(mA, mB, p);
-    return cudaGetLastError();
+    return launch_pdl(gemm_bf16_kernel, dim3(2 * pairs), THREADS, SMEM_TOTAL, st, mA, mB, p);
 }
 
 }  // namespace w8a8

@@ -400,6 +400,7 @@ gemm_gguf_kernel(const __grid_constant__ CUtensorMap tmX, const __grid_constant_
     const uint32_t peer_tmem = ld_shared_cluster_u32(mapa_shared(sb + L::OFF_TMEM, rank ^ 1u));
     const bool run_ok = (tmem == peer_tmem);
     if (!run_ok && threadIdx.x == 0) atomicOr(p.err, ERR_TMEM_PAIR);
+    wait_prior_grid();
     const WaitCtx wc{sb + L::OFF_ABORT, p.err, p.wait_limit_ns};
     const int NS = p.spans * STAGES_PER_SPAN;          // stages per tile
 
@@ -667,8 +668,7 @@ cudaError_t launch_fmt(const uint16_t *X, const uint8_t *Wraw, const float *bias
     p.wait_limit_ns = 2000000000ull;
     const int sms = device_sms();
     const int pairs = p.total_tiles < sms / 2 ? p.total_tiles : sms / 2;
-    gemm_gguf_kernel<FMT><<<2 * pairs, THREADS, L::SMEM_TOTAL, st>>>(mX, mW, p);
-    return cudaGetLastError();
+    return launch_pdl(gemm_gguf_kernel<FMT>, dim3(2 * pairs), THREADS, L::SMEM_TOTAL, st, mX, mW, p);
 }
 
 }  // namespace

@@ -358,6 +358,7 @@ gemm_tc2_kernel(const __grid_constant__ CUtensorMap tmA0, const __grid_constant_
     const uint32_t peer_tmem = ld_shared_cluster_u32(mapa_shared(sb + L::OFF_TMEM, rank ^ 1u));
     const bool run_ok = (tmem == peer_tmem);
     if (!run_ok && threadIdx.x == 0) atomicOr(p.err, ERR_TMEM_PAIR);
+    wait_prior_grid();
     const WaitCtx wc{sb + L::OFF_ABORT, p.err, p.wait_limit_ns};
     const int KB = p.k_blocks;
     const int NS = (KB + SUB - 1) / SUB;                  // pipeline stages per tile
@@ -688,8 +689,7 @@ cudaError_t launch_gemm_tc2(const GemmBranch *br, int nb, int N, int K, bool out
     p.err = err;
     p.wait_limit_ns = 2000000000ull;
     const int pairs = p.total_tiles < sms / 2 ? p.total_tiles : sms / 2;
-    kern<<<2 * pairs, THREADS, smem_total, st>>>(maps[0], maps[1], maps[2], maps[3], p);
-    return cudaGetLastError();
+    return launch_pdl(kern, dim3(2 * pairs), THREADS, smem_total, st, maps[0], maps[1], maps[2], maps[3], p);
 }
 
 }  // namespace w8a8

@@ -55,9 +55,6 @@ using namespace tc;
 #ifndef W8A8_TS_S8
 #define W8A8_TS_S8 4
 #endif
-#ifndef W8A8_TS_PDL
-#define W8A8_TS_PDL 1
-#endif
 constexpr int PAIR_F = 256, CTA_F = 128;             // output features per pair / CTA (MMA M)
 constexpr int PAIR_T = 256, CTA_T = 128;             // tokens per pair / CTA (MMA N)
 constexpr int BK = 64;                               // K per sub-block (one swizzle atom row)
@@ -551,13 +548,7 @@ gemm_ts_kernel(const __grid_constant__ CUtensorMap tmX0, const __grid_constant__
     const uint32_t peer_tmem = ld_shared_cluster_u32(mapa_shared(sb + OFF_TMEM, rank ^ 1u));
     const bool run_ok = (tmem == peer_tmem);
     if (!run_ok && threadIdx.x == 0) atomicOr(p.err, ERR_TMEM_PAIR);
-    // Launched as a programmatic dependent of the kernel before it in the
-    // stream: everything above (barriers, tensor memory, the descriptors)
-    // overlaps that kernel's last blocks; no operand, plan, sum, scale,
-    // workspace counter or output is touched before it has completed.  The
-    // kernel after this one may start its own set-up as SMs free up.
-    asm volatile("griddepcontrol.wait;" ::: "memory");
-    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    wait_prior_grid();
     const WaitCtx wc{sb + OFF_ABORT, p.err, p.wait_limit_ns};
     const int KB = p.k_blocks;                            // K=64 sub-blocks per tile
     const int NS = (KB + SUB - 1) / SUB;                  // stages per tile
@@ -1066,17 +1057,7 @@ cudaError_t launch_gemm_ts(const GemmBranch *br, int nb, int N, int K, bool out_
     cudaError_t e = out_i32 ? (grouped ? prepare_ts_kernel<true, true>() : prepare_ts_kernel<true, false>())
                             : (grouped ? prepare_ts_kernel<false, true>() : prepare_ts_kernel<false, false>());
     if (e != cudaSuccess) return e;
-    cudaLaunchConfig_t cfg = {};
-    cfg.gridDim = dim3(2 * pairs);
-    cfg.blockDim = dim3(THREADS);
-    cfg.dynamicSmemBytes = SMEM_TOTAL;
-    cfg.stream = st;
-    cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = W8A8_TS_PDL;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, kern, maps[0], maps[1], maps[2], maps[3], p);
+    return launch_pdl(kern, dim3(2 * pairs), THREADS, SMEM_TOTAL, st, maps[0], maps[1], maps[2], maps[3], p);
 }
 
 // The int8-code linear on this engine.  Workspace layout: the split-K area

@@ -92,6 +92,17 @@ __device__ __forceinline__ bool mbar_wait(uint32_t bar, uint32_t parity, const W
     return mbar_wait_slow(bar, parity, w, code, honor_abort);
 }
 
+// Programmatic dependent launch: wait until the kernel before this one in
+// the stream has completed and its writes are visible (a no-op for a kernel
+// launched the ordinary way), then let the kernel after this one start its
+// own set-up on SMs as they free up.  A GEMM calls it after its barriers,
+// tensor memory and descriptors are set up and before it touches any operand,
+// plan, sum, scale, workspace or output.
+__device__ __forceinline__ void wait_prior_grid() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+
 __device__ __forceinline__ void fence_barrier_init() {
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
 }
