@@ -831,6 +831,22 @@ def run_ours(args):
     if w8a8.device_status(stream) != 0:
         raise RuntimeError("device error word set while timing the block sweep")
 
+    # the GPU's native INT8 tensor path on the same shape, as the second
+    # roofline denominator: cuBLAS's int8 x int8 -> int32 GEMM through
+    # torch._int_mm (a comparator only, in a CUDA graph of back-to-back calls)
+    int8_ceiling = None
+    if hasattr(torch, "_int_mm"):
+        try:
+            A8 = torch.randint(-127, 128, (M, K), device=dev, dtype=torch.int8)
+            B8 = torch.randint(-127, 128, (N, K), device=dev, dtype=torch.int8).t()
+            ms_i8 = isolated(lambda i, st: torch._int_mm(A8, B8), 3)
+            int8_ceiling = {"tops": ops_step / (ms_i8 * 1e-3) / 1e12, "ms": ms_i8,
+                            "how": "torch._int_mm (cuBLAS INT8 tensor path), the same M, N, K, "
+                                   "three calls in a CUDA graph"}
+            del A8, B8
+        except (RuntimeError, TypeError) as exc:
+            int8_ceiling = {"unavailable": str(exc)[:200]}
+
     # the other benchmark configurations, each on its own seeded recipe
     configs = {"single_m256_k512_n512": config_single(w8a8, wl, dev) if rank == 0 else None,
                "ffn_pair_m4608": config_ffn_pair(w8a8, wl, dev, isolated, args.codes, rank == 0)}
@@ -949,6 +965,8 @@ def run_ours(args):
                           "how": "the timed graph replayed back to back for >= 2 s; the GEMM alone "
                                  "(a graph of 10 launches replayed) for >= 2 s"},
             "configs": configs,
+            "int8_ceiling": (dict(int8_ceiling, gemm_over_ceiling=gemm_tflops / int8_ceiling["tops"])
+                             if int8_ceiling and "tops" in int8_ceiling else int8_ceiling),
             "other_codes": {
                 "codes": "int8" if f16 else "f16",
                 "step_ms_isolated": other_quant + other_gemm,
