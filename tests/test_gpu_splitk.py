@@ -67,6 +67,7 @@ def codes_case(M, N, K, kind, seed):
 @pytest.mark.parametrize("M,N,K,kind", [
     (512, 1024, 4096, "random"),      # 8 tiles: fewer than the pairs, 4 chunks
     (2560, 2304, 4096, "random"),     # 90 tiles: a partial second round
+    (2560, 3072, 4096, "random"),     # 120 tiles: 44 left over, more than half the pairs: no split
     (300, 520, 3072, "random"),       # 6 tiles, 3 chunks, ragged M and N
     (1000, 1000, 2064, "random"),     # 16 tiles, ragged last chunk
     (600, 512, 4096, "extreme"),      # drains inside the parts
@@ -161,3 +162,26 @@ def test_workspace_size_and_checks(w8):
     with pytest.raises(ValueError):
         w8.debug_gemm_f16codes_i32(q16, Wq, workspace=torch.zeros(w8.gemm_workspace_size(), dtype=torch.int32,
                                                                    device=DEV))
+
+
+def test_split_dual_workload_equals_unsplit(w8):
+    # the dual-branch workload's shape: 576 tiles on 76 pairs leave 44, more
+    # than half the pairs, so the launch runs unsplit with the workspace too
+    M, N, K = 4608, 4096, 4096
+    g = torch.Generator(device=DEV).manual_seed(13)
+    brs = []
+    for b in range(2):
+        q16 = torch.randint(-127, 128, (M, K), generator=g, device=DEV, dtype=torch.int32).to(torch.float16)
+        Wq = torch.randint(-127, 128, (N, K), generator=g, device=DEV, dtype=torch.int32).to(torch.int8)
+        sx = torch.rand(M, generator=g, device=DEV) * 1e-3
+        sw = torch.rand(N, generator=g, device=DEV) * 1e-3
+        bias = torch.randn(N, generator=g, device=DEV)
+        ss = (q16.to(torch.int32) ** 2).sum(1, dtype=torch.int32)
+        brs.append((q16, sx, Wq, sw, bias, w8.chunk_plan(Wq), ss))
+    ws = w8.gemm_workspace()
+    Y1 = w8.linear_dual_f16codes(brs, workspace=ws)
+    Y0 = w8.linear_dual_f16codes(brs)
+    for a, b in zip(Y1, Y0):
+        assert torch.equal(a, b)
+    assert counters_zero(ws)
+    assert w8.device_status() == 0
