@@ -28,6 +28,27 @@ __device__ __forceinline__ int quantize_rne_clamp(float v) {
     return static_cast<int>(r);
 }
 
+// Two fp32 -> one bf16x2 word (lo in bits 0-15), both rounded to nearest
+// even by one conversion instruction: the same bits as two
+// f32_to_bf16_bits_rn calls for every input that is not a NaN (checked for
+// all 2^32 patterns in each half on GB300); a NaN becomes the canonical one
+// instead of keeping its payload, so callers use it only where no value can
+// be a NaN.
+__device__ __forceinline__ uint32_t pack_bf16x2_cvt(float lo, float hi) {
+    uint32_t w;
+    asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(w) : "f"(hi), "f"(lo));
+    return w;
+}
+
+// The epilogue's value before the rounding to bf16: (t * sx) * sw + b, each
+// step rounded to nearest even, no contraction.
+__device__ __forceinline__ float epilogue_f32(float t, float sx, float sw, float b, bool has_bias) {
+    t = __fmul_rn(t, sx);
+    t = __fmul_rn(t, sw);
+    if (has_bias) t = __fadd_rn(t, b);
+    return t;
+}
+
 // Dequantizing epilogue for one output from (float)acc: bf16((t * sx) * sw
 // + b), each step rounded to nearest even, no contraction.
 __device__ __forceinline__ uint32_t epilogue_value_f(float t, float sx, float sw, float b,

@@ -38,6 +38,7 @@
 // commits MMA completion to both CTAs' barriers by multicast.  All waits are
 // bounded in time.
 #include <cstdint>
+#include <type_traits>
 #include <cuda.h>
 #include <cuda_runtime.h>
 
@@ -442,6 +443,7 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
                 // broadcasts: a global load per token inside the store loop
                 // would wait a full memory latency per token
                 const uint32_t epi = sb + OFF_EPI + (warp - 8) * EPI_BYTES;
+                bool sx_ok;
                 {
                     const float *sxp = br.x_scale + tok0;
                     float4 s4;
@@ -455,42 +457,70 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
                     }
                     st_shared_v4(epi + 16 * lane, make_uint4(__float_as_uint(s4.x), __float_as_uint(s4.y),
                                                              __float_as_uint(s4.z), __float_as_uint(s4.w)));
+                    constexpr float kSxLimit = 0x1p96f;       // |acc| < 2^31: acc * sx stays finite
+                    sx_ok = fabsf(s4.x) <= kSxLimit && fabsf(s4.y) <= kSxLimit && fabsf(s4.z) <= kSxLimit &&
+                            fabsf(s4.w) <= kSxLimit;
                     __syncwarp();
                 }
                 // lanes 2i and 2i+1 (features f, f+1) swap one value per pair
                 // of tokens, so that each stores one 32-bit word: the even
                 // lane both features of the first token, the odd lane both of
-                // the second (N even: the word is 4-byte aligned)
+                // the second (N even: the word is 4-byte aligned).  No output
+                // of the tile can be a NaN when every scale and the bias are
+                // finite and |sx| <= 2^96 (a product may overflow, but inf
+                // times a finite nonzero scale plus a finite bias stays
+                // infinite): each pair is then rounded to bf16 by one
+                // conversion instruction.  The epilogue shares the SM's issue
+                // slots with the converters, and rounding every value with
+                // integer operations made the whole GEMM ~5 % slower; tiles
+                // that could hold a NaN keep that rounding, which preserves a
+                // NaN's payload.
                 const bool odd = lane & 1;
                 const int fw = f & ~1;
                 uint16_t *out = static_cast<uint16_t *>(br.out) + (size_t)tok0 * p.N + fw;
                 const bool paired = (p.N & 1) == 0;
+                const bool fast_cvt = __all_sync(0xffffffffu, sx_ok && fabsf(sw) <= 3.402823466e38f &&
+                                                                   (!hb || fabsf(b) <= 3.402823466e38f));
+                auto store_pairs = [&](auto fast_tag) {
+                    constexpr bool FAST = decltype(fast_tag)::value;
 #pragma unroll
-                for (int i = 0; i < RUN; i += 4) {
-                    const uint4 s4 = ld_shared_v4(epi + 4 * i);
-                    const float sxv[4] = {__uint_as_float(s4.x), __uint_as_float(s4.y), __uint_as_float(s4.z),
-                                          __uint_as_float(s4.w)};
+                    for (int i = 0; i < RUN; i += 4) {
+                        const uint4 s4 = ld_shared_v4(epi + 4 * i);
+                        const float sxv[4] = {__uint_as_float(s4.x), __uint_as_float(s4.y), __uint_as_float(s4.z),
+                                              __uint_as_float(s4.w)};
 #pragma unroll
-                    for (int u = 0; u < 4; u += 2) {
-                        const uint32_t y0 = epilogue_value_f(__uint_as_float(static_cast<uint32_t>(run[i + u])),
-                                                             sxv[u], sw, b, hb);
-                        const uint32_t y1 = epilogue_value_f(__uint_as_float(static_cast<uint32_t>(run[i + u + 1])),
-                                                             sxv[u + 1], sw, b, hb);
-                        const uint32_t other = __shfl_xor_sync(0xffffffffu, odd ? y0 : y1, 1);
-                        const int tk = i + u + (odd ? 1 : 0);
-                        if (paired) {
-                            const uint32_t word = odd ? (other | (y1 << 16)) : (y0 | (other << 16));
+                        for (int u = 0; u < 4; u += 2) {
+                            const float t0 = epilogue_f32(__uint_as_float(static_cast<uint32_t>(run[i + u])),
+                                                          sxv[u], sw, b, hb);
+                            const float t1 = epilogue_f32(__uint_as_float(static_cast<uint32_t>(run[i + u + 1])),
+                                                          sxv[u + 1], sw, b, hb);
+                            const float other = __shfl_xor_sync(0xffffffffu, odd ? t0 : t1, 1);
+                            const int tk = i + u + (odd ? 1 : 0);
+                            const float lo = odd ? other : t0, hi = odd ? t1 : other;
+                            const uint32_t word = FAST ? pack_bf16x2_cvt(lo, hi)
+                                                       : f32_to_bf16_bits_rn(lo) | (f32_to_bf16_bits_rn(hi) << 16);
                             // streaming store: Y is not read again here, and
                             // evicting it first lets L2 write it back while
                             // the GEMM leaves HBM idle (1 % faster steps)
-                            if (tk < ntok && fok)
-                                asm volatile("st.global.cs.u32 [%0], %1;" ::"l"(out + (size_t)tk * p.N),
-                                             "r"(word) : "memory");
-                        } else {
-                            uint16_t *o = out + (f - fw);
-                            if (fok && i + u < ntok) o[(size_t)(i + u) * p.N] = static_cast<uint16_t>(y0);
-                            if (fok && i + u + 1 < ntok)
-                                o[(size_t)(i + u + 1) * p.N] = static_cast<uint16_t>(y1);
+                            if (tk < ntok && fok) __stcs(reinterpret_cast<unsigned int *>(out + (size_t)tk * p.N), word);
+                        }
+                    }
+                };
+                if (paired) {
+                    if (fast_cvt) store_pairs(std::true_type{});
+                    else store_pairs(std::false_type{});
+                } else {
+#pragma unroll
+                    for (int i = 0; i < RUN; i += 4) {
+                        const uint4 s4 = ld_shared_v4(epi + 4 * i);
+                        const float sxv[4] = {__uint_as_float(s4.x), __uint_as_float(s4.y), __uint_as_float(s4.z),
+                                              __uint_as_float(s4.w)};
+                        uint16_t *o = out + (f - fw);
+#pragma unroll
+                        for (int u = 0; u < 4; ++u) {
+                            const uint32_t y = epilogue_value_f(__uint_as_float(static_cast<uint32_t>(run[i + u])),
+                                                                sxv[u], sw, b, hb);
+                            if (fok && i + u < ntok) o[(size_t)(i + u) * p.N] = static_cast<uint16_t>(y);
                         }
                     }
                 }

@@ -300,3 +300,37 @@ def test_dual_f16codes_equals_singles(w8, oracle_mod, M0, M1):
         assert torch.equal(Y1, Ys[b])
         Xq, wsx = oracle_mod.quant_act(X, lam)
         np.testing.assert_array_equal(u16(Ys[b]), oracle_mod.linear(Xq, wsx, Wq, sw, bias))
+
+
+@pytest.mark.parametrize("case", ["inf_scale", "huge_scale", "nan_bias", "finite"])
+def test_epilogue_non_finite_scales(w8, oracle_mod, case):
+    # The epilogue rounds pairs with one conversion instruction only where no
+    # output can be a NaN; tiles with a non-finite scale or bias, or a token
+    # scale above 2^96 (acc * sx may overflow), take the integer rounding.
+    # Either way Y matches the oracle: bit for bit where it is a number, and
+    # NaN where the oracle's is NaN.
+    M, N, K = 300, 520, 1040
+    rng = np.random.default_rng(7)
+    Xq = rng.integers(-127, 128, (M, K), dtype=np.int8)
+    Wq = rng.integers(-127, 128, (N, K), dtype=np.int8)
+    Xq[5] = 0                                             # acc = 0 rows: inf * 0 = NaN
+    sx = rng.random(M, dtype=np.float32) * 1e-3
+    sw = rng.random(N, dtype=np.float32) * 1e-3
+    b = rng.standard_normal(N).astype(np.float32)
+    if case == "inf_scale":
+        sx[[3, 5, 260]] = np.inf
+        sw[[7, 300]] = 0.0
+    elif case == "huge_scale":
+        sx[[4, 270]] = np.float32(2.0 ** 120)             # acc * sx overflows to inf
+        sw[[9, 400]] = 0.0                                # inf * 0 = NaN
+    elif case == "nan_bias":
+        b[[11, 500]] = np.nan
+    q16 = t(Xq.astype(np.float16))
+    Y = u16(w8.linear_f16codes(q16, t(sx), t(Wq), t(sw), t(b)))
+    want = oracle_mod.linear(Xq, sx, Wq, sw, b)
+    nan_g = (Y & 0x7fff) > 0x7f80
+    nan_w = (want & 0x7fff) > 0x7f80
+    np.testing.assert_array_equal(nan_g, nan_w)
+    np.testing.assert_array_equal(Y[~nan_g], want[~nan_w])
+    if case != "finite":
+        assert nan_w.any()
