@@ -120,11 +120,33 @@ cudaError_t build_gelu_table();
 // memory; values outside it (rare) read the global table.
 constexpr uint32_t kGeluLo = 0x3A80u, kGeluN = 0x4200u - 0x3A80u;
 
-__device__ __forceinline__ float gelu_hot(const float *tab, uint32_t h16) {
-    h16 &= 0xffffu;
-    const uint32_t t = (h16 & 0x7fffu) - kGeluLo;          // wraps below the range
-    if (t < kGeluN) return tab[t + ((h16 & 0x8000u) ? kGeluN : 0u)];
-    return gelu_of_bits(h16);
+// GELU of the 8 bf16 values of a chunk (word q holds columns 2q, 2q+1, the
+// low half first).  Each value's table index is computed without a branch
+// (a value outside the hot range reads entry 0 for now), the 8 lookups go
+// out together, and only a chunk holding a value outside the range (rare)
+// takes the branch that reads those from the global table: a branch per
+// value cost more issue slots than the lookups themselves.
+__device__ __forceinline__ void gelu_chunk(const float *tab, const uint32_t (&wd)[4], float2 (&out)[4]) {
+    uint32_t h[8], idx[8];
+    bool all_hot = true;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+        h[e] = (e & 1) ? (wd[e >> 1] >> 16) : (wd[e >> 1] & 0xffffu);
+        const uint32_t t = (h[e] & 0x7fffu) - kGeluLo;      // wraps below the range
+        const bool hot = t < kGeluN;
+        all_hot = all_hot && hot;
+        idx[e] = hot ? t + (h[e] >> 15) * kGeluN : 0u;
+    }
+    float v[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) v[e] = tab[idx[e]];
+    if (!all_hot) {
+#pragma unroll
+        for (int e = 0; e < 8; ++e)
+            if ((h[e] & 0x7fffu) - kGeluLo >= kGeluN) v[e] = gelu_of_bits(h[e]);
+    }
+#pragma unroll
+    for (int q = 0; q < 4; ++q) out[q] = make_float2(v[2 * q], v[2 * q + 1]);
 }
 
 // Element e of a chunk as the pass reads it: the value, or GELU of it.
@@ -486,7 +508,7 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
     const uint32_t ring = static_cast<uint32_t>(__cvta_generic_to_shared(ring_s)) +
                           static_cast<uint32_t>((warp * S * U * 32 + lane) * 16);
 
-    // GELU: the hot range of the table in shared memory (see gelu_hot)
+    // GELU: the hot range of the table in shared memory (see gelu_chunk)
     __shared__ float gtab[GELU ? 2 * kGeluN : 1];
     const int gteam = blockIdx.x * kTeams + team;
     const bool second = gteam >= p.teams0;
@@ -549,10 +571,13 @@ act_quant_team_kernel(const __grid_constant__ ActParams p) {
             asm volatile("ld.shared.v4.u32 {%0,%1,%2,%3}, [%4];"
                          : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(slot + u * 32 * 16));
             const uint32_t wd[4] = {v.x, v.y, v.z, v.w};
+            if (GELU) {
+                gelu_chunk(gtab, wd, xs[u]);
+            } else {
 #pragma unroll
-            for (int q = 0; q < 4; ++q)
-                xs[u][q] = GELU ? make_float2(gelu_hot(gtab, wd[q]), gelu_hot(gtab, wd[q] >> 16))
-                                : make_float2(__uint_as_float(wd[q] << 16), __uint_as_float(wd[q] & 0xffff0000u));
+                for (int q = 0; q < 4; ++q)
+                    xs[u][q] = make_float2(__uint_as_float(wd[q] << 16), __uint_as_float(wd[q] & 0xffff0000u));
+            }
         }
 #pragma unroll
         for (int u = 0; u < U; ++u) {
