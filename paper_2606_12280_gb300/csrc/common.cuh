@@ -30,8 +30,8 @@ __device__ __forceinline__ int quantize_rne_clamp(float v) {
 
 // Two fp32 -> one bf16x2 word (lo in bits 0-15), both rounded to nearest
 // even by one conversion instruction: the same bits as two
-// f32_to_bf16_bits_rn calls for every input that is not a NaN (checked for
-// all 2^32 patterns in each half on GB300); a NaN becomes the canonical one
+// f32_to_bf16_bits_rn calls for every input that is not a NaN (a GPU test
+// checks all 2^32 patterns in each half); a NaN becomes the canonical one
 // instead of keeping its payload, so callers use it only where no value can
 // be a NaN.
 __device__ __forceinline__ uint32_t pack_bf16x2_cvt(float lo, float hi) {
