@@ -19,6 +19,7 @@
 #include <cuda.h>
 #include <cuda_runtime.h>
 
+#include "common.cuh"
 #include "host_once.h"
 #include "launch.h"
 #include "tc_ptx.cuh"
@@ -91,12 +92,6 @@ __device__ __forceinline__ void tile_mn(const Params &p, int t, int &m0, int &n0
     n0 = ni * PAIR_N;
 }
 
-__device__ __forceinline__ uint32_t bf16_rne_bits(float f) {
-    uint32_t u = __float_as_uint(f);
-    if ((u & 0x7fffffffu) > 0x7f800000u) return (u >> 16) | 0x40u;
-    u += 0x7fffu + ((u >> 16) & 1u);
-    return u >> 16;
-}
 
 __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint32_t tmem,
                                               const WaitCtx &wc, int warp, int lane,
@@ -141,7 +136,9 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
                         for (int i = 0; i < 4; ++i) {
                             const float y0 = __fadd_rn(__uint_as_float(v[8 * h + 2 * i]), b[8 * h + 2 * i]);
                             const float y1 = __fadd_rn(__uint_as_float(v[8 * h + 2 * i + 1]), b[8 * h + 2 * i + 1]);
-                            w[i] = bf16_rne_bits(y0) | (bf16_rne_bits(y1) << 16);
+                            // one conversion instruction per pair (round to
+                            // nearest even; a NaN becomes the canonical one)
+                            w[i] = pack_bf16x2_cvt(y0, y1);
                         }
                         *reinterpret_cast<uint4 *>(out + cc * 16 + 8 * h) = make_uint4(w[0], w[1], w[2], w[3]);
                     }
