@@ -49,20 +49,11 @@ __device__ __forceinline__ float epilogue_f32(float t, float sx, float sw, float
     return t;
 }
 
-// Dequantizing epilogue for one output from (float)acc: bf16((t * sx) * sw
-// + b), each step rounded to nearest even, no contraction.
-__device__ __forceinline__ uint32_t epilogue_value_f(float t, float sx, float sw, float b,
-                                                     bool has_bias) {
-    t = __fmul_rn(t, sx);
-    t = __fmul_rn(t, sw);
-    if (has_bias) t = __fadd_rn(t, b);
-    return f32_to_bf16_bits_rn(t);
-}
-
-// The same from the int32 accumulator: bf16(((float)acc * sx) * sw + b).
+// Dequantizing epilogue for one output from the int32 accumulator:
+// bf16(((float)acc * sx) * sw + b), each step rounded to nearest even.
 __device__ __forceinline__ uint32_t epilogue_value(int32_t acc, float sx, float sw,
                                                    float b, bool has_bias) {
-    return epilogue_value_f(__int2float_rn(acc), sx, sw, b, has_bias);
+    return f32_to_bf16_bits_rn(epilogue_f32(__int2float_rn(acc), sx, sw, b, has_bias));
 }
 
 constexpr int kMaxK = W8A8_MAX_K;

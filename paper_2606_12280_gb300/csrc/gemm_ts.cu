@@ -465,7 +465,8 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
                 // lanes 2i and 2i+1 (features f, f+1) swap one value per pair
                 // of tokens, so that each stores one 32-bit word: the even
                 // lane both features of the first token, the odd lane both of
-                // the second (N even: the word is 4-byte aligned).  No output
+                // the second (N is a multiple of 8, so the word is 4-byte
+                // aligned and both features of a pair are inside).  No output
                 // of the tile can be a NaN when every scale and the bias are
                 // finite and |sx| <= 2^96 (a product may overflow, but inf
                 // times a finite nonzero scale plus a finite bias stays
@@ -478,7 +479,6 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
                 const bool odd = lane & 1;
                 const int fw = f & ~1;
                 uint16_t *out = static_cast<uint16_t *>(br.out) + (size_t)tok0 * p.N + fw;
-                const bool paired = (p.N & 1) == 0;
                 const bool fast_cvt = __all_sync(0xffffffffu, sx_ok && fabsf(sw) <= 3.402823466e38f &&
                                                                    (!hb || fabsf(b) <= 3.402823466e38f));
                 auto store_pairs = [&](auto fast_tag) {
@@ -506,24 +506,8 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
                         }
                     }
                 };
-                if (paired) {
-                    if (fast_cvt) store_pairs(std::true_type{});
-                    else store_pairs(std::false_type{});
-                } else {
-#pragma unroll
-                    for (int i = 0; i < RUN; i += 4) {
-                        const uint4 s4 = ld_shared_v4(epi + 4 * i);
-                        const float sxv[4] = {__uint_as_float(s4.x), __uint_as_float(s4.y), __uint_as_float(s4.z),
-                                              __uint_as_float(s4.w)};
-                        uint16_t *o = out + (f - fw);
-#pragma unroll
-                        for (int u = 0; u < 4; ++u) {
-                            const uint32_t y = epilogue_value_f(__uint_as_float(static_cast<uint32_t>(run[i + u])),
-                                                                sxv[u], sw, b, hb);
-                            if (fok && i + u < ntok) o[(size_t)(i + u) * p.N] = static_cast<uint16_t>(y);
-                        }
-                    }
-                }
+                if (fast_cvt) store_pairs(std::true_type{});
+                else store_pairs(std::false_type{});
             }
         }
         __syncwarp();
