@@ -468,9 +468,9 @@ __device__ __forceinline__ void epilogue_role(const Params &p, uint32_t sb, uint
                 // the second (N is a multiple of 8, so the word is 4-byte
                 // aligned and both features of a pair are inside).  No output
                 // of the tile can be a NaN when every scale and the bias are
-                // finite and |sx| <= 2^96 (a product may overflow, but inf
-                // times a finite nonzero scale plus a finite bias stays
-                // infinite): each pair is then rounded to bf16 by one
+                // finite and |sx| <= 2^96: acc * sx is then finite, times sw
+                // it may overflow to an infinity, and a finite bias leaves
+                // that infinite.  Each pair is then rounded to bf16 by one
                 // conversion instruction.  The epilogue shares the SM's issue
                 // slots with the converters, and rounding every value with
                 // integer operations made the whole GEMM ~5 % slower; tiles
