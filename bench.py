@@ -559,12 +559,18 @@ def run_ours(args):
     torch.cuda.synchronize()
     if ws > 1:
         torch.distributed.barrier()
-    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    a.record(runner.up)
-    runner.run([X_host] * e2e_steps, [Y_hosts[i % depth] for i in range(e2e_steps)])
-    b.record(runner.down)
-    torch.cuda.synchronize()
-    e2e_ms = max_over_ranks(a.elapsed_time(b), ws, dev)
+    # three passes, the median reported: the host link and the host's own
+    # memory are shared with the machine's other jobs, and one pass now and
+    # then ran at half speed
+    e2e_pass_ms = []
+    for _ in range(3):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(runner.up)
+        runner.run([X_host] * e2e_steps, [Y_hosts[i % depth] for i in range(e2e_steps)])
+        b.record(runner.down)
+        torch.cuda.synchronize()
+        e2e_pass_ms.append(a.elapsed_time(b))
+    e2e_ms = max_over_ranks(sorted(e2e_pass_ms)[1], ws, dev)
     e2e_value = sum_over_ranks(ops_step * e2e_steps, ws, dev) / (e2e_ms * 1e-3) / 1e12
     del runner
 
@@ -1033,6 +1039,7 @@ def run_ours(args):
             "cpu_baseline": cpu,
             "e2e": {"value": e2e_value, "unit": "TOPS", "h2d_bytes_per_step": 2 * M * K,
                     "d2h_bytes_per_step": 2 * M * N, "steps": e2e_steps,
+                    "pass_ms": e2e_pass_ms, "how": "median of three passes of the streamed steps",
                     "mode": "streamed: upload, compute, download on three streams, two buffer sets",
                     "serial_value": e2e_serial},
             "gpu_launches": 2 * args.steps,
