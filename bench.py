@@ -552,8 +552,8 @@ def run_ours(args):
     e2e_steps = max(4, args.steps)      # the same step count as the timed region
     depth = 2
     Y_hosts = [torch.empty(M, N, dtype=torch.bfloat16).pin_memory() for _ in range(depth)]
-    runner = StreamedLinear(M, K, N, lam, Wq, sw, bias, depth=depth, device=dev,
-                            plan=plan if f16 else None, codes=args.codes)
+    runner = StreamedLinear(M, K, N, lam, Wq, sw, bias, depth=depth, device=dev, plan=plan,
+                            codes=args.codes)
     runner.run([X_host] * depth, Y_hosts)
     runner.synchronize()
     torch.cuda.synchronize()
@@ -576,11 +576,12 @@ def run_ours(args):
 
     Y_host = Y_hosts[0]
     Xd = torch.empty(M, K, dtype=torch.bfloat16, device=dev)
+    serial_ws = _lin_ws(dev, M, K)
 
     def e2e_serial_step():
         Xd.copy_(X_host, non_blocking=True)
-        Y = w8a8.quantized_linear_forward(Xd, lam, Wq, sw, bias, plan=plan if f16 else None,
-                                          codes=args.codes, stream=stream)
+        Y = w8a8.quantized_linear_forward(Xd, lam, Wq, sw, bias, plan=plan, codes=args.codes,
+                                          workspace=serial_ws, stream=stream)
         Y_host.copy_(Y, non_blocking=True)
 
     for _ in range(2):

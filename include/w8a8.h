@@ -71,7 +71,9 @@ typedef enum {
     W8A8_ERR_TIMEOUT = 5
 } w8a8_status;
 
-/* Largest K for which K * 127 * 127 < 2^31. */
+/* A bound on K under which K * 127 * 127 < 2^31 (every |acc| of codes in
+ * [-127, 127] fits int32); with K a multiple of 16 the largest accepted K is
+ * 133136. */
 #define W8A8_MAX_K 133143
 
 /* Human-readable name of a status code (static storage, never NULL). */

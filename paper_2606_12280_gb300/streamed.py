@@ -26,7 +26,10 @@ class StreamedLinear:
     def __init__(self, M: int, K: int, N: int, smooth, Wq, w_scale, bias=None, depth: int = 2,
                  device=None, plan=None, codes: str = "f16"):
         """codes: "f16" (a3 writes the codes as fp16 values and the GEMM takes
-        them unconverted; plan = ``w8a8.chunk_plan(Wq)`` or None) or "int8"."""
+        them unconverted) or "int8" (the int8 container; the GEMM call gets a
+        workspace and expands the codes first).  plan: ``w8a8.chunk_plan(Wq)``
+        or None.  One workspace serves every buffer set: the GEMMs run in
+        order on one stream."""
         if codes not in ("f16", "int8"):
             raise ValueError("codes must be 'f16' or 'int8'")
         self.M, self.K, self.N = M, K, N
@@ -39,6 +42,7 @@ class StreamedLinear:
                    for _ in range(depth)]
         self.sx = [torch.empty(M, dtype=torch.float32, device=dev) for _ in range(depth)]
         self.ss = [torch.empty(M, dtype=torch.int32, device=dev) for _ in range(depth)] if self.f16 else None
+        self.ws = None if self.f16 else w8a8.linear_workspace(M, K, device=dev)
         self.Y = [torch.empty(M, N, dtype=torch.bfloat16, device=dev) for _ in range(depth)]
         self.up = torch.cuda.Stream(device=dev)
         self.comp = torch.cuda.Stream(device=dev)
@@ -81,7 +85,7 @@ class StreamedLinear:
                                          stream=self.comp)
                 else:
                     w8a8.linear(self.Xq[s], self.sx[s], self.Wq, self.w_scale, self.bias, Y=self.Y[s],
-                                stream=self.comp)
+                                plan=self.plan, workspace=self.ws, stream=self.comp)
                 self.y_ready[s].record(self.comp)
             with torch.cuda.stream(self.down):
                 self.down.wait_event(self.y_ready[s])

@@ -749,16 +749,25 @@ def select_protected(scores, n_protect: int):
     return [int(f) for f in flags]
 
 
-def quantized_linear_forward(X, smooth, Wq, w_scale, bias=None, plan=None, codes="f16", stream=None):
+def quantized_linear_forward(X, smooth, Wq, w_scale, bias=None, plan=None, codes="f16", workspace=None,
+                             stream=None):
     """The per-call hot path of one quantized linear: a3 then a4+a5.  codes:
     "f16" (the codes as fp16 values, the faster GEMM; K <= 16384, else the
-    int8 container is used) or "int8"; plan: ``chunk_plan(Wq)`` or None (used
-    with fp16 codes)."""
+    int8 container is used) or "int8"; plan: ``chunk_plan(Wq)`` or None;
+    workspace: None, or ``linear_workspace(M, K)`` (the int8 container's
+    faster GEMM; the fp16 codes use its split-K area).  Same bits in every
+    combination."""
     if codes not in ("f16", "int8"):
         raise ValueError("codes must be 'f16' or 'int8'")
-    if codes == "f16" and X.shape[1] <= 16384:
-        ss = torch.empty(X.shape[0], dtype=torch.int32, device=X.device) if plan is not None else None
+    M, K = X.shape
+    if codes == "f16" and K <= 16384:
+        ss = torch.empty(M, dtype=torch.int32, device=X.device) if plan is not None else None
         Xq16, sx = quant_act_f16codes(X, smooth, sumsq=ss, stream=stream)
-        return linear_f16codes(Xq16, sx, Wq, w_scale, bias, plan=plan, x_sumsq=ss, stream=stream)
+        gws = None
+        if workspace is not None:
+            _linear_ws(workspace, M, K)
+            gws = workspace
+        return linear_f16codes(Xq16, sx, Wq, w_scale, bias, plan=plan, x_sumsq=ss, workspace=gws,
+                               stream=stream)
     Xq, sx = quant_act(X, smooth, stream=stream)
-    return linear(Xq, sx, Wq, w_scale, bias, stream=stream)
+    return linear(Xq, sx, Wq, w_scale, bias, plan=plan, workspace=workspace, stream=stream)

@@ -8,8 +8,9 @@ on both engines, so the bar is bitwise: the int32 product equals the int64
 product of the codes (including -128, which a3 never writes but the int8
 container holds), Y equals the oracle and the call without a workspace, and
 the dual call equals two single calls.  The cases cover ragged M and N, a
-ragged last K chunk, K = 16384, partial sums near 2^24, fewer tiles than CTA
-pairs, an empty branch, and a workspace reused across calls.
+ragged last K chunk, K = 16384, the largest accepted K (products at the int32
+limit), partial sums near 2^24, fewer tiles than CTA pairs, an empty branch,
+and a workspace reused across calls.
 """
 
 import numpy as np
@@ -128,6 +129,53 @@ def test_qkv_shape_equals_unsplit(w8):
     assert torch.equal(acc1, acc0)
     assert split_counters_zero(w8, ws)
     assert w8.device_status() == 0
+
+
+@pytest.mark.parametrize("kind", ["random", "edge"])
+def test_int32_exact_largest_k(w8, kind):
+    # K = 133136, the largest accepted K: 127^2 K = 2147350544 is 133103 below
+    # 2^31 - 1, so the "edge" products sit at the int32 limit, of either sign
+    M, N, K = 130, 136, 133136
+    rng = np.random.default_rng(kind == "edge")
+    if kind == "random":
+        Xq = rng.integers(-127, 128, (M, K), dtype=np.int8)
+        Wq = rng.integers(-127, 128, (N, K), dtype=np.int8)
+    else:
+        Xq = np.full((M, K), 127, np.int8)
+        Xq[::2] = -127
+        Wq = np.full((N, K), 127, np.int8)
+        Wq[1::3] = -127
+    # every partial sum is an integer below 2^53: the float64 product is exact
+    want = (Xq.astype(np.float64) @ Wq.astype(np.float64).T).astype(np.int64)
+    if kind == "edge":
+        assert np.abs(want).max() == 127 * 127 * K and want.min() == -127 * 127 * K
+    plan = w8.chunk_plan(t(Wq))
+    ws = w8.linear_workspace(M, K)
+    for kw in ({}, {"plan": plan}, {"workspace": ws}, {"plan": plan, "workspace": ws}):
+        acc = w8.debug_gemm_i32(t(Xq), t(Wq), **kw)
+        np.testing.assert_array_equal(acc.cpu().numpy(), want)
+    assert split_counters_zero(w8, ws)
+    assert w8.device_status() == 0
+
+
+def test_layer_forward_largest_k(w8, oracle_mod):
+    # K > 16384: a3 writes int8 codes (fp16 codes are limited to K <= 16384)
+    # and the workspace call expands them before the GEMM
+    M, N, K = 70, 136, 133136
+    c = wl.make_case(M, K, N, seed=29, calib_tokens=32)
+    s = oracle_mod.channel_absmax(c.X_cal)
+    lam = oracle_mod.smooth_scales(s, c.W[0], c.alpha)
+    Wq, sw = oracle_mod.quantize_weights(c.W[0], lam)
+    Xq_ref, sx_ref = oracle_mod.quant_act(c.X[0], lam)
+    want = oracle_mod.linear(Xq_ref, sx_ref, Wq, sw, c.bias[0])
+    args = dict(smooth=t(lam), Wq=t(Wq), w_scale=t(sw), bias=t(c.bias[0]))
+    Y0 = w8.layer_forward(bf(c.X[0]), False, N, K, **args)
+    np.testing.assert_array_equal(u16(Y0), want)
+    ws = w8.linear_workspace(M, K)
+    for _ in range(2):                                          # the workspace is reused
+        Y1 = w8.layer_forward(bf(c.X[0]), False, N, K, plan=w8.chunk_plan(t(Wq)), workspace=ws, **args)
+        assert torch.equal(Y1, Y0)
+    assert split_counters_zero(w8, ws)
 
 
 @pytest.mark.parametrize("M0,M1", [(300, 130), (2000, 800), (0, 257), (513, 0)])

@@ -1,5 +1,6 @@
 """The streamed runner (three streams, double-buffered device tensors) gives
-bitwise the same outputs as calling the layer batch by batch."""
+bitwise the same outputs as calling the layer batch by batch, with either code
+container, with and without a drain plan and a workspace."""
 
 import numpy as np
 import pytest
@@ -10,8 +11,8 @@ from paper_2606_12280_gb300 import workloads as wl
 pytestmark = pytest.mark.gpu
 
 
-@pytest.mark.parametrize("codes", ["f16", "int8"])
-def test_streamed_matches_direct(codes):
+@pytest.mark.parametrize("codes,with_plan", [("f16", True), ("int8", True), ("int8", False)])
+def test_streamed_matches_direct(codes, with_plan):
     if not torch.cuda.is_available():
         pytest.skip("no CUDA device")
     from paper_2606_12280_gb300 import w8a8
@@ -27,7 +28,7 @@ def test_streamed_matches_direct(codes):
     batches = [torch.from_numpy(wl.random_bf16((M, K), seed=100 + i, scale=1.0 + i).view(np.int16))
                .view(torch.bfloat16).pin_memory() for i in range(5)]
     outs = [torch.empty(M, N, dtype=torch.bfloat16).pin_memory() for _ in range(5)]
-    plan = w8a8.chunk_plan(Wq) if codes == "f16" else None
+    plan = w8a8.chunk_plan(Wq) if with_plan else None
     r = StreamedLinear(M, K, N, lam, Wq, sw, bias, depth=2, plan=plan, codes=codes)
     r.run(batches, outs)
     r.synchronize()
@@ -35,6 +36,9 @@ def test_streamed_matches_direct(codes):
         want = w8a8.quantized_linear_forward(xh.to(dev), lam, Wq, sw, bias, plan=plan, codes=codes)
         other = w8a8.quantized_linear_forward(xh.to(dev), lam, Wq, sw, bias,
                                               codes="int8" if codes == "f16" else "f16")
+        with_ws = w8a8.quantized_linear_forward(xh.to(dev), lam, Wq, sw, bias, plan=plan, codes=codes,
+                                                workspace=w8a8.linear_workspace(M, K))
         torch.cuda.synchronize()
         assert torch.equal(yh, want.cpu())
         assert torch.equal(want, other)
+        assert torch.equal(want, with_ws)
