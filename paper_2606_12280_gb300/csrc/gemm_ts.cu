@@ -875,11 +875,13 @@ __global__ void __launch_bounds__(kExpandThreads)
 expand_codes_kernel(const __grid_constant__ ExpandBranch b0, const __grid_constant__ ExpandBranch b1, int K) {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
     const int lane = threadIdx.x & 31;
-    int row = (blockIdx.x * kExpandThreads + threadIdx.x) >> 5;
-    const bool second = row >= b0.M;
+    // one warp per row, the row index in 64 bits (the grid grows with M0 + M1)
+    long long r = (static_cast<long long>(blockIdx.x) * kExpandThreads + threadIdx.x) >> 5;
+    const bool second = r >= b0.M;
     const ExpandBranch &b = second ? b1 : b0;
-    if (second) row -= b0.M;
-    if (row >= b.M) return;                           // whole warps leave together
+    if (second) r -= b0.M;
+    if (r >= b.M) return;                             // whole warps leave together
+    const int row = static_cast<int>(r);
     const int n8 = K / 8;                             // 8-code groups per row
     const uint2 *src = reinterpret_cast<const uint2 *>(b.Xq + (size_t)row * K);
     uint4 *dst = reinterpret_cast<uint4 *>(b.Xq16 + (size_t)row * K);
