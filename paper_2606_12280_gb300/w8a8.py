@@ -245,11 +245,12 @@ def linear(Xq, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, workspace=Non
     _room(Y, M * N, "Y")
     if plan is not None:
         _room(plan, chunk_plan_size(N, K), "plan")
+    ws = _linear_ws(workspace, M, K)
     _check("w8a8_linear", lib().w8a8_linear(
         _ptr(Xq, torch.int8, "Xq"), _ptr(x_scale, torch.float32, "x_scale"),
         _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
         _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(Y, torch.bfloat16, "Y"),
-        _ptr(plan, torch.int32, "plan"), _linear_ws(workspace, M, K), _stream(stream)))
+        _ptr(plan, torch.int32, "plan"), ws, _stream(stream)))
     return Y
 
 
@@ -310,10 +311,10 @@ def linear_dual(branches, Ys=None, workspace=None, stream=None):
     ``linear_workspace(M0 + M1, K)``; returns [Y_cond, Y_uncond]."""
     if len(branches) != 2:
         raise ValueError("linear_dual takes exactly two branches")
-    arr, out, N, K = _branch_array(branches, Ys)
     tokens = sum(int(br[0].shape[0]) for br in branches)
-    _check("w8a8_linear_dual", lib().w8a8_linear_dual(arr, N, K, _linear_ws(workspace, tokens, K),
-                                                       _stream(stream)))
+    ws = _linear_ws(workspace, tokens, int(branches[0][0].shape[1]))
+    arr, out, N, K = _branch_array(branches, Ys)
+    _check("w8a8_linear_dual", lib().w8a8_linear_dual(arr, N, K, ws, _stream(stream)))
     return out
 
 
@@ -328,10 +329,10 @@ def debug_gemm_i32(Xq, Wq, acc=None, plan=None, workspace=None, stream=None):
     _room(acc, M * N, "acc")
     if plan is not None:
         _room(plan, chunk_plan_size(N, K), "plan")
+    ws = _linear_ws(workspace, M, K)
     _check("w8a8_debug_gemm_i32", lib().w8a8_debug_gemm_i32(
         _ptr(Xq, torch.int8, "Xq"), _ptr(Wq, torch.int8, "Wq"), M, N, K,
-        _ptr(acc, torch.int32, "acc"), _ptr(plan, torch.int32, "plan"), _linear_ws(workspace, M, K),
-        _stream(stream)))
+        _ptr(acc, torch.int32, "acc"), _ptr(plan, torch.int32, "plan"), ws, _stream(stream)))
     return acc
 
 
@@ -428,6 +429,7 @@ def linear_dual_f16codes(branches, Ys=None, workspace=None, stream=None):
     ``gemm_workspace()`` (see ``linear_f16codes``)."""
     if len(branches) != 2:
         raise ValueError("linear_dual_f16codes takes exactly two branches")
+    ws = _workspace(workspace)
     N, K = branches[0][2].shape
     arr = (Branch16 * 2)()
     out = []
@@ -449,8 +451,7 @@ def linear_dual_f16codes(branches, Ys=None, workspace=None, stream=None):
                           _ptr(b, torch.float32, "bias"), _ptr(Y, torch.bfloat16, "Y"), Xq16.shape[0],
                           _ptr(plan, torch.int32, "plan"), _ptr(ss, torch.int32, "x_sumsq"))
         out.append(Y)
-    _check("w8a8_linear_dual_f16codes", lib().w8a8_linear_dual_f16codes(arr, N, K, _workspace(workspace),
-                                                                         _stream(stream)))
+    _check("w8a8_linear_dual_f16codes", lib().w8a8_linear_dual_f16codes(arr, N, K, ws, _stream(stream)))
     return out
 
 
@@ -509,12 +510,12 @@ def linear_f16codes(Xq16, x_scale, Wq, w_scale, bias=None, Y=None, plan=None, x_
         _room(plan, chunk_plan_size(N, K), "plan")
     _room(x_sumsq, M, "x_sumsq")
     _room(Y, M * N, "Y")
+    ws = _workspace(workspace)
     _check("w8a8_linear_f16codes", lib().w8a8_linear_f16codes(
         _ptr(Xq16, torch.float16, "Xq16"), _ptr(x_scale, torch.float32, "x_scale"),
         _ptr(Wq, torch.int8, "Wq"), _ptr(w_scale, torch.float32, "w_scale"),
         _ptr(bias, torch.float32, "bias"), M, N, K, _ptr(plan, torch.int32, "plan"),
-        _ptr(x_sumsq, torch.int32, "x_sumsq"), _ptr(Y, torch.bfloat16, "Y"), _workspace(workspace),
-        _stream(stream)))
+        _ptr(x_sumsq, torch.int32, "x_sumsq"), _ptr(Y, torch.bfloat16, "Y"), ws, _stream(stream)))
     return Y
 
 
@@ -529,10 +530,11 @@ def debug_gemm_f16codes_i32(Xq16, Wq, plan=None, x_sumsq=None, acc=None, workspa
         _room(plan, chunk_plan_size(N, K), "plan")
     _room(x_sumsq, M, "x_sumsq")
     _room(acc, M * N, "acc")
+    ws = _workspace(workspace)
     _check("w8a8_debug_gemm_f16codes_i32", lib().w8a8_debug_gemm_f16codes_i32(
         _ptr(Xq16, torch.float16, "Xq16"), _ptr(Wq, torch.int8, "Wq"), M, N, K,
         _ptr(plan, torch.int32, "plan"), _ptr(x_sumsq, torch.int32, "x_sumsq"),
-        _ptr(acc, torch.int32, "acc"), _workspace(workspace), _stream(stream)))
+        _ptr(acc, torch.int32, "acc"), ws, _stream(stream)))
     return acc
 
 
@@ -760,14 +762,11 @@ def quantized_linear_forward(X, smooth, Wq, w_scale, bias=None, plan=None, codes
     if codes not in ("f16", "int8"):
         raise ValueError("codes must be 'f16' or 'int8'")
     M, K = X.shape
+    _linear_ws(workspace, M, K)                 # checked before anything is launched
     if codes == "f16" and K <= 16384:
         ss = torch.empty(M, dtype=torch.int32, device=X.device) if plan is not None else None
         Xq16, sx = quant_act_f16codes(X, smooth, sumsq=ss, stream=stream)
-        gws = None
-        if workspace is not None:
-            _linear_ws(workspace, M, K)
-            gws = workspace
-        return linear_f16codes(Xq16, sx, Wq, w_scale, bias, plan=plan, x_sumsq=ss, workspace=gws,
+        return linear_f16codes(Xq16, sx, Wq, w_scale, bias, plan=plan, x_sumsq=ss, workspace=workspace,
                                stream=stream)
     Xq, sx = quant_act(X, smooth, stream=stream)
     return linear(Xq, sx, Wq, w_scale, bias, plan=plan, workspace=workspace, stream=stream)

@@ -31,6 +31,9 @@ def e(n, dt):
 
 def cases(w8):
     P = w8.chunk_plan_size(N, K)
+    LW, GW = w8.linear_workspace_size(M, K), w8.gemm_workspace_size()
+    # the split-K area is sized by the device's SM count: 0 bytes without a GPU
+    gw = {"workspace": (GW, u8)} if GW > 0 else {}
     G0, G1 = N * (K // 32) * 34, N * (256 // 256) * 144
     X, W, Xq, Wq, X16 = e((M, K), bf16), e((N, K), f32), e((M, K), i8), e((N, K), i8), e((M, K), f16)
     # (function, positional args, {sized keyword: (numel, dtype)})
@@ -40,13 +43,16 @@ def cases(w8):
         (w8.quantize_weights, (W,), {"smooth": (K, f32), "Wq": (N * K, i8), "w_scale": (N, f32)}),
         (w8.quant_act, (X,), {"smooth": (K, f32), "Xq": (M * K, i8), "x_scale": (M, f32)}),
         (w8.linear, (Xq, e(M, f32), Wq, e(N, f32)), {"bias": (N, f32), "Y": (M * N, bf16)}),
+        (w8.linear, (Xq, e(M, f32), Wq, e(N, f32)), {"Y": (M * N, bf16), "plan": (P, i32), "workspace": (LW, u8)}),
         (w8.debug_gemm_i32, (Xq, Wq), {"acc": (M * N, i32)}),
+        (w8.debug_gemm_i32, (Xq, Wq), {"acc": (M * N, i32), "workspace": (LW, u8)}),
         (w8.gelu_quant_act, (X,), {"smooth": (K, f32), "Xq": (M * K, i8), "x_scale": (M, f32)}),
         (w8.quant_act_f16codes, (X,), {"smooth": (K, f32), "Xq16": (M * K, f16), "x_scale": (M, f32),
                                        "sumsq": (M, i32)}),
         (w8.linear_f16codes, (X16, e(M, f32), Wq, e(N, f32)), {"bias": (N, f32), "Y": (M * N, bf16),
-                                                             "plan": (P, i32), "x_sumsq": (M, i32)}),
-        (w8.debug_gemm_f16codes_i32, (X16, Wq), {"plan": (P, i32), "x_sumsq": (M, i32), "acc": (M * N, i32)}),
+                                                             "plan": (P, i32), "x_sumsq": (M, i32), **gw}),
+        (w8.debug_gemm_f16codes_i32, (X16, Wq), {"plan": (P, i32), "x_sumsq": (M, i32), "acc": (M * N, i32),
+                                                 **gw}),
         (w8.chunk_plan, (Wq,), {"plan": (P, i32)}),
         (w8.linear_gguf, (e((M, K), bf16), e(G0, u8), 0, N), {"bias": (N, f32), "Y": (M * N, bf16)}),
         (w8.linear_gguf, (e((M, 256), bf16), e(G1, u8), 1, N), {"Y": (M * N, bf16)}),
@@ -62,6 +68,10 @@ def cases(w8):
                                               "bias": (N, f32), "Xq_work": (M * K, i8),
                                               "x_scale_work": (M, f32), "Y": (M * N, bf16)}),
         (w8.layer_forward, (X, True, N, K), {"W_bf16": (N * K, bf16), "bias": (N, f32), "Y": (M * N, bf16)}),
+        (w8.layer_forward, (X, False, N, K), {"smooth": (K, f32), "Wq": (N * K, i8), "w_scale": (N, f32),
+                                              "x_scale_work": (M, f32), "Y": (M * N, bf16), "plan": (P, i32),
+                                              "workspace": (LW, u8)}),
+        (w8.quantized_linear_forward, (X, e(K, f32), Wq, e(N, f32)), {"workspace": (LW, u8)}),
     ]
 
 
